@@ -1,0 +1,22 @@
+"""Float64 CPU oracle for Jacap's eviction pass (test infrastructure only).
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU legs may
+import this package. The CUDA library never uses it.
+"""
+
+from .jacap_oracle import (  # noqa: F401
+    JacapParams,
+    window_stats,
+    pool_attention,
+    sensitivity,
+    response_variance,
+    head_weight,
+    unit_weights,
+    capacity_matrix,
+    jacap_scores,
+    select_topb,
+    compact,
+    oracle_unit,
+    oracle_pass,
+    unit_views,
+)
