@@ -1,0 +1,419 @@
+#!/usr/bin/env python
+"""Throughput of Jacap's prefill eviction pass on GB300; prints ONE JSON line.
+
+A step is one whole pass (jacap_score + jacap_select + jacap_compact: every
+row of the hot path) over one synthetic Llama-3-8B-shaped cache (32 layers,
+32 query / 8 KV heads, head_dim 128, n = 32768, w = 32, B = 512, bf16), with
+the inputs resident in HBM. The metric is evicted-cache tokens per second per
+layer-pass, sum_s n_s * L / t_step, summed over ranks.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--budget B] [--config C]
+  python bench.py --impl reference ...   # the float64 CPU oracle, bounded sample
+
+Under torchrun every rank evicts its own cache of the same shape (weak
+scaling, no collective on the data path); the time is the max over ranks.
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "evicted-cache tokens/s per layer-pass (1 GB300) and % of HBM roofline"
+UNIT = "tokens/s"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=500)
+    p.add_argument("--warmup", type=int, default=10)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--config", type=int, default=2)
+    p.add_argument("--budget", type=int, default=None)
+    p.add_argument("--e2e-steps", type=int, default=10)
+    p.add_argument("--cpu-seconds", type=float, default=15.0)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-e2e", action="store_true")
+    return p.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while running."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "20"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.1)
+        self.proc.terminate()
+        self.proc.wait()
+        rows = []
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) == 8:
+                rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+
+        sm = [num(r[0]) for r in rows if num(r[0]) is not None]
+        mx = [num(r[1]) for r in rows if num(r[1]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[4 + i].lower() == "active"})
+        pw = [num(r[2]) for r in rows if num(r[2]) is not None]
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows), "power_w_max": max(pw) if pw else None}
+
+
+def workload_config(wl, budget, gpus):
+    return {
+        "workload": wl.name,
+        "layers": wl.num_layers,
+        "q_heads": wl.num_q_heads,
+        "kv_heads": wl.num_kv_heads,
+        "head_dim": wl.head_dim,
+        "seqlens": list(wl.seqlens) if len(wl.seqlens) <= 4 else f"{len(wl.seqlens)} requests, sum {wl.total_tokens}",
+        "window": wl.window,
+        "budget": budget,
+        "tau": 10.0,
+        "cache_dtype": wl.dtype,
+        "l2": "inputs larger than L2: each step streams the whole cache (K and V alone are "
+              f"{2 * wl.num_layers * wl.num_kv_heads * wl.total_tokens * wl.head_dim * (2 if wl.dtype == 'bf16' else 4) / 1e9:.2f} GB)",
+        "parallelism": f"{gpus} independent replica(s), one cache per GPU",
+    }
+
+
+# ------------------------------------------------------------------ oracle --
+def oracle_sample(wl, budget, seconds, device, tensors=None):
+    """Time the float64 oracle on whole units of the workload for ~`seconds`.
+
+    Returns (tokens_layers_per_s, sample_description, wall_s)."""
+    from oracle import JacapParams, oracle_unit
+    from paper_2609_08131_gb300.workloads import fill_unit, unit_arrays
+
+    units = [(s, l, g) for l in range(wl.num_layers) for g in range(wl.num_kv_heads) for s in range(len(wl.seqlens))]
+    done, tok, t_total = 0, 0, 0.0
+    for (s, l, g) in units:
+        n = wl.seqlens[s]
+        if tensors is not None:
+            q, K, V = unit_arrays(tensors, wl.num_q_heads, s, l, g)
+        else:
+            k, v, qq = fill_unit(wl, s, l, g, n, "cpu")
+            dt = wl.torch_dtype
+            q = qq.to(dt).double().numpy()
+            K = k.to(dt).double().numpy()
+            V = v.to(dt).double().numpy()
+        t0 = time.perf_counter()
+        oracle_unit(q, K, V, budget, JacapParams())
+        t_total += time.perf_counter() - t0
+        done += 1
+        tok += n
+        if t_total >= seconds:
+            break
+    # tokens x layers: a unit is one (layer, KV head) of a request, i.e. 1/Hkv of a layer-pass
+    value = tok / wl.num_kv_heads / t_total
+    desc = f"{done} whole unit(s) (request, layer, KV head) of {tok} tokens in total, float64 numpy"
+    return value, desc, t_total
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    from oracle import JacapParams, oracle_unit
+    from paper_2609_08131_gb300.workloads import config, fill_unit
+
+    wl = config(args.config)
+    budget = args.budget or wl.budget
+    # per-step sample: a prefix of one unit, sized so K + W steps take ~150 s
+    n_full = wl.seqlens[0]
+    k, v, q = fill_unit(wl, 0, 0, 0, n_full, "cpu")
+    dt = wl.torch_dtype
+    K64, V64, Q64 = k.to(dt).double().numpy(), v.to(dt).double().numpy(), q.to(dt).double().numpy()
+    t0 = time.perf_counter()
+    oracle_unit(Q64, K64[:2048], V64[:2048], budget, JacapParams())
+    per_tok = (time.perf_counter() - t0) / 2048
+    target = 150.0 / max(1, args.steps + args.warmup)
+    m = int(max(256, min(n_full, target / per_tok)))
+    for _ in range(args.warmup):
+        oracle_unit(Q64, K64[:m], V64[:m], budget, JacapParams())
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        oracle_unit(Q64, K64[:m], V64[:m], budget, JacapParams())
+        times.append(time.perf_counter() - t0)
+    avg = sum(times) / len(times)
+    value = m / wl.num_kv_heads / avg
+    sample = (f"each step: the float64 oracle on the first {m} tokens of one (layer, KV head) unit of the workload "
+              f"(a sub-cache of {m} tokens); tokens x layers = {m}/{wl.num_kv_heads} per step")
+    line = {
+        "impl": "reference",
+        "metric": METRIC,
+        "value": value,
+        "unit": UNIT,
+        "n_gpus": args.gpus,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": avg * 1e3,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f64",
+        "data": "synthetic",
+        "config": workload_config(wl, budget, args.gpus),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
+# -------------------------------------------------------------------- ours --
+def run_ours(args):
+    import torch
+
+    from paper_2609_08131_gb300 import SCORE_KERNEL_NAMES
+    from paper_2609_08131_gb300.api import Cache, Evictor
+    from paper_2609_08131_gb300.workloads import config, generate
+    from dataclasses import replace
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+
+    wl = config(args.config)
+    budget = args.budget or wl.budget
+    wl = replace(wl, seed=wl.seed + 1000 * rank, budget=budget)
+    t = generate(wl, dev)
+    cache = Cache(t.q_win, t.k, t.v, t.cu_seqlens, t.seqlens, wl.num_q_heads)
+    ev = Evictor(cache, budget)
+    stream = torch.cuda.current_stream(dev)
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+
+    for _ in range(max(3, args.warmup)):
+        ev.run()
+    ev.check()
+
+    K = args.steps
+    nk = len(SCORE_KERNEL_NAMES)
+    ev_score = [[torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)] for _ in range(K)]
+    ev_tail = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(K)]
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(local)
+    barrier()
+    torch.cuda.synchronize()
+    sampler.start()
+    start.record(stream)
+    for i in range(K):
+        ev.score(events=ev_score[i])
+        ev.select()
+        ev_tail[i][0].record(stream)
+        ev.compact()
+        ev_tail[i][1].record(stream)
+    stop.record(stream)
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    barrier()
+    ev.check()
+    t_ms = start.elapsed_time(stop) / K
+    if dist is not None:
+        x = torch.tensor([t_ms], device=dev)
+        dist.all_reduce(x, op=dist.ReduceOp.MAX)
+        t_ms = float(x.item())
+
+    # per-kernel average durations inside the timed region
+    kern = {name: 0.0 for name in SCORE_KERNEL_NAMES}
+    kern["select"] = 0.0
+    kern["compact"] = 0.0
+    for i in range(K):
+        for j, name in enumerate(SCORE_KERNEL_NAMES):
+            kern[name] += ev_score[i][j].elapsed_time(ev_score[i][j + 1])
+        kern["select"] += ev_score[i][nk].elapsed_time(ev_tail[i][0])
+        kern["compact"] += ev_tail[i][0].elapsed_time(ev_tail[i][1])
+    kern = {k: v / K for k, v in kern.items()}
+
+    L, Hkv, N, d = t.k.shape
+    es = t.k.element_size()
+    kv_bytes = L * Hkv * N * d * es
+    kept_rows = L * Hkv * sum(min(n, budget) for n in t.seqlens)
+    alg_kernel = {
+        "k_pass": kv_bytes,                       # K read once
+        "weight_gram": kv_bytes,                  # V read once
+        "scores": kv_bytes + L * Hkv * N * 4,     # V read, scores written
+        "select": L * Hkv * N * 4,                # scores read
+        "compact": 4 * kept_rows * d * es,        # retained K, V read and written
+    }
+    dom = max(alg_kernel, key=lambda k: kern[k])
+    hbm, src = peaks()
+    achieved = alg_kernel[dom] / (kern[dom] * 1e-3) / 1e9
+    tokens_layers = sum(t.seqlens) * L
+    value = tokens_layers * world / (t_ms * 1e-3)
+    alg_pass = wl.algorithmic_bytes(budget)
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        v_cpu, desc, wall = oracle_sample(wl, budget, args.cpu_seconds, dev, tensors=t)
+        cpu = {"value": v_cpu, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+               "sample": desc + f"; {wall:.1f} s of CPU work; numpy BLAS threads left at their default"}
+
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, ev, t, stream, world, dist)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC,
+            "value": value,
+            "unit": UNIT,
+            "n_gpus": world,
+            "steps": K,
+            "warmup": args.warmup,
+            "ms_per_step": t_ms,
+            "higher_is_better": True,
+            "scaling": "weak",
+            "vs_baseline": None,
+            "dtype": "bf16" if wl.dtype == "bf16" else "f32",
+            "data": "synthetic",
+            "config": workload_config(wl, budget, world),
+            "roofline": {
+                "bound": "hbm",
+                "kernel": dom,
+                "achieved": achieved,
+                "peak": hbm,
+                "unit": "GB/s",
+                "frac": achieved / hbm,
+                "traffic": None,
+                "peak_source": f"{src} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)" if src == "measured" else "fallback",
+            },
+            "pass_roofline": {
+                "algorithmic_bytes": alg_pass,
+                "achieved_gbs": alg_pass / (t_ms * 1e-3) / 1e9,
+                "frac_of_8tbs": alg_pass / (t_ms * 1e-3) / 1e9 / NOMINAL_HBM_GBS,
+                "frac_of_measured": alg_pass / (t_ms * 1e-3) / 1e9 / hbm,
+            },
+            "kernel_ms": kern,
+            "gpu_launches": K * (len(SCORE_KERNEL_NAMES) + 2),
+            "clocks": clocks,
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+        }
+        print(json.dumps(line))
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def run_e2e(args, ev, t, stream, world, dist):
+    """Same metric through the public API with the inputs in pinned host memory:
+    every step copies the cache host->device, runs the pass and reads the kept
+    positions back."""
+    import torch
+
+    q_h = t.q_win.cpu().pin_memory()
+    k_h = t.k.cpu().pin_memory()
+    v_h = t.v.cpu().pin_memory()
+    cu_h = t.cu_seqlens.cpu().pin_memory()
+    idx_h = torch.empty(ev.idx.shape, dtype=ev.idx.dtype).pin_memory()
+    kept_h = torch.empty(ev.kept.shape, dtype=ev.kept.dtype).pin_memory()
+
+    def step():
+        t.q_win.copy_(q_h, non_blocking=True)
+        t.k.copy_(k_h, non_blocking=True)
+        t.v.copy_(v_h, non_blocking=True)
+        t.cu_seqlens.copy_(cu_h, non_blocking=True)
+        ev.run()
+        idx_h.copy_(ev.idx, non_blocking=True)
+        kept_h.copy_(ev.kept, non_blocking=True)
+
+    for _ in range(2):
+        step()
+    torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    n = max(1, args.e2e_steps)
+    for _ in range(n):
+        step()
+    b.record(stream)
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / n
+    if dist is not None:
+        x = torch.tensor([ms], device=t.k.device)
+        dist.all_reduce(x, op=dist.ReduceOp.MAX)
+        ms = float(x.item())
+    ev.check()
+    L = t.k.shape[0]
+    h2d = sum(x.numel() * x.element_size() for x in (q_h, k_h, v_h, cu_h))
+    d2h = idx_h.numel() * 4 + kept_h.numel() * 4
+    return {"value": sum(t.seqlens) * L * world / (ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": n}
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,202 @@
+/*
+ * jacap.h - C ABI of libjacap: the prefill-time KV-cache eviction pass of
+ * Jacap (Jacobian-capacity-aware eviction), Algorithm 1 of Sec. 3.4, on one
+ * NVIDIA GB300 (sm_103a).
+ *
+ * For every unit = (request s, layer l, KV head g) with n_s cached tokens the
+ * pass computes, per Algorithm 1 and Eqs. 8-10:
+ *
+ *   mu_h, lambda_h  mean and per-channel variance of the last w queries of
+ *                   every query head h served by KV head g (Sec. 3.4, last
+ *                   paragraph; diagonal Lambda_Q as in App. B.2);
+ *   alpha_bar_h,i   softmax_i(k_i . mu_h / (tau sqrt(d)))  over all n_s tokens;
+ *   w_i             (1/d) sum_h [alpha_bar_h,i (1 - alpha_bar_h,i)]^2 * kappa_h,i,
+ *                   kappa_h,i = sum_c lambda_h,c k_i,c^2          (Eq. 8);
+ *   A               I + sum_i w_i v_i v_i^T                     (Eq. 9);
+ *   score_i         w_i v_i^T A^{-1} v_i                         (Eq. 10);
+ *   C               the budget B highest scores (Alg. 1 step 5), ties to the
+ *                   lower token index, listed in ascending order;
+ *   K_out, V_out    the retained rows {(k_i, v_i)}_{i in C} (Sec. 3.1).
+ *
+ * Query head h is served by KV head h / (num_q_heads / num_kv_heads).
+ *
+ * Conventions for every entry point
+ *  - Pointers named *_host are host memory; every other data pointer is device
+ *    memory on the current CUDA device. The caller owns all memory; the library
+ *    allocates nothing and keeps no mutable global state.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *    All work is enqueued asynchronously on it; nothing synchronises except
+ *    jacap_device_status().
+ *  - Host-side validation happens before anything is enqueued; on any error
+ *    status nothing has been launched. A failed launch returns JACAP_ERR_CUDA.
+ *  - Problems only the device can see (a malformed cu_seqlens array, a
+ *    non-finite input or intermediate, a bounded wait that expired) are
+ *    recorded in the status word kept at the start of the workspace; kernels
+ *    that find it set return without work. Read it with jacap_device_status().
+ *    No kernel traps or asserts.
+ *  - Calls on different streams are safe when they use different workspaces.
+ */
+#ifndef JACAP_H
+#define JACAP_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  JACAP_OK = 0,
+  JACAP_ERR_INVALID_ARG = 1, /* bad pointer, size, stride, alignment or layout   */
+  JACAP_ERR_UNSUPPORTED = 2, /* head_dim != 128, group size not in {1,2,4,8},
+                                ridge = 0, or a device older than sm_103a       */
+  JACAP_ERR_WORKSPACE = 3,   /* workspace too small or misaligned               */
+  JACAP_ERR_CUDA = 4,        /* a CUDA runtime/driver call or launch failed     */
+  JACAP_ERR_NONFINITE = 5,   /* (device) NaN/Inf met in an input or intermediate */
+  JACAP_ERR_TIMEOUT = 6      /* (device) a bounded wait expired; the kernel quit */
+} jacap_status;
+
+typedef enum { JACAP_F32 = 0, JACAP_BF16 = 1 } jacap_dtype;
+
+/*
+ * Cache layout (Sec. 3.1: the KV cache {(k_i, v_i)} of every layer and head).
+ *
+ *  K, V    element (l, g, t, c) at  l*kv_stride_layer + g*kv_stride_head
+ *          + t*kv_stride_token + c  (elements; channel c contiguous), for
+ *          t in [0, total_tokens). Request s owns t in [cu[s], cu[s+1]).
+ *  Q_win   the last `window` queries of every request, layer and query head:
+ *          element (s, l, h, j, c) at s*q_stride_seq + l*q_stride_layer
+ *          + h*q_stride_head + j*q_stride_pos + c.
+ *  dtype   type of K, V and Q_win (all three share it).
+ *
+ * Requirements (else JACAP_ERR_INVALID_ARG / _UNSUPPORTED): head_dim == 128;
+ * num_q_heads % num_kv_heads == 0 with a ratio in {1,2,4,8}; window >= 1;
+ * every stride a multiple of 8 elements (16-byte rows) and K, V, Q_win 16-byte
+ * aligned; kv_stride_token >= head_dim; num_seqs >= 1; total_tokens >= 1 and
+ * < 2^31; max_seqlen >= every n_s. cu_seqlens must satisfy cu[0] = 0,
+ * cu[s] <= cu[s+1], cu[num_seqs] = total_tokens and n_s >= 1; the device
+ * checks this and reports JACAP_ERR_INVALID_ARG through the status word.
+ */
+typedef struct {
+  int32_t num_seqs;
+  const int32_t* cu_seqlens; /* device, [num_seqs + 1] token offsets           */
+  int32_t max_seqlen;        /* host upper bound of n_s                        */
+  int64_t total_tokens;      /* N_tot = cu_seqlens[num_seqs]                   */
+  int32_t num_layers;
+  int32_t num_q_heads;
+  int32_t num_kv_heads;
+  int32_t head_dim;          /* d_k = d_o = 128                                */
+  int32_t window;            /* w: queries per head used for (mu_Q, Lambda_Q)   */
+  jacap_dtype dtype;
+  int64_t kv_stride_layer, kv_stride_head, kv_stride_token;
+  int64_t q_stride_seq, q_stride_layer, q_stride_head, q_stride_pos;
+} jacap_layout;
+
+/*
+ * Method switches. Defaults {10.0f, 1, 1, 0}:
+ *  tau            temperature of the pool softmax (Sec. 3.4; Sec. 4.4 reports
+ *                 the best accuracy near 10). Must be finite and > 0.
+ *  weight_div_dk  1: keep the 1/d_k factor of Eq. 8; 0: drop it (Alg. 1 step 2
+ *                 prints the weight without it).
+ *  ridge          must be 1: the identity term of Eq. 9. (0 is an oracle-only
+ *                 variant and returns JACAP_ERR_UNSUPPORTED.)
+ *  cov_unbiased   0: lambda = population variance over the window (divide by
+ *                 w); 1: divide by w - 1 (needs window >= 2).
+ */
+typedef struct {
+  float tau;
+  int32_t weight_div_dk;
+  int32_t ridge;
+  int32_t cov_unbiased;
+} jacap_params;
+
+/* Bytes of device workspace jacap_score/jacap_select need for `layout`
+ * (budget is accepted for forward compatibility and may be any value >= 1).
+ * Returns 0 if the layout is invalid. The workspace must be 256-byte aligned;
+ * it holds the status word and every intermediate (mu, lambda, logits, kappa,
+ * w, partial Grams, the factor of A). */
+size_t jacap_workspace_size(const jacap_layout* layout, int32_t budget);
+
+/*
+ * Scores of every cached token (Algorithm 1 steps 1-4; Eqs. 8-10).
+ *  q_win, k, v  device, layout above.
+ *  scores       device float32 [num_layers][num_kv_heads][total_tokens]:
+ *               score of token t of plane (l, g); r_i of Eq. 10.
+ *  ws, ws_bytes device workspace of at least jacap_workspace_size() bytes.
+ * Resets the status word, then enqueues: query statistics, a streaming pass
+ * over K (logits, kappa, softmax statistics), a fused weight + weighted-Gram
+ * pass over V (tensor cores for bf16), the Cholesky factor and inverse of A,
+ * and the quadratic forms.
+ */
+jacap_status jacap_score(const jacap_layout* layout, const jacap_params* params,
+                         const void* q_win, const void* k, const void* v, float* scores,
+                         void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * jacap_score with timing hooks, for benchmarks: identical work, plus
+ * cudaEventRecord(events[i], stream) before the i-th kernel of the pass and
+ * events[num_events - 1] after the last one. `events` holds cudaEvent_t
+ * handles (as void*) created by the caller; num_events must be 0 (no hooks)
+ * or JACAP_SCORE_KERNELS + 1. Kernel order: plan, query statistics, K pass,
+ * weight + Gram, factor, scores.
+ */
+#define JACAP_SCORE_KERNELS 6
+jacap_status jacap_score_timed(const jacap_layout* layout, const jacap_params* params,
+                               const void* q_win, const void* k, const void* v, float* scores,
+                               void* ws, size_t ws_bytes, void* stream,
+                               void* const* events, int32_t num_events);
+
+/*
+ * TOP-B per unit (Algorithm 1 step 5). Reads `scores` as written by
+ * jacap_score (non-negative float32). For unit (l, g, s):
+ *  idx   device int32 [num_layers][num_kv_heads][num_seqs][budget]: the chosen
+ *        token positions RELATIVE to the request start cu[s], ascending; ties
+ *        in score go to the lower position; when n_s < budget all n_s
+ *        positions are listed and the rest is -1.
+ *  kept  device int32 [num_seqs]: min(n_s, budget).
+ * budget >= 1. ws: the workspace used by jacap_score (its status word is
+ * honoured and updated).
+ */
+jacap_status jacap_select(const jacap_layout* layout, const float* scores, int32_t budget,
+                          int32_t* idx, int32_t* kept, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * Retained cache Z_C (Sec. 3.1): for every unit, copies rows idx[r] (relative
+ * to cu[s]) of K and V, bit for bit, into
+ *  k_out, v_out  device, dtype of the cache, dense [num_layers][num_kv_heads]
+ *                [num_seqs][budget][head_dim]; rows whose idx is -1 are zeroed.
+ * idx as produced by jacap_select; an entry that is -1 or not a position of
+ * the request yields a zero row (no index value reads out of bounds). k_out and
+ * v_out must be 16-byte aligned and
+ * must not overlap k or v.
+ */
+jacap_status jacap_compact(const jacap_layout* layout, const void* k, const void* v,
+                           const int32_t* idx, int32_t budget, void* k_out, void* v_out,
+                           void* stream);
+
+/* Synchronises `stream`, then reads the workspace status word: JACAP_OK or the
+ * first device-side error recorded since the last jacap_score on `ws`. */
+jacap_status jacap_device_status(const void* ws, void* stream);
+
+/* Static English text for a status code (never NULL). */
+const char* jacap_status_string(jacap_status status);
+
+/* Byte offsets of the intermediates inside the workspace, for tests and
+ * debugging (all float32, row-major):
+ *  mu_scaled  [num_seqs][num_layers][num_q_heads][128]   mu_h / (tau sqrt(d))
+ *  lambda     [num_seqs][num_layers][num_q_heads][128]   diagonal of Lambda_Q
+ *  weights    [num_layers][num_kv_heads][total_tokens]   w_i (Eq. 8 summed over the group)
+ *  gram       [num_layers][num_kv_heads][num_seqs][128][128]  sum_i w_i v_i v_i^T
+ *  chol_inv   [num_layers][num_kv_heads][num_seqs][128][128]  L^{-1}, A = L L^T
+ * Returns JACAP_ERR_INVALID_ARG for an invalid layout. */
+typedef struct {
+  size_t mu_scaled, lambda, weights, gram, chol_inv;
+} jacap_ws_offsets;
+jacap_status jacap_workspace_offsets(const jacap_layout* layout, int32_t budget, jacap_ws_offsets* out);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* JACAP_H */

@@ -1,0 +1,146 @@
+"""Jacap's prefill-time KV-cache eviction pass on one GB300 (sm_103a).
+
+Thin Python binding of ``libjacap.so`` (C ABI in ``include/jacap.h``). The
+functions ``jacap_*`` below carry the same names and arguments as the C entry
+points and do argument marshalling only: every step of the pass runs in the
+library's CUDA kernels. There is no CPU fallback; if the library is missing
+the calls raise.
+
+``api`` adds a torch-facing convenience layer (layouts from tensors,
+workspace allocation, errors as exceptions, host-buffer end-to-end calls).
+"""
+
+from __future__ import annotations
+
+import ctypes
+
+from . import _lib
+
+JACAP_OK = 0
+JACAP_ERR_INVALID_ARG = 1
+JACAP_ERR_UNSUPPORTED = 2
+JACAP_ERR_WORKSPACE = 3
+JACAP_ERR_CUDA = 4
+JACAP_ERR_NONFINITE = 5
+JACAP_ERR_TIMEOUT = 6
+
+JACAP_F32 = 0
+JACAP_BF16 = 1
+
+
+class jacap_layout(ctypes.Structure):
+    """Mirror of ``jacap_layout`` (include/jacap.h)."""
+
+    _fields_ = [
+        ("num_seqs", ctypes.c_int32),
+        ("cu_seqlens", ctypes.c_void_p),
+        ("max_seqlen", ctypes.c_int32),
+        ("total_tokens", ctypes.c_int64),
+        ("num_layers", ctypes.c_int32),
+        ("num_q_heads", ctypes.c_int32),
+        ("num_kv_heads", ctypes.c_int32),
+        ("head_dim", ctypes.c_int32),
+        ("window", ctypes.c_int32),
+        ("dtype", ctypes.c_int32),
+        ("kv_stride_layer", ctypes.c_int64),
+        ("kv_stride_head", ctypes.c_int64),
+        ("kv_stride_token", ctypes.c_int64),
+        ("q_stride_seq", ctypes.c_int64),
+        ("q_stride_layer", ctypes.c_int64),
+        ("q_stride_head", ctypes.c_int64),
+        ("q_stride_pos", ctypes.c_int64),
+    ]
+
+
+class jacap_params(ctypes.Structure):
+    """Mirror of ``jacap_params``; defaults are the method's (tau = 10)."""
+
+    _fields_ = [
+        ("tau", ctypes.c_float),
+        ("weight_div_dk", ctypes.c_int32),
+        ("ridge", ctypes.c_int32),
+        ("cov_unbiased", ctypes.c_int32),
+    ]
+
+    def __init__(self, tau=10.0, weight_div_dk=1, ridge=1, cov_unbiased=0):
+        super().__init__(tau, weight_div_dk, ridge, cov_unbiased)
+
+
+class jacap_ws_offsets(ctypes.Structure):
+    _fields_ = [
+        ("mu_scaled", ctypes.c_size_t),
+        ("lambda_", ctypes.c_size_t),
+        ("weights", ctypes.c_size_t),
+        ("gram", ctypes.c_size_t),
+        ("chol_inv", ctypes.c_size_t),
+    ]
+
+
+_P = ctypes.c_void_p
+_SIGS = {
+    "jacap_workspace_size": (ctypes.c_size_t, [ctypes.POINTER(jacap_layout), ctypes.c_int32]),
+    "jacap_score": (ctypes.c_int, [ctypes.POINTER(jacap_layout), ctypes.POINTER(jacap_params), _P, _P, _P, _P, _P,
+                                   ctypes.c_size_t, _P]),
+    "jacap_score_timed": (ctypes.c_int, [ctypes.POINTER(jacap_layout), ctypes.POINTER(jacap_params), _P, _P, _P, _P,
+                                         _P, ctypes.c_size_t, _P, ctypes.POINTER(ctypes.c_void_p), ctypes.c_int32]),
+    "jacap_select": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, ctypes.c_int32, _P, _P, _P, ctypes.c_size_t,
+                                    _P]),
+    "jacap_compact": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, _P, _P, ctypes.c_int32, _P, _P, _P]),
+    "jacap_device_status": (ctypes.c_int, [_P, _P]),
+    "jacap_status_string": (ctypes.c_char_p, [ctypes.c_int]),
+    "jacap_workspace_offsets": (ctypes.c_int, [ctypes.POINTER(jacap_layout), ctypes.c_int32,
+                                               ctypes.POINTER(jacap_ws_offsets)]),
+}
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded C library with argument types declared."""
+    h = _lib.load(build_if_missing=True)
+    if not getattr(h, "_jacap_typed", False):
+        for name, (res, args) in _SIGS.items():
+            fn = getattr(h, name)
+            fn.restype = res
+            fn.argtypes = args
+        h._jacap_typed = True
+    return h
+
+
+def jacap_workspace_size(layout: jacap_layout, budget: int) -> int:
+    return lib().jacap_workspace_size(ctypes.byref(layout), budget)
+
+
+def jacap_score(layout, params, q_win, k, v, scores, ws, ws_bytes, stream) -> int:
+    return lib().jacap_score(ctypes.byref(layout), ctypes.byref(params), q_win, k, v, scores, ws, ws_bytes, stream)
+
+
+JACAP_SCORE_KERNELS = 6
+SCORE_KERNEL_NAMES = ("plan", "query_stats", "k_pass", "weight_gram", "factor", "scores")
+
+
+def jacap_score_timed(layout, params, q_win, k, v, scores, ws, ws_bytes, stream, events) -> int:
+    """``events``: sequence of cudaEvent_t handles (ints), length 0 or 7."""
+    arr = (ctypes.c_void_p * max(1, len(events)))(*[ctypes.c_void_p(e) for e in events])
+    return lib().jacap_score_timed(ctypes.byref(layout), ctypes.byref(params), q_win, k, v, scores, ws, ws_bytes,
+                                   stream, arr, len(events))
+
+
+def jacap_select(layout, scores, budget, idx, kept, ws, ws_bytes, stream) -> int:
+    return lib().jacap_select(ctypes.byref(layout), scores, budget, idx, kept, ws, ws_bytes, stream)
+
+
+def jacap_compact(layout, k, v, idx, budget, k_out, v_out, stream) -> int:
+    return lib().jacap_compact(ctypes.byref(layout), k, v, idx, budget, k_out, v_out, stream)
+
+
+def jacap_device_status(ws, stream) -> int:
+    return lib().jacap_device_status(ws, stream)
+
+
+def jacap_status_string(status: int) -> str:
+    return lib().jacap_status_string(status).decode()
+
+
+def jacap_workspace_offsets(layout: jacap_layout, budget: int):
+    out = jacap_ws_offsets()
+    st = lib().jacap_workspace_offsets(ctypes.byref(layout), budget, ctypes.byref(out))
+    return st, out

@@ -1,0 +1,325 @@
+// jacap_api.cu - host side of the libjacap C ABI (declared in include/jacap.h).
+//
+// Validates arguments on the host before anything is enqueued, carves the
+// caller's workspace, encodes the TMA tensor maps of K and V, and enqueues the
+// kernels of the eviction pass on the caller's stream. Allocates nothing.
+#include <cudaTypedefs.h>
+#include <math.h>
+#include <string.h>
+
+#include "jacap.h"
+#include "jacap_dev.cuh"
+#include "jacap_internal.h"
+
+using namespace jacap;
+
+namespace {
+
+constexpr size_t ALIGN = 1024;
+inline size_t align_up(size_t x) { return (x + ALIGN - 1) & ~(ALIGN - 1); }
+
+struct Carve {
+  size_t status, plan, counters, mu, lam, lk, cstats, w, gpart, gram, minv, minv_img, total;
+};
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+// Argument checks that need no GPU. Returns JACAP_OK or the error.
+jacap_status check_layout(const jacap_layout* L) {
+  if (L == nullptr || L->cu_seqlens == nullptr) return JACAP_ERR_INVALID_ARG;
+  if (L->num_seqs < 1 || L->num_layers < 1 || L->num_kv_heads < 1 || L->num_q_heads < 1) return JACAP_ERR_INVALID_ARG;
+  if (L->total_tokens < 1 || L->total_tokens >= ((int64_t)1 << 31)) return JACAP_ERR_INVALID_ARG;
+  if (L->max_seqlen < 1 || (int64_t)L->max_seqlen > L->total_tokens) return JACAP_ERR_INVALID_ARG;
+  if (L->window < 1) return JACAP_ERR_INVALID_ARG;
+  if (L->dtype != JACAP_F32 && L->dtype != JACAP_BF16) return JACAP_ERR_INVALID_ARG;
+  if (L->num_q_heads % L->num_kv_heads != 0) return JACAP_ERR_INVALID_ARG;
+  const int G = L->num_q_heads / L->num_kv_heads;
+  if (L->head_dim != D) return JACAP_ERR_UNSUPPORTED;
+  if (G != 1 && G != 2 && G != 4 && G != 8) return JACAP_ERR_UNSUPPORTED;
+  const int64_t el16 = L->dtype == JACAP_BF16 ? 8 : 4;  // elements per 16 bytes
+  const int64_t kv[3] = {L->kv_stride_layer, L->kv_stride_head, L->kv_stride_token};
+  const int64_t qs[4] = {L->q_stride_seq, L->q_stride_layer, L->q_stride_head, L->q_stride_pos};
+  for (int64_t s : kv)
+    if (s < D || s % el16 != 0) return JACAP_ERR_INVALID_ARG;
+  for (int64_t s : qs)
+    if (s < D || s % el16 != 0) return JACAP_ERR_INVALID_ARG;
+  const int64_t es = L->dtype == JACAP_BF16 ? 2 : 4;
+  if ((uint64_t)L->kv_stride_layer * es >= (1ull << 40) || (uint64_t)L->kv_stride_head * es >= (1ull << 40) ||
+      (uint64_t)L->kv_stride_token * es >= (1ull << 40))
+    return JACAP_ERR_INVALID_ARG;
+  return JACAP_OK;
+}
+
+// Tokens per work item: the largest of 4096..128 that still yields enough
+// items to fill the GPU several times over (independent of the device so the
+// workspace size is a pure function of the layout).
+int pick_chunk(const jacap_layout* L) {
+  const int64_t planes = (int64_t)L->num_layers * L->num_kv_heads;
+  for (int c = 4096; c > TILE; c >>= 1) {
+    const int64_t items = planes * (L->total_tokens / c + L->num_seqs);
+    if (items >= 1024) return c;
+  }
+  return TILE;
+}
+
+void make_dims(const jacap_layout* L, const jacap_params* P, Dims& dm) {
+  memset(&dm, 0, sizeof(dm));
+  dm.S = L->num_seqs;
+  dm.L = L->num_layers;
+  dm.Hq = L->num_q_heads;
+  dm.Hkv = L->num_kv_heads;
+  dm.G = L->num_q_heads / L->num_kv_heads;
+  dm.window = L->window;
+  dm.Ntot = L->total_tokens;
+  dm.chunk = pick_chunk(L);
+  dm.c_cap = L->total_tokens / dm.chunk + L->num_seqs;
+  dm.kv_sl = L->kv_stride_layer;
+  dm.kv_sh = L->kv_stride_head;
+  dm.kv_st = L->kv_stride_token;
+  dm.q_ss = L->q_stride_seq;
+  dm.q_sl = L->q_stride_layer;
+  dm.q_sh = L->q_stride_head;
+  dm.q_sp = L->q_stride_pos;
+  if (P != nullptr) {
+    dm.inv_scale = (float)(1.0 / ((double)P->tau * sqrt((double)D)));
+    dm.wdiv = P->weight_div_dk ? 1.0f / (float)D : 1.0f;
+    dm.cov_unbiased = P->cov_unbiased;
+  }
+}
+
+Carve carve(const Dims& dm) {
+  Carve c;
+  const size_t planes = (size_t)dm.L * dm.Hkv;
+  const size_t units = planes * dm.S;
+  size_t o = 0;
+  c.status = o; o = align_up(o + 64);
+  c.plan = o; o = align_up(o + ((size_t)dm.S + 2) * 4);
+  c.counters = o; o = align_up(o + units * 4);
+  c.mu = o; o = align_up(o + (size_t)dm.S * dm.L * dm.Hq * D * 4);
+  c.lam = o; o = align_up(o + (size_t)dm.S * dm.L * dm.Hq * D * 4);
+  c.lk = o; o = align_up(o + planes * (size_t)dm.Ntot * 2 * dm.G * 4);
+  c.cstats = o; o = align_up(o + planes * (size_t)dm.c_cap * dm.G * 2 * 4);
+  c.w = o; o = align_up(o + planes * (size_t)dm.Ntot * 4);
+  c.gpart = o; o = align_up(o + planes * (size_t)dm.c_cap * D * D * 4);
+  c.gram = o; o = align_up(o + units * D * D * 4);
+  c.minv = o; o = align_up(o + units * D * D * 4);
+  c.minv_img = o; o = align_up(o + units * 65536);
+  c.total = o;
+  return c;
+}
+
+Ws make_ws(void* base, const Carve& c) {
+  uint8_t* b = (uint8_t*)base;
+  Ws ws;
+  ws.status = (uint32_t*)(b + c.status);
+  ws.plan = (int32_t*)(b + c.plan);
+  ws.counters = (int32_t*)(b + c.counters);
+  ws.mu = (float*)(b + c.mu);
+  ws.lam = (float*)(b + c.lam);
+  ws.lk = (float*)(b + c.lk);
+  ws.cstats = (float*)(b + c.cstats);
+  ws.w = (float*)(b + c.w);
+  ws.gpart = (float*)(b + c.gpart);
+  ws.gram = (float*)(b + c.gram);
+  ws.minv = (float*)(b + c.minv);
+  ws.minv_img = b + c.minv_img;
+  return ws;
+}
+
+// Current device must be sm_103 (GB300). Returns its SM count via *sms.
+jacap_status check_device(int* sms) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return JACAP_ERR_CUDA;
+  int major = 0, minor = 0;
+  if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return JACAP_ERR_CUDA;
+  if (major != 10 || minor != 3) return JACAP_ERR_UNSUPPORTED;
+  return JACAP_OK;
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (fn == nullptr) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = (PFN_cuTensorMapEncodeTiled_v12000)p;
+  }
+  return fn;
+}
+
+// 4-D map over (channel, token, kv head, layer) with {128 B, 128 tokens} boxes
+// and the 128-byte swizzle; out-of-range tokens read as zero.
+bool encode_kv_map(CUtensorMap* map, const jacap_layout* L, const void* base) {
+  PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
+  if (fn == nullptr) return false;
+  const bool bf = L->dtype == JACAP_BF16;
+  const cuuint64_t es = bf ? 2 : 4;
+  const cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)L->total_tokens, (cuuint64_t)L->num_kv_heads,
+                              (cuuint64_t)L->num_layers};
+  const cuuint64_t strides[3] = {(cuuint64_t)L->kv_stride_token * es, (cuuint64_t)L->kv_stride_head * es,
+                                 (cuuint64_t)L->kv_stride_layer * es};
+  const cuuint32_t box[4] = {(cuuint32_t)(128 / es), (cuuint32_t)TILE, 1, 1};
+  const cuuint32_t estr[4] = {1, 1, 1, 1};
+  const CUresult r = fn(map, bf ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4,
+                        const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+jacap_status map_cuda(cudaError_t e) { return e == cudaSuccess ? JACAP_OK : JACAP_ERR_CUDA; }
+
+int persistent_grid(int64_t items, int sms, int per_sm) {
+  const int64_t cap = (int64_t)sms * per_sm;
+  const int64_t g = items < cap ? items : cap;
+  return g < 1 ? 1 : (int)g;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t jacap_workspace_size(const jacap_layout* layout, int32_t budget) {
+  if (check_layout(layout) != JACAP_OK || budget < 1) return 0;
+  Dims dm;
+  make_dims(layout, nullptr, dm);
+  return carve(dm).total;
+}
+
+jacap_status jacap_workspace_offsets(const jacap_layout* layout, int32_t budget, jacap_ws_offsets* out) {
+  if (out == nullptr || budget < 1) return JACAP_ERR_INVALID_ARG;
+  const jacap_status st = check_layout(layout);
+  if (st != JACAP_OK) return st;
+  Dims dm;
+  make_dims(layout, nullptr, dm);
+  const Carve c = carve(dm);
+  out->mu_scaled = c.mu;
+  out->lambda = c.lam;
+  out->weights = c.w;
+  out->gram = c.gram;
+  out->chol_inv = c.minv;
+  return JACAP_OK;
+}
+
+jacap_status jacap_score(const jacap_layout* layout, const jacap_params* params, const void* q_win,
+                         const void* k, const void* v, float* scores, void* ws, size_t ws_bytes, void* stream) {
+  return jacap_score_timed(layout, params, q_win, k, v, scores, ws, ws_bytes, stream, nullptr, 0);
+}
+
+jacap_status jacap_score_timed(const jacap_layout* layout, const jacap_params* params, const void* q_win,
+                               const void* k, const void* v, float* scores, void* ws, size_t ws_bytes,
+                               void* stream, void* const* events, int32_t num_events) {
+  if (num_events != 0 && (num_events != JACAP_SCORE_KERNELS + 1 || events == nullptr)) return JACAP_ERR_INVALID_ARG;
+  jacap_status st = check_layout(layout);
+  if (st != JACAP_OK) return st;
+  if (params == nullptr || q_win == nullptr || k == nullptr || v == nullptr || scores == nullptr || ws == nullptr)
+    return JACAP_ERR_INVALID_ARG;
+  if (!(params->tau > 0.f) || !isfinite(params->tau)) return JACAP_ERR_INVALID_ARG;
+  if (params->weight_div_dk != 0 && params->weight_div_dk != 1) return JACAP_ERR_INVALID_ARG;
+  if (params->cov_unbiased != 0 && params->cov_unbiased != 1) return JACAP_ERR_INVALID_ARG;
+  if (params->cov_unbiased && layout->window < 2) return JACAP_ERR_INVALID_ARG;
+  if (params->ridge != 1) return JACAP_ERR_UNSUPPORTED;
+  if (!aligned16(q_win) || !aligned16(k) || !aligned16(v) || ((uintptr_t)scores & 3u) != 0)
+    return JACAP_ERR_INVALID_ARG;
+  Dims dm;
+  make_dims(layout, params, dm);
+  const Carve c = carve(dm);
+  if (((uintptr_t)ws & 255u) != 0 || ws_bytes < c.total) return JACAP_ERR_WORKSPACE;
+  int sms = 0;
+  if ((st = check_device(&sms)) != JACAP_OK) return st;
+  cudaStream_t s = (cudaStream_t)stream;
+  const Ws w = make_ws(ws, c);
+  CUtensorMap kmap, vmap;
+  const bool bf = layout->dtype == JACAP_BF16;
+  if (!encode_kv_map(&kmap, layout, k) || !encode_kv_map(&vmap, layout, v)) return JACAP_ERR_CUDA;
+  const int64_t items = (int64_t)dm.L * dm.Hkv * dm.c_cap;
+  const int dt = bf ? 1 : 0;
+  const int32_t* cu = layout->cu_seqlens;
+  auto hook = [&](int i) -> jacap_status {
+    if (num_events == 0) return JACAP_OK;
+    return map_cuda(cudaEventRecord((cudaEvent_t)events[i], s));
+  };
+  if ((st = map_cuda(cudaMemsetAsync(w.status, 0, 64, s))) != JACAP_OK) return st;
+  if ((st = hook(0)) != JACAP_OK || (st = map_cuda(launch_plan(dm, w, cu, s))) != JACAP_OK) return st;
+  if ((st = hook(1)) != JACAP_OK || (st = map_cuda(launch_window_stats(dm, w, dt, q_win, s))) != JACAP_OK) return st;
+  if ((st = hook(2)) != JACAP_OK ||
+      (st = map_cuda(launch_kpass(kmap, dm, w, dt, cu, persistent_grid(items, sms, 1), s))) != JACAP_OK)
+    return st;
+  if ((st = hook(3)) != JACAP_OK ||
+      (st = map_cuda(launch_gram(vmap, dm, w, dt, v, cu, persistent_grid(items, sms, bf ? 1 : 4), s))) != JACAP_OK)
+    return st;
+  if ((st = hook(4)) != JACAP_OK || (st = map_cuda(launch_factor(dm, w, s))) != JACAP_OK) return st;
+  if ((st = hook(5)) != JACAP_OK ||
+      (st = map_cuda(launch_score(vmap, dm, w, dt, v, cu, scores, persistent_grid(items, sms, bf ? 1 : 2), s))) !=
+          JACAP_OK)
+    return st;
+  if ((st = hook(6)) != JACAP_OK) return st;
+  return JACAP_OK;
+}
+
+jacap_status jacap_select(const jacap_layout* layout, const float* scores, int32_t budget, int32_t* idx,
+                          int32_t* kept, void* ws, size_t ws_bytes, void* stream) {
+  jacap_status st = check_layout(layout);
+  if (st != JACAP_OK) return st;
+  if (scores == nullptr || idx == nullptr || kept == nullptr || ws == nullptr || budget < 1)
+    return JACAP_ERR_INVALID_ARG;
+  if (((uintptr_t)scores & 3u) != 0 || ((uintptr_t)idx & 3u) != 0 || ((uintptr_t)kept & 3u) != 0)
+    return JACAP_ERR_INVALID_ARG;
+  Dims dm;
+  make_dims(layout, nullptr, dm);
+  const Carve c = carve(dm);
+  if (((uintptr_t)ws & 255u) != 0 || ws_bytes < c.total) return JACAP_ERR_WORKSPACE;
+  int sms = 0;
+  if ((st = check_device(&sms)) != JACAP_OK) return st;
+  const Ws w = make_ws(ws, c);
+  const int64_t units = (int64_t)dm.L * dm.Hkv * dm.S;
+  return map_cuda(launch_select(dm, w, layout->cu_seqlens, scores, budget, idx, kept,
+                                persistent_grid(units, sms, 2), (cudaStream_t)stream));
+}
+
+jacap_status jacap_compact(const jacap_layout* layout, const void* k, const void* v, const int32_t* idx,
+                           int32_t budget, void* k_out, void* v_out, void* stream) {
+  jacap_status st = check_layout(layout);
+  if (st != JACAP_OK) return st;
+  if (k == nullptr || v == nullptr || idx == nullptr || k_out == nullptr || v_out == nullptr || budget < 1)
+    return JACAP_ERR_INVALID_ARG;
+  if (!aligned16(k) || !aligned16(v) || !aligned16(k_out) || !aligned16(v_out) || ((uintptr_t)idx & 3u) != 0)
+    return JACAP_ERR_INVALID_ARG;
+  int sms = 0;
+  if ((st = check_device(&sms)) != JACAP_OK) return st;
+  Dims dm;
+  make_dims(layout, nullptr, dm);
+  return map_cuda(launch_compact(dm, layout->dtype == JACAP_BF16 ? 1 : 0, layout->cu_seqlens, k, v, idx, budget,
+                                 k_out, v_out, (cudaStream_t)stream));
+}
+
+jacap_status jacap_device_status(const void* ws, void* stream) {
+  if (ws == nullptr) return JACAP_ERR_INVALID_ARG;
+  if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess) return JACAP_ERR_CUDA;
+  uint32_t word = 0;
+  if (cudaMemcpy(&word, ws, sizeof(word), cudaMemcpyDeviceToHost) != cudaSuccess) return JACAP_ERR_CUDA;
+  if (word & ST_INVALID) return JACAP_ERR_INVALID_ARG;
+  if (word & ST_TIMEOUT) return JACAP_ERR_TIMEOUT;
+  if (word & ST_NONFINITE) return JACAP_ERR_NONFINITE;
+  return JACAP_OK;
+}
+
+const char* jacap_status_string(jacap_status status) {
+  switch (status) {
+    case JACAP_OK: return "ok";
+    case JACAP_ERR_INVALID_ARG: return "invalid argument";
+    case JACAP_ERR_UNSUPPORTED: return "unsupported configuration or device";
+    case JACAP_ERR_WORKSPACE: return "workspace too small or misaligned";
+    case JACAP_ERR_CUDA: return "CUDA runtime or launch error";
+    case JACAP_ERR_NONFINITE: return "non-finite value in an input or intermediate";
+    case JACAP_ERR_TIMEOUT: return "a bounded device wait expired";
+    default: return "unknown status";
+  }
+}
+
+}  // extern "C"

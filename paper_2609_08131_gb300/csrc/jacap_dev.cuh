@@ -1,0 +1,280 @@
+// jacap_dev.cuh - shared definitions of the libjacap kernels (sm_103a).
+//
+// Problem shapes, the workspace map, the work-item plan, and thin inline-PTX
+// wrappers for mbarriers, TMA (cp.async.bulk.tensor), bulk copies and the
+// tcgen05 tensor-core / tensor-memory instructions. Every wait on an mbarrier
+// is bounded by wall-clock time (%globaltimer); on expiry the waiter records
+// JACAP status bit ST_TIMEOUT in the workspace status word and reports failure
+// to its caller, which then winds the CTA down instead of spinning forever.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace jacap {
+
+constexpr int D = 128;     // head_dim d_k = d_o
+constexpr int TILE = 128;  // tokens per tile (one TMA box row count, one MMA M)
+
+// Status word bits (word 0 of the workspace). Host maps them to jacap_status.
+enum : uint32_t {
+  ST_INVALID = 1u,    // malformed cu_seqlens
+  ST_NONFINITE = 2u,  // NaN/Inf in an input or intermediate
+  ST_TIMEOUT = 4u,    // a bounded wait expired
+};
+
+constexpr unsigned long long WAIT_LIMIT_NS = 2000000000ull;  // 2 s per wait
+
+// Shapes and method constants of one call, passed by value to every kernel.
+struct Dims {
+  int S, L, Hq, Hkv, G, window;
+  int64_t Ntot;
+  int chunk;          // tokens per work item (multiple of TILE)
+  int64_t c_cap;      // capacity of per-plane chunk arrays (>= sum_s ceil(n_s/chunk))
+  int64_t kv_sl, kv_sh, kv_st;  // K/V strides (elements)
+  int64_t q_ss, q_sl, q_sh, q_sp;
+  float inv_scale;    // 1 / (tau sqrt(d))
+  float wdiv;         // 1/d (Eq. 8) or 1 (weight_div_dk = 0)
+  int cov_unbiased;
+};
+
+// Workspace map (device pointers into the caller's workspace).
+struct Ws {
+  uint32_t* status;   // [16] status word + first failing unit
+  int32_t* plan;      // [0] = chunks per plane C_tot, [1 .. S+1] = chunk prefix per request
+  int32_t* counters;  // [units] per-unit completion counters (reserved)
+  float* mu;          // [S][L][Hq][D]  mu / (tau sqrt d)
+  float* lam;         // [S][L][Hq][D]  diagonal of Lambda_Q
+  float* lk;          // [L*Hkv][Ntot][2G]  logits then kappa per query head of the group
+  float* cstats;      // [L*Hkv][c_cap][G][2]  per-chunk (max, sum exp(l - max))
+  float* w;           // [L*Hkv][Ntot]  Eq. 8 weights summed over the group
+  float* gpart;       // [L*Hkv][c_cap][D][D]  per-chunk partial Grams
+  float* gram;        // [units][D][D]  sum_i w_i v_i v_i^T
+  float* minv;        // [units][D][D]  L^{-1} (float32, lower triangular)
+  uint8_t* minv_img;  // [units][65536]  L^{-1} as bf16 hi/lo, shared-memory image for the score MMA
+};
+
+// A unit is (plane p = l*Hkv + g, request s); its index is p*S + s.
+struct Item {
+  int plane, seq, chunk;  // chunk index within the request
+  int64_t t0, t1;         // token range [t0, t1) on the plane's token axis
+  int64_t seq_start;      // cu[s]
+  int cidx;               // chunk index within the plane (prefix[s] + chunk)
+};
+
+__device__ __forceinline__ bool decode_item(const Dims& dm, const int32_t* plan, const int32_t* cu,
+                                            int64_t item, Item& it) {
+  const int ctot = plan[0];
+  const int64_t total = (int64_t)dm.L * dm.Hkv * ctot;
+  if (item >= total) return false;
+  it.plane = (int)(item / ctot);
+  const int r = (int)(item - (int64_t)it.plane * ctot);
+  // largest s with prefix[s] <= r (prefix is plan[1 .. S+1], nondecreasing)
+  int lo = 0, hi = dm.S - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (plan[1 + mid] <= r) lo = mid; else hi = mid - 1;
+  }
+  it.seq = lo;
+  it.chunk = r - plan[1 + lo];
+  it.cidx = r;
+  it.seq_start = cu[lo];
+  const int64_t end = cu[lo + 1];
+  it.t0 = it.seq_start + (int64_t)it.chunk * dm.chunk;
+  it.t1 = min(end, it.t0 + (int64_t)dm.chunk);
+  return true;
+}
+
+__device__ __forceinline__ bool status_failed(const Ws& ws) {
+  return *((volatile uint32_t*)ws.status) != 0u;
+}
+
+__device__ __forceinline__ void flag(const Ws& ws, uint32_t bit) { atomicOr(ws.status, bit); }
+
+// ------------------------------------------------------------------ PTX ----
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ unsigned long long globaltimer() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.release.cta.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cta.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait for the phase with the given parity to complete. Returns false
+// (after flagging ST_TIMEOUT) if it did not complete within WAIT_LIMIT_NS, or
+// if *abort became nonzero while waiting.
+static __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, const Ws& ws,
+                                            volatile int* abort) {
+  const unsigned long long t0 = globaltimer();
+  for (uint32_t it = 0;; ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 63u) == 63u) {
+      if (abort != nullptr && *abort) return false;
+      if (globaltimer() - t0 > WAIT_LIMIT_NS) {
+        flag(ws, ST_TIMEOUT);
+        if (abort != nullptr) *abort = 1;
+        return false;
+      }
+    }
+  }
+}
+
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const Ws& ws,
+                                          volatile int* abort) {
+  if (mbar_try_wait(bar, parity)) return true;
+  return mbar_wait_slow(bar, parity, ws, abort);
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// 4-D tiled TMA load into shared memory, completion counted on `bar`.
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* map, int c0, int c1, int c2,
+                                            int c3, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cta.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(dst),
+      "l"(map), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(bar)
+      : "memory");
+}
+
+// Linear bulk copy global -> shared (16-byte aligned, size multiple of 16).
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cta.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+      "l"(src), "r"(bytes), "r"(bar)
+      : "memory");
+}
+
+__device__ __forceinline__ void prefetch_tmap(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(map) : "memory");
+}
+
+// ------------------------------------------------------------ tcgen05 ----
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// D[tmem] (+)= A[smem desc] * B[smem desc], kind::f16 (bf16 inputs, f32 accumulate).
+__device__ __forceinline__ void umma_f16_ss(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                            uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrive on `bar` once every tcgen05 op issued so far by this thread completed.
+__device__ __forceinline__ void umma_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+               : "memory");
+}
+
+// Load 32 consecutive f32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
+        "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
+        "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),
+        "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Shared-memory matrix descriptor (tcgen05 format): start address, leading-
+// and stride-dimension byte offsets, version 1, 128-byte swizzle.
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr, uint32_t lbo_bytes, uint32_t sbo_bytes) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((lbo_bytes >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo_bytes >> 4) & 0x3FFFu) << 32;
+  d |= (uint64_t)1 << 46;  // descriptor version for tcgen05
+  d |= (uint64_t)2 << 61;  // 128-byte swizzle
+  return d;
+}
+
+// Instruction descriptor of kind::f16: bf16 A and B, f32 D, dense.
+// a_mn / b_mn: 1 if that operand is MN-major (transposed), 0 if K-major.
+__host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N, int a_mn, int b_mn) {
+  return (1u << 4)                      // D format f32
+         | (1u << 7)                    // A format bf16
+         | (1u << 10)                   // B format bf16
+         | ((uint32_t)a_mn << 15)       // A major
+         | ((uint32_t)b_mn << 16)       // B major
+         | ((uint32_t)(N >> 3) << 17)   // N / 8
+         | ((uint32_t)(M >> 4) << 24);  // M / 16
+}
+
+// Byte offset of element (row, col) in a [rows][64]-element bf16 block stored
+// with the 128-byte swizzle (the layout TMA writes for a {64, rows} box).
+__device__ __forceinline__ uint32_t sw128_off(uint32_t row, uint32_t chunk16) {
+  return row * 128u + ((chunk16 ^ (row & 7u)) << 4);
+}
+
+__device__ __forceinline__ float bf16lo(uint32_t x) { return __uint_as_float(x << 16); }
+__device__ __forceinline__ float bf16hi(uint32_t x) { return __uint_as_float(x & 0xFFFF0000u); }
+
+// Round two floats to bf16 (nearest even) and pack (a in the low half).
+__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(b), "f"(a));
+  return r;
+}
+
+}  // namespace jacap

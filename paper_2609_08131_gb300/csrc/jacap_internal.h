@@ -1,0 +1,24 @@
+// jacap_internal.h - host-side launchers of the libjacap kernels.
+// All launchers enqueue on `st` and return the launch error (cudaSuccess if
+// the kernel was enqueued).
+#pragma once
+
+#include "jacap_dev.cuh"
+
+namespace jacap {
+
+cudaError_t launch_plan(const Dims& dm, const Ws& ws, const int32_t* cu, cudaStream_t st);
+cudaError_t launch_window_stats(const Dims& dm, const Ws& ws, int dtype, const void* q, cudaStream_t st);
+cudaError_t launch_kpass(const CUtensorMap& kmap, const Dims& dm, const Ws& ws, int dtype, const int32_t* cu,
+                         int grid, cudaStream_t st);
+cudaError_t launch_gram(const CUtensorMap& vmap, const Dims& dm, const Ws& ws, int dtype, const void* v,
+                        const int32_t* cu, int grid, cudaStream_t st);
+cudaError_t launch_factor(const Dims& dm, const Ws& ws, cudaStream_t st);
+cudaError_t launch_score(const CUtensorMap& vmap, const Dims& dm, const Ws& ws, int dtype, const void* v,
+                         const int32_t* cu, float* scores, int grid, cudaStream_t st);
+cudaError_t launch_select(const Dims& dm, const Ws& ws, const int32_t* cu, const float* scores, int budget,
+                          int32_t* idx, int32_t* kept, int grid, cudaStream_t st);
+cudaError_t launch_compact(const Dims& dm, int dtype, const int32_t* cu, const void* k, const void* v,
+                           const int32_t* idx, int budget, void* k_out, void* v_out, cudaStream_t st);
+
+}  // namespace jacap

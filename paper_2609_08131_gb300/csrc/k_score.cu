@@ -1,0 +1,266 @@
+// k_score.cu - Jacap scores r_i = w_i v_i^T A^{-1} v_i = w_i ||L^{-1} v_i||^2 (Eq. 10).
+//
+// bf16 caches: the tensor cores form Y = V (L^{-1})^T for a 128-token tile with
+// one kind::f16 MMA chain of N = 256: columns 0-127 use hi(L^{-1}), columns
+// 128-255 lo(L^{-1}), both K-major from a 64 KB shared-memory image written by
+// the factor kernel; V comes straight from the TMA-staged tile. Each epilogue
+// thread owns one token (one TMEM lane) and reduces ||y||^2 = sum_j (D[j] +
+// D[128+j])^2 in fp32, then multiplies by w_i. The tensor-memory accumulator
+// is double-buffered so the epilogue of tile i overlaps the MMAs of tile i+1.
+// float32 caches: SIMT forward products with L^{-1} held in shared memory.
+#include "jacap_dev.cuh"
+#include "jacap_internal.h"
+
+namespace jacap {
+
+constexpr int SC_THREADS = 192;  // warp 0: TMA, warp 1: MMA, warps 2-5: epilogue
+constexpr int SC_STAGES = 4;
+constexpr int SC_BOX = 16384;
+constexpr int SC_TILE_BYTES = 2 * SC_BOX;
+constexpr int SC_M_BYTES = 65536;
+constexpr uint32_t SC_TMEM_COLS = 512;
+// M = 128 tokens, N = 256 (hi | lo rows of L^{-1}), both operands K-major.
+constexpr uint32_t SC_IDESC = idesc_bf16_f32(128, 256, 0, 0);
+
+constexpr size_t score_bf16_smem_bytes() { return 1024 + SC_M_BYTES + SC_STAGES * SC_TILE_BYTES + 256; }
+
+__global__ void __launch_bounds__(SC_THREADS, 1)
+    score_bf16_kernel(const __grid_constant__ CUtensorMap vmap, Dims dm, Ws ws, const int32_t* __restrict__ cu,
+                      float* __restrict__ scores) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint8_t* mimg = smem;
+  uint8_t* stages = smem + SC_M_BYTES;
+  uint64_t* vfull = (uint64_t*)(stages + SC_STAGES * SC_TILE_BYTES);
+  uint64_t* vempty = vfull + SC_STAGES;
+  uint64_t* accfull = vempty + SC_STAGES;
+  uint64_t* accempty = accfull + 2;
+  uint64_t* mfull = accempty + 2;
+  uint64_t* mempty = mfull + 1;
+  uint64_t* mdone = mempty + 1;
+  __shared__ uint32_t s_tmem;
+  __shared__ int s_abort, s_skip;
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  if (tid == 0) {
+    s_abort = 0;
+    s_skip = status_failed(ws) ? 1 : 0;
+    for (int i = 0; i < SC_STAGES; ++i) {
+      mbar_init(smem_u32(&vfull[i]), 1);
+      mbar_init(smem_u32(&vempty[i]), 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(smem_u32(&accfull[i]), 1);
+      mbar_init(smem_u32(&accempty[i]), 4);
+    }
+    mbar_init(smem_u32(mfull), 1);
+    mbar_init(smem_u32(mempty), 1);
+    mbar_init(smem_u32(mdone), 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (s_skip) return;
+  if (warp == 1) {
+    tmem_alloc(smem_u32(&s_tmem), SC_TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = s_tmem;
+  volatile int* abort = &s_abort;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      prefetch_tmap(&vmap);
+      uint32_t it = 0, nitem = 0;
+      bool ok = true;
+      Item item;
+      for (int64_t i = blockIdx.x; ok && decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+        const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
+        const int64_t u = (int64_t)item.plane * dm.S + item.seq;
+        if (nitem > 0 && !mbar_wait(smem_u32(mempty), (nitem - 1) & 1, ws, abort)) break;
+        mbar_arrive_expect_tx(smem_u32(mfull), SC_M_BYTES);
+        bulk_g2s(smem_u32(mimg), ws.minv_img + u * SC_M_BYTES, SC_M_BYTES, smem_u32(mfull));
+        ++nitem;
+        for (int64_t t = item.t0; t < item.t1; t += TILE) {
+          const int st = it % SC_STAGES;
+          if (it >= (uint32_t)SC_STAGES &&
+              !mbar_wait(smem_u32(&vempty[st]), ((it / SC_STAGES) & 1) ^ 1, ws, abort)) {
+            ok = false;
+            break;
+          }
+          uint8_t* vt = stages + st * SC_TILE_BYTES;
+          mbar_arrive_expect_tx(smem_u32(&vfull[st]), SC_TILE_BYTES);
+          tma_load_4d(smem_u32(vt), &vmap, 0, (int)t, g, l, smem_u32(&vfull[st]));
+          tma_load_4d(smem_u32(vt + SC_BOX), &vmap, 64, (int)t, g, l, smem_u32(&vfull[st]));
+          ++it;
+        }
+      }
+      for (uint32_t k = (it > (uint32_t)SC_STAGES ? it - SC_STAGES : 0); k < it; ++k)
+        mbar_wait(smem_u32(&vfull[k % SC_STAGES]), (k / SC_STAGES) & 1, ws, nullptr);
+      if (nitem > 0) mbar_wait(smem_u32(mfull), (nitem - 1) & 1, ws, nullptr);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      uint32_t it = 0, nitem = 0;
+      bool ok = true;
+      Item item;
+      for (int64_t i = blockIdx.x; ok && decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+        if (!mbar_wait(smem_u32(mfull), nitem & 1, ws, abort)) break;
+        tc_fence_after();
+        const uint32_t ma = smem_u32(mimg);
+        for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
+          const int st = it % SC_STAGES;
+          const int ab = it & 1;
+          if (it >= 2 && !mbar_wait(smem_u32(&accempty[ab]), ((it >> 1) & 1) ^ 1, ws, abort)) {
+            ok = false;
+            break;
+          }
+          if (!mbar_wait(smem_u32(&vfull[st]), (it / SC_STAGES) & 1, ws, abort)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t va = smem_u32(stages + st * SC_TILE_BYTES);
+#pragma unroll
+          for (int k = 0; k < D / 16; ++k) {  // 16 channels per MMA
+            const uint32_t koff = (k >> 2) * SC_BOX + (k & 3) * 32;
+            const uint64_t ad = smem_desc_sw128(va + koff, 16, 1024);
+            const uint64_t bd = smem_desc_sw128(ma + (k >> 2) * 32768 + (k & 3) * 32, 16, 1024);
+            umma_f16_ss(tmem + ab * 256, ad, bd, SC_IDESC, k > 0 ? 1u : 0u);
+          }
+          umma_commit(smem_u32(&vempty[st]));
+          umma_commit(smem_u32(&accfull[ab]));
+        }
+        if (!ok) break;
+        umma_commit(smem_u32(mempty));
+        ++nitem;
+      }
+      // every MMA issued by this thread has completed before teardown
+      umma_commit(smem_u32(mdone));
+      mbar_wait(smem_u32(mdone), 0, ws, nullptr);
+    }
+  } else {
+    const int quarter = warp & 3;
+    const int y = quarter * 32 + lane;  // token row of the tile == TMEM lane
+    uint32_t it = 0;
+    bool bad = false;
+    Item item;
+    for (int64_t i = blockIdx.x; decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+      for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
+        const int ab = it & 1;
+        if (!mbar_wait(smem_u32(&accfull[ab]), (it >> 1) & 1, ws, abort)) goto epi_done;
+        tc_fence_after();
+        const uint32_t trow = tmem + ab * 256 + ((uint32_t)(quarter * 32) << 16);
+        float ssq = 0.f;
+#pragma unroll 1
+        for (int cb = 0; cb < 4; ++cb) {
+          float a[32], b[32];
+          tmem_ld32(trow + cb * 32, a);
+          tmem_ld32(trow + 128 + cb * 32, b);
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            const float yv = a[j] + b[j];
+            ssq = fmaf(yv, yv, ssq);
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&accempty[ab]));
+        const int64_t tok = t + y;
+        if (tok < item.t1) {
+          const int64_t o = (int64_t)item.plane * dm.Ntot + tok;
+          const float sc = ws.w[o] * ssq;
+          scores[o] = sc;
+          bad |= !isfinite(sc);
+        }
+      }
+    }
+  epi_done:
+    if (bad) flag(ws, ST_NONFINITE);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, SC_TMEM_COLS);
+  }
+}
+
+// ------------------------------------------------------------ SIMT fp32 ---
+constexpr int SF_THREADS = 128;
+constexpr int SF_LD = D + 1;
+constexpr size_t score_f32_smem_bytes() { return (size_t)(D * D + TILE * SF_LD) * sizeof(float); }
+
+__global__ void __launch_bounds__(SF_THREADS)
+    score_f32_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu, const float* __restrict__ v,
+                     float* __restrict__ scores) {
+  extern __shared__ float ssm[];
+  float* Mi = ssm;               // [D][D] L^{-1}
+  float* vt = ssm + D * D;       // [TILE][SF_LD]
+  __shared__ int s_skip;
+  const int tid = threadIdx.x;
+  if (tid == 0) s_skip = status_failed(ws) ? 1 : 0;
+  __syncthreads();
+  if (s_skip) return;
+  bool bad = false;
+  int64_t loaded = -1;
+  Item item;
+  for (int64_t i = blockIdx.x; decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+    const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
+    const int64_t u = (int64_t)item.plane * dm.S + item.seq;
+    const float* vbase = v + (int64_t)l * dm.kv_sl + (int64_t)g * dm.kv_sh;
+    __syncthreads();
+    if (u != loaded) {
+      const float* src = ws.minv + u * D * D;
+      for (int e = tid * 4; e < D * D; e += SF_THREADS * 4) *(float4*)(Mi + e) = *(const float4*)(src + e);
+      loaded = u;
+    }
+    for (int64_t t = item.t0; t < item.t1; t += TILE) {
+      __syncthreads();
+      for (int e = tid; e < TILE * (D / 4); e += SF_THREADS) {
+        const int r = e / (D / 4), c4 = (e % (D / 4)) * 4;
+        float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (t + r < item.t1) x = *(const float4*)(vbase + (t + r) * dm.kv_st + c4);
+        vt[r * SF_LD + c4] = x.x; vt[r * SF_LD + c4 + 1] = x.y;
+        vt[r * SF_LD + c4 + 2] = x.z; vt[r * SF_LD + c4 + 3] = x.w;
+      }
+      __syncthreads();
+      const int64_t tok = t + tid;
+      if (tok < item.t1) {
+        const float* vr = vt + tid * SF_LD;
+        float ssq = 0.f;
+        for (int r = 0; r < D; ++r) {
+          float yv = 0.f;
+          const float* mr = Mi + r * D;
+          for (int c = 0; c <= r; ++c) yv = fmaf(mr[c], vr[c], yv);
+          ssq = fmaf(yv, yv, ssq);
+        }
+        const int64_t o = (int64_t)item.plane * dm.Ntot + tok;
+        const float sc = ws.w[o] * ssq;
+        scores[o] = sc;
+        bad |= !isfinite(sc);
+      }
+    }
+  }
+  if (bad) flag(ws, ST_NONFINITE);
+}
+
+cudaError_t launch_score(const CUtensorMap& vmap, const Dims& dm, const Ws& ws, int dtype, const void* v,
+                         const int32_t* cu, float* scores, int grid, cudaStream_t st) {
+  if (dtype == 1) {
+    constexpr size_t smem = score_bf16_smem_bytes();
+    cudaError_t e = cudaFuncSetAttribute(score_bf16_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    score_bf16_kernel<<<grid, SC_THREADS, smem, st>>>(vmap, dm, ws, cu, scores);
+  } else {
+    constexpr size_t smem = score_f32_smem_bytes();
+    cudaError_t e = cudaFuncSetAttribute(score_f32_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    score_f32_kernel<<<grid, SF_THREADS, smem, st>>>(dm, ws, cu, (const float*)v, scores);
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace jacap

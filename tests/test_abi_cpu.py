@@ -1,0 +1,132 @@
+"""The C-ABI library builds, loads, exports every declared symbol, and rejects
+bad arguments on the host before touching a GPU. No compute call here."""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2609_08131_gb300 as J
+from paper_2609_08131_gb300 import _lib
+
+HEADER = os.path.join(_lib.INCLUDE, "jacap.h")
+
+
+def declared_symbols():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(jacap_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_symbols()
+    for n in ["jacap_score", "jacap_select", "jacap_compact", "jacap_workspace_size", "jacap_device_status",
+              "jacap_status_string", "jacap_workspace_offsets"]:
+        assert n in names
+    assert set(names) == set(_lib.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol(jacap_lib):
+    for name in declared_symbols():
+        assert hasattr(jacap_lib, name), name
+
+
+def good_layout(**kw):
+    lay = J.jacap_layout()
+    lay.num_seqs = 2
+    lay.cu_seqlens = 0x1000  # never dereferenced on the host
+    lay.max_seqlen = 300
+    lay.total_tokens = 500
+    lay.num_layers = 2
+    lay.num_q_heads = 8
+    lay.num_kv_heads = 2
+    lay.head_dim = 128
+    lay.window = 16
+    lay.dtype = J.JACAP_BF16
+    lay.kv_stride_layer = 2 * 500 * 128
+    lay.kv_stride_head = 500 * 128
+    lay.kv_stride_token = 128
+    lay.q_stride_seq = 2 * 8 * 16 * 128
+    lay.q_stride_layer = 8 * 16 * 128
+    lay.q_stride_head = 16 * 128
+    lay.q_stride_pos = 128
+    for k, v in kw.items():
+        setattr(lay, k, v)
+    return lay
+
+
+def test_workspace_size_is_positive_and_monotone():
+    a = J.jacap_workspace_size(good_layout(), 64)
+    b = J.jacap_workspace_size(good_layout(total_tokens=5000, max_seqlen=4000,
+                                           kv_stride_head=5000 * 128, kv_stride_layer=2 * 5000 * 128), 64)
+    assert 0 < a < b
+    assert a % 1024 == 0
+
+
+@pytest.mark.parametrize("field,value,expect", [
+    ("head_dim", 64, J.JACAP_ERR_UNSUPPORTED),
+    ("num_q_heads", 6, J.JACAP_ERR_UNSUPPORTED),       # G = 3
+    ("num_q_heads", 7, J.JACAP_ERR_INVALID_ARG),       # not a multiple
+    ("num_q_heads", 32, J.JACAP_ERR_UNSUPPORTED),      # G = 16
+    ("window", 0, J.JACAP_ERR_INVALID_ARG),
+    ("num_seqs", 0, J.JACAP_ERR_INVALID_ARG),
+    ("total_tokens", 0, J.JACAP_ERR_INVALID_ARG),
+    ("total_tokens", 1 << 31, J.JACAP_ERR_INVALID_ARG),
+    ("max_seqlen", 0, J.JACAP_ERR_INVALID_ARG),
+    ("kv_stride_token", 100, J.JACAP_ERR_INVALID_ARG),  # < head_dim
+    ("kv_stride_token", 132, J.JACAP_ERR_INVALID_ARG),  # not 16-byte aligned rows (bf16)
+    ("q_stride_pos", 130, J.JACAP_ERR_INVALID_ARG),
+    ("dtype", 7, J.JACAP_ERR_INVALID_ARG),
+    ("cu_seqlens", 0, J.JACAP_ERR_INVALID_ARG),
+])
+def test_invalid_layouts_are_rejected_on_the_host(field, value, expect):
+    lay = good_layout(**{field: value})
+    assert J.jacap_workspace_size(lay, 8) == 0
+    p = ctypes.c_void_p(0x1000)
+    st = J.jacap_score(lay, J.jacap_params(), p, p, p, p, p, 1 << 40, None)
+    assert st == expect
+    st = J.jacap_select(lay, p, 8, p, p, p, 1 << 40, None)
+    assert st == expect
+    st = J.jacap_compact(lay, p, p, p, 8, p, p, None)
+    assert st == expect
+
+
+def test_bad_params_and_buffers_are_rejected_on_the_host():
+    lay = good_layout()
+    p = ctypes.c_void_p(0x1000)
+    big = J.jacap_workspace_size(lay, 8)
+    assert J.jacap_score(lay, J.jacap_params(tau=0.0), p, p, p, p, p, big, None) == J.JACAP_ERR_INVALID_ARG
+    assert J.jacap_score(lay, J.jacap_params(tau=float("nan")), p, p, p, p, p, big, None) == J.JACAP_ERR_INVALID_ARG
+    assert J.jacap_score(lay, J.jacap_params(ridge=0), p, p, p, p, p, big, None) == J.JACAP_ERR_UNSUPPORTED
+    assert J.jacap_score(lay, J.jacap_params(weight_div_dk=2), p, p, p, p, p, big, None) == J.JACAP_ERR_INVALID_ARG
+    lay1 = good_layout(window=1)
+    assert J.jacap_score(lay1, J.jacap_params(cov_unbiased=1), p, p, p, p, p, big, None) == J.JACAP_ERR_INVALID_ARG
+    mis = ctypes.c_void_p(0x1008)  # 8-byte aligned only
+    assert J.jacap_score(lay, J.jacap_params(), mis, p, p, p, p, big, None) == J.JACAP_ERR_INVALID_ARG
+    assert J.jacap_score(lay, J.jacap_params(), p, p, p, p, p, big - 1, None) == J.JACAP_ERR_WORKSPACE
+    assert J.jacap_score(lay, J.jacap_params(), p, p, p, p, ctypes.c_void_p(0x1010), big, None) == J.JACAP_ERR_WORKSPACE
+    assert J.jacap_select(lay, p, 0, p, p, p, big, None) == J.JACAP_ERR_INVALID_ARG
+    assert J.jacap_compact(lay, p, p, p, 8, mis, p, None) == J.JACAP_ERR_INVALID_ARG
+    assert J.jacap_device_status(None, None) == J.JACAP_ERR_INVALID_ARG
+
+
+def test_status_strings():
+    for s in range(0, 8):
+        assert isinstance(J.jacap_status_string(s), str) and J.jacap_status_string(s)
+    assert J.jacap_status_string(0) == "ok"
+
+
+def test_workspace_offsets_are_inside_the_workspace():
+    lay = good_layout()
+    st, off = J.jacap_workspace_offsets(lay, 8)
+    assert st == J.JACAP_OK
+    total = J.jacap_workspace_size(lay, 8)
+    for name in ["mu_scaled", "lambda_", "weights", "gram", "chol_inv"]:
+        assert 0 < getattr(off, name) < total
+    assert J.jacap_workspace_offsets(good_layout(head_dim=64), 8)[0] == J.JACAP_ERR_UNSUPPORTED
+
+
+def test_python_binding_names_match_the_c_abi():
+    for name in _lib.EXPORTS:
+        assert callable(getattr(J, name))

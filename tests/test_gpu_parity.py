@@ -1,0 +1,209 @@
+"""GPU parity of the CUDA eviction pass against the float64 oracle.
+
+Every test calls the library through the C ABI (via the ctypes binding) and
+compares with ``oracle.oracle_unit`` on the same bytes (the oracle reads the
+device tensors back exactly). Small cases compare every unit and every
+intermediate; the five evaluation configurations run at full size, in the
+launch configuration bench.py times, with sampled units checked against the
+oracle and size-independent properties checked on every unit.
+"""
+
+from dataclasses import replace
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import JacapParams, oracle_unit
+from paper_2609_08131_gb300 import jacap_params
+from paper_2609_08131_gb300.api import Cache, Evictor, evict
+from paper_2609_08131_gb300.workloads import Workload, config, generate, unit_arrays
+
+from parity import assert_rows_bitwise, assert_scores_close, assert_selection, gpu_selection_properties
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda:0"
+
+
+def make_cache(t, wl):
+    return Cache(t.q_win, t.k, t.v, t.cu_seqlens, t.seqlens, wl.num_q_heads)
+
+
+def check_unit(ev, t, wl, params, s, layer, g, check_w=True):
+    q, K, V = unit_arrays(t, wl.num_q_heads, s, layer, g)
+    ora = oracle_unit(q, K, V, ev.budget, JacapParams(tau=params.tau, weight_div_dk=bool(params.weight_div_dk),
+                                                       cov_unbiased=bool(params.cov_unbiased)))
+    cu = t.cu_seqlens.cpu().tolist()
+    a, b = cu[s], cu[s + 1]
+    n = b - a
+    gs = ev.scores[layer, g, a:b].double().cpu().numpy()
+    if check_w:
+        gw = ev.intermediates()["weights"][layer, g, a:b].double().cpu().numpy()
+        assert_scores_close(gw, ora["w"], "weights")
+    assert_scores_close(gs, ora["scores"])
+    gidx = ev.idx[layer, g, s].cpu().numpy()
+    assert_selection(gidx, n, ev.budget, ora["scores"], ora["idx"])
+    kept = min(n, ev.budget)
+    sel = torch.as_tensor(gidx[:kept], dtype=torch.long, device=t.k.device)
+    assert_rows_bitwise(t.k[layer, g, a:b][sel], ev.k_out[layer, g, s, :kept])
+    assert_rows_bitwise(t.v[layer, g, a:b][sel], ev.v_out[layer, g, s, :kept])
+    if kept < ev.budget:
+        assert bool((ev.k_out[layer, g, s, kept:] == 0).all()) and bool((ev.v_out[layer, g, s, kept:] == 0).all())
+    return ora
+
+
+SMALL = {
+    # name: (workload, params)
+    "bf16_gqa4_ragged_tails": (Workload("t", 2, 8, 2, (1000, 300, 129), 16, 64, seed=11), jacap_params()),
+    "bf16_mha_tau1": (Workload("t", 1, 4, 4, (777,), 8, 100, seed=12), jacap_params(tau=1.0)),
+    "bf16_gqa2_peaky_tiny_seq": (Workload("t", 1, 4, 2, (500, 1, 2), 16, 32, seed=13), jacap_params(tau=0.3)),
+    "bf16_gqa8_one_past_tile": (Workload("t", 1, 8, 1, (4101,), 32, 256, seed=14), jacap_params()),
+    "bf16_sinks_unbiased_nodiv": (Workload("t", 1, 8, 2, (2048, 1500), 64, 200, seed=15, sink_tokens=4,
+                                           sink_scale=4.0), jacap_params(tau=2.0, weight_div_dk=0, cov_unbiased=1)),
+    "f32_outlier_mha": (Workload("t", 1, 4, 4, (1500, 2049), 32, 128, dtype="f32", dist="outlier", seed=16,
+                                 outlier_channels=4, outlier_scale=8.0), jacap_params()),
+    "f32_gqa4_peaky": (Workload("t", 2, 8, 2, (600, 130), 8, 50, dtype="f32", seed=17), jacap_params(tau=0.5)),
+    "bf16_budget_exceeds_all": (Workload("t", 1, 4, 2, (100, 257), 8, 300, seed=18), jacap_params()),
+}
+
+
+@pytest.mark.parametrize("name", list(SMALL))
+def test_small_caches_every_unit(name):
+    wl, params = SMALL[name]
+    t = generate(wl, DEV)
+    ev = evict(make_cache(t, wl), wl.budget, params)
+    for s in range(len(wl.seqlens)):
+        for layer in range(wl.num_layers):
+            for g in range(wl.num_kv_heads):
+                check_unit(ev, t, wl, params, s, layer, g)
+    gpu_selection_properties(ev.scores, ev.idx, ev.kept, wl.seqlens, wl.budget)
+
+
+def test_intermediates_match_the_oracle():
+    wl = Workload("t", 2, 8, 2, (900, 333), 16, 64, seed=21)
+    params = jacap_params(tau=1.5)
+    t = generate(wl, DEV)
+    ev = evict(make_cache(t, wl), wl.budget, params)
+    inter = ev.intermediates()
+    G = wl.num_q_heads // wl.num_kv_heads
+    import oracle.jacap_oracle as O
+    for s in range(2):
+        for layer in range(2):
+            for g in range(2):
+                q, K, V = unit_arrays(t, wl.num_q_heads, s, layer, g)
+                for j in range(G):
+                    mu, lam = O.window_stats(q[j])
+                    h = g * G + j
+                    np.testing.assert_allclose(inter["mu_scaled"][s, layer, h].double().cpu().numpy(),
+                                               mu / (params.tau * np.sqrt(128)), rtol=1e-5, atol=1e-7)
+                    np.testing.assert_allclose(inter["lambda"][s, layer, h].double().cpu().numpy(), lam,
+                                               rtol=1e-5, atol=1e-7)
+                w = O.unit_weights(K, q, JacapParams(tau=params.tau))
+                A = O.capacity_matrix(V, w)
+                G_ora = A - np.eye(128)
+                G_gpu = inter["gram"][layer, g, s].double().cpu().numpy()
+                np.testing.assert_allclose(G_gpu, G_ora, rtol=1e-4, atol=1e-5 * np.abs(G_ora).max())
+                Lc = np.linalg.cholesky(A)
+                Minv = np.linalg.inv(Lc)
+                np.testing.assert_allclose(inter["chol_inv"][layer, g, s].double().cpu().numpy(), Minv,
+                                           rtol=1e-4, atol=1e-6)
+
+
+def test_repeat_calls_are_bitwise_deterministic():
+    wl = Workload("t", 2, 8, 2, (1500, 700), 16, 64, seed=22)
+    t = generate(wl, DEV)
+    ev = Evictor(make_cache(t, wl), wl.budget)
+    ev.run()
+    ev.check()
+    s1, i1 = ev.scores.clone(), ev.idx.clone()
+    ev.run()
+    ev.check()
+    assert torch.equal(ev.scores, s1) and torch.equal(ev.idx, i1)
+
+
+def test_strided_cache_views():
+    # K/V as views into a padded buffer (token stride 136) and a head-major
+    # buffer; the TMA maps and the gather must follow the strides.
+    wl = Workload("t", 2, 8, 2, (700, 260), 16, 64, seed=23)
+    t = generate(wl, DEV)
+    L, Hkv, N, d = t.k.shape
+    kb = torch.zeros((Hkv, L, N, 136), dtype=t.k.dtype, device=DEV)
+    vb = torch.zeros_like(kb)
+    kb[..., :d] = t.k.transpose(0, 1)
+    vb[..., :d] = t.v.transpose(0, 1)
+    k2 = kb.transpose(0, 1)[..., :d]
+    v2 = vb.transpose(0, 1)[..., :d]
+    ev_ref = evict(make_cache(t, wl), wl.budget)
+    t2 = replace(t, k=k2, v=v2)
+    ev = evict(Cache(t.q_win, k2, v2, t.cu_seqlens, t.seqlens, wl.num_q_heads), wl.budget)
+    assert torch.equal(ev.scores, ev_ref.scores)
+    assert torch.equal(ev.idx, ev_ref.idx)
+    assert torch.equal(ev.k_out, ev_ref.k_out) and torch.equal(ev.v_out, ev_ref.v_out)
+    check_unit(ev, t2, wl, jacap_params(), 1, 1, 1)
+
+
+def test_window_of_one_gives_zero_scores_and_first_positions():
+    wl = Workload("t", 1, 4, 2, (600,), 1, 40, seed=24)
+    t = generate(wl, DEV)
+    ev = evict(make_cache(t, wl), wl.budget)
+    assert bool((ev.scores == 0).all())
+    assert ev.idx[0, 0, 0].cpu().tolist() == list(range(40))
+
+
+def test_malformed_cu_seqlens_is_reported_on_the_device():
+    wl = Workload("t", 1, 4, 2, (300, 200), 8, 32, seed=25)
+    t = generate(wl, DEV)
+    bad = torch.tensor([0, 300, 400], dtype=torch.int32, device=DEV)  # does not end at N_tot
+    ev = Evictor(Cache(t.q_win, t.k, t.v, bad, [300, 100], wl.num_q_heads), wl.budget)
+    ev.run()
+    assert ev.device_status() == 1  # JACAP_ERR_INVALID_ARG
+
+
+def test_nonfinite_input_is_reported_on_the_device():
+    wl = Workload("t", 1, 4, 2, (300,), 8, 32, seed=26)
+    t = generate(wl, DEV)
+    t.k[0, 1, 17, 5] = float("nan")
+    ev = Evictor(make_cache(t, wl), wl.budget)
+    ev.run()
+    assert ev.device_status() == 5  # JACAP_ERR_NONFINITE
+
+
+def test_config1_every_unit():
+    wl = config(1)
+    t = generate(wl, DEV)
+    ev = evict(make_cache(t, wl), wl.budget)
+    for g in range(wl.num_kv_heads):
+        check_unit(ev, t, wl, jacap_params(), 0, 0, g)
+    gpu_selection_properties(ev.scores, ev.idx, ev.kept, wl.seqlens, wl.budget)
+
+
+def _sample_units(wl, count):
+    S = len(wl.seqlens)
+    cands = [(0, 0, 0), (S - 1, wl.num_layers - 1, wl.num_kv_heads - 1),
+             (S // 2, wl.num_layers // 2, wl.num_kv_heads // 2), (S // 3, 7 % wl.num_layers, 3 % wl.num_kv_heads)]
+    out = []
+    for c in cands:
+        if c not in out:
+            out.append(c)
+    return out[:count]
+
+
+@pytest.mark.parametrize("index,samples", [(2, 3), (3, 2), (4, 2), (5, 3)])
+def test_full_size_config(index, samples):
+    wl = config(index)
+    t = generate(wl, DEV)
+    ev = evict(make_cache(t, wl), wl.budget)
+    gpu_selection_properties(ev.scores, ev.idx, ev.kept, wl.seqlens, wl.budget)
+    for (s, layer, g) in _sample_units(wl, samples):
+        check_unit(ev, t, wl, jacap_params(), s, layer, g, check_w=False)
+    if index == 2:
+        for b in (128, 2048):
+            ev2 = Evictor(make_cache(t, wl), b)
+            ev2.scores.copy_(ev.scores)
+            ev2.ws[:64].zero_()  # status word: select honours the one jacap_score leaves
+            ev2.select()
+            ev2.compact()
+            gpu_selection_properties(ev2.scores, ev2.idx, ev2.kept, wl.seqlens, b)
+    del ev, t
+    torch.cuda.empty_cache()
