@@ -257,6 +257,10 @@ def run_ours(args):
     ev_score = [[torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)] for _ in range(K)]
     ev_tail = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(K)]
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    # torch creates the CUDA event lazily: record each once so its handle exists
+    for e in [x for row in ev_score + ev_tail for x in row] + [start, stop]:
+        e.record(stream)
+    torch.cuda.synchronize()
     sampler = ClockSampler(local)
     barrier()
     torch.cuda.synchronize()
