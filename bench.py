@@ -46,6 +46,8 @@ def parse():
     p.add_argument("--cpu-seconds", type=float, default=15.0)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--layers", type=int, default=None,
+                   help="override the layer count (small profiling captures; the line reports it)")
     return p.parse_args()
 
 
@@ -57,6 +59,40 @@ def peaks():
         return float(d["hbm_gbs"]), "measured"
     except Exception:
         return FALLBACK_HBM_GBS, "fallback"
+
+
+def aggregate_ranks(t_ms: float, tokens_layers: int, dist=None, device=None):
+    """Whole-job throughput over ranks: every rank processed `tokens_layers`
+    in `t_ms`; the job time is the max over ranks (weak scaling, replicas)."""
+    world = 1
+    if dist is not None and dist.is_initialized():
+        import torch
+
+        world = dist.get_world_size()
+        x = torch.tensor([float(t_ms)], dtype=torch.float64, device=device)
+        dist.all_reduce(x, op=dist.ReduceOp.MAX)
+        t_ms = float(x.item())
+        n = torch.tensor([int(tokens_layers)], dtype=torch.int64, device=device)
+        dist.all_reduce(n, op=dist.ReduceOp.SUM)
+        tokens_layers = int(n.item())
+    return tokens_layers / (t_ms * 1e-3), t_ms, world
+
+
+def recorded_traffic(kernel: str):
+    """DRAM bytes per launch of `kernel` from the committed ncu record, or None
+    when there is no record or the kernel's sources changed since the capture."""
+    import hashlib
+
+    try:
+        with open(os.path.join(ROOT, "profiles", "dram_traffic.json")) as f:
+            rec = json.load(f)["kernels"][kernel]
+        h = hashlib.sha256()
+        for src in rec["sources"]:
+            with open(os.path.join(ROOT, src), "rb") as f:
+                h.update(f.read())
+        return int(rec["traffic_bytes_per_launch"]) if h.hexdigest() == rec["source_sha256"] else None
+    except Exception:
+        return None
 
 
 class ClockSampler:
@@ -239,6 +275,8 @@ def run_ours(args):
     wl = config(args.config)
     budget = args.budget or wl.budget
     wl = replace(wl, seed=wl.seed + 1000 * rank, budget=budget)
+    if args.layers:
+        wl = replace(wl, num_layers=args.layers, name=wl.name + f", {args.layers} layers")
     t = generate(wl, dev)
     cache = Cache(t.q_win, t.k, t.v, t.cu_seqlens, t.seqlens, wl.num_q_heads)
     ev = Evictor(cache, budget)
@@ -278,10 +316,7 @@ def run_ours(args):
     barrier()
     ev.check()
     t_ms = start.elapsed_time(stop) / K
-    if dist is not None:
-        x = torch.tensor([t_ms], device=dev)
-        dist.all_reduce(x, op=dist.ReduceOp.MAX)
-        t_ms = float(x.item())
+    value, t_ms, _ = aggregate_ranks(t_ms, sum(t.seqlens) * t.k.shape[0], dist, dev)
 
     # per-kernel average durations inside the timed region
     kern = {name: 0.0 for name in SCORE_KERNEL_NAMES}
@@ -309,7 +344,6 @@ def run_ours(args):
     hbm, src = peaks()
     achieved = alg_kernel[dom] / (kern[dom] * 1e-3) / 1e9
     tokens_layers = sum(t.seqlens) * L
-    value = tokens_layers * world / (t_ms * 1e-3)
     alg_pass = wl.algorithmic_bytes(budget)
 
     cpu = None
@@ -344,7 +378,7 @@ def run_ours(args):
                 "peak": hbm,
                 "unit": "GB/s",
                 "frac": achieved / hbm,
-                "traffic": None,
+                "traffic": recorded_traffic(dom) if wl.num_layers == 32 and wl.seqlens == (32768,) else None,
                 "peak_source": f"{src} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)" if src == "measured" else "fallback",
             },
             "pass_roofline": {

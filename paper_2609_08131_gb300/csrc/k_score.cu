@@ -150,6 +150,9 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
     for (int64_t i = blockIdx.x; decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
       for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
         const int ab = it & 1;
+        const int64_t tok = t + y;
+        const int64_t o = (int64_t)item.plane * dm.Ntot + tok;
+        const float wt = tok < item.t1 ? ws.w[o] : 0.f;  // issued before the wait: hides its latency
         if (!mbar_wait(smem_u32(&accfull[ab]), (it >> 1) & 1, ws, abort)) goto epi_done;
         tc_fence_after();
         const uint32_t trow = tmem + ab * 256 + ((uint32_t)(quarter * 32) << 16);
@@ -168,10 +171,8 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_u32(&accempty[ab]));
-        const int64_t tok = t + y;
         if (tok < item.t1) {
-          const int64_t o = (int64_t)item.plane * dm.Ntot + tok;
-          const float sc = ws.w[o] * ssq;
+          const float sc = wt * ssq;
           scores[o] = sc;
           bad |= !isfinite(sc);
         }

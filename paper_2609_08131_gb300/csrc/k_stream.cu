@@ -4,7 +4,8 @@
 //                       (chunks of `chunk` tokens that never straddle requests).
 //  window_stats_kernel  mu_h and the diagonal of Lambda_Q from the last w queries
 //                       of each query head (Sec. 3.4 last paragraph; App. B.2).
-//  kpass_kernel         one streaming pass over K with TMA-staged 128-token
+//  kpass_kernel         (float32 caches; bf16 caches use k_kpass.cu) one
+//                       streaming pass over K with TMA-staged 128-token
 //                       tiles: for each token and each query head h of its group
 //                       the pool logit l = k.mu_h/(tau sqrt d) (Sec. 3.4, Alg. 1
 //                       step 1) and kappa = sum_c lambda_h,c k_c^2 (Sec. 3.4),
@@ -310,8 +311,8 @@ static cudaError_t launch_kpass_t(const CUtensorMap& kmap, const Dims& dm, const
 
 cudaError_t launch_kpass(const CUtensorMap& kmap, const Dims& dm, const Ws& ws, int dtype, const int32_t* cu,
                          int grid, cudaStream_t st) {
-  return dtype == 1 ? launch_kpass_t<__nv_bfloat16>(kmap, dm, ws, cu, grid, st)
-                    : launch_kpass_t<float>(kmap, dm, ws, cu, grid, st);
+  // bf16: logits on the tensor cores (k_kpass.cu); float32: the SIMT pass above
+  return dtype == 1 ? launch_kpass_bf16(kmap, dm, ws, cu, grid, st) : launch_kpass_t<float>(kmap, dm, ws, cu, grid, st);
 }
 
 }  // namespace jacap
