@@ -9,12 +9,13 @@
 //      w for the score pass;
 //   3. accumulates the chunk's partial Gram  sum_i w_i v_i v_i^T  (Eq. 9).
 //
-// bf16 caches use the 5th-generation tensor cores: A = V^T straight from the
-// TMA-staged tile (bf16 is exact), B = [hi | lo] where w_i v_i = hi + lo is
-// split into two bf16 halves by the scaling warps (residual error ~2^-17
-// relative per product), so one kind::f16 MMA with N = 256 yields
-// D[:, :128] + D[:, 128:] = sum_i v_i (w_i v_i)^T accumulated in fp32 in
-// tensor memory. float32 caches take a SIMT fp32 kernel of the same contract.
+// bf16 caches use the 5th-generation tensor cores. B = V straight from the
+// TMA-staged tile (bf16 is exact); the scaled operand w_i v_i = hi + lo is
+// split into two bf16 halves (residual ~2^-17 relative per product) by the
+// scaling warps and written to tensor memory as two A operands, so
+// D = sum_i (hi_i + lo_i) v_i^T accumulates in fp32 in tensor memory without
+// passing the scaled operand through shared memory. float32 caches take a
+// SIMT fp32 kernel of the same contract.
 #include "jacap_dev.cuh"
 #include "jacap_internal.h"
 
@@ -80,58 +81,71 @@ __device__ __forceinline__ float weight_from_lk(const Dims& dm, const float* ust
   return wt * dm.wdiv;
 }
 
+// Logits and kappa of heads h0 .. h0 + NH - 1 of one token (src points at
+// the token's row + h0).
+template <int G, int NH>
+__device__ __forceinline__ void load_lk_part(const float* src, float (&l)[NH], float (&k)[NH]) {
+#pragma unroll
+  for (int j = 0; j < NH; ++j) {
+    l[j] = src[j];
+    k[j] = src[G + j];
+  }
+}
+
+// Partial Eq. 8 sum over heads h0 .. h0 + NH - 1 from the logits/kappa row;
+// uinv = [M_0..M_{G-1}, 1/Z_0..1/Z_{G-1}] (the reciprocal saves a divide per head).
+template <int G, int NH>
+__device__ __forceinline__ float weight_part(const float* l, const float* kap, const float* uinv, int h0) {
+  float wt = 0.f;
+#pragma unroll
+  for (int j = 0; j < NH; ++j) {
+    const float a = expf(l[j] - uinv[h0 + j]) * uinv[G + h0 + j];  // alpha_bar
+    const float rho = a * (1.f - a);                                  // diagonal of S
+    wt = fmaf(rho * rho, kap[j], wt);                                 // rho^2 kappa
+  }
+  return wt;
+}
+
 template <int G>
 __device__ __forceinline__ float jacobian_weight(const Dims& dm, const Ws& ws, const float* ustat, int plane,
                                                  int64_t tok) {
-  const float* src = ws.lk + ((int64_t)plane * dm.Ntot + tok) * (2 * G);
   float lk[2 * G];
-  if constexpr ((2 * G) % 4 == 0) {
-#pragma unroll
-    for (int e = 0; e < 2 * G; e += 4) {
-      const float4 q4 = *(const float4*)(src + e);
-      lk[e] = q4.x; lk[e + 1] = q4.y; lk[e + 2] = q4.z; lk[e + 3] = q4.w;
-    }
-  } else {
-#pragma unroll
-    for (int e = 0; e < 2 * G; ++e) lk[e] = src[e];
-  }
-  float wt = 0.f;
-#pragma unroll
-  for (int h = 0; h < G; ++h) {
-    const float a = expf(lk[h] - ustat[h]) / ustat[G + h];  // alpha_bar
-    const float rho = a * (1.f - a);                           // diagonal of S
-    wt = fmaf(rho * rho, lk[G + h], wt);                       // rho^2 kappa
-  }
-  return wt * dm.wdiv;
+  load_lk<G>(dm, ws, plane, tok, lk);
+  return weight_from_lk<G>(dm, ustat, lk);
 }
 
 // --------------------------------------------------------------- tcgen05 ---
-constexpr int GR_THREADS = 320;  // warp 0: TMA, warp 1: MMA, warps 2-9: scale + epilogue
-constexpr int GR_SCALERS = 256;  // two threads per token row, interleaved 16-byte chunks
-constexpr int GR_VST = 3;                     // V tiles in flight (TMA ring)
-constexpr int GR_BST = 2;                     // hi/lo operand buffers
-constexpr int GR_BOX = 16384;                 // {64 channels, 128 tokens} bf16, 128-byte swizzle
-constexpr int GR_V_BYTES = 2 * GR_BOX;        // V tile
-constexpr int GR_B_BYTES = 4 * GR_BOX;        // hi (2 boxes) + lo (2 boxes)
-constexpr uint32_t GR_TMEM_COLS = 256;
-// M = 128 (channels of V^T), N = 256 (hi | lo), both operands MN-major.
-constexpr uint32_t GR_IDESC = idesc_bf16_f32(128, 256, 1, 1);
+// G = sum_i v_i (w_i v_i)^T on the tensor cores with the scaled operand in
+// tensor memory: D (128 x 128, fp32) += A (128 channels x 16 tokens, TMEM)
+// * B (16 tokens x 128 channels, the TMA-staged V tile, MN-major). Per tile
+// the scaling warps read V transposed with ldmatrix, multiply by w_i, split
+// w_i v_i = hi + lo (bf16 each) and store hi and lo as two A operands; two
+// MMAs per 16 tokens accumulate v (hi + lo)^T.
+constexpr int GR_THREADS = 320;   // warp 0: TMA, warp 1: MMA, warps 2-9: scale + epilogue
+constexpr int GR_SCALERS = 256;
+constexpr int GR_VST = 6;          // V tiles in flight
+constexpr int GR_BOX = 16384;      // {64 channels, 128 tokens} bf16, 128-byte swizzle
+constexpr int GR_V_BYTES = 2 * GR_BOX;
+constexpr uint32_t GR_TMEM_COLS = 512;
+constexpr uint32_t GR_ACOL = 128;  // A buffers: [128 + 128 ab, +64) hi, [+64, +128) lo
+// M = 128 (channels), N = 128 (channels), A in TMEM (K-major), B MN-major.
+constexpr uint32_t GR_IDESC = idesc_bf16_f32(128, 128, 0, 1);
 
-constexpr size_t gram_bf16_smem_bytes() { return 1024 + GR_VST * GR_V_BYTES + GR_BST * GR_B_BYTES + 256; }
+constexpr size_t gram_bf16_smem_bytes() { return 1024 + GR_VST * GR_V_BYTES + GR_VST * TILE * 4 + 256; }
 
 template <int G>
 __global__ void __launch_bounds__(GR_THREADS, 1)
     gram_bf16_kernel(const __grid_constant__ CUtensorMap vmap, Dims dm, Ws ws, const int32_t* __restrict__ cu) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint8_t* vring = smem;                                   // [GR_VST][GR_V_BYTES]
-  uint8_t* bring = smem + GR_VST * GR_V_BYTES;             // [GR_BST][GR_B_BYTES]
-  float* ustat = (float*)(bring + GR_BST * GR_B_BYTES);    // [2G] (<= 16 floats)
+  uint8_t* vring = smem;                                        // [GR_VST][GR_V_BYTES]
+  float* wbuf = (float*)(vring + GR_VST * GR_V_BYTES);          // [GR_VST][TILE] weights of the tile
+  float* ustat = wbuf + GR_VST * TILE;                          // [2G] (<= 16 floats)
   uint64_t* vfull = (uint64_t*)(ustat + 16);
   uint64_t* vempty = vfull + GR_VST;
-  uint64_t* bfull = vempty + GR_VST;
-  uint64_t* bempty = bfull + GR_BST;
-  uint64_t* accfull = bempty + GR_BST;
+  uint64_t* afull = vempty + GR_VST;
+  uint64_t* aempty = afull + 2;
+  uint64_t* accfull = aempty + 2;
   uint64_t* accempty = accfull + 1;
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort, s_skip;
@@ -144,9 +158,9 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
       mbar_init(smem_u32(&vfull[i]), 1);
       mbar_init(smem_u32(&vempty[i]), 1);
     }
-    for (int i = 0; i < GR_BST; ++i) {
-      mbar_init(smem_u32(&bfull[i]), GR_SCALERS / 32);
-      mbar_init(smem_u32(&bempty[i]), 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(smem_u32(&afull[i]), GR_SCALERS / 32);
+      mbar_init(smem_u32(&aempty[i]), 1);
     }
     mbar_init(smem_u32(accfull), 1);
     mbar_init(smem_u32(accempty), GR_SCALERS / 32);
@@ -201,38 +215,39 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
         tc_fence_after();
         bool first = true;
         for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
-          const int vs = it % GR_VST, bs = it % GR_BST;
+          const int vs = it % GR_VST, ab = it & 1;
           if (!mbar_wait(smem_u32(&vfull[vs]), (it / GR_VST) & 1, ws, abort) ||
-              !mbar_wait(smem_u32(&bfull[bs]), (it / GR_BST) & 1, ws, abort)) {
+              !mbar_wait(smem_u32(&afull[ab]), (it >> 1) & 1, ws, abort)) {
             ok = false;
             break;
           }
           tc_fence_after();
           const uint32_t va = smem_u32(vring + vs * GR_V_BYTES);
-          const uint32_t ba = smem_u32(bring + bs * GR_B_BYTES);
+          const uint32_t acol = tmem + GR_ACOL + 128 * ab;
 #pragma unroll
           for (int k = 0; k < TILE / 16; ++k) {  // 16 tokens per MMA
-            const uint64_t ad = smem_desc_sw128(va + k * 2048, GR_BOX, 1024);
-            const uint64_t bd = smem_desc_sw128(ba + k * 2048, GR_BOX, 1024);
-            umma_f16_ss(tmem, ad, bd, GR_IDESC, (first && k == 0) ? 0u : 1u);
+            const uint64_t bd = smem_desc_sw128(va + k * 2048, GR_BOX, 1024);
+            umma_f16_ts(tmem, acol + 8 * k, bd, GR_IDESC, (first && k == 0) ? 0u : 1u);
+            umma_f16_ts(tmem, acol + 64 + 8 * k, bd, GR_IDESC, 1u);
           }
           first = false;
           umma_commit(smem_u32(&vempty[vs]));
-          umma_commit(smem_u32(&bempty[bs]));
+          umma_commit(smem_u32(&aempty[ab]));
         }
         if (!ok) break;
         umma_commit(smem_u32(accfull));
         ++nitem;
       }
+      if (it > 0) mbar_wait(smem_u32(&aempty[(it - 1) & 1]), ((it - 1) >> 1) & 1, ws, nullptr);
     }
   } else {
     // ------------------------------------- scaling warps + epilogue -------
-    const int sidx = tid - 64;                    // 0..255
-    const int y = sidx >> 1;                      // token row 0..127 of each tile
-    const int half = sidx & 1;                    // owns the 16-byte chunks cc with cc % 2 == half
-    const int quarter = warp & 3;                 // TMEM lane quarter of this warp
-    const int m = quarter * 32 + lane;            // Gram row (channel) owned in the epilogue
-    const int colh = (warp - 2) >> 2;             // Gram columns [64 colh, 64 colh + 64) in the epilogue
+    const int sidx = tid - 64;           // 0..255
+    const int quarter = warp & 3;        // TMEM lane quarter == channels 32 quarter .. +31
+    const int th = (warp - 2) >> 2;      // token half of each tile (blocks 4 th .. 4 th + 3)
+    const int m = quarter * 32 + lane;   // Gram row (channel) owned in the epilogue
+    // ldmatrix row addresses: lane l -> matrix l / 8, row l % 8
+    const int lm = lane >> 3, lr = lane & 7;
     uint32_t it = 0, nitem = 0;
     bool bad = false;
     Item item;
@@ -248,75 +263,106 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
         }
       }
       asm volatile("bar.sync 1, 256;" ::: "memory");
-      float us[2 * G];
+      float us[2 * G];  // M_h, then 1/Z_h
 #pragma unroll
-      for (int e = 0; e < 2 * G; ++e) us[e] = ustat[e];
-      float lkc[2 * G];  // logits/kappa of this thread's token in the current tile
-      if (item.t0 + y < item.t1) load_lk<G>(dm, ws, item.plane, item.t0 + y, lkc);
+      for (int e = 0; e < G; ++e) {
+        us[e] = ustat[e];
+        us[G + e] = 1.f / ustat[G + e];
+      }
+      // weights: thread pair (2 y2, 2 y2 + 1) shares token y2; thread `part`
+      // sums heads part*NH .. part*NH + NH - 1 and one shuffle adds the halves
+      constexpr int NH = G >= 2 ? G / 2 : 1;
+      const int y2 = sidx >> 1, part = sidx & 1;
+      const bool wact = G >= 2 || part == 0;
+      const int h0 = G >= 2 ? part * NH : 0;
+      float up[2 * NH];  // [M_h, then 1/Z_h] of this thread's heads (compile-time indices)
+#pragma unroll
+      for (int j = 0; j < NH; ++j) {
+        up[j] = (G >= 2 && part) ? us[NH + j] : us[j];
+        up[NH + j] = (G >= 2 && part) ? us[G + NH + j] : us[G + j];
+      }
+      float lc[NH], kc[NH];  // this thread's logits/kappa for the current tile
+      const float* lkp = ws.lk + (int64_t)item.plane * dm.Ntot * (2 * G) + h0;
+      if (wact && item.t0 + y2 < item.t1) load_lk_part<G, NH>(lkp + (item.t0 + y2) * (2 * G), lc, kc);
 
       for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
-        const int vs = it % GR_VST, bs = it % GR_BST;
+        const int vs = it % GR_VST, ab = it & 1;
         if (!mbar_wait(smem_u32(&vfull[vs]), (it / GR_VST) & 1, ws, abort)) goto scale_done;
-        if (it >= (uint32_t)GR_BST && !mbar_wait(smem_u32(&bempty[bs]), ((it / GR_BST) & 1) ^ 1, ws, abort))
-          goto scale_done;
-        const int64_t tok = t + y;
-        const bool valid = tok < item.t1;
-        // logits/kappa of the next tile's token: issued now, used one tile later
-        float lkn[2 * G];
-        if (t + TILE + y < item.t1) load_lk<G>(dm, ws, item.plane, t + TILE + y, lkn);
-        float wt = 0.f;
-        if (valid) {
-          wt = weight_from_lk<G>(dm, us, lkc);
-          if (half == 0) {
+        float* wt_s = wbuf + vs * TILE;
+        {  // Eq. 8 weight of token t + y2
+          const int64_t tok = t + y2;
+          float ln[NH], kn[NH];
+          if (wact && t + TILE + y2 < item.t1) load_lk_part<G, NH>(lkp + (t + TILE + y2) * (2 * G), ln, kn);
+          float wp = 0.f;
+          if (wact && tok < item.t1) wp = weight_part<NH, NH>(lc, kc, up, 0);
+          const float wt = (wp + __shfl_xor_sync(0xffffffffu, wp, 1)) * dm.wdiv;
+          if (part == 0 && tok < item.t1) {
             ws.w[(int64_t)item.plane * dm.Ntot + tok] = wt;
             bad |= !isfinite(wt);
           }
-        }
+          if (part == 0) wt_s[y2] = tok < item.t1 ? wt : 0.f;
 #pragma unroll
-        for (int e = 0; e < 2 * G; ++e) lkc[e] = lkn[e];
-        const uint8_t* vt = vring + vs * GR_V_BYTES;
-        uint8_t* bt = bring + bs * GR_B_BYTES;
-        // half h owns box h (channels 64h..64h+63); at step q it takes 16-byte
-        // chunk q ^ 4h, so the 8 lanes of each shared-memory phase (4 rows x 2
-        // halves) touch 8 distinct bank groups under the 128-byte swizzle
-        uint4 raw[8];
-#pragma unroll
-        for (int q = 0; q < 8; ++q)
-          raw[q] = valid ? *(const uint4*)(vt + half * GR_BOX + sw128_off(y, q ^ (4 * half))) : make_uint4(0, 0, 0, 0);
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          const uint32_t off = half * GR_BOX + sw128_off(y, q ^ (4 * half));
-          const uint32_t rw[4] = {raw[q].x, raw[q].y, raw[q].z, raw[q].w};
-          uint32_t hw[4], lw[4];
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float x0 = wt * bf16lo(rw[e]);
-            const float x1 = wt * bf16hi(rw[e]);
-            hw[e] = pack_bf16x2(x0, x1);
-            lw[e] = pack_bf16x2(x0 - bf16lo(hw[e]), x1 - bf16hi(hw[e]));
+          for (int j = 0; j < NH; ++j) {
+            lc[j] = ln[j];
+            kc[j] = kn[j];
           }
-          *(uint4*)(bt + off) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-          *(uint4*)(bt + 2 * GR_BOX + off) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
         }
-        fence_proxy_async_smem();
+        asm volatile("bar.sync 1, 256;" ::: "memory");
+        if (it >= 2 && !mbar_wait(smem_u32(&aempty[ab]), ((it >> 1) & 1) ^ 1, ws, abort)) goto scale_done;
+        tc_fence_after();
+        const uint32_t vt = smem_u32(vring + vs * GR_V_BYTES);
+        const uint32_t acol = tmem + GR_ACOL + 128 * ab;
+#pragma unroll
+        for (int lh = 0; lh < 2; ++lh) {
+          // one 32-column slab (this warp's 4 token blocks) of hi and of lo,
+          // built in registers and written with one wide store each
+          uint32_t hi[16], lo[16];
+#pragma unroll
+          for (int blk = 0; blk < 4; ++blk) {
+            const int b = 4 * th + blk;  // 16-token block of the tile
+            // weights of this thread's token pairs: rows 2(t%4), 2(t%4)+1 of each 8-token half
+            const float2 wa = *(const float2*)(wt_s + 16 * b + 2 * (lane & 3));
+            const float2 wb = *(const float2*)(wt_s + 16 * b + 8 + 2 * (lane & 3));
+            // matrices: 0 = (tokens 0-7, ch c0..c0+7), 1 = (tokens 0-7, c0+8..), 2 = (8-15, c0..), 3 = (8-15, c0+8..)
+            const int c0 = quarter * 32 + lh * 16 + (lm & 1) * 8;
+            const int tokr = 16 * b + (lm >> 1) * 8 + lr;
+            const uint32_t addr = vt + (c0 >> 6) * GR_BOX + sw128_off(tokr, (c0 & 63) >> 3);
+            uint32_t r[4];
+            ldsm_x4_trans(addr, r[0], r[1], r[2], r[3]);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              // x = w v (exact fp32 products), hi = bf16(x), lo = bf16(x - hi)
+              const float2 x = __fmul2_rn(q < 2 ? wa : wb, make_float2(bf16lo(r[q]), bf16hi(r[q])));
+              const uint32_t h = pack_bf16x2(x.x, x.y);
+              const float2 res = __ffma2_rn(make_float2(bf16lo(h), bf16hi(h)), make_float2(-1.f, -1.f), x);
+              // registers (r0 = lanes 0-7, r1 = lanes 8-15) of columns 8 blk + 4 (q / 2) ..
+              hi[4 * blk + 2 * (q >> 1) + (q & 1)] = h;
+              lo[4 * blk + 2 * (q >> 1) + (q & 1)] = pack_bf16x2(res.x, res.y);
+            }
+          }
+          const uint32_t lanes = (uint32_t)(quarter * 32 + lh * 16) << 16;
+          tmem_st_16x128b_x8(acol + lanes + 32 * th, hi);
+          tmem_st_16x128b_x8(acol + lanes + 64 + 32 * th, lo);
+        }
+        tmem_wait_st();
+        tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(smem_u32(&bfull[bs]));
+        if (lane == 0) mbar_arrive(smem_u32(&afull[ab]));
       }
-      // epilogue: D[:, :128] + D[:, 128:] is this chunk's partial Gram
+      // epilogue: D is this chunk's partial Gram; warp (quarter, th) writes rows
+      // 32 quarter .. +31, columns 64 th .. 64 th + 63
       if (!mbar_wait(smem_u32(accfull), nitem & 1, ws, abort)) goto scale_done;
       tc_fence_after();
       {
-        const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16) + 64 * colh;
-        float* dst = ws.gpart + (((int64_t)item.plane * dm.c_cap + item.cidx) * D + m) * D + 64 * colh;
+        const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16) + 64 * th;
+        float* dst = ws.gpart + (((int64_t)item.plane * dm.c_cap + item.cidx) * D + m) * D + 64 * th;
 #pragma unroll 1
         for (int cb = 0; cb < 2; ++cb) {
-          float a[32], b[32];
+          float a[32];
           tmem_ld32(trow + cb * 32, a);
-          tmem_ld32(trow + 128 + cb * 32, b);
 #pragma unroll
           for (int j = 0; j < 32; j += 4)
-            *(float4*)(dst + cb * 32 + j) = make_float4(a[j] + b[j], a[j + 1] + b[j + 1], a[j + 2] + b[j + 2],
-                                                        a[j + 3] + b[j + 3]);
+            *(float4*)(dst + cb * 32 + j) = make_float4(a[j], a[j + 1], a[j + 2], a[j + 3]);
         }
       }
       tc_fence_before();

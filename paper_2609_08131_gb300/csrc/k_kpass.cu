@@ -6,52 +6,140 @@
 // plus an online (max, sum exp(l - max)) per work item and head, which the
 // weight pass combines into the softmax normaliser.
 //
-// Layout of the work: TMA streams 128-token K tiles (128-byte swizzle) through
-// a 6-stage ring. The logits are a 128 x 128 x N contraction per tile and run
-// on the tensor cores: B holds mu' = mu/(tau sqrt d) split exactly into three
-// bf16 parts (hi + mid + lo carries ~24 significant bits) for the G heads, and
-// the fp32 result lands in tensor memory. kappa needs elementwise squares and
-// runs on the CUDA cores: eight lanes share a token, each keeps its 16
-// channels of lambda in registers and the G partial sums are combined with a
-// reduce-scatter over the eight lanes. Two groups of four warps take
-// alternate tiles; each reads back the logits of its tile from tensor memory
-// (one thread per token), writes l and kappa, and keeps the online statistics.
+// Both sums are 128 x 128 x N contractions per 128-token tile and run on the
+// tensor cores, with fp32 accumulation in tensor memory:
+//   logits: A = the TMA-staged K tile (shared memory, K-major), B = mu' =
+//           mu / (tau sqrt d) split exactly into three bf16 parts (hi + mid +
+//           lo carries ~24 significant bits) for the G heads;
+//   kappa:  A = k^2 in tensor memory, B = lambda split the same way. A bf16
+//           k has 8 significant bits, so k^2 is exact in fp32 and splits
+//           exactly into hi = k^2 truncated to bf16 plus lo = k^2 - hi (at
+//           most 8 significant bits, exact in bf16); two MMA chains add hi
+//           and lo.
+// Each thread of a compute group owns one token row (its tensor-memory lane):
+// it reads the row once from shared memory, writes hi and lo of k^2 into
+// tensor memory with wide stores, and reads the logits and kappa back. Three
+// groups of four warps (two for G = 8) take tiles round-robin, each with its
+// own k^2 buffer, so one group's MMAs run while the others build; a group
+// reads a tile back only after building its next one. TMA keeps six tiles in
+// flight.
 #include "jacap_dev.cuh"
 #include "jacap_internal.h"
 
 namespace jacap {
 
-constexpr int KB_THREADS = 320;  // warp 0: TMA, warp 1: mu image + MMA, warps 2-9: two compute groups
 constexpr int KB_STAGES = 6;
 constexpr int KB_BOX = 16384;    // {64 channels, 128 tokens} bf16
 constexpr int KB_TILE_BYTES = 2 * KB_BOX;
-constexpr int KB_NACC = 4;       // tensor-memory logit buffers
-constexpr uint32_t KB_TMEM_COLS = 128;
+constexpr int KB_NACC = 4;       // tensor-memory result buffers
+constexpr uint32_t KB_TMEM_COLS = 512;
 
 template <int G>
 struct KbCfg {
-  static constexpr int NB = (3 * G <= 16) ? 16 : 32;  // MMA N = rows of the mu image
+  static constexpr int NB = (3 * G <= 16) ? 16 : 32;  // MMA N = rows of each B image
+  static constexpr int DC = 2 * NB;                    // result columns per buffer: logits, then kappa
+  static constexpr int NG = G == 8 ? 2 : 3;            // compute groups (each 4 warps + a k^2 buffer)
+  static constexpr int THREADS = 64 + 128 * NG;        // warp 0: TMA, warp 1: B images + MMA, then groups
+  static constexpr uint32_t ACOL = KB_TMEM_COLS - 128 * NG;  // k^2 of group g: [ACOL + 128 g, +64) hi, [+64, +128) lo
+  static_assert(KB_NACC * DC <= (int)ACOL, "tensor memory budget");
   static constexpr int IMG_ATOM = NB * 128;            // bytes per 64-channel atom
   static constexpr int IMG_BYTES = 2 * IMG_ATOM;
   static constexpr uint32_t IDESC = idesc_bf16_f32(128, NB, 0, 0);
-  static constexpr size_t SMEM = 1024 + (size_t)KB_STAGES * KB_TILE_BYTES + 2 * IMG_BYTES +
-                                 (size_t)2 * 128 * 2 * G * 4 + 256;
+  static constexpr size_t SMEM = 1024 + (size_t)KB_STAGES * KB_TILE_BYTES + 4 * IMG_BYTES + 4 * NG * 2 * G * 4 + 256;
 };
 
+// B image of one item: rows n = part * G + h hold part (0 hi, 1 mid, 2 lo) of
+// src[h][0..127], K-major with the 128-byte swizzle (two 64-channel atoms).
 template <int G>
-__global__ void __launch_bounds__(KB_THREADS, 1)
+__device__ __forceinline__ void build_split_image(uint8_t* im, const float* src, int lane) {
+  using C = KbCfg<G>;
+  for (int e = lane; e < C::NB * 16; e += 32) {
+    const int n = e >> 4, cc = e & 15;
+    uint32_t wv[4] = {0u, 0u, 0u, 0u};
+    if (n < 3 * G) {
+      const int part = n / G, h = n % G;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        float x[2];
+#pragma unroll
+        for (int z = 0; z < 2; ++z) {
+          const float v = src[h * D + cc * 8 + 2 * q + z];
+          const float hi = __bfloat162float(__float2bfloat16_rn(v));
+          const float r1 = v - hi;
+          const float mid = __bfloat162float(__float2bfloat16_rn(r1));
+          x[z] = part == 0 ? hi : (part == 1 ? mid : r1 - mid);
+        }
+        wv[q] = pack_bf16x2(x[0], x[1]);
+      }
+    }
+    *(uint4*)(im + (cc >> 3) * C::IMG_ATOM + sw128_off(n, cc & 7)) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+  }
+}
+
+// Read back the logits and kappa of own tile `pit` (token row y of the tile
+// starting at `pt`), release its result buffer, write l and kappa, and fold
+// the logits into the running softmax statistics. False after an abort.
+template <int G>
+__device__ __forceinline__ bool kb_readout(uint32_t tmem, uint32_t lanes, uint64_t* accfull, uint64_t* accempty,
+                                           uint32_t pit, int64_t pt, const Item& item, int y, int lane,
+                                           const Dims& dm, const Ws& ws, volatile int* abort, float (&run_m)[G],
+                                           float (&run_s)[G], bool& bad) {
+  using C = KbCfg<G>;
+  const int ab = pit % KB_NACC;
+  if (!mbar_wait(smem_u32(&accfull[ab]), (pit / KB_NACC) & 1, ws, abort)) return false;
+  tc_fence_after();
+  float dv[C::DC];
+  const uint32_t ta = tmem + ab * C::DC + lanes;
+  tmem_ld32(ta, dv);
+  if constexpr (C::DC == 64) tmem_ld32(ta + 32, dv + 32);
+  tc_fence_before();
+  __syncwarp();
+  if (lane == 0) mbar_arrive(smem_u32(&accempty[ab]));
+  const int64_t tok = pt + y;
+  if (tok < item.t1) {
+    float out[2 * G];
+#pragma unroll
+    for (int h = 0; h < G; ++h) {
+      const float lg = dv[h] + dv[G + h] + dv[2 * G + h];
+      const float kp = dv[C::NB + h] + dv[C::NB + G + h] + dv[C::NB + 2 * G + h];
+      out[h] = lg;
+      out[G + h] = kp;
+      bad |= !isfinite(lg) || !isfinite(kp);
+      if (lg > run_m[h]) {
+        run_s[h] = run_s[h] * expf(run_m[h] - lg) + 1.f;
+        run_m[h] = lg;
+      } else {
+        run_s[h] += expf(lg - run_m[h]);
+      }
+    }
+    float* dst = ws.lk + ((int64_t)item.plane * dm.Ntot + tok) * (2 * G);
+    if constexpr ((2 * G) % 4 == 0) {
+#pragma unroll
+      for (int e = 0; e < 2 * G; e += 4) *(float4*)(dst + e) = make_float4(out[e], out[e + 1], out[e + 2], out[e + 3]);
+    } else {
+#pragma unroll
+      for (int e = 0; e < 2 * G; ++e) dst[e] = out[e];
+    }
+  }
+  return true;
+}
+
+template <int G>
+__global__ void __launch_bounds__(KbCfg<G>::THREADS, 1)
     kpass_bf16_kernel(const __grid_constant__ CUtensorMap kmap, Dims dm, Ws ws, const int32_t* __restrict__ cu) {
   using C = KbCfg<G>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t* tiles = smem;
-  uint8_t* img = tiles + KB_STAGES * KB_TILE_BYTES;                  // [2][IMG_BYTES]
-  float* red = (float*)(img + 2 * C::IMG_BYTES);                      // [2 groups][128][2G]
-  uint64_t* full = (uint64_t*)(red + 2 * 128 * 2 * G);
+  uint8_t* img = tiles + KB_STAGES * KB_TILE_BYTES;  // [parity][mu, lambda][IMG_BYTES]
+  float* red = (float*)(img + 4 * C::IMG_BYTES);      // [compute warps][2G]
+  uint64_t* full = (uint64_t*)(red + 4 * C::NG * 2 * G);
   uint64_t* empty = full + KB_STAGES;
   uint64_t* accfull = empty + KB_STAGES;
   uint64_t* accempty = accfull + KB_NACC;
-  uint64_t* imgfree = accempty + KB_NACC;
+  uint64_t* afull = accempty + KB_NACC;
+  uint64_t* aempty = afull + 3;
+  uint64_t* imgfree = aempty + 3;
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort, s_skip;
 
@@ -66,6 +154,10 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
     for (int i = 0; i < KB_NACC; ++i) {
       mbar_init(smem_u32(&accfull[i]), 1);
       mbar_init(smem_u32(&accempty[i]), 4);
+    }
+    for (int i = 0; i < C::NG; ++i) {
+      mbar_init(smem_u32(&afull[i]), 4);
+      mbar_init(smem_u32(&aempty[i]), 1);
     }
     mbar_init(smem_u32(&imgfree[0]), 1);
     mbar_init(smem_u32(&imgfree[1]), 1);
@@ -110,7 +202,7 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
         mbar_wait(smem_u32(&full[k % KB_STAGES]), (k / KB_STAGES) & 1, ws, nullptr);
     }
   } else if (warp == 1) {
-    // ------------------------------------ mu image builder + MMA issuer ---
+    // ------------------------------------------ B images + MMA issuer -----
     uint32_t it = 0, nitem = 0;
     bool ok = true;
     Item item;
@@ -118,39 +210,22 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
       const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
       const int p = nitem & 1;
       if (nitem >= 2 && !mbar_wait(smem_u32(&imgfree[p]), ((nitem >> 1) - 1) & 1, ws, abort)) break;
-      // B image rows n = part * G + h (part 0/1/2 = hi/mid/lo of mu'_h), K-major, 128-byte swizzle
-      uint8_t* im = img + p * C::IMG_BYTES;
-      const float* mu = ws.mu + (((int64_t)item.seq * dm.L + l) * dm.Hq + (int64_t)g * G) * D;
-      for (int e = lane; e < C::NB * 16; e += 32) {
-        const int n = e >> 4, cc = e & 15;
-        uint32_t wv[4] = {0u, 0u, 0u, 0u};
-        if (n < 3 * G) {
-          const int part = n / G, h = n % G;
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            float x[2];
-#pragma unroll
-            for (int z = 0; z < 2; ++z) {
-              const float v = mu[h * D + cc * 8 + 2 * q + z];
-              const float hi = __bfloat162float(__float2bfloat16_rn(v));
-              const float r1 = v - hi;
-              const float mid = __bfloat162float(__float2bfloat16_rn(r1));
-              x[z] = part == 0 ? hi : (part == 1 ? mid : r1 - mid);
-            }
-            wv[q] = pack_bf16x2(x[0], x[1]);
-          }
-        }
-        *(uint4*)(im + (cc >> 3) * C::IMG_ATOM + sw128_off(n, cc & 7)) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
-      }
+      uint8_t* im_mu = img + (2 * p) * C::IMG_BYTES;
+      uint8_t* im_lam = img + (2 * p + 1) * C::IMG_BYTES;
+      const int64_t qb = (((int64_t)item.seq * dm.L + l) * dm.Hq + (int64_t)g * G) * D;
+      build_split_image<G>(im_mu, ws.mu + qb, lane);
+      build_split_image<G>(im_lam, ws.lam + qb, lane);
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) {
         tc_fence_after();
-        const uint32_t ia = smem_u32(im);
+        const uint32_t ia = smem_u32(im_mu), il = smem_u32(im_lam);
         for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
           const int st = it % KB_STAGES;
           const int ab = it % KB_NACC;
+          const int grp = it % C::NG;
           if (!mbar_wait(smem_u32(&full[st]), (it / KB_STAGES) & 1, ws, abort) ||
+              !mbar_wait(smem_u32(&afull[grp]), (it / C::NG) & 1, ws, abort) ||
               (it >= (uint32_t)KB_NACC &&
                !mbar_wait(smem_u32(&accempty[ab]), ((it / KB_NACC) & 1) ^ 1, ws, abort))) {
             ok = false;
@@ -158,13 +233,20 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
           }
           tc_fence_after();
           const uint32_t ka = smem_u32(tiles + st * KB_TILE_BYTES);
+          const uint32_t dl = tmem + ab * C::DC;  // logits
+          const uint32_t dk = dl + C::NB;         // kappa: hi and lo parts of k^2 accumulate here
+          const uint32_t aq = tmem + C::ACOL + 128 * grp;
 #pragma unroll
-          for (int k = 0; k < D / 16; ++k) {  // 16 channels per MMA
+          for (int k = 0; k < D / 16; ++k) {  // 16 channels per MMA; three chains interleaved
             const uint64_t ad = smem_desc_sw128(ka + (k >> 2) * KB_BOX + (k & 3) * 32, 16, 1024);
-            const uint64_t bd = smem_desc_sw128(ia + (k >> 2) * C::IMG_ATOM + (k & 3) * 32, 16, 1024);
-            umma_f16_ss(tmem + ab * 32, ad, bd, C::IDESC, k > 0 ? 1u : 0u);
+            const uint64_t bm = smem_desc_sw128(ia + (k >> 2) * C::IMG_ATOM + (k & 3) * 32, 16, 1024);
+            const uint64_t bl = smem_desc_sw128(il + (k >> 2) * C::IMG_ATOM + (k & 3) * 32, 16, 1024);
+            umma_f16_ss(dl, ad, bm, C::IDESC, k > 0 ? 1u : 0u);
+            umma_f16_ts(dk, aq + 8 * k, bl, C::IDESC, k > 0 ? 1u : 0u);
+            umma_f16_ts(dk, aq + 64 + 8 * k, bl, C::IDESC, 1u);
           }
           umma_commit(smem_u32(&empty[st]));
+          umma_commit(smem_u32(&aempty[grp]));
           umma_commit(smem_u32(&accfull[ab]));
         }
         if (ok) umma_commit(smem_u32(&imgfree[p]));
@@ -178,152 +260,94 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
       mbar_wait(smem_u32(&accfull[(it - 1) % KB_NACC]), ((it - 1) / KB_NACC) & 1, ws, nullptr);
   } else {
     // ---------------------------------------------- compute groups --------
-    const int grp = (warp - 2) >> 2;        // tiles with it % 2 == grp
-    const int wg = (warp - 2) & 3;          // warp index within the group == TMEM lane quarter
+    const int grp = (warp - 2) >> 2;        // tiles with it % NG == grp
     const int quarter = warp & 3;
-    const int y = quarter * 32 + lane;      // token row owned for the logits (TMEM lane)
-    const int sub = lane & 7;               // kappa: lane within the 8-lane token group
-    const int tg = wg * 4 + (lane >> 3);    // kappa: token group 0..15 of the group
-    const int gidx = tid - 64;              // 0..255 across both groups
+    const int y = quarter * 32 + lane;      // token row owned (tensor-memory lane)
+    const uint32_t lanes = (uint32_t)(quarter * 32) << 16;
+    const uint32_t aq = tmem + C::ACOL + 128 * grp + lanes;
     uint32_t it = 0;
     bool bad = false;
     Item item;
     for (int64_t i = blockIdx.x; decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
-      const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
-      // lambda of this lane's 16 channels (8 sub..8 sub+7 and 64+8 sub..), all heads
-      float lam[G][16];
-      {
-        const float* lp = ws.lam + (((int64_t)item.seq * dm.L + l) * dm.Hq + (int64_t)g * G) * D;
-#pragma unroll
-        for (int h = 0; h < G; ++h) {
-#pragma unroll
-          for (int q = 0; q < 8; q += 4) {
-            const float4 a = *(const float4*)(lp + h * D + 8 * sub + q);
-            const float4 b = *(const float4*)(lp + h * D + 64 + 8 * sub + q);
-            lam[h][q] = a.x; lam[h][q + 1] = a.y; lam[h][q + 2] = a.z; lam[h][q + 3] = a.w;
-            lam[h][8 + q] = b.x; lam[h][8 + q + 1] = b.y; lam[h][8 + q + 2] = b.z; lam[h][8 + q + 3] = b.w;
-          }
-        }
-      }
       float run_m[G], run_s[G];
 #pragma unroll
       for (int h = 0; h < G; ++h) {
         run_m[h] = -INFINITY;
         run_s[h] = 0.f;
       }
+      // The readout of an own tile is deferred until the group has built the
+      // k^2 operand of its next own tile, so the tile's MMAs run meanwhile.
+      bool have = false;
+      uint32_t p_it = 0;
+      int64_t p_t = 0;
       for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
-        if ((int)(it & 1) != grp) continue;
+        if ((int)(it % C::NG) != grp) continue;
         const int st = it % KB_STAGES;
-        const int ab = it % KB_NACC;
         if (!mbar_wait(smem_u32(&full[st]), (it / KB_STAGES) & 1, ws, abort)) goto compute_done;
+        if (it >= (uint32_t)C::NG &&
+            !mbar_wait(smem_u32(&aempty[grp]), ((it / C::NG) & 1) ^ 1, ws, abort))
+          goto compute_done;
+        tc_fence_after();
         const uint8_t* kt = tiles + st * KB_TILE_BYTES;
-        // ---- kappa: 8 steps of 16 tokens, 8 lanes per token ----
-        uint4 rr[16];  // this lane's two 16-byte chunks of its token row, all 8 steps
+        // ---- k^2 = hi + lo (exact) into tensor memory, 32 channels at a time ----
 #pragma unroll
-        for (int s8 = 0; s8 < 8; ++s8) {
-          const int yk = 16 * s8 + tg;
-          rr[2 * s8] = *(const uint4*)(kt + sw128_off(yk, sub));
-          rr[2 * s8 + 1] = *(const uint4*)(kt + KB_BOX + sw128_off(yk, sub));
-        }
+        for (int cq = 0; cq < 4; ++cq) {
+          uint32_t hi[16], lo[16];
 #pragma unroll
-        for (int s8 = 0; s8 < 8; ++s8) {
-          const int yk = 16 * s8 + tg;
-          const uint32_t rw[8] = {rr[2 * s8].x, rr[2 * s8].y, rr[2 * s8].z, rr[2 * s8].w,
-                                  rr[2 * s8 + 1].x, rr[2 * s8 + 1].y, rr[2 * s8 + 1].z, rr[2 * s8 + 1].w};
-          float2 acc[G];
+          for (int j = 0; j < 4; ++j) {
+            const int ch = 4 * cq + j;  // 16-byte chunk: channels 8 ch .. 8 ch + 7
+            const uint4 raw = *(const uint4*)(kt + (ch >> 3) * KB_BOX + sw128_off(y, ch & 7));
+            const uint32_t rw[4] = {raw.x, raw.y, raw.z, raw.w};
 #pragma unroll
-          for (int h = 0; h < G; ++h) acc[h] = make_float2(0.f, 0.f);
-#pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            const float2 kk = make_float2(bf16lo(rw[q]), bf16hi(rw[q]));
-            const float2 sq = __fmul2_rn(kk, kk);
-#pragma unroll
-            for (int h = 0; h < G; ++h) acc[h] = __ffma2_rn(sq, make_float2(lam[h][2 * q], lam[h][2 * q + 1]), acc[h]);
-          }
-          float v[G];
-#pragma unroll
-          for (int h = 0; h < G; ++h) v[h] = acc[h].x + acc[h].y;
-          // reduce-scatter of the G sums over the 8 lanes of the token group
-          int base = 0;  // first head index this lane still holds
-#pragma unroll
-          for (int span = G, bit = 4; bit >= 1; bit >>= 1) {
-            if (span > 1) {
-              const int halfspan = span >> 1;
-              const bool upper = (sub & bit) != 0;
-#pragma unroll
-              for (int j = 0; j < halfspan; ++j) {
-                const float send = upper ? v[j] : v[halfspan + j];
-                const float recv = __shfl_xor_sync(0xffffffffu, send, bit);
-                v[j] = (upper ? v[halfspan + j] : v[j]) + recv;
-              }
-              if (upper) base += halfspan;
-              span = halfspan;
-            } else {
-              v[0] += __shfl_xor_sync(0xffffffffu, v[0], bit);
+            for (int q = 0; q < 4; ++q) {
+              const float2 kk = make_float2(bf16lo(rw[q]), bf16hi(rw[q]));
+              const float2 sq = __fmul2_rn(kk, kk);
+              const uint32_t s0 = __float_as_uint(sq.x), s1 = __float_as_uint(sq.y);
+              const float2 ht = make_float2(__uint_as_float(s0 & 0xFFFF0000u), __uint_as_float(s1 & 0xFFFF0000u));
+              const float2 rr = __ffma2_rn(ht, make_float2(-1.f, -1.f), sq);
+              hi[4 * j + q] = __byte_perm(s0, s1, 0x7632);
+              lo[4 * j + q] = __byte_perm(__float_as_uint(rr.x), __float_as_uint(rr.y), 0x7632);
             }
           }
-          // lanes that end with the same head hold equal sums; the lowest writes
-          const int64_t tokk = t + yk;
-          constexpr int REP = G >= 8 ? 1 : 8 / G;  // lanes per finished head
-          if (tokk < item.t1 && (sub % REP) == 0) {
-            ws.lk[((int64_t)item.plane * dm.Ntot + tokk) * (2 * G) + G + base] = v[0];
-            bad |= !isfinite(v[0]);
-          }
+          tmem_st_32x32b_x16(aq + 16 * cq, hi);
+          tmem_st_32x32b_x16(aq + 64 + 16 * cq, lo);
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_u32(&empty[st]));
-        // ---- logits from tensor memory: one thread per token ----
-        if (!mbar_wait(smem_u32(&accfull[ab]), (it / KB_NACC) & 1, ws, abort)) goto compute_done;
-        tc_fence_after();
-        float dv[C::NB];
-        const uint32_t ta = tmem + ab * 32 + ((uint32_t)(quarter * 32) << 16);
-        if constexpr (C::NB == 16) tmem_ld16(ta, dv); else tmem_ld32(ta, dv);
+        tmem_wait_st();
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(smem_u32(&accempty[ab]));
-        const int64_t tok = t + y;
-        if (tok < item.t1) {
-          float lg[G];
-#pragma unroll
-          for (int h = 0; h < G; ++h) {
-            lg[h] = dv[h] + dv[G + h] + dv[2 * G + h];
-            bad |= !isfinite(lg[h]);
-            if (lg[h] > run_m[h]) {
-              run_s[h] = run_s[h] * expf(run_m[h] - lg[h]) + 1.f;
-              run_m[h] = lg[h];
-            } else {
-              run_s[h] += expf(lg[h] - run_m[h]);
-            }
-          }
-          float* dst = ws.lk + ((int64_t)item.plane * dm.Ntot + tok) * (2 * G);
-          if constexpr (G % 4 == 0) {
-#pragma unroll
-            for (int h = 0; h < G; h += 4) *(float4*)(dst + h) = make_float4(lg[h], lg[h + 1], lg[h + 2], lg[h + 3]);
-          } else {
-#pragma unroll
-            for (int h = 0; h < G; ++h) dst[h] = lg[h];
-          }
-        }
+        if (lane == 0) mbar_arrive(smem_u32(&afull[grp]));
+        if (have && !kb_readout<G>(tmem, lanes, accfull, accempty, p_it, p_t, item, y, lane, dm, ws, abort, run_m,
+                                   run_s, bad))
+          goto compute_done;
+        have = true;
+        p_it = it;
+        p_t = t;
       }
+      if (have && !kb_readout<G>(tmem, lanes, accfull, accempty, p_it, p_t, item, y, lane, dm, ws, abort, run_m,
+                                 run_s, bad))
+        goto compute_done;
       // ---- per-item softmax statistics: warp butterflies, then 8 warps ----
+      const int cw = warp - 2;
 #pragma unroll
       for (int h = 0; h < G; ++h) {
         softmax_warp_merge(run_m[h], run_s[h]);
         if (lane == 0) {
-          red[(gidx >> 5) * 2 * G + h] = run_m[h];
-          red[(gidx >> 5) * 2 * G + G + h] = run_s[h];
+          red[cw * 2 * G + h] = run_m[h];
+          red[cw * 2 * G + G + h] = run_s[h];
         }
       }
-      asm volatile("bar.sync 1, 256;" ::: "memory");
-      if (gidx < G) {
-        const int h = gidx;
+      named_barrier_sync(1, 128 * C::NG);
+      if (tid - 64 < G) {
+        const int h = tid - 64;
         float m = -INFINITY, ssum = 0.f;
-        for (int j = 0; j < 8; ++j) softmax_merge(m, ssum, red[j * 2 * G + h], red[j * 2 * G + G + h]);
+        for (int j = 0; j < 4 * C::NG; ++j) softmax_merge(m, ssum, red[j * 2 * G + h], red[j * 2 * G + G + h]);
         float* cs = ws.cstats + (((int64_t)item.plane * dm.c_cap + item.cidx) * G + h) * 2;
         cs[0] = m;
         cs[1] = ssum;
       }
-      asm volatile("bar.sync 1, 256;" ::: "memory");
+      named_barrier_sync(1, 128 * C::NG);
     }
   compute_done:
     if (bad) flag(ws, ST_NONFINITE);
@@ -343,7 +367,7 @@ static cudaError_t launch_g(const CUtensorMap& kmap, const Dims& dm, const Ws& w
   static_assert(smem <= 232448, "shared memory budget");
   cudaError_t e = cudaFuncSetAttribute(kpass_bf16_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  kpass_bf16_kernel<G><<<grid, KB_THREADS, smem, st>>>(kmap, dm, ws, cu);
+  kpass_bf16_kernel<G><<<grid, KbCfg<G>::THREADS, smem, st>>>(kmap, dm, ws, cu);
   return cudaGetLastError();
 }
 
