@@ -23,7 +23,8 @@
  * Conventions for every entry point
  *  - Pointers named *_host are host memory; every other data pointer is device
  *    memory on the current CUDA device. The caller owns all memory; the library
- *    allocates nothing and keeps no mutable global state.
+ *    allocates nothing and keeps no mutable global state (the one exception is
+ *    the static scratch of jacap_score_static).
  *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
  *    All work is enqueued asynchronously on it; nothing synchronises except
  *    jacap_device_status().
@@ -146,6 +147,31 @@ jacap_status jacap_score_timed(const jacap_layout* layout, const jacap_params* p
                                const void* q_win, const void* k, const void* v, float* scores,
                                void* ws, size_t ws_bytes, void* stream,
                                void* const* events, int32_t num_events);
+
+/*
+ * jacap_score for callers that cannot allocate device memory (the paper has no
+ * counterpart; this is a deployment convenience). The workspace is a fixed
+ * library-owned array of JACAP_STATIC_SCRATCH_BYTES in static device memory,
+ * one per device; no call allocates. The work and results are those of
+ * jacap_score with a caller workspace.
+ *  - Layouts whose jacap_workspace_size() exceeds JACAP_STATIC_SCRATCH_BYTES
+ *    are refused with JACAP_ERR_WORKSPACE before any CUDA call; an invalid
+ *    or unsupported layout gives the status jacap_score would.
+ *  - The first call on a device (that device current) looks up the scratch
+ *    address with cudaGetSymbolAddress, which loads the module's static memory;
+ *    make that first call before capturing the stream into a graph.
+ *  - scratch_out (may be NULL) receives the scratch's device address; it is
+ *    laid out as a workspace (see jacap_workspace_offsets) and can be passed
+ *    as `ws` to jacap_select and jacap_device_status. Its status word is reset
+ *    by every call; nothing else needs to start at zero.
+ *  - Every call on a device shares that one scratch: calls (and any use of the
+ *    returned address) that overlap in time race and corrupt each other's
+ *    results. Serialise them, e.g. on one stream.
+ */
+#define JACAP_STATIC_SCRATCH_BYTES ((size_t)64 << 20)
+jacap_status jacap_score_static(const jacap_layout* layout, const jacap_params* params,
+                                const void* q_win, const void* k, const void* v, float* scores,
+                                void* stream, void** scratch_out);
 
 /*
  * TOP-B per unit (Algorithm 1 step 5). Reads `scores` as written by

@@ -83,6 +83,8 @@ _SIGS = {
                                    ctypes.c_size_t, _P]),
     "jacap_score_timed": (ctypes.c_int, [ctypes.POINTER(jacap_layout), ctypes.POINTER(jacap_params), _P, _P, _P, _P,
                                          _P, ctypes.c_size_t, _P, ctypes.POINTER(ctypes.c_void_p), ctypes.c_int32]),
+    "jacap_score_static": (ctypes.c_int, [ctypes.POINTER(jacap_layout), ctypes.POINTER(jacap_params), _P, _P, _P,
+                                          _P, _P, ctypes.POINTER(ctypes.c_void_p)]),
     "jacap_select": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, ctypes.c_int32, _P, _P, _P, ctypes.c_size_t,
                                     _P]),
     "jacap_compact": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, _P, _P, ctypes.c_int32, _P, _P, _P]),
@@ -122,6 +124,18 @@ def jacap_score_timed(layout, params, q_win, k, v, scores, ws, ws_bytes, stream,
     arr = (ctypes.c_void_p * max(1, len(events)))(*[ctypes.c_void_p(e) for e in events])
     return lib().jacap_score_timed(ctypes.byref(layout), ctypes.byref(params), q_win, k, v, scores, ws, ws_bytes,
                                    stream, arr, len(events))
+
+
+JACAP_STATIC_SCRATCH_BYTES = 64 << 20
+
+
+def jacap_score_static(layout, params, q_win, k, v, scores, stream):
+    """Returns ``(status, scratch)``: ``scratch`` is the device address of the
+    library-owned workspace the call used (0 when it was refused)."""
+    out = ctypes.c_void_p(0)
+    st = lib().jacap_score_static(ctypes.byref(layout), ctypes.byref(params), q_win, k, v, scores, stream,
+                                  ctypes.byref(out))
+    return st, out.value or 0
 
 
 def jacap_select(layout, scores, budget, idx, kept, ws, ws_bytes, stream) -> int:

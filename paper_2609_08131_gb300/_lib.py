@@ -22,7 +22,8 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libjacap.so")
 
-SOURCES = ["jacap_api.cu", "k_stream.cu", "k_kpass.cu", "k_gram.cu", "k_factor.cu", "k_score.cu", "k_select.cu"]
+SOURCES = ["jacap_api.cu", "k_stream.cu", "k_kpass.cu", "k_gram.cu", "k_factor.cu", "k_score.cu", "k_select.cu",
+           "jacap_static.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
           "-I" + INCLUDE, "-I" + CSRC]
@@ -89,6 +90,7 @@ EXPORTS = [
     "jacap_workspace_size",
     "jacap_score",
     "jacap_score_timed",
+    "jacap_score_static",
     "jacap_select",
     "jacap_compact",
     "jacap_device_status",
