@@ -333,9 +333,11 @@ def run_ours(args):
     es = t.k.element_size()
     kv_bytes = L * Hkv * N * d * es
     kept_rows = L * Hkv * sum(min(n, budget) for n in t.seqlens)
+    G = wl.num_q_heads // wl.num_kv_heads
     alg_kernel = {
         "k_pass": kv_bytes,                       # K read once
-        "weight_gram": kv_bytes,                  # V read once
+        "weights": L * Hkv * N * (8 * G + 8),     # logits + kappa read, w and its bf16 split written
+        "gram": kv_bytes,                         # V read once
         "scores": kv_bytes + L * Hkv * N * 4,     # V read, scores written
         "select": L * Hkv * N * 4,                # scores read
         "compact": 4 * kept_rows * d * es,        # retained K, V read and written

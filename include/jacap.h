@@ -126,9 +126,9 @@ size_t jacap_workspace_size(const jacap_layout* layout, int32_t budget);
  *               score of token t of plane (l, g); r_i of Eq. 10.
  *  ws, ws_bytes device workspace of at least jacap_workspace_size() bytes.
  * Resets the status word, then enqueues: query statistics, a streaming pass
- * over K (logits, kappa, softmax statistics), a fused weight + weighted-Gram
- * pass over V (tensor cores for bf16), the Cholesky factor and inverse of A,
- * and the quadratic forms.
+ * over K (logits, kappa, softmax statistics), the Eq. 8 weights, the
+ * weighted-Gram pass over V (tensor cores for bf16), the Cholesky factor and
+ * inverse of A, and the quadratic forms.
  */
 jacap_status jacap_score(const jacap_layout* layout, const jacap_params* params,
                          const void* q_win, const void* k, const void* v, float* scores,
@@ -140,9 +140,9 @@ jacap_status jacap_score(const jacap_layout* layout, const jacap_params* params,
  * events[num_events - 1] after the last one. `events` holds cudaEvent_t
  * handles (as void*) created by the caller; num_events must be 0 (no hooks)
  * or JACAP_SCORE_KERNELS + 1. Kernel order: plan, query statistics, K pass,
- * weight + Gram, factor, scores.
+ * weights, Gram, factor, scores.
  */
-#define JACAP_SCORE_KERNELS 6
+#define JACAP_SCORE_KERNELS 7
 jacap_status jacap_score_timed(const jacap_layout* layout, const jacap_params* params,
                                const void* q_win, const void* k, const void* v, float* scores,
                                void* ws, size_t ws_bytes, void* stream,

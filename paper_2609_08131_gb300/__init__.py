@@ -115,12 +115,12 @@ def jacap_score(layout, params, q_win, k, v, scores, ws, ws_bytes, stream) -> in
     return lib().jacap_score(ctypes.byref(layout), ctypes.byref(params), q_win, k, v, scores, ws, ws_bytes, stream)
 
 
-JACAP_SCORE_KERNELS = 6
-SCORE_KERNEL_NAMES = ("plan", "query_stats", "k_pass", "weight_gram", "factor", "scores")
+JACAP_SCORE_KERNELS = 7
+SCORE_KERNEL_NAMES = ("plan", "query_stats", "k_pass", "weights", "gram", "factor", "scores")
 
 
 def jacap_score_timed(layout, params, q_win, k, v, scores, ws, ws_bytes, stream, events) -> int:
-    """``events``: sequence of cudaEvent_t handles (ints), length 0 or 7."""
+    """``events``: sequence of cudaEvent_t handles (ints), length 0 or JACAP_SCORE_KERNELS + 1."""
     arr = (ctypes.c_void_p * max(1, len(events)))(*[ctypes.c_void_p(e) for e in events])
     return lib().jacap_score_timed(ctypes.byref(layout), ctypes.byref(params), q_win, k, v, scores, ws, ws_bytes,
                                    stream, arr, len(events))

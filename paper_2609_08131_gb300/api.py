@@ -114,8 +114,8 @@ class Evictor:
         self.v_out = torch.empty_like(self.k_out)
 
     def score(self, stream=None, events=None):
-        """jacap_score; with ``events`` (7 torch.cuda.Event objects) the timed
-        variant records them around the six kernels of the pass."""
+        """jacap_score; with ``events`` (JACAP_SCORE_KERNELS + 1 torch.cuda.Event
+        objects) the timed variant records them around the kernels of the pass."""
         c = self.cache
         if events is None:
             _check(jacap_score(self.lay, self.params, _ptr(c.q_win), _ptr(c.k), _ptr(c.v), _ptr(self.scores),

@@ -19,7 +19,7 @@ constexpr size_t ALIGN = 1024;
 inline size_t align_up(size_t x) { return (x + ALIGN - 1) & ~(ALIGN - 1); }
 
 struct Carve {
-  size_t status, plan, counters, mu, lam, lk, cstats, w, gpart, gram, minv, minv_img, total;
+  size_t status, plan, counters, mu, lam, lk, cstats, w, wsplit, gpart, gram, minv, minv_img, total;
 };
 
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
@@ -100,6 +100,7 @@ Carve carve(const Dims& dm) {
   c.lk = o; o = align_up(o + planes * (size_t)dm.Ntot * 2 * dm.G * 4);
   c.cstats = o; o = align_up(o + planes * (size_t)dm.c_cap * dm.G * 2 * 4);
   c.w = o; o = align_up(o + planes * (size_t)dm.Ntot * 4);
+  c.wsplit = o; o = align_up(o + planes * (size_t)dm.Ntot * 4 + 64);  // + tail read by 16-byte rounded copies
   c.gpart = o; o = align_up(o + planes * (size_t)dm.c_cap * D * D * 4);
   c.gram = o; o = align_up(o + units * D * D * 4);
   c.minv = o; o = align_up(o + units * D * D * 4);
@@ -119,6 +120,7 @@ Ws make_ws(void* base, const Carve& c) {
   ws.lk = (float*)(b + c.lk);
   ws.cstats = (float*)(b + c.cstats);
   ws.w = (float*)(b + c.w);
+  ws.wsplit = (uint32_t*)(b + c.wsplit);
   ws.gpart = (float*)(b + c.gpart);
   ws.gram = (float*)(b + c.gram);
   ws.minv = (float*)(b + c.minv);
@@ -251,14 +253,17 @@ jacap_status jacap_score_timed(const jacap_layout* layout, const jacap_params* p
       (st = map_cuda(launch_kpass(kmap, dm, w, dt, cu, persistent_grid(items, sms, 1), s))) != JACAP_OK)
     return st;
   if ((st = hook(3)) != JACAP_OK ||
+      (st = map_cuda(launch_weights(dm, w, cu, persistent_grid(items, sms, 8), s))) != JACAP_OK)
+    return st;
+  if ((st = hook(4)) != JACAP_OK ||
       (st = map_cuda(launch_gram(vmap, dm, w, dt, v, cu, persistent_grid(items, sms, bf ? 1 : 4), s))) != JACAP_OK)
     return st;
-  if ((st = hook(4)) != JACAP_OK || (st = map_cuda(launch_factor(dm, w, s))) != JACAP_OK) return st;
-  if ((st = hook(5)) != JACAP_OK ||
+  if ((st = hook(5)) != JACAP_OK || (st = map_cuda(launch_factor(dm, w, s))) != JACAP_OK) return st;
+  if ((st = hook(6)) != JACAP_OK ||
       (st = map_cuda(launch_score(vmap, dm, w, dt, v, cu, scores, persistent_grid(items, sms, bf ? 1 : 2), s))) !=
           JACAP_OK)
     return st;
-  if ((st = hook(6)) != JACAP_OK) return st;
+  if ((st = hook(7)) != JACAP_OK) return st;
   return JACAP_OK;
 }
 

@@ -50,6 +50,7 @@ struct Ws {
   float* lk;          // [L*Hkv][Ntot][2G]  logits then kappa per query head of the group
   float* cstats;      // [L*Hkv][c_cap][G][2]  per-chunk (max, sum exp(l - max))
   float* w;           // [L*Hkv][Ntot]  Eq. 8 weights summed over the group
+  uint32_t* wsplit;   // [L*Hkv][Ntot]  w as bf16 hi (low half) + bf16 lo = w - hi (high half)
   float* gpart;       // [L*Hkv][c_cap][D][D]  per-chunk partial Grams
   float* gram;        // [units][D][D]  sum_i w_i v_i v_i^T
   float* minv;        // [units][D][D]  L^{-1} (float32, lower triangular)
@@ -380,6 +381,32 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
   uint32_t r;
   asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(b), "f"(a));
   return r;
+}
+
+// Packed bf16 arithmetic on two lanes (low half, high half), one rounding each.
+__device__ __forceinline__ uint32_t bf16x2_mul(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("mul.rn.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
+}
+__device__ __forceinline__ uint32_t bf16x2_fma(uint32_t a, uint32_t b, uint32_t c) {
+  uint32_t d;
+  asm("fma.rn.bf16x2 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+  return d;
+}
+__device__ __forceinline__ uint32_t bf16x2_neg(uint32_t a) {
+  uint32_t d;
+  asm("neg.bf16x2 %0, %1;" : "=r"(d) : "r"(a));
+  return d;
+}
+// x * v as hi + lo (bf16 pairs) for a weight given as whi + wlo (bf16 pairs):
+// hi = RN(whi v); the residual whi v - hi has at most 8 significant bits and is
+// exact in bf16 (one fused multiply-add); lo = RN(wlo v + residual).
+// |hi + lo - (whi + wlo) v| <= 2^-9 |lo| ~ 2^-17 |x v|.
+__device__ __forceinline__ void bf16x2_scale_split(uint32_t whi, uint32_t wlo, uint32_t v, uint32_t& hi,
+                                                   uint32_t& lo) {
+  hi = bf16x2_mul(whi, v);
+  lo = bf16x2_fma(wlo, v, bf16x2_fma(whi, v, bf16x2_neg(hi)));
 }
 
 }  // namespace jacap

@@ -1,18 +1,20 @@
-// k_gram.cu - fused Jacobian weight + weighted Gram pass over V.
+// k_gram.cu - Jacobian weights and the weighted Gram pass over V.
 //
-// For every work item (a chunk of one unit's tokens) this pass
+// Weight pass (one streaming pass over the K pass's logits/kappa rows), per
+// work item (a chunk of one unit's tokens):
 //   1. combines the K pass's per-chunk (max, sum exp) into the pool-softmax
 //      normaliser (M_h, Z_h) of each query head h of the group (Sec. 3.4,
 //      display after Algorithm 1);
 //   2. forms w_i = (1/d) sum_h [alpha_bar (1 - alpha_bar)]^2 kappa_h,i with
 //      alpha_bar = exp(l_h,i - M_h) / Z_h (Eq. 8; GQA heads summed) and stores
-//      w for the score pass;
-//   3. accumulates the chunk's partial Gram  sum_i w_i v_i v_i^T  (Eq. 9).
+//      w for the score pass and as a bf16 pair hi + lo for the Gram pass.
+// Gram pass: accumulates the chunk's partial Gram  sum_i w_i v_i v_i^T  (Eq. 9).
 //
 // bf16 caches use the 5th-generation tensor cores. B = V straight from the
 // TMA-staged tile (bf16 is exact); the scaled operand w_i v_i = hi + lo is
 // split into two bf16 halves (residual ~2^-17 relative per product) by the
-// scaling warps and written to tensor memory as two A operands, so
+// scaling warps with packed bf16 arithmetic on w_i = whi + wlo, and written to
+// tensor memory as two A operands, so
 // D = sum_i (hi_i + lo_i) v_i^T accumulates in fp32 in tensor memory without
 // passing the scaled operand through shared memory. float32 caches take a
 // SIMT fp32 kernel of the same contract.
@@ -21,10 +23,10 @@
 
 namespace jacap {
 
-// Pool-softmax normaliser of the unit (plane, seq) for G heads: M_h = max of the
-// chunk maxima, Z_h = sum_c s_c exp(m_c - M_h), combined in chunk order.
-// Same normaliser computed by one warp: lanes take chunks c0 + lane + 32 k and
-// a butterfly merges them (fixed order, so every CTA of the unit agrees).
+// Pool-softmax normaliser of the unit (plane, seq) for query head h of the
+// group: M_h = max of the chunk maxima, Z_h = sum_c s_c exp(m_c - M_h). One
+// warp: lanes take chunks c0 + lane + 32 k and a butterfly merges them in a
+// fixed order, so every CTA that needs the unit's normaliser gets the same bits.
 template <int G>
 __device__ __forceinline__ void unit_softmax_stats_warp(const Dims& dm, const Ws& ws, int plane, int seq, int h,
                                                         float& M, float& Z) {
@@ -38,110 +40,117 @@ __device__ __forceinline__ void unit_softmax_stats_warp(const Dims& dm, const Ws
   Z = s;
 }
 
-template <int G>
-__device__ __forceinline__ void unit_softmax_stats(const Dims& dm, const Ws& ws, int plane, int seq, int h,
-                                                   float& M, float& Z) {
-  const int c0 = ws.plan[1 + seq], c1 = ws.plan[2 + seq];
-  const float* cs = ws.cstats + ((int64_t)plane * dm.c_cap) * G * 2;
-  M = -INFINITY;
-  for (int c = c0; c < c1; ++c) M = fmaxf(M, cs[((int64_t)c * G + h) * 2]);
-  Z = 0.f;
-  for (int c = c0; c < c1; ++c) {
-    const float m = cs[((int64_t)c * G + h) * 2];
-    if (m > -INFINITY) Z += cs[((int64_t)c * G + h) * 2 + 1] * expf(m - M);
-  }
-}
+// ---------------------------------------------------------------- weights --
+// w_i of Eq. 8 summed over the G query heads of the group (GQA heads add their
+// weights): w_i = wdiv * sum_h [alpha_bar (1 - alpha_bar)]^2 kappa_h,i with
+// alpha_bar = exp(l_h,i - M_h) / Z_h. One streaming pass over the K pass's
+// logits/kappa rows; writes w (float32, for the score pass) and w as a bf16
+// pair hi + lo (for the tensor-core Gram, whose scaling is done in bf16).
+constexpr int WT_THREADS = 256;
 
-// w_i of Eq. 8 summed over the G query heads of the group (reading: GQA heads
-// add their weights). ustat = [M_0..M_{G-1}, Z_0..Z_{G-1}].
 template <int G>
-__device__ __forceinline__ void load_lk(const Dims& dm, const Ws& ws, int plane, int64_t tok, float* lk) {
-  const float* src = ws.lk + ((int64_t)plane * dm.Ntot + tok) * (2 * G);
-  if constexpr ((2 * G) % 4 == 0) {
-#pragma unroll
-    for (int e = 0; e < 2 * G; e += 4) {
-      const float4 q4 = *(const float4*)(src + e);
-      lk[e] = q4.x; lk[e + 1] = q4.y; lk[e + 2] = q4.z; lk[e + 3] = q4.w;
+__global__ void __launch_bounds__(WT_THREADS) weight_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu) {
+  __shared__ float us[2 * G];  // M_h, then 1 / Z_h
+  __shared__ int s_skip;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  if (tid == 0) s_skip = status_failed(ws) ? 1 : 0;
+  __syncthreads();
+  if (s_skip) return;
+  bool bad = false;
+  Item item;
+  for (int64_t i = blockIdx.x; decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+    __syncthreads();
+    if (warp < G) {
+      float M, Z;
+      unit_softmax_stats_warp<G>(dm, ws, item.plane, item.seq, warp, M, Z);
+      if (lane == 0) {
+        us[warp] = M;
+        us[G + warp] = 1.f / Z;
+      }
     }
-  } else {
+    __syncthreads();
+    float u[2 * G];
 #pragma unroll
-    for (int e = 0; e < 2 * G; ++e) lk[e] = src[e];
-  }
-}
-
-template <int G>
-__device__ __forceinline__ float weight_from_lk(const Dims& dm, const float* ustat, const float* lk) {
-  float wt = 0.f;
+    for (int e = 0; e < 2 * G; ++e) u[e] = us[e];
+    const int64_t base = (int64_t)item.plane * dm.Ntot;
+    for (int64_t tok = item.t0 + tid; tok < item.t1; tok += WT_THREADS) {
+      const float* src = ws.lk + (base + tok) * (2 * G);
+      float lk[2 * G];
+      if constexpr ((2 * G) % 4 == 0) {
 #pragma unroll
-  for (int h = 0; h < G; ++h) {
-    const float a = expf(lk[h] - ustat[h]) / ustat[G + h];  // alpha_bar
-    const float rho = a * (1.f - a);                           // diagonal of S
-    wt = fmaf(rho * rho, lk[G + h], wt);                       // rho^2 kappa
-  }
-  return wt * dm.wdiv;
-}
-
-// Logits and kappa of heads h0 .. h0 + NH - 1 of one token (src points at
-// the token's row + h0).
-template <int G, int NH>
-__device__ __forceinline__ void load_lk_part(const float* src, float (&l)[NH], float (&k)[NH]) {
+        for (int e = 0; e < 2 * G; e += 4) {
+          const float4 q4 = *(const float4*)(src + e);
+          lk[e] = q4.x; lk[e + 1] = q4.y; lk[e + 2] = q4.z; lk[e + 3] = q4.w;
+        }
+      } else {
+        const float2 q2 = *(const float2*)src;
+        lk[0] = q2.x;
+        lk[1] = q2.y;
+      }
+      float wt = 0.f;
 #pragma unroll
-  for (int j = 0; j < NH; ++j) {
-    l[j] = src[j];
-    k[j] = src[G + j];
+      for (int h = 0; h < G; ++h) {
+        const float a = expf(lk[h] - u[h]) * u[G + h];  // alpha_bar
+        const float rho = a * (1.f - a);                 // diagonal of the softmax Jacobian
+        wt = fmaf(rho * rho, lk[G + h], wt);             // rho^2 kappa
+      }
+      wt *= dm.wdiv;
+      bad |= !isfinite(wt);
+      ws.w[base + tok] = wt;
+      // hi = RN(w), lo = RN(w - hi) (w - hi is exact in float32)
+      ws.wsplit[base + tok] = pack_bf16x2(wt, wt - bf16lo(pack_bf16x2(wt, 0.f)));
+    }
   }
-}
-
-// Partial Eq. 8 sum over heads h0 .. h0 + NH - 1 from the logits/kappa row;
-// uinv = [M_0..M_{G-1}, 1/Z_0..1/Z_{G-1}] (the reciprocal saves a divide per head).
-template <int G, int NH>
-__device__ __forceinline__ float weight_part(const float* l, const float* kap, const float* uinv, int h0) {
-  float wt = 0.f;
-#pragma unroll
-  for (int j = 0; j < NH; ++j) {
-    const float a = expf(l[j] - uinv[h0 + j]) * uinv[G + h0 + j];  // alpha_bar
-    const float rho = a * (1.f - a);                                  // diagonal of S
-    wt = fmaf(rho * rho, kap[j], wt);                                 // rho^2 kappa
-  }
-  return wt;
-}
-
-template <int G>
-__device__ __forceinline__ float jacobian_weight(const Dims& dm, const Ws& ws, const float* ustat, int plane,
-                                                 int64_t tok) {
-  float lk[2 * G];
-  load_lk<G>(dm, ws, plane, tok, lk);
-  return weight_from_lk<G>(dm, ustat, lk);
+  if (bad) flag(ws, ST_NONFINITE);
 }
 
 // --------------------------------------------------------------- tcgen05 ---
 // G = sum_i v_i (w_i v_i)^T on the tensor cores with the scaled operand in
 // tensor memory: D (128 x 128, fp32) += A (128 channels x 16 tokens, TMEM)
-// * B (16 tokens x 128 channels, the TMA-staged V tile, MN-major). Per tile
-// the scaling warps read V transposed with ldmatrix, multiply by w_i, split
-// w_i v_i = hi + lo (bf16 each) and store hi and lo as two A operands; two
-// MMAs per 16 tokens accumulate v (hi + lo)^T.
+// * B (16 tokens x 128 channels, the TMA-staged V tile, MN-major). The TMA
+// warp stages each V tile together with the tile's weights (bf16 pairs
+// hi + lo from the weight pass). The scaling warps read V transposed with
+// ldmatrix, form w_i v_i = hi + lo with packed bf16 arithmetic and store hi
+// and lo as two A operands; two MMAs per 16 tokens accumulate v (hi + lo)^T.
+// The scaling warps share nothing but the mbarriers of the pipeline.
 constexpr int GR_THREADS = 320;   // warp 0: TMA, warp 1: MMA, warps 2-9: scale + epilogue
 constexpr int GR_SCALERS = 256;
 constexpr int GR_VST = 6;          // V tiles in flight
 constexpr int GR_BOX = 16384;      // {64 channels, 128 tokens} bf16, 128-byte swizzle
 constexpr int GR_V_BYTES = 2 * GR_BOX;
+constexpr int GR_W_BYTES = 640;    // weight words of a tile: <= 3 + 128, rounded to 16-byte copies
 constexpr uint32_t GR_TMEM_COLS = 512;
 constexpr uint32_t GR_ACOL = 128;  // A buffers: [128 + 128 ab, +64) hi, [+64, +128) lo
 // M = 128 (channels), N = 128 (channels), A in TMEM (K-major), B MN-major.
 constexpr uint32_t GR_IDESC = idesc_bf16_f32(128, 128, 0, 1);
 
-constexpr size_t gram_bf16_smem_bytes() { return 1024 + GR_VST * GR_V_BYTES + GR_VST * TILE * 4 + 256; }
+constexpr size_t gram_bf16_smem_bytes() { return 1024 + GR_VST * (GR_V_BYTES + GR_W_BYTES) + 256; }
 
-template <int G>
+// Weight words of the tile starting at token t of the plane: the copy starts
+// at the 16-byte boundary at or below the tile's first word (`off` words
+// before it) and covers the tile's `nvalid` tokens, rounded up to 16 bytes.
+struct WTile {
+  int64_t word0;  // first copied word (multiple of 4)
+  int off, nvalid;
+  uint32_t bytes;
+};
+__device__ __forceinline__ WTile weight_tile(const Dims& dm, const Item& item, int64_t t) {
+  WTile w;
+  const int64_t a = (int64_t)item.plane * dm.Ntot + t;
+  w.word0 = a & ~(int64_t)3;
+  w.off = (int)(a - w.word0);
+  w.nvalid = (int)(item.t1 - t < TILE ? item.t1 - t : TILE);
+  w.bytes = (uint32_t)(((w.off + w.nvalid + 3) & ~3) * 4);
+  return w;
+}
+
 __global__ void __launch_bounds__(GR_THREADS, 1)
     gram_bf16_kernel(const __grid_constant__ CUtensorMap vmap, Dims dm, Ws ws, const int32_t* __restrict__ cu) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint8_t* vring = smem;                                        // [GR_VST][GR_V_BYTES]
-  float* wbuf = (float*)(vring + GR_VST * GR_V_BYTES);          // [GR_VST][TILE] weights of the tile
-  float* ustat = wbuf + GR_VST * TILE;                          // [2G] (<= 16 floats)
-  uint64_t* vfull = (uint64_t*)(ustat + 16);
+  uint8_t* vring = smem;                                   // [GR_VST][GR_V_BYTES]
+  uint8_t* wring = vring + GR_VST * GR_V_BYTES;            // [GR_VST][GR_W_BYTES] weight words
+  uint64_t* vfull = (uint64_t*)(wring + GR_VST * GR_W_BYTES);
   uint64_t* vempty = vfull + GR_VST;
   uint64_t* afull = vempty + GR_VST;
   uint64_t* aempty = afull + 2;
@@ -195,9 +204,12 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
             break;
           }
           uint8_t* vt = vring + st * GR_V_BYTES;
-          mbar_arrive_expect_tx(smem_u32(&vfull[st]), GR_V_BYTES);
-          tma_load_4d(smem_u32(vt), &vmap, 0, (int)t, g, l, smem_u32(&vfull[st]));
-          tma_load_4d(smem_u32(vt + GR_BOX), &vmap, 64, (int)t, g, l, smem_u32(&vfull[st]));
+          const WTile wt = weight_tile(dm, item, t);
+          const uint32_t bar = smem_u32(&vfull[st]);
+          mbar_arrive_expect_tx(bar, GR_V_BYTES + wt.bytes);
+          tma_load_4d(smem_u32(vt), &vmap, 0, (int)t, g, l, bar);
+          tma_load_4d(smem_u32(vt + GR_BOX), &vmap, 64, (int)t, g, l, bar);
+          bulk_g2s(smem_u32(wring + st * GR_W_BYTES), ws.wsplit + wt.word0, wt.bytes, bar);
           ++it;
         }
       }
@@ -242,72 +254,33 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
     }
   } else {
     // ------------------------------------- scaling warps + epilogue -------
-    const int sidx = tid - 64;           // 0..255
     const int quarter = warp & 3;        // TMEM lane quarter == channels 32 quarter .. +31
     const int th = (warp - 2) >> 2;      // token half of each tile (blocks 4 th .. 4 th + 3)
     const int m = quarter * 32 + lane;   // Gram row (channel) owned in the epilogue
     // ldmatrix row addresses: lane l -> matrix l / 8, row l % 8
     const int lm = lane >> 3, lr = lane & 7;
     uint32_t it = 0, nitem = 0;
-    bool bad = false;
     Item item;
     for (int64_t i = blockIdx.x; decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
-      asm volatile("bar.sync 1, 256;" ::: "memory");
-      if ((sidx >> 5) < G) {  // scaler warp h computes head h's normaliser
-        const int h = sidx >> 5;
-        float M, Z;
-        unit_softmax_stats_warp<G>(dm, ws, item.plane, item.seq, h, M, Z);
-        if (lane == 0) {
-          ustat[h] = M;
-          ustat[G + h] = Z;
-        }
-      }
-      asm volatile("bar.sync 1, 256;" ::: "memory");
-      float us[2 * G];  // M_h, then 1/Z_h
-#pragma unroll
-      for (int e = 0; e < G; ++e) {
-        us[e] = ustat[e];
-        us[G + e] = 1.f / ustat[G + e];
-      }
-      // weights: thread pair (2 y2, 2 y2 + 1) shares token y2; thread `part`
-      // sums heads part*NH .. part*NH + NH - 1 and one shuffle adds the halves
-      constexpr int NH = G >= 2 ? G / 2 : 1;
-      const int y2 = sidx >> 1, part = sidx & 1;
-      const bool wact = G >= 2 || part == 0;
-      const int h0 = G >= 2 ? part * NH : 0;
-      float up[2 * NH];  // [M_h, then 1/Z_h] of this thread's heads (compile-time indices)
-#pragma unroll
-      for (int j = 0; j < NH; ++j) {
-        up[j] = (G >= 2 && part) ? us[NH + j] : us[j];
-        up[NH + j] = (G >= 2 && part) ? us[G + NH + j] : us[G + j];
-      }
-      float lc[NH], kc[NH];  // this thread's logits/kappa for the current tile
-      const float* lkp = ws.lk + (int64_t)item.plane * dm.Ntot * (2 * G) + h0;
-      if (wact && item.t0 + y2 < item.t1) load_lk_part<G, NH>(lkp + (item.t0 + y2) * (2 * G), lc, kc);
-
       for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
         const int vs = it % GR_VST, ab = it & 1;
         if (!mbar_wait(smem_u32(&vfull[vs]), (it / GR_VST) & 1, ws, abort)) goto scale_done;
-        float* wt_s = wbuf + vs * TILE;
-        {  // Eq. 8 weight of token t + y2
-          const int64_t tok = t + y2;
-          float ln[NH], kn[NH];
-          if (wact && t + TILE + y2 < item.t1) load_lk_part<G, NH>(lkp + (t + TILE + y2) * (2 * G), ln, kn);
-          float wp = 0.f;
-          if (wact && tok < item.t1) wp = weight_part<NH, NH>(lc, kc, up, 0);
-          const float wt = (wp + __shfl_xor_sync(0xffffffffu, wp, 1)) * dm.wdiv;
-          if (part == 0 && tok < item.t1) {
-            ws.w[(int64_t)item.plane * dm.Ntot + tok] = wt;
-            bad |= !isfinite(wt);
-          }
-          if (part == 0) wt_s[y2] = tok < item.t1 ? wt : 0.f;
+        // weights of this lane's token pairs (rows 2(l%4), 2(l%4)+1 of each
+        // 8-token half of its 4 blocks) as bf16 pairs; tokens past the item
+        // weigh zero
+        uint32_t wph[8], wpl[8];
+        {
+          const WTile wt = weight_tile(dm, item, t);
+          const uint32_t* wsl = (const uint32_t*)(wring + vs * GR_W_BYTES) + wt.off;
 #pragma unroll
-          for (int j = 0; j < NH; ++j) {
-            lc[j] = ln[j];
-            kc[j] = kn[j];
+          for (int e = 0; e < 8; ++e) {
+            const int i0 = 16 * (4 * th + (e >> 1)) + 8 * (e & 1) + 2 * (lane & 3);
+            const uint32_t x0 = i0 < wt.nvalid ? wsl[i0] : 0u;
+            const uint32_t x1 = i0 + 1 < wt.nvalid ? wsl[i0 + 1] : 0u;
+            wph[e] = __byte_perm(x0, x1, 0x5410);  // (hi of token i0, hi of i0 + 1)
+            wpl[e] = __byte_perm(x0, x1, 0x7632);  // (lo, lo)
           }
         }
-        asm volatile("bar.sync 1, 256;" ::: "memory");
         if (it >= 2 && !mbar_wait(smem_u32(&aempty[ab]), ((it >> 1) & 1) ^ 1, ws, abort)) goto scale_done;
         tc_fence_after();
         const uint32_t vt = smem_u32(vring + vs * GR_V_BYTES);
@@ -320,9 +293,6 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
 #pragma unroll
           for (int blk = 0; blk < 4; ++blk) {
             const int b = 4 * th + blk;  // 16-token block of the tile
-            // weights of this thread's token pairs: rows 2(t%4), 2(t%4)+1 of each 8-token half
-            const float2 wa = *(const float2*)(wt_s + 16 * b + 2 * (lane & 3));
-            const float2 wb = *(const float2*)(wt_s + 16 * b + 8 + 2 * (lane & 3));
             // matrices: 0 = (tokens 0-7, ch c0..c0+7), 1 = (tokens 0-7, c0+8..), 2 = (8-15, c0..), 3 = (8-15, c0+8..)
             const int c0 = quarter * 32 + lh * 16 + (lm & 1) * 8;
             const int tokr = 16 * b + (lm >> 1) * 8 + lr;
@@ -331,13 +301,10 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
             ldsm_x4_trans(addr, r[0], r[1], r[2], r[3]);
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
-              // x = w v (exact fp32 products), hi = bf16(x), lo = bf16(x - hi)
-              const float2 x = __fmul2_rn(q < 2 ? wa : wb, make_float2(bf16lo(r[q]), bf16hi(r[q])));
-              const uint32_t h = pack_bf16x2(x.x, x.y);
-              const float2 res = __ffma2_rn(make_float2(bf16lo(h), bf16hi(h)), make_float2(-1.f, -1.f), x);
-              // registers (r0 = lanes 0-7, r1 = lanes 8-15) of columns 8 blk + 4 (q / 2) ..
-              hi[4 * blk + 2 * (q >> 1) + (q & 1)] = h;
-              lo[4 * blk + 2 * (q >> 1) + (q & 1)] = pack_bf16x2(res.x, res.y);
+              // w v = hi + lo; registers (r0 = lanes 0-7, r1 = lanes 8-15) of
+              // columns 8 blk + 4 (q / 2) ..
+              const int e = 4 * blk + 2 * (q >> 1) + (q & 1);
+              bf16x2_scale_split(wph[2 * blk + (q >> 1)], wpl[2 * blk + (q >> 1)], r[q], hi[e], lo[e]);
             }
           }
           const uint32_t lanes = (uint32_t)(quarter * 32 + lh * 16) << 16;
@@ -370,8 +337,7 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
       if (lane == 0) mbar_arrive(smem_u32(accempty));
       ++nitem;
     }
-  scale_done:
-    if (bad) flag(ws, ST_NONFINITE);
+  scale_done:;
   }
   tc_fence_before();
   __syncthreads();
@@ -388,32 +354,21 @@ constexpr int GF_THREADS = 256;
 constexpr int GF_SLAB = 32;
 constexpr int GF_LD = D + 4;
 
-template <int G>
 __global__ void __launch_bounds__(GF_THREADS)
     gram_f32_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu, const float* __restrict__ v) {
   __shared__ float xs[GF_SLAB][GF_LD];  // w_i v_i
   __shared__ float vs[GF_SLAB][GF_LD];  // v_i
   __shared__ float wsl[GF_SLAB];
-  __shared__ float ustat[2 * G];
   __shared__ int s_skip;
   const int tid = threadIdx.x;
   if (tid == 0) s_skip = status_failed(ws) ? 1 : 0;
   __syncthreads();
   if (s_skip) return;
   const int rb = tid / 16, cb = tid % 16;
-  bool bad = false;
   Item item;
   for (int64_t i = blockIdx.x; decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
     const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
     const float* vbase = v + (int64_t)l * dm.kv_sl + (int64_t)g * dm.kv_sh;
-    __syncthreads();
-    if (tid < G) {
-      float M, Z;
-      unit_softmax_stats<G>(dm, ws, item.plane, item.seq, tid, M, Z);
-      ustat[tid] = M;
-      ustat[G + tid] = Z;
-    }
-    __syncthreads();
     float acc[8][8];
 #pragma unroll
     for (int a = 0; a < 8; ++a)
@@ -422,13 +377,7 @@ __global__ void __launch_bounds__(GF_THREADS)
     for (int64_t t = item.t0; t < item.t1; t += GF_SLAB) {
       if (tid < GF_SLAB) {
         const int64_t tok = t + tid;
-        float wt = 0.f;
-        if (tok < item.t1) {
-          wt = jacobian_weight<G>(dm, ws, ustat, item.plane, tok);
-          ws.w[(int64_t)item.plane * dm.Ntot + tok] = wt;
-          bad |= !isfinite(wt);
-        }
-        wsl[tid] = wt;
+        wsl[tid] = tok < item.t1 ? ws.w[(int64_t)item.plane * dm.Ntot + tok] : 0.f;
       }
       __syncthreads();
       for (int e = tid; e < GF_SLAB * (D / 4); e += GF_THREADS) {
@@ -464,34 +413,36 @@ __global__ void __launch_bounds__(GF_THREADS)
       *(float4*)(row + 4) = make_float4(acc[p][4], acc[p][5], acc[p][6], acc[p][7]);
     }
   }
-  if (bad) flag(ws, ST_NONFINITE);
 }
 
 // ------------------------------------------------------------ launchers ----
 template <int G>
-static cudaError_t launch_gram_g(const CUtensorMap& vmap, const Dims& dm, const Ws& ws, int dtype, const void* v,
-                                 const int32_t* cu, int grid, cudaStream_t st) {
-  if (dtype == 1) {
-    constexpr size_t smem = gram_bf16_smem_bytes();
-    cudaError_t e =
-        cudaFuncSetAttribute(gram_bf16_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    gram_bf16_kernel<G><<<grid, GR_THREADS, smem, st>>>(vmap, dm, ws, cu);
-  } else {
-    gram_f32_kernel<G><<<grid, GF_THREADS, 0, st>>>(dm, ws, cu, (const float*)v);
-  }
+static cudaError_t launch_weights_g(const Dims& dm, const Ws& ws, const int32_t* cu, int grid, cudaStream_t st) {
+  weight_kernel<G><<<grid, WT_THREADS, 0, st>>>(dm, ws, cu);
   return cudaGetLastError();
+}
+
+cudaError_t launch_weights(const Dims& dm, const Ws& ws, const int32_t* cu, int grid, cudaStream_t st) {
+  switch (dm.G) {
+    case 1: return launch_weights_g<1>(dm, ws, cu, grid, st);
+    case 2: return launch_weights_g<2>(dm, ws, cu, grid, st);
+    case 4: return launch_weights_g<4>(dm, ws, cu, grid, st);
+    case 8: return launch_weights_g<8>(dm, ws, cu, grid, st);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 cudaError_t launch_gram(const CUtensorMap& vmap, const Dims& dm, const Ws& ws, int dtype, const void* v,
                         const int32_t* cu, int grid, cudaStream_t st) {
-  switch (dm.G) {
-    case 1: return launch_gram_g<1>(vmap, dm, ws, dtype, v, cu, grid, st);
-    case 2: return launch_gram_g<2>(vmap, dm, ws, dtype, v, cu, grid, st);
-    case 4: return launch_gram_g<4>(vmap, dm, ws, dtype, v, cu, grid, st);
-    case 8: return launch_gram_g<8>(vmap, dm, ws, dtype, v, cu, grid, st);
-    default: return cudaErrorInvalidValue;
+  if (dtype == 1) {
+    constexpr size_t smem = gram_bf16_smem_bytes();
+    cudaError_t e = cudaFuncSetAttribute(gram_bf16_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    gram_bf16_kernel<<<grid, GR_THREADS, smem, st>>>(vmap, dm, ws, cu);
+  } else {
+    gram_f32_kernel<<<grid, GF_THREADS, 0, st>>>(dm, ws, cu, (const float*)v);
   }
+  return cudaGetLastError();
 }
 
 }  // namespace jacap
