@@ -121,6 +121,7 @@ constexpr int GR_V_BYTES = 2 * GR_BOX;
 constexpr int GR_W_BYTES = 640;    // weight words of a tile: <= 3 + 128, rounded to 16-byte copies
 constexpr uint32_t GR_TMEM_COLS = 512;
 constexpr uint32_t GR_ACOL = 128;  // A buffers: [128 + 128 ab, +64) hi, [+64, +128) lo
+constexpr uint32_t GR_DCOL1 = 384; // accumulators: columns [0, 128) and [384, 512), alternating by item
 // M = 128 (channels), N = 128 (channels), A in TMEM (K-major), B MN-major.
 constexpr uint32_t GR_IDESC = idesc_bf16_f32(128, 128, 0, 1);
 
@@ -154,8 +155,8 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
   uint64_t* vempty = vfull + GR_VST;
   uint64_t* afull = vempty + GR_VST;
   uint64_t* aempty = afull + 2;
-  uint64_t* accfull = aempty + 2;
-  uint64_t* accempty = accfull + 1;
+  uint64_t* accfull = aempty + 2;   // [2]
+  uint64_t* accempty = accfull + 2; // [2]
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort, s_skip;
 
@@ -171,8 +172,10 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
       mbar_init(smem_u32(&afull[i]), GR_SCALERS / 32);
       mbar_init(smem_u32(&aempty[i]), 1);
     }
-    mbar_init(smem_u32(accfull), 1);
-    mbar_init(smem_u32(accempty), GR_SCALERS / 32);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(smem_u32(&accfull[i]), 1);
+      mbar_init(smem_u32(&accempty[i]), GR_SCALERS / 32);
+    }
     fence_mbar_init();
   }
   __syncthreads();
@@ -223,7 +226,10 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
       bool ok = true;
       Item item;
       for (int64_t i = blockIdx.x; ok && decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
-        if (nitem > 0 && !mbar_wait(smem_u32(accempty), (nitem - 1) & 1, ws, abort)) break;
+        // accumulator of this item; its previous item's epilogue must be done
+        const int db = nitem & 1;
+        const uint32_t dacc = tmem + (db ? GR_DCOL1 : 0u);
+        if (nitem >= 2 && !mbar_wait(smem_u32(&accempty[db]), ((nitem >> 1) & 1) ^ 1, ws, abort)) break;
         tc_fence_after();
         bool first = true;
         for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
@@ -239,15 +245,15 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
 #pragma unroll
           for (int k = 0; k < TILE / 16; ++k) {  // 16 tokens per MMA
             const uint64_t bd = smem_desc_sw128(va + k * 2048, GR_BOX, 1024);
-            umma_f16_ts(tmem, acol + 8 * k, bd, GR_IDESC, (first && k == 0) ? 0u : 1u);
-            umma_f16_ts(tmem, acol + 64 + 8 * k, bd, GR_IDESC, 1u);
+            umma_f16_ts(dacc, acol + 8 * k, bd, GR_IDESC, (first && k == 0) ? 0u : 1u);
+            umma_f16_ts(dacc, acol + 64 + 8 * k, bd, GR_IDESC, 1u);
           }
           first = false;
           umma_commit(smem_u32(&vempty[vs]));
           umma_commit(smem_u32(&aempty[ab]));
         }
         if (!ok) break;
-        umma_commit(smem_u32(accfull));
+        umma_commit(smem_u32(&accfull[db]));
         ++nitem;
       }
       if (it > 0) mbar_wait(smem_u32(&aempty[(it - 1) & 1]), ((it - 1) >> 1) & 1, ws, nullptr);
@@ -318,10 +324,11 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
       }
       // epilogue: D is this chunk's partial Gram; warp (quarter, th) writes rows
       // 32 quarter .. +31, columns 64 th .. 64 th + 63
-      if (!mbar_wait(smem_u32(accfull), nitem & 1, ws, abort)) goto scale_done;
+      const int db = nitem & 1;
+      if (!mbar_wait(smem_u32(&accfull[db]), (nitem >> 1) & 1, ws, abort)) goto scale_done;
       tc_fence_after();
       {
-        const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16) + 64 * th;
+        const uint32_t trow = tmem + (db ? GR_DCOL1 : 0u) + ((uint32_t)(quarter * 32) << 16) + 64 * th;
         float* dst = ws.gpart + (((int64_t)item.plane * dm.c_cap + item.cidx) * D + m) * D + 64 * th;
 #pragma unroll 1
         for (int cb = 0; cb < 2; ++cb) {
@@ -334,7 +341,7 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(accempty));
+      if (lane == 0) mbar_arrive(smem_u32(&accempty[db]));
       ++nitem;
     }
   scale_done:;
