@@ -159,6 +159,23 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   return ok != 0;
 }
 
+// Same test, but a thread whose phase is not complete may be suspended for up
+// to `hint_ns` (it resumes as soon as the phase completes), so waiting warps
+// stop competing for issue slots and shared-memory bandwidth.
+__device__ __forceinline__ bool mbar_try_wait_suspend(uint32_t bar, uint32_t parity, uint32_t hint_ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cta.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity), "r"(hint_ns)
+      : "memory");
+  return ok != 0;
+}
+
+constexpr uint32_t WAIT_SUSPEND_NS = 1000;
+
 // Bounded wait for the phase with the given parity to complete. Returns false
 // (after flagging ST_TIMEOUT) if it did not complete within WAIT_LIMIT_NS, or
 // if *abort became nonzero while waiting.
@@ -166,8 +183,8 @@ static __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity
                                             volatile int* abort) {
   const unsigned long long t0 = globaltimer();
   for (uint32_t it = 0;; ++it) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 63u) == 63u) {
+    if (mbar_try_wait_suspend(bar, parity, WAIT_SUSPEND_NS)) return true;
+    if ((it & 7u) == 7u) {
       if (abort != nullptr && *abort) return false;
       if (globaltimer() - t0 > WAIT_LIMIT_NS) {
         flag(ws, ST_TIMEOUT);
@@ -381,6 +398,25 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
   uint32_t r;
   asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(b), "f"(a));
   return r;
+}
+
+// Explicit shared-memory loads from 32-bit shared addresses (the aligned views
+// of the dynamic shared buffer are plain pointers to the compiler, which would
+// otherwise emit generic loads).
+__device__ __forceinline__ uint4 lds_u128(uint32_t addr) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
+  return v;
+}
+__device__ __forceinline__ float4 lds_f128(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr));
+  return v;
+}
+__device__ __forceinline__ uint32_t lds_u32(uint32_t addr) {
+  uint32_t v;
+  asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr));
+  return v;
 }
 
 // Packed bf16 arithmetic on two lanes (low half, high half), one rounding each.

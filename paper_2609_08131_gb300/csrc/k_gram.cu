@@ -277,12 +277,12 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
         uint32_t wph[8], wpl[8];
         {
           const WTile wt = weight_tile(dm, item, t);
-          const uint32_t* wsl = (const uint32_t*)(wring + vs * GR_W_BYTES) + wt.off;
+          const uint32_t wsl = smem_u32(wring + vs * GR_W_BYTES) + 4 * wt.off;
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
             const int i0 = 16 * (4 * th + (e >> 1)) + 8 * (e & 1) + 2 * (lane & 3);
-            const uint32_t x0 = i0 < wt.nvalid ? wsl[i0] : 0u;
-            const uint32_t x1 = i0 + 1 < wt.nvalid ? wsl[i0 + 1] : 0u;
+            const uint32_t x0 = i0 < wt.nvalid ? lds_u32(wsl + 4 * i0) : 0u;
+            const uint32_t x1 = i0 + 1 < wt.nvalid ? lds_u32(wsl + 4 * i0 + 4) : 0u;
             wph[e] = __byte_perm(x0, x1, 0x5410);  // (hi of token i0, hi of i0 + 1)
             wpl[e] = __byte_perm(x0, x1, 0x7632);  // (lo, lo)
           }

@@ -16,34 +16,37 @@
 // fp32 and is weighted by lambda (fp32, broadcast from shared memory) with
 // packed fp32x2 multiply-adds.
 //
-// Warp roles: 0 TMA producer (six tiles in flight); 1 builds the mu' image
-// and lambda of each item and issues the logits MMAs; 2-5 kappa (a pair of
-// warps per tile, two tokens per lane, the pairs alternate tiles); 6-9 read the
-// logits back from tensor memory (one lane quarter each) and keep the online
-// softmax statistics.
+// Warp roles: 0 TMA producer; 1 issues the logits MMAs; 14 builds the mu'
+// image and lambda of each item (double-buffered, one item ahead); 2-9 kappa (two groups of four warps alternate
+// tiles; in a group each warp takes one quarter of the channels for all 128
+// tokens, four per lane, so every lambda value read from shared memory serves
+// four tokens; the quarters are reduce-scattered through shared memory);
+// 10-13 read the logits back from tensor memory (one lane quarter each) and
+// keep the online softmax statistics.
 #include "jacap_dev.cuh"
 #include "jacap_internal.h"
 
 namespace jacap {
 
-constexpr int KB_STAGES = 6;
 constexpr int KB_BOX = 16384;    // {64 channels, 128 tokens} bf16
 constexpr int KB_TILE_BYTES = 2 * KB_BOX;
 constexpr int KB_NACC = 4;       // tensor-memory logits buffers
 constexpr uint32_t KB_TMEM_COLS = 128;
-constexpr int KB_THREADS = 320;
-constexpr int KB_KAPPA_WARP0 = 2, KB_READ_WARP0 = 6;
+constexpr int KB_THREADS = 480;
+constexpr int KB_KAPPA_WARP0 = 2, KB_READ_WARP0 = 10, KB_BUILD_WARP = 14;
 
 template <int G>
 struct KbCfg {
+  static constexpr int STAGES = G == 8 ? 5 : 6;        // K tiles in flight
   static constexpr int NB = (3 * G <= 16) ? 16 : 32;  // MMA N = rows of the mu' image
   static constexpr int IMG_ATOM = NB * 128;            // bytes per 64-channel atom
   static constexpr int IMG_BYTES = 2 * IMG_ATOM;
   static constexpr int LAM_BYTES = G * D * 4;          // lambda, fp32 [G][128]
+  static constexpr int KRED_FLOATS = 2 * 4 * 4 * G * 32;  // [group][token subset][writer][G][32]
   static constexpr uint32_t IDESC = idesc_bf16_f32(128, NB, 0, 0);
   static_assert(KB_NACC * NB <= (int)KB_TMEM_COLS, "tensor memory budget");
-  static constexpr size_t SMEM =
-      1024 + (size_t)KB_STAGES * KB_TILE_BYTES + 2 * IMG_BYTES + 2 * LAM_BYTES + 4 * 2 * G * 4 + 512;
+  static constexpr size_t SMEM = 1024 + (size_t)STAGES * KB_TILE_BYTES + 2 * IMG_BYTES + 2 * LAM_BYTES +
+                                 KRED_FLOATS * 4 + 4 * 2 * G * 4 + 512;
 };
 
 // mu' image of one item: rows n = part * G + h hold part (0 hi, 1 mid, 2 lo) of
@@ -74,51 +77,47 @@ __device__ __forceinline__ void build_split_image(uint8_t* im, const float* src,
   }
 }
 
-// kappa of two token rows (ya, yb) of a staged tile: sum over the 16 chunks of
-// 8 channels of lambda_h,c k_c^2, two independent fp32x2 chains per token and
-// head.
+// Partial kappa over channel quarter `cq` (chunks 4 cq .. 4 cq + 3 of 8
+// channels) for the four token rows lane + 32 j of a staged tile:
+// part[j][h] = sum_c lambda_h,c k_c^2. Each lambda load feeds four tokens.
 template <int G>
-__device__ __forceinline__ void kappa_two_rows(const uint8_t* kt, const float* lam, int ya, int yb, float (&ka)[G],
-                                               float (&kb)[G]) {
-  float2 aa[G][2], ab[G][2];
+__device__ __forceinline__ void kappa_quarter(uint32_t kt, uint32_t lam, int lane, int cq, float (&part)[4][G]) {
+  float2 acc[4][G];
 #pragma unroll
-  for (int h = 0; h < G; ++h) {
-    aa[h][0] = aa[h][1] = ab[h][0] = ab[h][1] = make_float2(0.f, 0.f);
-  }
-#pragma unroll 2
-  for (int cc = 0; cc < 16; ++cc) {
-    const uint4 ra = *(const uint4*)(kt + (cc >> 3) * KB_BOX + sw128_off(ya, cc & 7));
-    const uint4 rb = *(const uint4*)(kt + (cc >> 3) * KB_BOX + sw128_off(yb, cc & 7));
-    const uint32_t wa[4] = {ra.x, ra.y, ra.z, ra.w}, wb[4] = {rb.x, rb.y, rb.z, rb.w};
-    float2 sa[4], sb[4];
+  for (int j = 0; j < 4; ++j)
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const float2 xa = make_float2(bf16lo(wa[q]), bf16hi(wa[q]));
-      const float2 xb = make_float2(bf16lo(wb[q]), bf16hi(wb[q]));
-      sa[q] = __fmul2_rn(xa, xa);  // exact: 8-bit significands
-      sb[q] = __fmul2_rn(xb, xb);
-    }
+    for (int h = 0; h < G; ++h) acc[j][h] = make_float2(0.f, 0.f);
+#pragma unroll 1
+  for (int cc = 4 * cq; cc < 4 * cq + 4; ++cc) {
+    float4 l0[G], l1[G];
 #pragma unroll
     for (int h = 0; h < G; ++h) {
-      const float4 l0 = *(const float4*)(lam + h * D + 8 * cc);
-      const float4 l1 = *(const float4*)(lam + h * D + 8 * cc + 4);
-      const float2 p0 = make_float2(l0.x, l0.y), p1 = make_float2(l0.z, l0.w);
-      const float2 p2 = make_float2(l1.x, l1.y), p3 = make_float2(l1.z, l1.w);
-      aa[h][0] = __ffma2_rn(sa[0], p0, aa[h][0]);
-      aa[h][1] = __ffma2_rn(sa[1], p1, aa[h][1]);
-      ab[h][0] = __ffma2_rn(sb[0], p0, ab[h][0]);
-      ab[h][1] = __ffma2_rn(sb[1], p1, ab[h][1]);
-      aa[h][0] = __ffma2_rn(sa[2], p2, aa[h][0]);
-      aa[h][1] = __ffma2_rn(sa[3], p3, aa[h][1]);
-      ab[h][0] = __ffma2_rn(sb[2], p2, ab[h][0]);
-      ab[h][1] = __ffma2_rn(sb[3], p3, ab[h][1]);
+      l0[h] = lds_f128(lam + (h * D + 8 * cc) * 4);
+      l1[h] = lds_f128(lam + (h * D + 8 * cc + 4) * 4);
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const uint4 r = lds_u128(kt + (cc >> 3) * KB_BOX + sw128_off(lane + 32 * j, cc & 7));
+      const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+      float2 sq[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float2 x = make_float2(bf16lo(w[q]), bf16hi(w[q]));
+        sq[q] = __fmul2_rn(x, x);  // exact: 8-bit significands
+      }
+#pragma unroll
+      for (int h = 0; h < G; ++h) {
+        acc[j][h] = __ffma2_rn(sq[0], make_float2(l0[h].x, l0[h].y), acc[j][h]);
+        acc[j][h] = __ffma2_rn(sq[1], make_float2(l0[h].z, l0[h].w), acc[j][h]);
+        acc[j][h] = __ffma2_rn(sq[2], make_float2(l1[h].x, l1[h].y), acc[j][h]);
+        acc[j][h] = __ffma2_rn(sq[3], make_float2(l1[h].z, l1[h].w), acc[j][h]);
+      }
     }
   }
 #pragma unroll
-  for (int h = 0; h < G; ++h) {
-    ka[h] = (aa[h][0].x + aa[h][1].x) + (aa[h][0].y + aa[h][1].y);
-    kb[h] = (ab[h][0].x + ab[h][1].x) + (ab[h][0].y + ab[h][1].y);
-  }
+  for (int j = 0; j < 4; ++j)
+#pragma unroll
+    for (int h = 0; h < G; ++h) part[j][h] = acc[j][h].x + acc[j][h].y;
 }
 
 template <int G>
@@ -139,10 +138,12 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
   using C = KbCfg<G>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  constexpr int KB_STAGES = C::STAGES;
   uint8_t* tiles = smem;
   uint8_t* img = tiles + KB_STAGES * KB_TILE_BYTES;    // [parity][IMG_BYTES] mu' images
   float* lams = (float*)(img + 2 * C::IMG_BYTES);       // [parity][G][128] lambda
-  float* red = lams + 2 * G * D;                         // [4 readout warps][2G]
+  float* kred = lams + 2 * G * D;                        // partial kappa of the upper channel half
+  float* red = kred + C::KRED_FLOATS;                    // [4 readout warps][2G]
   uint64_t* full = (uint64_t*)(red + 4 * 2 * G);
   uint64_t* empty = full + KB_STAGES;
   uint64_t* accfull = empty + KB_STAGES;
@@ -158,7 +159,7 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
     s_skip = status_failed(ws) ? 1 : 0;
     for (int i = 0; i < KB_STAGES; ++i) {
       mbar_init(smem_u32(&full[i]), 1);
-      mbar_init(smem_u32(&empty[i]), 3);  // MMA commit + the two kappa warps of the tile
+      mbar_init(smem_u32(&empty[i]), 5);  // MMA commit + the four kappa warps of the tile
     }
     for (int i = 0; i < KB_NACC; ++i) {
       mbar_init(smem_u32(&accfull[i]), 1);
@@ -166,7 +167,7 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&imgready[i]), 1);
-      mbar_init(smem_u32(&imgfree[i]), 5);  // MMA commit + the four kappa warps
+      mbar_init(smem_u32(&imgfree[i]), 9);  // MMA commit + the eight kappa warps
     }
     fence_mbar_init();
   }
@@ -209,25 +210,16 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
         mbar_wait(smem_u32(&full[k % KB_STAGES]), (k / KB_STAGES) & 1, ws, nullptr);
     }
   } else if (warp == 1) {
-    // ------------------------------- mu' image, lambda, logits MMA issuer --
-    uint32_t it = 0, nitem = 0;
-    bool ok = true;
-    Item item;
-    for (int64_t i = blockIdx.x; ok && decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
-      const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
-      const int p = nitem & 1;
-      if (nitem >= 2 && !mbar_wait(smem_u32(&imgfree[p]), ((nitem >> 1) - 1) & 1, ws, abort)) break;
-      uint8_t* im_mu = img + p * C::IMG_BYTES;
-      float* lam_s = lams + p * G * D;
-      const int64_t qb = (((int64_t)item.seq * dm.L + l) * dm.Hq + (int64_t)g * G) * D;
-      build_split_image<G>(im_mu, ws.mu + qb, lane);
-      for (int e = lane; e < G * D / 4; e += 32) ((float4*)lam_s)[e] = ((const float4*)(ws.lam + qb))[e];
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(smem_u32(&imgready[p]));
+    // ------------------------------------------------ logits MMA issuer ---
+    if (lane == 0) {
+      uint32_t it = 0, nitem = 0;
+      bool ok = true;
+      Item item;
+      for (int64_t i = blockIdx.x; ok && decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+        const int p = nitem & 1;
+        if (!mbar_wait(smem_u32(&imgready[p]), (nitem >> 1) & 1, ws, abort)) break;
         tc_fence_after();
-        const uint32_t ia = smem_u32(im_mu);
+        const uint32_t ia = smem_u32(img + p * C::IMG_BYTES);
         for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
           const int st = it % KB_STAGES;
           const int ab = it % KB_NACC;
@@ -250,41 +242,86 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
           umma_commit(smem_u32(&accfull[ab]));
         }
         if (ok) umma_commit(smem_u32(&imgfree[p]));
+        ++nitem;
       }
-      it = __shfl_sync(0xffffffffu, it, 0);
-      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      // every MMA issued here completes before the CTA tears down tensor memory
+      if (it > 0) mbar_wait(smem_u32(&accfull[(it - 1) % KB_NACC]), ((it - 1) / KB_NACC) & 1, ws, nullptr);
+    }
+  } else if (warp == KB_BUILD_WARP) {
+    // ---------------------------------- mu' image and lambda, one item ahead
+    uint32_t nitem = 0;
+    Item item;
+    for (int64_t i = blockIdx.x; decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+      const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
+      const int p = nitem & 1;
+      if (nitem >= 2 && !mbar_wait(smem_u32(&imgfree[p]), ((nitem >> 1) - 1) & 1, ws, abort)) break;
+      const int64_t qb = (((int64_t)item.seq * dm.L + l) * dm.Hq + (int64_t)g * G) * D;
+      build_split_image<G>(img + p * C::IMG_BYTES, ws.mu + qb, lane);
+      float* lam_s = lams + p * G * D;
+      for (int e = lane; e < G * D / 4; e += 32) ((float4*)lam_s)[e] = ((const float4*)(ws.lam + qb))[e];
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&imgready[p]));
       ++nitem;
     }
-    // every MMA issued here completes before the CTA tears down tensor memory
-    if (lane == 0 && it > 0)
-      mbar_wait(smem_u32(&accfull[(it - 1) % KB_NACC]), ((it - 1) / KB_NACC) & 1, ws, nullptr);
-  } else if (warp < KB_READ_WARP0) {
+  } else if (warp >= KB_KAPPA_WARP0 && warp < KB_READ_WARP0) {
     // ------------------------------------------------------ kappa ---------
     const int kw = warp - KB_KAPPA_WARP0;
-    const int pair = kw >> 1;                 // tiles with it % 2 == pair
-    const int ya = 64 * (kw & 1) + lane;      // token rows ya and ya + 32 of the tile
-    const int yb = ya + 32;
+    const int grp = kw >> 2;                  // tiles with it % 2 == grp
+    const int cq = kw & 3;                    // channel quarter; also the token subset finished here
+    const int bar_id = 2 + grp;               // the four warps of the group
+    float* slot = kred + grp * (4 * 4 * G * 32);
     uint32_t it = 0, nitem = 0;
     bool bad = false;
     Item item;
+    // A failed wait (which means the abort flag is set) still arrives at the
+    // group's named barriers, and the four warps leave together after them.
     for (int64_t i = blockIdx.x; decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
       const int p = nitem & 1;
-      if (!mbar_wait(smem_u32(&imgready[p]), (nitem >> 1) & 1, ws, abort)) goto kappa_done;
+      mbar_wait(smem_u32(&imgready[p]), (nitem >> 1) & 1, ws, abort);
+      named_barrier_sync(bar_id, 128);
+      if (*abort) goto kappa_done;
       {
-        const float* lam_s = lams + p * G * D;
+        const uint32_t lam_s = smem_u32(lams + p * G * D);
         float* lkp = ws.lk + (int64_t)item.plane * dm.Ntot * (2 * G) + G;
         for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
-          if ((int)(it & 1) != pair) continue;
+          if ((int)(it & 1) != grp) continue;
           const int st = it % KB_STAGES;
-          if (!mbar_wait(smem_u32(&full[st]), (it / KB_STAGES) & 1, ws, abort)) goto kappa_done;
-          float ka[G], kb[G];
-          kappa_two_rows<G>(tiles + st * KB_TILE_BYTES, lam_s, ya, yb, ka, kb);
-          __syncwarp();
-          if (lane == 0) mbar_arrive(smem_u32(&empty[st]));
+          float part[4][G];
+          if (mbar_wait(smem_u32(&full[st]), (it / KB_STAGES) & 1, ws, abort)) {
+            kappa_quarter<G>(smem_u32(tiles + st * KB_TILE_BYTES), lam_s, lane, cq, part);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&empty[st]));
+            // hand the other three token subsets to their owners
 #pragma unroll
-          for (int h = 0; h < G; ++h) bad |= !isfinite(ka[h]) || !isfinite(kb[h]);
-          if (t + ya < item.t1) store_part<G>(lkp + (t + ya) * (2 * G), ka);
-          if (t + yb < item.t1) store_part<G>(lkp + (t + yb) * (2 * G), kb);
+            for (int j = 0; j < 4; ++j)
+              if (j != cq)
+#pragma unroll
+                for (int h = 0; h < G; ++h) slot[((j * 4 + cq) * G + h) * 32 + lane] = part[j][h];
+          }
+          named_barrier_sync(bar_id, 128);
+          if (*abort) goto kappa_done;
+          float kap[G];
+#pragma unroll
+          for (int h = 0; h < G; ++h) {
+            // own subset cq: add the other quarters' partial sums in writer order
+            float v = 0.f;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              float x;
+              if (q == cq) {
+                x = part[cq][h];
+              } else {
+                x = slot[((cq * 4 + q) * G + h) * 32 + lane];
+              }
+              v += x;
+            }
+            kap[h] = v;
+            bad |= !isfinite(v);
+          }
+          named_barrier_sync(bar_id, 128);  // the slots may be rewritten after this
+          const int64_t tok = t + lane + 32 * cq;
+          if (tok < item.t1) store_part<G>(lkp + tok * (2 * G), kap);
         }
       }
       __syncwarp();
@@ -293,7 +330,7 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
     }
   kappa_done:
     if (bad) flag(ws, ST_NONFINITE);
-  } else {
+  } else if (warp >= KB_READ_WARP0 && warp < KB_READ_WARP0 + 4) {
     // ------------------------------------------ logits readout + stats ----
     const int quarter = warp & 3;
     const int y = quarter * 32 + lane;        // token row (tensor-memory lane)
@@ -312,7 +349,7 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
       float* lkp = ws.lk + (int64_t)item.plane * dm.Ntot * (2 * G);
       for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
         const int ab = it % KB_NACC;
-        if (!mbar_wait(smem_u32(&accfull[ab]), (it / KB_NACC) & 1, ws, abort)) goto read_done;
+        if (!mbar_wait(smem_u32(&accfull[ab]), (it / KB_NACC) & 1, ws, abort)) break;  // abort: see below
         tc_fence_after();
         float dv[C::NB];
         if constexpr (C::NB == 16) tmem_ld16(tmem + ab * C::NB + lanes, dv);
@@ -346,7 +383,9 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
           red[rw * 2 * G + G + h] = run_s[h];
         }
       }
+      // a warp that met an abort still arrives here; all four leave together
       named_barrier_sync(1, 128);
+      if (*abort) goto read_done;
       if (rw == 0 && lane < G) {
         const int h = lane;
         float m = -INFINITY, ssum = 0.f;
