@@ -19,7 +19,7 @@ constexpr size_t ALIGN = 1024;
 inline size_t align_up(size_t x) { return (x + ALIGN - 1) & ~(ALIGN - 1); }
 
 struct Carve {
-  size_t status, plan, counters, mu, lam, lk, cstats, w, wsplit, gpart, gram, minv, minv_img, total;
+  size_t status, plan, chunks, counters, mu, lam, lk, cstats, w, wsplit, gpart, gram, minv, minv_img, total;
 };
 
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
@@ -94,6 +94,7 @@ Carve carve(const Dims& dm) {
   size_t o = 0;
   c.status = o; o = align_up(o + 64);
   c.plan = o; o = align_up(o + ((size_t)dm.S + 2) * 4);
+  c.chunks = o; o = align_up(o + (size_t)dm.c_cap * 16);
   c.counters = o; o = align_up(o + units * 4);
   c.mu = o; o = align_up(o + (size_t)dm.S * dm.L * dm.Hq * D * 4);
   c.lam = o; o = align_up(o + (size_t)dm.S * dm.L * dm.Hq * D * 4);
@@ -114,6 +115,7 @@ Ws make_ws(void* base, const Carve& c) {
   Ws ws;
   ws.status = (uint32_t*)(b + c.status);
   ws.plan = (int32_t*)(b + c.plan);
+  ws.chunks = (int4*)(b + c.chunks);
   ws.counters = (int32_t*)(b + c.counters);
   ws.mu = (float*)(b + c.mu);
   ws.lam = (float*)(b + c.lam);

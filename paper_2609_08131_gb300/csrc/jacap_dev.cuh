@@ -44,6 +44,7 @@ struct Dims {
 struct Ws {
   uint32_t* status;   // [16] status word + first failing unit
   int32_t* plan;      // [0] = chunks per plane C_tot, [1 .. S+1] = chunk prefix per request
+  int4* chunks;       // [c_cap] chunk r of every plane: {t0, t1, request, r}
   int32_t* counters;  // [units] per-unit completion counters (reserved)
   float* mu;          // [S][L][Hq][D]  mu / (tau sqrt d)
   float* lam;         // [S][L][Hq][D]  diagonal of Lambda_Q
@@ -59,34 +60,39 @@ struct Ws {
 
 // A unit is (plane p = l*Hkv + g, request s); its index is p*S + s.
 struct Item {
-  int plane, seq, chunk;  // chunk index within the request
+  int plane, seq;         // plane and request
   int64_t t0, t1;         // token range [t0, t1) on the plane's token axis
-  int64_t seq_start;      // cu[s]
-  int cidx;               // chunk index within the plane (prefix[s] + chunk)
+  int cidx;               // chunk index within the plane
 };
 
-__device__ __forceinline__ bool decode_item(const Dims& dm, const int32_t* plan, const int32_t* cu,
-                                            int64_t item, Item& it) {
-  const int ctot = plan[0];
-  const int64_t total = (int64_t)dm.L * dm.Hkv * ctot;
-  if (item >= total) return false;
-  it.plane = (int)(item / ctot);
-  const int r = (int)(item - (int64_t)it.plane * ctot);
-  // largest s with prefix[s] <= r (prefix is plan[1 .. S+1], nondecreasing)
-  int lo = 0, hi = dm.S - 1;
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (plan[1 + mid] <= r) lo = mid; else hi = mid - 1;
+// The work items of a persistent CTA: items start, start + stride, ... where
+// item i = plane * C_tot + r is chunk r of the plane (chunks never straddle
+// requests; the chunk table is the same for every plane). The record of the
+// next item is loaded while the current one is processed, so an item
+// boundary costs no dependent global loads.
+struct ItemStream {
+  const int4* tab;
+  int64_t total, i, step;
+  int ctot;
+  int4 rec;
+  __device__ __forceinline__ ItemStream(const Dims& dm, const Ws& ws, int64_t start, int64_t stride)
+      : tab(ws.chunks), i(start), step(stride) {
+    ctot = ws.plan[0];
+    total = (int64_t)dm.L * dm.Hkv * ctot;
+    if (i < total) rec = tab[i % ctot];
   }
-  it.seq = lo;
-  it.chunk = r - plan[1 + lo];
-  it.cidx = r;
-  it.seq_start = cu[lo];
-  const int64_t end = cu[lo + 1];
-  it.t0 = it.seq_start + (int64_t)it.chunk * dm.chunk;
-  it.t1 = min(end, it.t0 + (int64_t)dm.chunk);
-  return true;
-}
+  __device__ __forceinline__ bool next(Item& it) {
+    if (i >= total) return false;
+    it.plane = (int)(i / ctot);
+    it.t0 = rec.x;
+    it.t1 = rec.y;
+    it.seq = rec.z;
+    it.cidx = rec.w;
+    i += step;
+    if (i < total) rec = tab[i % ctot];
+    return true;
+  }
+};
 
 __device__ __forceinline__ bool status_failed(const Ws& ws) {
   return *((volatile uint32_t*)ws.status) != 0u;
@@ -181,6 +187,7 @@ constexpr uint32_t WAIT_SUSPEND_NS = 1000;
 // if *abort became nonzero while waiting.
 static __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, const Ws& ws,
                                             volatile int* abort) {
+  if (abort != nullptr && *abort) return false;
   const unsigned long long t0 = globaltimer();
   for (uint32_t it = 0;; ++it) {
     if (mbar_try_wait_suspend(bar, parity, WAIT_SUSPEND_NS)) return true;

@@ -58,7 +58,7 @@ __global__ void __launch_bounds__(WT_THREADS) weight_kernel(Dims dm, Ws ws, cons
   if (s_skip) return;
   bool bad = false;
   Item item;
-  for (int64_t i = blockIdx.x; decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+  for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
     __syncthreads();
     if (warp < G) {
       float M, Z;
@@ -197,7 +197,7 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
       uint32_t it = 0;
       bool ok = true;
       Item item;
-      for (int64_t i = blockIdx.x; ok && decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+      for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); ok && is.next(item);) {
         const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
         for (int64_t t = item.t0; t < item.t1; t += TILE) {
           const int st = it % GR_VST;
@@ -225,7 +225,7 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
       uint32_t it = 0, nitem = 0;
       bool ok = true;
       Item item;
-      for (int64_t i = blockIdx.x; ok && decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+      for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); ok && is.next(item);) {
         // accumulator of this item; its previous item's epilogue must be done
         const int db = nitem & 1;
         const uint32_t dacc = tmem + (db ? GR_DCOL1 : 0u);
@@ -267,7 +267,7 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
     const int lm = lane >> 3, lr = lane & 7;
     uint32_t it = 0, nitem = 0;
     Item item;
-    for (int64_t i = blockIdx.x; decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+    for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
       for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
         const int vs = it % GR_VST, ab = it & 1;
         if (!mbar_wait(smem_u32(&vfull[vs]), (it / GR_VST) & 1, ws, abort)) goto scale_done;
@@ -373,7 +373,7 @@ __global__ void __launch_bounds__(GF_THREADS)
   if (s_skip) return;
   const int rb = tid / 16, cb = tid % 16;
   Item item;
-  for (int64_t i = blockIdx.x; decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+  for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
     const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
     const float* vbase = v + (int64_t)l * dm.kv_sl + (int64_t)g * dm.kv_sh;
     float acc[8][8];

@@ -190,7 +190,7 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
       uint32_t it = 0;
       bool ok = true;
       Item item;
-      for (int64_t i = blockIdx.x; ok && decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+      for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); ok && is.next(item);) {
         const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
         for (int64_t t = item.t0; t < item.t1; t += TILE) {
           const int st = it % KB_STAGES;
@@ -215,11 +215,11 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
       uint32_t it = 0, nitem = 0;
       bool ok = true;
       Item item;
-      for (int64_t i = blockIdx.x; ok && decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+      for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); ok && is.next(item);) {
         const int p = nitem & 1;
         if (!mbar_wait(smem_u32(&imgready[p]), (nitem >> 1) & 1, ws, abort)) break;
         tc_fence_after();
-        const uint32_t ia = smem_u32(img + p * C::IMG_BYTES);
+        const uint64_t b0 = smem_desc_sw128(smem_u32(img + p * C::IMG_BYTES), 16, 1024);
         for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
           const int st = it % KB_STAGES;
           const int ab = it % KB_NACC;
@@ -230,12 +230,13 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t ka = smem_u32(tiles + st * KB_TILE_BYTES);
+          // descriptors advance by (byte offset >> 4) in their address field
+          const uint64_t a0 = smem_desc_sw128(smem_u32(tiles + st * KB_TILE_BYTES), 16, 1024);
           const uint32_t dl = tmem + ab * C::NB;
 #pragma unroll
           for (int k = 0; k < D / 16; ++k) {  // 16 channels per MMA
-            const uint64_t ad = smem_desc_sw128(ka + (k >> 2) * KB_BOX + (k & 3) * 32, 16, 1024);
-            const uint64_t bm = smem_desc_sw128(ia + (k >> 2) * C::IMG_ATOM + (k & 3) * 32, 16, 1024);
+            const uint64_t ad = a0 + (uint64_t)((((k >> 2) * KB_BOX) + (k & 3) * 32) >> 4);
+            const uint64_t bm = b0 + (uint64_t)((((k >> 2) * C::IMG_ATOM) + (k & 3) * 32) >> 4);
             umma_f16_ss(dl, ad, bm, C::IDESC, k > 0 ? 1u : 0u);
           }
           umma_commit(smem_u32(&empty[st]));
@@ -251,7 +252,7 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
     // ---------------------------------- mu' image and lambda, one item ahead
     uint32_t nitem = 0;
     Item item;
-    for (int64_t i = blockIdx.x; decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+    for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
       const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
       const int p = nitem & 1;
       if (nitem >= 2 && !mbar_wait(smem_u32(&imgfree[p]), ((nitem >> 1) - 1) & 1, ws, abort)) break;
@@ -276,7 +277,7 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
     Item item;
     // A failed wait (which means the abort flag is set) still arrives at the
     // group's named barriers, and the four warps leave together after them.
-    for (int64_t i = blockIdx.x; decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+    for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
       const int p = nitem & 1;
       mbar_wait(smem_u32(&imgready[p]), (nitem >> 1) & 1, ws, abort);
       named_barrier_sync(bar_id, 128);
@@ -339,7 +340,7 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
     uint32_t it = 0;
     bool bad = false;
     Item item;
-    for (int64_t i = blockIdx.x; decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+    for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
       float run_m[G], run_s[G];
 #pragma unroll
       for (int h = 0; h < G; ++h) {
@@ -364,12 +365,10 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
           for (int h = 0; h < G; ++h) {
             lg[h] = dv[h] + dv[G + h] + dv[2 * G + h];
             bad |= !isfinite(lg[h]);
-            if (lg[h] > run_m[h]) {
-              run_s[h] = run_s[h] * expf(run_m[h] - lg[h]) + 1.f;
-              run_m[h] = lg[h];
-            } else {
-              run_s[h] += expf(lg[h] - run_m[h]);
-            }
+            // branch-free online update: one of the two exponentials is exp(0)
+            const float mn = fmaxf(run_m[h], lg[h]);
+            run_s[h] = run_s[h] * expf(run_m[h] - mn) + expf(lg[h] - mn);
+            run_m[h] = mn;
           }
           store_part<G>(lkp + tok * (2 * G), lg);
         }

@@ -6,7 +6,9 @@
 // the factor kernel; V comes straight from the TMA-staged tile. Each epilogue
 // thread owns one token (one TMEM lane) and reduces ||y||^2 = sum_j (D[j] +
 // D[128+j])^2 in fp32, then multiplies by w_i. The tensor-memory accumulator
-// is double-buffered so the epilogue of tile i overlaps the MMAs of tile i+1.
+// is double-buffered so the epilogue of tile i overlaps the MMAs of tile i+1,
+// and so is the L^{-1} image, so the next item's image streams in while the
+// current item's tiles run.
 // float32 caches: SIMT forward products with L^{-1} held in shared memory.
 #include "jacap_dev.cuh"
 #include "jacap_internal.h"
@@ -14,7 +16,7 @@
 namespace jacap {
 
 constexpr int SC_THREADS = 192;  // warp 0: TMA, warp 1: MMA, warps 2-5: epilogue
-constexpr int SC_STAGES = 4;
+constexpr int SC_STAGES = 3;
 constexpr int SC_BOX = 16384;
 constexpr int SC_TILE_BYTES = 2 * SC_BOX;
 constexpr int SC_M_BYTES = 65536;
@@ -22,22 +24,22 @@ constexpr uint32_t SC_TMEM_COLS = 512;
 // M = 128 tokens, N = 256 (hi | lo rows of L^{-1}), both operands K-major.
 constexpr uint32_t SC_IDESC = idesc_bf16_f32(128, 256, 0, 0);
 
-constexpr size_t score_bf16_smem_bytes() { return 1024 + SC_M_BYTES + SC_STAGES * SC_TILE_BYTES + 256; }
+constexpr size_t score_bf16_smem_bytes() { return 1024 + 2 * SC_M_BYTES + SC_STAGES * SC_TILE_BYTES + 256; }
 
 __global__ void __launch_bounds__(SC_THREADS, 1)
     score_bf16_kernel(const __grid_constant__ CUtensorMap vmap, Dims dm, Ws ws, const int32_t* __restrict__ cu,
                       float* __restrict__ scores) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint8_t* mimg = smem;
-  uint8_t* stages = smem + SC_M_BYTES;
+  uint8_t* mimg = smem;                       // [2][SC_M_BYTES], by item parity
+  uint8_t* stages = smem + 2 * SC_M_BYTES;
   uint64_t* vfull = (uint64_t*)(stages + SC_STAGES * SC_TILE_BYTES);
   uint64_t* vempty = vfull + SC_STAGES;
   uint64_t* accfull = vempty + SC_STAGES;
   uint64_t* accempty = accfull + 2;
-  uint64_t* mfull = accempty + 2;
-  uint64_t* mempty = mfull + 1;
-  uint64_t* mdone = mempty + 1;
+  uint64_t* mfull = accempty + 2;   // [2]
+  uint64_t* mempty = mfull + 2;     // [2]
+  uint64_t* mdone = mempty + 2;
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort, s_skip;
 
@@ -53,8 +55,10 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
       mbar_init(smem_u32(&accfull[i]), 1);
       mbar_init(smem_u32(&accempty[i]), 4);
     }
-    mbar_init(smem_u32(mfull), 1);
-    mbar_init(smem_u32(mempty), 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(smem_u32(&mfull[i]), 1);
+      mbar_init(smem_u32(&mempty[i]), 1);
+    }
     mbar_init(smem_u32(mdone), 1);
     fence_mbar_init();
   }
@@ -76,12 +80,13 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
       uint32_t it = 0, nitem = 0;
       bool ok = true;
       Item item;
-      for (int64_t i = blockIdx.x; ok && decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+      for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); ok && is.next(item);) {
         const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
         const int64_t u = (int64_t)item.plane * dm.S + item.seq;
-        if (nitem > 0 && !mbar_wait(smem_u32(mempty), (nitem - 1) & 1, ws, abort)) break;
-        mbar_arrive_expect_tx(smem_u32(mfull), SC_M_BYTES);
-        bulk_g2s(smem_u32(mimg), ws.minv_img + u * SC_M_BYTES, SC_M_BYTES, smem_u32(mfull));
+        const int mp = nitem & 1;
+        if (nitem >= 2 && !mbar_wait(smem_u32(&mempty[mp]), ((nitem >> 1) & 1) ^ 1, ws, abort)) break;
+        mbar_arrive_expect_tx(smem_u32(&mfull[mp]), SC_M_BYTES);
+        bulk_g2s(smem_u32(mimg + mp * SC_M_BYTES), ws.minv_img + u * SC_M_BYTES, SC_M_BYTES, smem_u32(&mfull[mp]));
         ++nitem;
         for (int64_t t = item.t0; t < item.t1; t += TILE) {
           const int st = it % SC_STAGES;
@@ -99,17 +104,19 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
       }
       for (uint32_t k = (it > (uint32_t)SC_STAGES ? it - SC_STAGES : 0); k < it; ++k)
         mbar_wait(smem_u32(&vfull[k % SC_STAGES]), (k / SC_STAGES) & 1, ws, nullptr);
-      if (nitem > 0) mbar_wait(smem_u32(mfull), (nitem - 1) & 1, ws, nullptr);
+      for (uint32_t k = (nitem > 2 ? nitem - 2 : 0); k < nitem; ++k)
+        mbar_wait(smem_u32(&mfull[k & 1]), (k >> 1) & 1, ws, nullptr);
     }
   } else if (warp == 1) {
     if (lane == 0) {
       uint32_t it = 0, nitem = 0;
       bool ok = true;
       Item item;
-      for (int64_t i = blockIdx.x; ok && decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
-        if (!mbar_wait(smem_u32(mfull), nitem & 1, ws, abort)) break;
+      for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); ok && is.next(item);) {
+        const int mp = nitem & 1;
+        if (!mbar_wait(smem_u32(&mfull[mp]), (nitem >> 1) & 1, ws, abort)) break;
         tc_fence_after();
-        const uint32_t ma = smem_u32(mimg);
+        const uint32_t ma = smem_u32(mimg + mp * SC_M_BYTES);
         for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
           const int st = it % SC_STAGES;
           const int ab = it & 1;
@@ -134,7 +141,7 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
           umma_commit(smem_u32(&accfull[ab]));
         }
         if (!ok) break;
-        umma_commit(smem_u32(mempty));
+        umma_commit(smem_u32(&mempty[mp]));
         ++nitem;
       }
       // every MMA issued by this thread has completed before teardown
@@ -147,7 +154,7 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
     uint32_t it = 0;
     bool bad = false;
     Item item;
-    for (int64_t i = blockIdx.x; decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+    for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
       for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
         const int ab = it & 1;
         const int64_t tok = t + y;
@@ -208,7 +215,7 @@ __global__ void __launch_bounds__(SF_THREADS)
   bool bad = false;
   int64_t loaded = -1;
   Item item;
-  for (int64_t i = blockIdx.x; decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+  for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
     const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
     const int64_t u = (int64_t)item.plane * dm.S + item.seq;
     const float* vbase = v + (int64_t)l * dm.kv_sl + (int64_t)g * dm.kv_sh;

@@ -35,6 +35,22 @@ __global__ void plan_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu) {
   ws.plan[0] = acc;
 }
 
+// Chunk table: record r = {t0, t1, request, r} for the C_tot chunks of a plane.
+__global__ void chunk_table_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu) {
+  const int ctot = ws.plan[0];
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= ctot) return;
+  // largest s with prefix[s] <= r (prefix is plan[1 .. S+1], nondecreasing)
+  int lo = 0, hi = dm.S - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (ws.plan[1 + mid] <= r) lo = mid; else hi = mid - 1;
+  }
+  const int64_t t0 = (int64_t)cu[lo] + (int64_t)(r - ws.plan[1 + lo]) * dm.chunk;
+  const int64_t t1 = min((int64_t)cu[lo + 1], t0 + (int64_t)dm.chunk);
+  ws.chunks[r] = make_int4((int)t0, (int)t1, lo, r);
+}
+
 template <typename T>
 __device__ __forceinline__ float ld_elem(const T* p);
 template <>
@@ -126,7 +142,7 @@ __global__ void __launch_bounds__(KP_THREADS, 1)
       uint32_t it = 0;
       bool ok = true;
       Item item;
-      for (int64_t i = blockIdx.x; ok && decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+      for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); ok && is.next(item);) {
         const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
         for (int64_t t = item.t0; t < item.t1; t += TILE) {
           const int st = it % C::STAGES;
@@ -156,7 +172,7 @@ __global__ void __launch_bounds__(KP_THREADS, 1)
   uint32_t it = 0;
   bool bad = false;
   Item item;
-  for (int64_t i = blockIdx.x; decode_item(dm, ws.plan, cu, i, item); i += gridDim.x) {
+  for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
     const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
     // query statistics of the G heads of this KV head
     asm volatile("bar.sync 1, 128;" ::: "memory");
@@ -279,6 +295,9 @@ static cudaError_t launch_window_stats_t(const Dims& dm, const Ws& ws, const voi
 
 cudaError_t launch_plan(const Dims& dm, const Ws& ws, const int32_t* cu, cudaStream_t st) {
   plan_kernel<<<1, 32, 0, st>>>(dm, ws, cu);
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  chunk_table_kernel<<<(unsigned)((dm.c_cap + 255) / 256), 256, 0, st>>>(dm, ws, cu);
   return cudaGetLastError();
 }
 
