@@ -52,7 +52,7 @@ struct Ws {
   float* cstats;      // [L*Hkv][c_cap][G][2]  per-chunk (max, sum exp(l - max))
   float* w;           // [L*Hkv][Ntot]  Eq. 8 weights summed over the group
   uint32_t* wsplit;   // [L*Hkv][Ntot]  w as bf16 hi (low half) + bf16 lo = w - hi (high half)
-  float* gpart;       // [L*Hkv][c_cap][D][D]  per-chunk partial Grams
+  float* gpart;       // [L*Hkv][c_cap][D/32][D][32]  per-chunk partial Grams: (m, n) at ((n/32) D + m) 32 + n%32
   float* gram;        // [units][D][D]  sum_i w_i v_i v_i^T
   float* minv;        // [units][D][D]  L^{-1} (float32, lower triangular)
   uint8_t* minv_img;  // [units][65536]  L^{-1} as bf16 hi/lo, shared-memory image for the score MMA

@@ -57,11 +57,13 @@ __global__ void __launch_bounds__(FA_THREADS, 1) factor_kernel(Dims dm, Ws ws) {
 #pragma unroll
       for (int b = 0; b < 4; ++b) ar[a][b] = 0.f;
     for (int ch = c0; ch < c1; ++ch) {  // 32 independent loads in flight per chunk
+      // partial layout: (m, n) at ((n / 32) D + m) 32 + n % 32, so a warp
+      // (fixed row, 32 consecutive columns) reads 128 contiguous bytes
       const float* src = gp + (int64_t)ch * D * D;
 #pragma unroll
       for (int a = 0; a < 8; ++a)
 #pragma unroll
-        for (int b = 0; b < 4; ++b) ar[a][b] += src[(ty + 16 * a) * D + tx + 32 * b];
+        for (int b = 0; b < 4; ++b) ar[a][b] += src[(b * D + ty + 16 * a) * 32 + tx];
     }
 #pragma unroll
     for (int a = 0; a < 8; ++a)

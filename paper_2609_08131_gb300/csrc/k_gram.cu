@@ -112,8 +112,10 @@ __global__ void __launch_bounds__(WT_THREADS) weight_kernel(Dims dm, Ws ws, cons
 // hi + lo from the weight pass). The scaling warps read V transposed with
 // ldmatrix, form w_i v_i = hi + lo with packed bf16 arithmetic and store hi
 // and lo as two A operands; two MMAs per 16 tokens accumulate v (hi + lo)^T.
-// The scaling warps share nothing but the mbarriers of the pipeline.
-constexpr int GR_THREADS = 320;   // warp 0: TMA, warp 1: MMA, warps 2-9: scale + epilogue
+// The scaling warps share nothing but the mbarriers of the pipeline; four
+// epilogue warps copy each finished chunk Gram out of tensor memory while the
+// next chunk accumulates in the other buffer.
+constexpr int GR_THREADS = 448;   // warp 0: TMA, warp 1: MMA, warps 2-9: scale, warps 10-13: epilogue
 constexpr int GR_SCALERS = 256;
 constexpr int GR_VST = 6;          // V tiles in flight
 constexpr int GR_BOX = 16384;      // {64 channels, 128 tokens} bf16, 128-byte swizzle
@@ -174,7 +176,7 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&accfull[i]), 1);
-      mbar_init(smem_u32(&accempty[i]), GR_SCALERS / 32);
+      mbar_init(smem_u32(&accempty[i]), 4);  // the epilogue warps
     }
     fence_mbar_init();
   }
@@ -240,11 +242,12 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t va = smem_u32(vring + vs * GR_V_BYTES);
+          // B descriptors advance by (byte offset >> 4) in their address field
+          const uint64_t b0 = smem_desc_sw128(smem_u32(vring + vs * GR_V_BYTES), GR_BOX, 1024);
           const uint32_t acol = tmem + GR_ACOL + 128 * ab;
 #pragma unroll
           for (int k = 0; k < TILE / 16; ++k) {  // 16 tokens per MMA
-            const uint64_t bd = smem_desc_sw128(va + k * 2048, GR_BOX, 1024);
+            const uint64_t bd = b0 + (uint64_t)((k * 2048) >> 4);
             umma_f16_ts(dacc, acol + 8 * k, bd, GR_IDESC, (first && k == 0) ? 0u : 1u);
             umma_f16_ts(dacc, acol + 64 + 8 * k, bd, GR_IDESC, 1u);
           }
@@ -258,14 +261,13 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
       }
       if (it > 0) mbar_wait(smem_u32(&aempty[(it - 1) & 1]), ((it - 1) >> 1) & 1, ws, nullptr);
     }
-  } else {
-    // ------------------------------------- scaling warps + epilogue -------
+  } else if (warp < 10) {
+    // ------------------------------------------------- scaling warps ------
     const int quarter = warp & 3;        // TMEM lane quarter == channels 32 quarter .. +31
     const int th = (warp - 2) >> 2;      // token half of each tile (blocks 4 th .. 4 th + 3)
-    const int m = quarter * 32 + lane;   // Gram row (channel) owned in the epilogue
     // ldmatrix row addresses: lane l -> matrix l / 8, row l % 8
     const int lm = lane >> 3, lr = lane & 7;
-    uint32_t it = 0, nitem = 0;
+    uint32_t it = 0;
     Item item;
     for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
       for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
@@ -322,29 +324,36 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_u32(&afull[ab]));
       }
-      // epilogue: D is this chunk's partial Gram; warp (quarter, th) writes rows
-      // 32 quarter .. +31, columns 64 th .. 64 th + 63
+    }
+  scale_done:;
+  } else {
+    // ------------------------------------------------------ epilogue ------
+    // D is a chunk's partial Gram; warp (quarter q) copies rows 32 q .. +31,
+    // each lane its row: 32 consecutive floats per column block, so a lane
+    // writes 128 contiguous bytes per block.
+    const int quarter = warp & 3;
+    const int m = quarter * 32 + lane;
+    uint32_t nitem = 0;
+    Item item;
+    for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
       const int db = nitem & 1;
-      if (!mbar_wait(smem_u32(&accfull[db]), (nitem >> 1) & 1, ws, abort)) goto scale_done;
+      if (!mbar_wait(smem_u32(&accfull[db]), (nitem >> 1) & 1, ws, abort)) break;
       tc_fence_after();
-      {
-        const uint32_t trow = tmem + (db ? GR_DCOL1 : 0u) + ((uint32_t)(quarter * 32) << 16) + 64 * th;
-        float* dst = ws.gpart + (((int64_t)item.plane * dm.c_cap + item.cidx) * D + m) * D + 64 * th;
+      const uint32_t trow = tmem + (db ? GR_DCOL1 : 0u) + ((uint32_t)(quarter * 32) << 16);
+      float* dst = ws.gpart + ((int64_t)item.plane * dm.c_cap + item.cidx) * D * D + (int64_t)m * 32;
 #pragma unroll 1
-        for (int cb = 0; cb < 2; ++cb) {
-          float a[32];
-          tmem_ld32(trow + cb * 32, a);
+      for (int cb = 0; cb < D / 32; ++cb) {
+        float a[32];
+        tmem_ld32(trow + cb * 32, a);
 #pragma unroll
-          for (int j = 0; j < 32; j += 4)
-            *(float4*)(dst + cb * 32 + j) = make_float4(a[j], a[j + 1], a[j + 2], a[j + 3]);
-        }
+        for (int j = 0; j < 32; j += 4)
+          *(float4*)(dst + cb * D * 32 + j) = make_float4(a[j], a[j + 1], a[j + 2], a[j + 3]);
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&accempty[db]));
       ++nitem;
     }
-  scale_done:;
   }
   tc_fence_before();
   __syncthreads();
@@ -415,7 +424,9 @@ __global__ void __launch_bounds__(GF_THREADS)
     float* dst = ws.gpart + ((int64_t)item.plane * dm.c_cap + item.cidx) * D * D;
 #pragma unroll
     for (int p = 0; p < 8; ++p) {
-      float* row = dst + (rb * 8 + p) * D + cb * 8;
+      // (m, n) at ((n / 32) D + m) 32 + n % 32; the 8 columns share one block
+      const int m = rb * 8 + p, n0 = cb * 8;
+      float* row = dst + ((n0 >> 5) * D + m) * 32 + (n0 & 31);
       *(float4*)row = make_float4(acc[p][0], acc[p][1], acc[p][2], acc[p][3]);
       *(float4*)(row + 4) = make_float4(acc[p][4], acc[p][5], acc[p][6], acc[p][7]);
     }

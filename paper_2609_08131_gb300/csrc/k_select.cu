@@ -3,12 +3,17 @@
 //
 // select_kernel: one 1024-thread CTA per unit (grid-stride). Scores are
 // non-negative float32, so their bit patterns order like unsigned integers.
-// Four 8-bit radix passes (most significant digit first, shared-memory
-// histograms) find the B-th largest key T and how many keys equal to T are
-// still needed; one ordered pass then keeps every key > T and the first
-// `need` keys == T by position (ties go to the lower position), writing the
-// kept positions in ascending order through block-wide ballot scans. All of
-// it is deterministic.
+// Three radix passes (digits of 11, 11 and 10 bits, most significant first,
+// shared-memory histograms; a pass counts only keys that match the digits
+// found so far) find the B-th largest key T and how many keys equal to T are
+// still needed. The keys are read in slabs of 32768 into registers (32 per
+// lane, all loads in flight together); a request of up to 32768 tokens is
+// read once and every pass works on registers. Emission walks the slabs in
+// order; in a slab each warp owns 1024 consecutive positions, counts its keys
+// > T and == T with ballots, and the warp totals give where its kept
+// positions go and which of its keys == T are among the first `need` by
+// position (ties go to the lower position); kept positions come out in
+// ascending order. All of it is deterministic.
 //
 // compact_kernel: 16-byte vector copies of the kept K and V rows into the
 // dense [L][Hkv][S][B][d] output; rows of -1 (or of a position outside the
@@ -20,44 +25,34 @@ namespace jacap {
 
 constexpr int SE_THREADS = 1024;
 
-// Exclusive block-wide prefix count of `pred`; returns the prefix for this
-// thread and writes the block total to *total. Uses wsum[32] in smem.
-__device__ __forceinline__ int block_excl_count(bool pred, int* wsum, int* total) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const unsigned bal = __ballot_sync(0xffffffffu, pred);
-  const int in_warp = __popc(bal & ((1u << lane) - 1u));
-  if (lane == 0) wsum[warp] = __popc(bal);
-  __syncthreads();
-  if (warp == 0) {
-    const int x = wsum[lane];
-    int incl = x;
+constexpr int SE_BINS = 2048;
+constexpr int SE_KPT = 32;                       // keys per lane of a slab
+constexpr int SE_SLAB = SE_THREADS * SE_KPT;     // 32768 keys: warp w holds positions 1024 w .. +1023
+
+// Keys of slab `sl` into registers: lane's register j holds position
+// sl * SE_SLAB + 1024 w + 32 j + lane (coalesced; all loads in flight at once).
+__device__ __forceinline__ void load_slab(const uint32_t* key, int n, int sl, int warp, int lane,
+                                          uint32_t (&kr)[SE_KPT]) {
+  const int base = sl * SE_SLAB + warp * (32 * SE_KPT) + lane;
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += y;
-    }
-    wsum[lane] = incl - x;  // exclusive
-    if (lane == 31) wsum[32] = incl;
+  for (int j = 0; j < SE_KPT; ++j) {
+    const int i = base + 32 * j;
+    kr[j] = i < n ? __ldg(key + i) : 0u;
   }
-  __syncthreads();
-  const int r = wsum[warp] + in_warp;
-  *total = wsum[32];
-  __syncthreads();
-  return r;
 }
 
 __global__ void __launch_bounds__(SE_THREADS)
     select_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu, const float* __restrict__ scores, int B,
                   int32_t* __restrict__ idx, int32_t* __restrict__ kept) {
-  __shared__ uint32_t hist[256];
-  __shared__ int wsum[33];
+  __shared__ uint32_t hist[SE_BINS];
   __shared__ uint32_t s_digit, s_need;
   __shared__ int s_skip;
-  const int tid = threadIdx.x;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   if (tid == 0) s_skip = status_failed(ws) ? 1 : 0;
   __syncthreads();
   if (s_skip) return;
   const int units = dm.L * dm.Hkv * dm.S;
+  const uint32_t lt = (1u << lane) - 1u;
   for (int u = blockIdx.x; u < units; u += gridDim.x) {
     const int plane = u / dm.S, s = u % dm.S;
     const int64_t start = cu[s];
@@ -78,51 +73,104 @@ __global__ void __launch_bounds__(SE_THREADS)
       for (int r = tid; r < B; r += SE_THREADS) out[r] = r < n ? r : -1;
       continue;
     }
-    // ---- radix select of the B-th largest key ----
+    const int nslab = (n + SE_SLAB - 1) / SE_SLAB;
+    uint32_t kr[SE_KPT];
+    if (nslab == 1) load_slab(key, n, 0, warp, lane, kr);  // register-resident for all passes
+    // ---- radix select of the B-th largest key: digits [31:21], [20:10], [9:0] ----
     uint32_t prefix = 0, mask = 0, need = (uint32_t)B;
-    for (int pass = 0; pass < 4; ++pass) {
-      const int shift = 24 - 8 * pass;
-      for (int b = tid; b < 256; b += SE_THREADS) hist[b] = 0;
+#pragma unroll 1
+    for (int pass = 0; pass < 3; ++pass) {
+      const int shift = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
+      const uint32_t dmask = pass == 2 ? 1023u : 2047u;
+      for (int b = tid; b < SE_BINS; b += SE_THREADS) hist[b] = 0;
       __syncthreads();
-      for (int i = tid; i < n; i += SE_THREADS) {
-        const uint32_t k = key[i];
-        if ((k & mask) == prefix) atomicAdd(&hist[(k >> shift) & 255u], 1u);
+#pragma unroll 1
+      for (int sl = 0; sl < nslab; ++sl) {
+        if (nslab > 1) load_slab(key, n, sl, warp, lane, kr);
+        const int base = sl * SE_SLAB + warp * (32 * SE_KPT) + lane;
+#pragma unroll
+        for (int j = 0; j < SE_KPT; ++j)
+          if (base + 32 * j < n && (kr[j] & mask) == prefix) atomicAdd(&hist[(kr[j] >> shift) & dmask], 1u);
       }
       __syncthreads();
-      if (tid == 0) {
-        uint32_t above = 0;
-        int d = 255;
-        for (; d > 0; --d) {
-          if (above + hist[d] >= need) break;
-          above += hist[d];
+      if (warp == 0) {
+        // lane l sums bins 64 l .. 64 l + 63; suffix sums over lanes locate the
+        // bin holding the need-th largest key, which that lane then finds
+        uint32_t c = 0;
+        for (int b = 0; b < 64; ++b) c += hist[64 * lane + b];
+        uint32_t suf = c;  // sum over lanes >= lane
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const uint32_t y = __shfl_down_sync(0xffffffffu, suf, o);
+          if (lane + o < 32) suf += y;
         }
-        s_digit = (uint32_t)d;
-        s_need = need - above;
+        const uint32_t above = suf - c;  // keys in bins of higher lanes
+        if (above < need && suf >= need) {  // exactly one lane
+          uint32_t acc = above;
+          int d = 64 * lane + 63;
+          for (; d > 64 * lane; --d) {
+            if (acc + hist[d] >= need) break;
+            acc += hist[d];
+          }
+          s_digit = (uint32_t)d;
+          s_need = need - acc;
+        }
       }
       __syncthreads();
       prefix |= s_digit << shift;
-      mask |= 255u << shift;
+      mask |= dmask << shift;
       need = s_need;
       __syncthreads();
     }
-    const uint32_t T = prefix;  // the B-th largest key; `need` keys == T are kept
-    // ---- ordered emission ----
-    int written = 0, eq_seen = 0;
-    for (int base = 0; base < n && written < B; base += SE_THREADS) {
-      const int i = base + tid;
-      const uint32_t k = i < n ? key[i] : 0u;
-      const bool gt = i < n && k > T;
-      const bool eq = i < n && k == T;
-      int eq_total;
-      const int eq_rank = eq_seen + block_excl_count(eq, wsum, &eq_total);
-      const bool sel = gt || (eq && eq_rank < (int)need);
-      int sel_total;
-      const int pos = written + block_excl_count(sel, wsum, &sel_total);
-      if (sel && pos < B) out[pos] = i;
-      written += sel_total;
-      eq_seen += eq_total;
+    const uint32_t T = prefix;  // the B-th largest key; the first `need` keys == T are kept
+    // ---- emission, slab by slab; in a slab warp w owns positions 1024 w .. +1023 ----
+    uint32_t gt_run = 0, eq_run = 0;  // kept-greater and equal keys before this slab
+#pragma unroll 1
+    for (int sl = 0; sl < nslab; ++sl) {
+      if (nslab > 1) load_slab(key, n, sl, warp, lane, kr);
+      const int base = sl * SE_SLAB + warp * (32 * SE_KPT) + lane;
+      uint32_t gt = 0, eq = 0;
+#pragma unroll
+      for (int j = 0; j < SE_KPT; ++j) {
+        const bool v = base + 32 * j < n;
+        gt += __popc(__ballot_sync(0xffffffffu, v && kr[j] > T));
+        eq += __popc(__ballot_sync(0xffffffffu, v && kr[j] == T));
+      }
+      if (lane == 0) {
+        hist[warp] = gt;  // the histogram is free again: it holds the warp totals
+        hist[32 + warp] = eq;
+      }
+      __syncthreads();
+      uint32_t gt_before = gt_run, eq_before = eq_run, gt_all = 0, eq_all = 0;
+      for (int w = 0; w < 32; ++w) {
+        const uint32_t g = hist[w], e = hist[32 + w];
+        if (w < warp) {
+          gt_before += g;
+          eq_before += e;
+        }
+        gt_all += g;
+        eq_all += e;
+      }
+      // kept before this warp's block: all greater keys plus the equal ones of rank < need
+      uint32_t pos = gt_before + min(eq_before, need);
+      uint32_t er = eq_before;
+#pragma unroll
+      for (int j = 0; j < SE_KPT; ++j) {
+        const int i = base + 32 * j;
+        const bool v = i < n;
+        const uint32_t beq = __ballot_sync(0xffffffffu, v && kr[j] == T);
+        const uint32_t my_er = er + __popc(beq & lt);
+        const bool sel = v && (kr[j] > T || (kr[j] == T && my_er < need));
+        const uint32_t bsel = __ballot_sync(0xffffffffu, sel);
+        const uint32_t my_pos = pos + __popc(bsel & lt);
+        if (sel && my_pos < (uint32_t)B) out[my_pos] = i;
+        pos += __popc(bsel);
+        er += __popc(beq);
+      }
+      gt_run += gt_all;
+      eq_run += eq_all;
+      __syncthreads();  // the totals in hist are read before the next slab rewrites them
     }
-    __syncthreads();
   }
 }
 
