@@ -50,12 +50,13 @@ jacap_status check_layout(const jacap_layout* L) {
   return JACAP_OK;
 }
 
-// Tokens per work item: the largest of 4096..128 that still yields enough
+// Tokens per work item: the largest of 16384..128 that still yields enough
 // items to fill the GPU several times over (independent of the device so the
-// workspace size is a pure function of the layout).
+// workspace size is a pure function of the layout). Larger items mean fewer
+// partial Grams to write and re-read and fewer item boundaries.
 int pick_chunk(const jacap_layout* L) {
   const int64_t planes = (int64_t)L->num_layers * L->num_kv_heads;
-  for (int c = 4096; c > TILE; c >>= 1) {
+  for (int c = 16384; c > TILE; c >>= 1) {
     const int64_t items = planes * (L->total_tokens / c + L->num_seqs);
     if (items >= 1024) return c;
   }

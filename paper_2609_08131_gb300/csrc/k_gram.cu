@@ -236,8 +236,8 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
         bool first = true;
         for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
           const int vs = it % GR_VST, ab = it & 1;
-          if (!mbar_wait(smem_u32(&vfull[vs]), (it / GR_VST) & 1, ws, abort) ||
-              !mbar_wait(smem_u32(&afull[ab]), (it >> 1) & 1, ws, abort)) {
+          // the scaling warps arrive on afull only after the tile's V landed
+          if (!mbar_wait(smem_u32(&afull[ab]), (it >> 1) & 1, ws, abort)) {
             ok = false;
             break;
           }

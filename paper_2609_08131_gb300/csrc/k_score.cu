@@ -1,11 +1,13 @@
 // k_score.cu - Jacap scores r_i = w_i v_i^T A^{-1} v_i = w_i ||L^{-1} v_i||^2 (Eq. 10).
 //
-// bf16 caches: the tensor cores form Y = V (L^{-1})^T for a 128-token tile with
-// one kind::f16 MMA chain of N = 256: columns 0-127 use hi(L^{-1}), columns
-// 128-255 lo(L^{-1}), both K-major from a 64 KB shared-memory image written by
-// the factor kernel; V comes straight from the TMA-staged tile. Each epilogue
-// thread owns one token (one TMEM lane) and reduces ||y||^2 = sum_j (D[j] +
-// D[128+j])^2 in fp32, then multiplies by w_i. The tensor-memory accumulator
+// bf16 caches: the tensor cores form Y = V (L^{-1})^T for a 128-token tile:
+// hi(L^{-1}) and lo(L^{-1}) (K-major, from a 64 KB shared-memory image written
+// by the factor kernel) accumulate into the same 128 fp32 columns, so
+// y = V (hi + lo)^T. L^{-1} is lower triangular, so output columns 0-63 need
+// only channels 0-63: the first four K-steps are N = 128 MMAs, the last four
+// N = 64 MMAs into columns 64-127. V comes straight from the TMA-staged tile.
+// Each epilogue thread owns one token (one TMEM lane) and reduces
+// ||y||^2 = sum_j D[j]^2 in fp32, then multiplies by w_i. The tensor-memory accumulator
 // is double-buffered so the epilogue of tile i overlaps the MMAs of tile i+1,
 // and so is the L^{-1} image, so the next item's image streams in while the
 // current item's tiles run.
@@ -20,9 +22,10 @@ constexpr int SC_STAGES = 3;
 constexpr int SC_BOX = 16384;
 constexpr int SC_TILE_BYTES = 2 * SC_BOX;
 constexpr int SC_M_BYTES = 65536;
-constexpr uint32_t SC_TMEM_COLS = 512;
-// M = 128 tokens, N = 256 (hi | lo rows of L^{-1}), both operands K-major.
-constexpr uint32_t SC_IDESC = idesc_bf16_f32(128, 256, 0, 0);
+constexpr uint32_t SC_TMEM_COLS = 256;  // two 128-column accumulators
+// M = 128 tokens, N = 128 or 64 rows of the L^{-1} image, both operands K-major.
+constexpr uint32_t SC_IDESC128 = idesc_bf16_f32(128, 128, 0, 0);
+constexpr uint32_t SC_IDESC64 = idesc_bf16_f32(128, 64, 0, 0);
 
 constexpr size_t score_bf16_smem_bytes() { return 1024 + 2 * SC_M_BYTES + SC_STAGES * SC_TILE_BYTES + 256; }
 
@@ -129,13 +132,22 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t va = smem_u32(stages + st * SC_TILE_BYTES);
+          // descriptors advance by (byte offset >> 4); image rows: hi at row n,
+          // lo at row 128 + n (16 KB further) of each 32 KB channel atom
+          const uint64_t a0 = smem_desc_sw128(smem_u32(stages + st * SC_TILE_BYTES), 16, 1024);
+          const uint64_t b0 = smem_desc_sw128(ma, 16, 1024);
+          const uint32_t dacc = tmem + ab * 128;
 #pragma unroll
-          for (int k = 0; k < D / 16; ++k) {  // 16 channels per MMA
-            const uint32_t koff = (k >> 2) * SC_BOX + (k & 3) * 32;
-            const uint64_t ad = smem_desc_sw128(va + koff, 16, 1024);
-            const uint64_t bd = smem_desc_sw128(ma + (k >> 2) * 32768 + (k & 3) * 32, 16, 1024);
-            umma_f16_ss(tmem + ab * 256, ad, bd, SC_IDESC, k > 0 ? 1u : 0u);
+          for (int k = 0; k < D / 16; ++k) {  // 16 channels per K-step
+            const uint64_t ad = a0 + (uint64_t)((((k >> 2) * SC_BOX) + (k & 3) * 32) >> 4);
+            const uint64_t bk = b0 + (uint64_t)((((k >> 2) * 32768) + (k & 3) * 32) >> 4);
+            if (k < 4) {  // channels 0-63: all 128 output columns
+              umma_f16_ss(dacc, ad, bk, SC_IDESC128, k > 0 ? 1u : 0u);
+              umma_f16_ss(dacc, ad, bk + (16384 >> 4), SC_IDESC128, 1u);
+            } else {      // channels 64-127: only columns (rows of L^{-1}) 64-127 are nonzero
+              umma_f16_ss(dacc + 64, ad, bk + (8192 >> 4), SC_IDESC64, 1u);
+              umma_f16_ss(dacc + 64, ad, bk + (24576 >> 4), SC_IDESC64, 1u);
+            }
           }
           umma_commit(smem_u32(&vempty[st]));
           umma_commit(smem_u32(&accfull[ab]));
@@ -162,18 +174,14 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
         const float wt = tok < item.t1 ? ws.w[o] : 0.f;  // issued before the wait: hides its latency
         if (!mbar_wait(smem_u32(&accfull[ab]), (it >> 1) & 1, ws, abort)) goto epi_done;
         tc_fence_after();
-        const uint32_t trow = tmem + ab * 256 + ((uint32_t)(quarter * 32) << 16);
+        const uint32_t trow = tmem + ab * 128 + ((uint32_t)(quarter * 32) << 16);
         float ssq = 0.f;
 #pragma unroll 1
         for (int cb = 0; cb < 4; ++cb) {
-          float a[32], b[32];
+          float a[32];
           tmem_ld32(trow + cb * 32, a);
-          tmem_ld32(trow + 128 + cb * 32, b);
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            const float yv = a[j] + b[j];
-            ssq = fmaf(yv, yv, ssq);
-          }
+          for (int j = 0; j < 32; ++j) ssq = fmaf(a[j], a[j], ssq);
         }
         tc_fence_before();
         __syncwarp();
