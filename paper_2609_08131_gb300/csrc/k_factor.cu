@@ -8,13 +8,21 @@
 // Since v^T A^{-1} v = ||L^{-1} v||^2, the score pass needs only L^{-1}
 // (Eq. 10). It is obtained by Gaussian forward elimination of [A | I] without
 // pivoting (safe: A is symmetric positive definite): after step j the pivot
-// d_j = A_jj and the right block holds X = Lt^{-1}, where A = Lt U with Lt
-// unit lower triangular and U = Diag(d) Lt^T, so L = Lt Diag(d)^{1/2} and
-// L^{-1} = Diag(d)^{-1/2} X. Both blocks live in registers: thread (ty, tx)
-// of the 16 x 32 thread grid owns rows ty + 16a and columns tx + 32b of A and
-// X; each step broadcasts column j of A (equal to row j by symmetry of every
-// Schur complement) and row j of X through double-buffered shared memory, so
-// a step costs one barrier and at most 64 fused multiply-adds per thread.
+// p_j = A_jj and the right block holds X = Lt^{-1}, where A = Lt U with Lt
+// unit lower triangular and U = Diag(p) Lt^T, so L = Lt Diag(p)^{1/2} and
+// L^{-1} = Diag(p)^{-1/2} X.
+//
+// Both blocks share one 128 x 128 register array Z: column c holds A until
+// step c eliminates it, and afterwards Y_c = -p_c X_{., c}. In that scaling
+// the eliminated value A_ic (= m_i p_c with m_i = A_ic / p_c) already equals
+// Y_ic, so step j updates every active row i > j by the same fused
+// multiply-add Z_i. -= m_i r with r_c = A_cj (c > j, lower triangle of A by
+// symmetry), r_j = 0 and r_c = Z_jc (c < j, row j of Y): one barrier and at
+// most 64 multiply-adds per thread. At the end X_ic = -Y_ic / p_c. Thread
+// (ty, tx) of the 8 x 32 grid owns rows ty + 8 a and columns 4 tx .. 4 tx + 3;
+// with 256 threads two units share an SM, so their barrier latencies overlap.
+// The multipliers use 1/p_j from the approximate hardware reciprocal refined by
+// one Newton-Raphson step (x <- x (2 - p x)), which is accurate to about one ulp.
 //
 // L^{-1} is written twice: as float32 (used by the float32 score pass and
 // exposed for tests) and as a bf16 hi/lo pair laid out exactly as the
@@ -27,13 +35,23 @@
 
 namespace jacap {
 
-constexpr int FA_THREADS = 512;
+constexpr int FA_THREADS = 256;
+constexpr int FA_ROWS = D * 32 / FA_THREADS;  // 16 rows per thread
+
+// 1/p: approximate reciprocal refined by one Newton-Raphson step.
+__device__ __forceinline__ float recip_nr(float p) {
+  float x;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(x) : "f"(p));
+  return x * fmaf(-p, x, 2.f);
+}
 constexpr int FA_LD = D + 1;
 constexpr size_t factor_smem_bytes() { return (size_t)D * FA_LD * sizeof(float); }
 
-__global__ void __launch_bounds__(FA_THREADS, 1) factor_kernel(Dims dm, Ws ws) {
+__global__ void __launch_bounds__(FA_THREADS, 2) factor_kernel(Dims dm, Ws ws) {
   extern __shared__ float Ms[];  // [D][FA_LD]: L^{-1} staged for the bf16 image
-  __shared__ float colA[2][D], rowX[2][D], piv[D];
+  __shared__ __align__(16) float colA[2][D];
+  __shared__ __align__(16) float rowY[2][D];
+  __shared__ float piv[D];
   __shared__ int s_skip, s_bad;
   const int tid = threadIdx.x;
   if (tid == 0) {
@@ -44,102 +62,112 @@ __global__ void __launch_bounds__(FA_THREADS, 1) factor_kernel(Dims dm, Ws ws) {
   if (s_skip) return;
   const int u = blockIdx.x;
   const int plane = u / dm.S, s = u % dm.S;
-  const int c0 = ws.plan[1 + s], c1 = ws.plan[2 + s];
+  const int ch0 = ws.plan[1 + s], ch1 = ws.plan[2 + s];
   const int ty = tid >> 5, tx = tid & 31;
+  const int c0 = 4 * tx;
 
-  // A = I + sum of partial Grams (chunk order); X = I
-  float ar[8][4], xr[8][4];
+  // A = I + sum of partial Grams (chunk order)
+  float z[FA_ROWS][4];
   {
     const float* gp = ws.gpart + ((int64_t)plane * dm.c_cap) * D * D;
     float* gout = ws.gram + (int64_t)u * D * D;
 #pragma unroll
-    for (int a = 0; a < 8; ++a)
+    for (int a = 0; a < FA_ROWS; ++a)
 #pragma unroll
-      for (int b = 0; b < 4; ++b) ar[a][b] = 0.f;
-    for (int ch = c0; ch < c1; ++ch) {  // 32 independent loads in flight per chunk
-      // partial layout: (m, n) at ((n / 32) D + m) 32 + n % 32, so a warp
-      // (fixed row, 32 consecutive columns) reads 128 contiguous bytes
-      const float* src = gp + (int64_t)ch * D * D;
+      for (int b = 0; b < 4; ++b) z[a][b] = 0.f;
+    for (int ch = ch0; ch < ch1; ++ch) {  // 16 independent 16-byte loads in flight per chunk
+      // partial layout: (m, n) at ((n / 32) D + m) 32 + n % 32
+      const float* src = gp + (int64_t)ch * D * D + (c0 >> 5) * D * 32 + (c0 & 31);
 #pragma unroll
-      for (int a = 0; a < 8; ++a)
-#pragma unroll
-        for (int b = 0; b < 4; ++b) ar[a][b] += src[(b * D + ty + 16 * a) * 32 + tx];
+      for (int a = 0; a < FA_ROWS; ++a) {
+        const float4 v = *(const float4*)(src + (ty + 8 * a) * 32);
+        z[a][0] += v.x;
+        z[a][1] += v.y;
+        z[a][2] += v.z;
+        z[a][3] += v.w;
+      }
     }
 #pragma unroll
-    for (int a = 0; a < 8; ++a)
+    for (int a = 0; a < FA_ROWS; ++a) {
+      const int i = ty + 8 * a;
+      *(float4*)(gout + i * D + c0) = make_float4(z[a][0], z[a][1], z[a][2], z[a][3]);
 #pragma unroll
-      for (int b = 0; b < 4; ++b) {
-        const int i = ty + 16 * a, c = tx + 32 * b;
-        gout[i * D + c] = ar[a][b];
-        ar[a][b] += (i == c ? 1.f : 0.f);
-        xr[a][b] = i == c ? 1.f : 0.f;
-      }
+      for (int b = 0; b < 4; ++b) z[a][b] += (i == c0 + b ? 1.f : 0.f);
+    }
   }
 
-  // forward elimination, step j = 32 jb + 16 jh + jj (jb, jh unrolled so the
-  // register indices of the pivot column and row are compile-time constants)
-#pragma unroll
-  for (int jb = 0; jb < 4; ++jb) {
-#pragma unroll
-    for (int jh = 0; jh < 2; ++jh) {
+  // forward elimination, step j = 8 jh + jl (jl unrolled so the register
+  // column of the pivot column is a compile-time constant)
 #pragma unroll 1
-      for (int jj = 0; jj < 16; ++jj) {
-        const int j = 32 * jb + 16 * jh + jj;
-        const int buf = j & 1;
-        if (tx == (j & 31)) {  // owners of column j of A (register column jb)
+  for (int jh = 0; jh < 16; ++jh) {
 #pragma unroll
-          for (int a = 0; a < 8; ++a) colA[buf][ty + 16 * a] = ar[a][jb];
-          if (ty == (j & 15)) piv[j] = ar[2 * jb + jh][jb];
-        }
-        if (ty == (j & 15)) {  // owners of row j of X (register row 2 jb + jh)
+    for (int jl = 0; jl < 8; ++jl) {
+      const int j = 8 * jh + jl;
+      const int buf = j & 1;
+      if (tx == (j >> 2)) {  // owners of column j: rows ty + 8 a, register column j % 4 = jl % 4
 #pragma unroll
-          for (int b = 0; b < 4; ++b) rowX[buf][tx + 32 * b] = xr[2 * jb + jh][b];
-        }
-        __syncthreads();
-        const float inv_p = 1.f / colA[buf][j];
-        float ck[4], rx[4];
+        for (int a = 0; a < FA_ROWS; ++a) colA[buf][ty + 8 * a] = z[a][jl & 3];
+      }
+      if (ty == jl) {  // owners of row j (register row jh)
+        float r0 = 0.f, r1 = 0.f, r2 = 0.f, r3 = 0.f;
 #pragma unroll
-        for (int b = 0; b < 4; ++b) {
-          ck[b] = colA[buf][tx + 32 * b];
-          rx[b] = rowX[buf][tx + 32 * b];
-        }
-#pragma unroll
-        for (int a = 0; a < 8; ++a) {
-          const int i = ty + 16 * a;
-          if (i > j) {
-            const float m = colA[buf][i] * inv_p;
-#pragma unroll
-            for (int b = 0; b < 4; ++b) {
-              const int c = tx + 32 * b;
-              if (c > j) {
-                if (c <= i) ar[a][b] = fmaf(-m, ck[b], ar[a][b]);
-              } else {
-                xr[a][b] = fmaf(-m, rx[b], xr[a][b]);
-              }
-            }
+        for (int a = 0; a < FA_ROWS; ++a)
+          if (a == jh) {
+            r0 = z[a][0];
+            r1 = z[a][1];
+            r2 = z[a][2];
+            r3 = z[a][3];
           }
+        *(float4*)&rowY[buf][c0] = make_float4(r0, r1, r2, r3);
+      }
+      __syncthreads();
+      const float pj = colA[buf][j];
+      if (tid == 0) piv[j] = pj;
+      const float inv_p = recip_nr(pj);
+      const float4 ca = *(const float4*)&colA[buf][c0];
+      const float4 ry = *(const float4*)&rowY[buf][c0];
+      const float cav[4] = {ca.x, ca.y, ca.z, ca.w}, ryv[4] = {ry.x, ry.y, ry.z, ry.w};
+      float r[4];
+#pragma unroll
+      for (int b = 0; b < 4; ++b) r[b] = c0 + b > j ? cav[b] : (c0 + b == j ? 0.f : ryv[b]);
+      const float2 r01 = make_float2(r[0], r[1]), r23 = make_float2(r[2], r[3]);
+#pragma unroll
+      for (int a = 0; a < FA_ROWS; ++a) {
+        if (ty + 8 * a > j) {  // active rows (uniform over the warp)
+          const float m = colA[buf][ty + 8 * a] * inv_p;
+          const float2 nm = make_float2(-m, -m);
+          const float2 z01 = __ffma2_rn(nm, r01, make_float2(z[a][0], z[a][1]));
+          const float2 z23 = __ffma2_rn(nm, r23, make_float2(z[a][2], z[a][3]));
+          z[a][0] = z01.x;
+          z[a][1] = z01.y;
+          z[a][2] = z23.x;
+          z[a][3] = z23.y;
         }
       }
     }
   }
   __syncthreads();
 
-  // L^{-1} = Diag(d)^{-1/2} X
+  // L^{-1}_ic = X_ic / sqrt(p_i) with X_ic = -Y_ic / p_c (c < i), X_ii = 1
   float* mout = ws.minv + (int64_t)u * D * D;
+  float ipc[4];
 #pragma unroll
-  for (int a = 0; a < 8; ++a) {
-    const int i = ty + 16 * a;
+  for (int b = 0; b < 4; ++b) ipc[b] = 1.f / piv[c0 + b];
+#pragma unroll
+  for (int a = 0; a < FA_ROWS; ++a) {
+    const int i = ty + 8 * a;
     const float d = piv[i];
     if (!(d > 0.f) || !isfinite(d)) s_bad = 1;
     const float sc = 1.f / sqrtf(fmaxf(d, 1e-30f));
+    float x[4];
 #pragma unroll
     for (int b = 0; b < 4; ++b) {
-      const int c = tx + 32 * b;
-      const float x = xr[a][b] * sc;
-      if (!isfinite(x)) s_bad = 1;
-      mout[i * D + c] = x;
-      Ms[i * FA_LD + c] = x;
+      const int c = c0 + b;
+      x[b] = c < i ? (-z[a][b] * ipc[b]) * sc : (c == i ? sc : 0.f);
+      if (!isfinite(x[b])) s_bad = 1;
+      Ms[i * FA_LD + c] = x[b];
     }
+    *(float4*)(mout + i * D + c0) = make_float4(x[0], x[1], x[2], x[3]);
   }
   __syncthreads();
   // bf16 hi/lo image: 2 K-atoms (channels 0-63, 64-127) x 256 rows x 128 B
