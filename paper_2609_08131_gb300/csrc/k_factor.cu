@@ -67,32 +67,32 @@ __global__ void __launch_bounds__(FA_THREADS, 2) factor_kernel(Dims dm, Ws ws) {
   const int c0 = 4 * tx;
 
   // A = I + sum of partial Grams (chunk order)
-  float z[FA_ROWS][4];
+  float2 z[FA_ROWS][2];  // columns (c0, c0+1) and (c0+2, c0+3) as packed pairs
   {
     const float* gp = ws.gpart + ((int64_t)plane * dm.c_cap) * D * D;
     float* gout = ws.gram + (int64_t)u * D * D;
 #pragma unroll
-    for (int a = 0; a < FA_ROWS; ++a)
-#pragma unroll
-      for (int b = 0; b < 4; ++b) z[a][b] = 0.f;
+    for (int a = 0; a < FA_ROWS; ++a) z[a][0] = z[a][1] = make_float2(0.f, 0.f);
     for (int ch = ch0; ch < ch1; ++ch) {  // 16 independent 16-byte loads in flight per chunk
       // partial layout: (m, n) at ((n / 32) D + m) 32 + n % 32
       const float* src = gp + (int64_t)ch * D * D + (c0 >> 5) * D * 32 + (c0 & 31);
 #pragma unroll
       for (int a = 0; a < FA_ROWS; ++a) {
         const float4 v = *(const float4*)(src + (ty + 8 * a) * 32);
-        z[a][0] += v.x;
-        z[a][1] += v.y;
-        z[a][2] += v.z;
-        z[a][3] += v.w;
+        z[a][0].x += v.x;
+        z[a][0].y += v.y;
+        z[a][1].x += v.z;
+        z[a][1].y += v.w;
       }
     }
 #pragma unroll
     for (int a = 0; a < FA_ROWS; ++a) {
       const int i = ty + 8 * a;
-      *(float4*)(gout + i * D + c0) = make_float4(z[a][0], z[a][1], z[a][2], z[a][3]);
-#pragma unroll
-      for (int b = 0; b < 4; ++b) z[a][b] += (i == c0 + b ? 1.f : 0.f);
+      *(float4*)(gout + i * D + c0) = make_float4(z[a][0].x, z[a][0].y, z[a][1].x, z[a][1].y);
+      z[a][0].x += (i == c0 ? 1.f : 0.f);
+      z[a][0].y += (i == c0 + 1 ? 1.f : 0.f);
+      z[a][1].x += (i == c0 + 2 ? 1.f : 0.f);
+      z[a][1].y += (i == c0 + 3 ? 1.f : 0.f);
     }
   }
 
@@ -106,19 +106,20 @@ __global__ void __launch_bounds__(FA_THREADS, 2) factor_kernel(Dims dm, Ws ws) {
       const int buf = j & 1;
       if (tx == (j >> 2)) {  // owners of column j: rows ty + 8 a, register column j % 4 = jl % 4
 #pragma unroll
-        for (int a = 0; a < FA_ROWS; ++a) colA[buf][ty + 8 * a] = z[a][jl & 3];
+        for (int a = 0; a < FA_ROWS; ++a) {
+          const float2 zp = z[a][(jl & 3) >> 1];
+          colA[buf][ty + 8 * a] = (jl & 1) ? zp.y : zp.x;
+        }
       }
       if (ty == jl) {  // owners of row j (register row jh)
-        float r0 = 0.f, r1 = 0.f, r2 = 0.f, r3 = 0.f;
+        float2 r01 = make_float2(0.f, 0.f), r23 = r01;
 #pragma unroll
         for (int a = 0; a < FA_ROWS; ++a)
           if (a == jh) {
-            r0 = z[a][0];
-            r1 = z[a][1];
-            r2 = z[a][2];
-            r3 = z[a][3];
+            r01 = z[a][0];
+            r23 = z[a][1];
           }
-        *(float4*)&rowY[buf][c0] = make_float4(r0, r1, r2, r3);
+        *(float4*)&rowY[buf][c0] = make_float4(r01.x, r01.y, r23.x, r23.y);
       }
       __syncthreads();
       const float pj = colA[buf][j];
@@ -136,12 +137,8 @@ __global__ void __launch_bounds__(FA_THREADS, 2) factor_kernel(Dims dm, Ws ws) {
         if (ty + 8 * a > j) {  // active rows (uniform over the warp)
           const float m = colA[buf][ty + 8 * a] * inv_p;
           const float2 nm = make_float2(-m, -m);
-          const float2 z01 = __ffma2_rn(nm, r01, make_float2(z[a][0], z[a][1]));
-          const float2 z23 = __ffma2_rn(nm, r23, make_float2(z[a][2], z[a][3]));
-          z[a][0] = z01.x;
-          z[a][1] = z01.y;
-          z[a][2] = z23.x;
-          z[a][3] = z23.y;
+          z[a][0] = __ffma2_rn(nm, r01, z[a][0]);
+          z[a][1] = __ffma2_rn(nm, r23, z[a][1]);
         }
       }
     }
@@ -159,11 +156,12 @@ __global__ void __launch_bounds__(FA_THREADS, 2) factor_kernel(Dims dm, Ws ws) {
     const float d = piv[i];
     if (!(d > 0.f) || !isfinite(d)) s_bad = 1;
     const float sc = 1.f / sqrtf(fmaxf(d, 1e-30f));
+    const float zv[4] = {z[a][0].x, z[a][0].y, z[a][1].x, z[a][1].y};
     float x[4];
 #pragma unroll
     for (int b = 0; b < 4; ++b) {
       const int c = c0 + b;
-      x[b] = c < i ? (-z[a][b] * ipc[b]) * sc : (c == i ? sc : 0.f);
+      x[b] = c < i ? (-zv[b] * ipc[b]) * sc : (c == i ? sc : 0.f);
       if (!isfinite(x[b])) s_bad = 1;
       Ms[i * FA_LD + c] = x[b];
     }
