@@ -46,6 +46,17 @@ switch so the alternatives stay testable):
 * R8  when n <= B every token is kept (kept = n) and the index list is padded
       with -1 up to B.
 * R10 Sigma_noise = I (isotropic noise with sigma^2 absorbed, App. B.1).
+* R13 ``linear_weighting=True`` replaces S_C by the identity, the linear
+      Gaussian surrogate the paper contrasts Jacap with (App. A, end of the
+      discussion of S_C): rho_i = 1, so w_i = kappa_i / d_k.
+* R14 ``full_covariance=True`` uses the full window covariance Lambda_Q (the
+      O(N d^2) variant of App. B.2's complexity analysis) instead of its
+      diagonal: kappa_i = k_i^T Lambda_Q k_i, Lambda_Q = (1/w) sum_j
+      (q_j - mu)(q_j - mu)^T (1/(w-1) with ``cov_unbiased``).
+
+Also here, as a quality reference only (no GPU counterpart):
+``greedy_logdet_select`` picks B tokens one at a time, each maximising the
+increase of the App. B.1 objective log det(I + sum_{i in C} w_i u_i u_i^T).
 """
 
 from __future__ import annotations
@@ -58,12 +69,14 @@ import numpy as np
 
 @dataclass(frozen=True)
 class JacapParams:
-    """Switches for the readings R1-R4 above; defaults are the method's."""
+    """Switches for the readings R1-R4, R13, R14 above; defaults are the method's."""
 
     tau: float = 10.0
     weight_div_dk: bool = True
     ridge: bool = True
     cov_unbiased: bool = False
+    linear_weighting: bool = False
+    full_covariance: bool = False
 
 
 def _f64(x) -> np.ndarray:
@@ -87,6 +100,17 @@ def window_stats(q_win, cov_unbiased: bool = False):
     denom = (w - 1) if cov_unbiased else w
     lam = (dev * dev).sum(axis=0) / denom
     return mu, lam
+
+
+def window_covariance(q_win, cov_unbiased: bool = False):
+    """Full Lambda_Q of one query head's window (reading R14): the covariance
+    of the w window queries, (w, d) in, (d, d) out."""
+    q = _f64(q_win)
+    w = q.shape[0]
+    if w < 1 or (cov_unbiased and w < 2):
+        raise ValueError("window too short for the requested estimator")
+    dev = q - q.sum(axis=0) / w
+    return (dev.T @ dev) / ((w - 1) if cov_unbiased else w)
 
 
 # --------------------------------------------------------------------------
@@ -120,15 +144,28 @@ def response_variance(K, lam):
     return (K * K) @ _f64(lam)
 
 
+def response_variance_full(K, Lam):
+    """kappa_i = k_i^T Lambda_Q k_i for a full Lambda_Q (App. B.2, reading R14)."""
+    K = _f64(K)
+    return np.einsum("nc,cd,nd->n", K, _f64(Lam), K)
+
+
 # --------------------------------------------------------------------------
 # Step 4: Jacobian importance weight (Eq. 8), GQA sum (reading R5)
 # --------------------------------------------------------------------------
 def head_weight(K, mu, lam, params: JacapParams = JacapParams()):
-    """w_i = rho_i^2 kappa_i / d_k for one query head (Eq. 8)."""
+    """w_i = rho_i^2 kappa_i / d_k for one query head (Eq. 8).
+
+    ``lam`` is the diagonal of Lambda_Q, or the full (d, d) matrix when
+    ``params.full_covariance`` (R14). With ``params.linear_weighting`` S_C is
+    the identity and rho_i = 1 (R13)."""
     K = _f64(K)
     d = K.shape[1]
-    rho = sensitivity(pool_attention(K, mu, params.tau))
-    kappa = response_variance(K, lam)
+    if params.linear_weighting:
+        rho = np.ones(K.shape[0])
+    else:
+        rho = sensitivity(pool_attention(K, mu, params.tau))
+    kappa = response_variance_full(K, lam) if params.full_covariance else response_variance(K, lam)
     w = rho * rho * kappa
     if params.weight_div_dk:
         w = w / d
@@ -146,6 +183,8 @@ def unit_weights(K, q_group, params: JacapParams = JacapParams()):
     w = np.zeros(K.shape[0])
     for h in range(q_group.shape[0]):
         mu, lam = window_stats(q_group[h], params.cov_unbiased)
+        if params.full_covariance:
+            lam = window_covariance(q_group[h], params.cov_unbiased)
         w = w + head_weight(K, mu, lam, params)
     return w
 
@@ -205,6 +244,37 @@ def compact(K, V, idx, kept: int):
 
 
 # --------------------------------------------------------------------------
+# Quality reference: greedy log-determinant selection (App. B.1 objective)
+# --------------------------------------------------------------------------
+def greedy_logdet_select(U, w, budget: int):
+    """Greedy maximiser of log det(I + sum_{i in C} w_i u_i u_i^T) over |C| = B.
+
+    Each round adds the token with the largest gain log(1 + w_i u_i^T A^{-1} u_i)
+    (matrix determinant lemma, App. B.1), A being I plus the chosen terms so far;
+    ties go to the lower index. Returns the chosen indices in pick order and the
+    objective after each pick. Plain float64; a reference for selection quality,
+    not part of the GPU pass.
+    """
+    U = _f64(U)
+    w = _f64(w)
+    n, d = U.shape
+    A = np.eye(d)
+    chosen, objective = [], []
+    free = np.ones(n, dtype=bool)
+    for _ in range(min(budget, n)):
+        Ainv = np.linalg.inv(A)
+        gain = np.full(n, -np.inf)
+        q = np.einsum("nc,cd,nd->n", U, Ainv, U)
+        gain[free] = np.log1p(w[free] * q[free])
+        i = int(np.argmax(gain))  # first maximum: the lower index on ties
+        chosen.append(i)
+        free[i] = False
+        A = A + w[i] * np.outer(U[i], U[i])
+        objective.append(float(np.linalg.slogdet(A)[1]))
+    return np.array(chosen, dtype=np.int64), np.array(objective)
+
+
+# --------------------------------------------------------------------------
 # Whole unit and whole cache
 # --------------------------------------------------------------------------
 def oracle_unit(q_group, K, V, budget: int, params: JacapParams = JacapParams()):
@@ -217,7 +287,7 @@ def oracle_unit(q_group, K, V, budget: int, params: JacapParams = JacapParams())
     for h in range(G):
         mu, lam = window_stats(q_group[h], params.cov_unbiased)
         mus.append(mu)
-        lams.append(lam)
+        lams.append(lam)  # the diagonal of Lambda_Q, also under R14
         alphas.append(pool_attention(K64, mu, params.tau))
     w = unit_weights(K64, q_group, params)
     scores = jacap_scores(V64, w, params.ridge)
