@@ -95,7 +95,7 @@ typedef struct {
 } jacap_layout;
 
 /*
- * Method switches. Defaults {10.0f, 1, 1, 0}:
+ * Method switches. Defaults {10.0f, 1, 1, 0, 0, 0}:
  *  tau            temperature of the pool softmax (Sec. 3.4; Sec. 4.4 reports
  *                 the best accuracy near 10). Must be finite and > 0.
  *  weight_div_dk  1: keep the 1/d_k factor of Eq. 8; 0: drop it (Alg. 1 step 2
@@ -104,12 +104,21 @@ typedef struct {
  *                 variant and returns JACAP_ERR_UNSUPPORTED.)
  *  cov_unbiased   0: lambda = population variance over the window (divide by
  *                 w); 1: divide by w - 1 (needs window >= 2).
+ *  linear_weighting  0: the softmax-aware weight of Eq. 8; 1: the linear
+ *                 surrogate S_C = I that App. A contrasts Jacap with, i.e.
+ *                 rho_i = 1 and w_i = (1/d) sum_h kappa_h,i (a CapKV-style
+ *                 weight; the logits and softmax statistics are then unused).
+ *  full_covariance  must be 0 (the diagonal Lambda_Q of App. B.2);
+ *                 1 returns JACAP_ERR_UNSUPPORTED.
+ * Callers that zero-initialise the two trailing fields get the method.
  */
 typedef struct {
   float tau;
   int32_t weight_div_dk;
   int32_t ridge;
   int32_t cov_unbiased;
+  int32_t linear_weighting;
+  int32_t full_covariance;
 } jacap_params;
 
 /* Bytes of device workspace jacap_score/jacap_select need for `layout`

@@ -53,17 +53,19 @@ class jacap_layout(ctypes.Structure):
 
 
 class jacap_params(ctypes.Structure):
-    """Mirror of ``jacap_params``; defaults are the method's (tau = 10)."""
+    """Mirror of ``jacap_params``; defaults are the method's (tau = 10, Eq. 8 weights)."""
 
     _fields_ = [
         ("tau", ctypes.c_float),
         ("weight_div_dk", ctypes.c_int32),
         ("ridge", ctypes.c_int32),
         ("cov_unbiased", ctypes.c_int32),
+        ("linear_weighting", ctypes.c_int32),
+        ("full_covariance", ctypes.c_int32),
     ]
 
-    def __init__(self, tau=10.0, weight_div_dk=1, ridge=1, cov_unbiased=0):
-        super().__init__(tau, weight_div_dk, ridge, cov_unbiased)
+    def __init__(self, tau=10.0, weight_div_dk=1, ridge=1, cov_unbiased=0, linear_weighting=0, full_covariance=0):
+        super().__init__(tau, weight_div_dk, ridge, cov_unbiased, linear_weighting, full_covariance)
 
 
 class jacap_ws_offsets(ctypes.Structure):

@@ -85,6 +85,7 @@ void make_dims(const jacap_layout* L, const jacap_params* P, Dims& dm) {
     dm.inv_scale = (float)(1.0 / ((double)P->tau * sqrt((double)D)));
     dm.wdiv = P->weight_div_dk ? 1.0f / (float)D : 1.0f;
     dm.cov_unbiased = P->cov_unbiased;
+    dm.linear = P->linear_weighting;
   }
 }
 
@@ -228,7 +229,9 @@ jacap_status jacap_score_timed(const jacap_layout* layout, const jacap_params* p
   if (params->weight_div_dk != 0 && params->weight_div_dk != 1) return JACAP_ERR_INVALID_ARG;
   if (params->cov_unbiased != 0 && params->cov_unbiased != 1) return JACAP_ERR_INVALID_ARG;
   if (params->cov_unbiased && layout->window < 2) return JACAP_ERR_INVALID_ARG;
-  if (params->ridge != 1) return JACAP_ERR_UNSUPPORTED;
+  if (params->linear_weighting != 0 && params->linear_weighting != 1) return JACAP_ERR_INVALID_ARG;
+  if (params->full_covariance != 0 && params->full_covariance != 1) return JACAP_ERR_INVALID_ARG;
+  if (params->ridge != 1 || params->full_covariance != 0) return JACAP_ERR_UNSUPPORTED;
   if (!aligned16(q_win) || !aligned16(k) || !aligned16(v) || ((uintptr_t)scores & 3u) != 0)
     return JACAP_ERR_INVALID_ARG;
   Dims dm;

@@ -38,6 +38,7 @@ struct Dims {
   float inv_scale;    // 1 / (tau sqrt(d))
   float wdiv;         // 1/d (Eq. 8) or 1 (weight_div_dk = 0)
   int cov_unbiased;
+  int linear;         // 1: S_C = I, rho = 1 (linear surrogate weight)
 };
 
 // Workspace map (device pointers into the caller's workspace).

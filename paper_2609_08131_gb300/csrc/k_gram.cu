@@ -43,7 +43,8 @@ __device__ __forceinline__ void unit_softmax_stats_warp(const Dims& dm, const Ws
 // ---------------------------------------------------------------- weights --
 // w_i of Eq. 8 summed over the G query heads of the group (GQA heads add their
 // weights): w_i = wdiv * sum_h [alpha_bar (1 - alpha_bar)]^2 kappa_h,i with
-// alpha_bar = exp(l_h,i - M_h) / Z_h. One streaming pass over the K pass's
+// alpha_bar = exp(l_h,i - M_h) / Z_h; with the linear surrogate (S_C = I)
+// rho = 1 and w_i = wdiv * sum_h kappa_h,i. One streaming pass over the K pass's
 // logits/kappa rows; writes w (float32, for the score pass) and w as a bf16
 // pair hi + lo (for the tensor-core Gram, whose scaling is done in bf16).
 constexpr int WT_THREADS = 256;
@@ -88,11 +89,16 @@ __global__ void __launch_bounds__(WT_THREADS) weight_kernel(Dims dm, Ws ws, cons
         lk[1] = q2.y;
       }
       float wt = 0.f;
+      if (dm.linear) {  // S_C = I: rho = 1
 #pragma unroll
-      for (int h = 0; h < G; ++h) {
-        const float a = expf(lk[h] - u[h]) * u[G + h];  // alpha_bar
-        const float rho = a * (1.f - a);                 // diagonal of the softmax Jacobian
-        wt = fmaf(rho * rho, lk[G + h], wt);             // rho^2 kappa
+        for (int h = 0; h < G; ++h) wt += lk[G + h];
+      } else {
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+          const float a = expf(lk[h] - u[h]) * u[G + h];  // alpha_bar
+          const float rho = a * (1.f - a);                 // diagonal of the softmax Jacobian
+          wt = fmaf(rho * rho, lk[G + h], wt);             // rho^2 kappa
+        }
       }
       wt *= dm.wdiv;
       bad |= !isfinite(wt);

@@ -33,7 +33,8 @@ def make_cache(t, wl):
 def check_unit(ev, t, wl, params, s, layer, g, check_w=True):
     q, K, V = unit_arrays(t, wl.num_q_heads, s, layer, g)
     ora = oracle_unit(q, K, V, ev.budget, JacapParams(tau=params.tau, weight_div_dk=bool(params.weight_div_dk),
-                                                       cov_unbiased=bool(params.cov_unbiased)))
+                                                       cov_unbiased=bool(params.cov_unbiased),
+                                                       linear_weighting=bool(params.linear_weighting)))
     cu = t.cu_seqlens.cpu().tolist()
     a, b = cu[s], cu[s + 1]
     n = b - a
@@ -65,6 +66,10 @@ SMALL = {
                                  outlier_channels=4, outlier_scale=8.0), jacap_params()),
     "f32_gqa4_peaky": (Workload("t", 2, 8, 2, (600, 130), 8, 50, dtype="f32", seed=17), jacap_params(tau=0.5)),
     "bf16_budget_exceeds_all": (Workload("t", 1, 4, 2, (100, 257), 8, 300, seed=18), jacap_params()),
+    "bf16_gqa4_linear_weighting": (Workload("t", 2, 8, 2, (1500, 700), 16, 128, seed=19),
+                                   jacap_params(linear_weighting=1)),
+    "f32_mha_linear_weighting": (Workload("t", 1, 4, 4, (900,), 8, 64, dtype="f32", seed=20),
+                                 jacap_params(linear_weighting=1, cov_unbiased=1)),
 }
 
 
