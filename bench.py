@@ -42,6 +42,8 @@ def parse():
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--config", type=int, default=2)
     p.add_argument("--budget", type=int, default=None)
+    p.add_argument("--weighting", default="jacobian", choices=["jacobian", "linear"],
+                   help="Eq. 8 softmax-aware weights (the method) or the linear S = I surrogate")
     p.add_argument("--e2e-steps", type=int, default=10)
     p.add_argument("--cpu-seconds", type=float, default=15.0)
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -148,7 +150,7 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows), "power_w_max": max(pw) if pw else None}
 
 
-def workload_config(wl, budget, gpus):
+def workload_config(wl, budget, gpus, weighting="jacobian"):
     return {
         "workload": wl.name,
         "layers": wl.num_layers,
@@ -159,6 +161,7 @@ def workload_config(wl, budget, gpus):
         "window": wl.window,
         "budget": budget,
         "tau": 10.0,
+        "weighting": weighting,
         "cache_dtype": wl.dtype,
         "l2": "inputs larger than L2: each step streams the whole cache (K and V alone are "
               f"{2 * wl.num_layers * wl.num_kv_heads * wl.total_tokens * wl.head_dim * (2 if wl.dtype == 'bf16' else 4) / 1e9:.2f} GB)",
@@ -167,7 +170,7 @@ def workload_config(wl, budget, gpus):
 
 
 # ------------------------------------------------------------------ oracle --
-def oracle_sample(wl, budget, seconds, device, tensors=None):
+def oracle_sample(wl, budget, seconds, device, tensors=None, weighting="jacobian"):
     """Time the float64 oracle on whole units of the workload for ~`seconds`.
 
     Returns (tokens_layers_per_s, sample_description, wall_s)."""
@@ -187,7 +190,7 @@ def oracle_sample(wl, budget, seconds, device, tensors=None):
             K = k.to(dt).double().numpy()
             V = v.to(dt).double().numpy()
         t0 = time.perf_counter()
-        oracle_unit(q, K, V, budget, JacapParams())
+        oracle_unit(q, K, V, budget, JacapParams(linear_weighting=weighting == "linear"))
         t_total += time.perf_counter() - t0
         done += 1
         tok += n
@@ -214,16 +217,17 @@ def run_reference(args):
     dt = wl.torch_dtype
     K64, V64, Q64 = k.to(dt).double().numpy(), v.to(dt).double().numpy(), q.to(dt).double().numpy()
     t0 = time.perf_counter()
-    oracle_unit(Q64, K64[:2048], V64[:2048], budget, JacapParams())
+    P = JacapParams(linear_weighting=args.weighting == "linear")
+    oracle_unit(Q64, K64[:2048], V64[:2048], budget, P)
     per_tok = (time.perf_counter() - t0) / 2048
     target = 150.0 / max(1, args.steps + args.warmup)
     m = int(max(256, min(n_full, target / per_tok)))
     for _ in range(args.warmup):
-        oracle_unit(Q64, K64[:m], V64[:m], budget, JacapParams())
+        oracle_unit(Q64, K64[:m], V64[:m], budget, P)
     times = []
     for _ in range(args.steps):
         t0 = time.perf_counter()
-        oracle_unit(Q64, K64[:m], V64[:m], budget, JacapParams())
+        oracle_unit(Q64, K64[:m], V64[:m], budget, P)
         times.append(time.perf_counter() - t0)
     avg = sum(times) / len(times)
     value = m / wl.num_kv_heads / avg
@@ -243,7 +247,7 @@ def run_reference(args):
         "vs_baseline": None,
         "dtype": "f64",
         "data": "synthetic",
-        "config": workload_config(wl, budget, args.gpus),
+        "config": workload_config(wl, budget, args.gpus, args.weighting),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
@@ -279,7 +283,9 @@ def run_ours(args):
         wl = replace(wl, num_layers=args.layers, name=wl.name + f", {args.layers} layers")
     t = generate(wl, dev)
     cache = Cache(t.q_win, t.k, t.v, t.cu_seqlens, t.seqlens, wl.num_q_heads)
-    ev = Evictor(cache, budget)
+    from paper_2609_08131_gb300 import jacap_params
+
+    ev = Evictor(cache, budget, jacap_params(linear_weighting=1 if args.weighting == "linear" else 0))
     stream = torch.cuda.current_stream(dev)
 
     def barrier():
@@ -350,7 +356,7 @@ def run_ours(args):
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
-        v_cpu, desc, wall = oracle_sample(wl, budget, args.cpu_seconds, dev, tensors=t)
+        v_cpu, desc, wall = oracle_sample(wl, budget, args.cpu_seconds, dev, tensors=t, weighting=args.weighting)
         cpu = {"value": v_cpu, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
                "sample": desc + f"; {wall:.1f} s of CPU work; numpy BLAS threads left at their default"}
 
@@ -372,7 +378,7 @@ def run_ours(args):
             "vs_baseline": None,
             "dtype": "bf16" if wl.dtype == "bf16" else "f32",
             "data": "synthetic",
-            "config": workload_config(wl, budget, world),
+            "config": workload_config(wl, budget, world, args.weighting),
             "roofline": {
                 "bound": "hbm",
                 "kernel": dom,

@@ -54,6 +54,12 @@ switch so the alternatives stay testable):
       diagonal: kappa_i = k_i^T Lambda_Q k_i, Lambda_Q = (1/w) sum_j
       (q_j - mu)(q_j - mu)^T (1/(w-1) with ``cov_unbiased``).
 
+* R15 true output directions (Sec. 3.1: u_i = W_O v_i; Sec. 3.4 uses v_i as a
+      proxy): ``oracle_unit(..., out_proj=W)`` takes one output map W
+      (d_o x d) per unit -- for a KV head shared by G query heads the caller
+      chooses how the heads' W_O slices combine (e.g. stacked) -- and uses
+      u_i = W v_i in A = I + sum_j w_j u_j u_j^T (d_o x d_o) and in the score.
+
 Also here, as a quality reference only (no GPU counterpart):
 ``greedy_logdet_select`` picks B tokens one at a time, each maximising the
 increase of the App. B.1 objective log det(I + sum_{i in C} w_i u_i u_i^T).
@@ -277,10 +283,14 @@ def greedy_logdet_select(U, w, budget: int):
 # --------------------------------------------------------------------------
 # Whole unit and whole cache
 # --------------------------------------------------------------------------
-def oracle_unit(q_group, K, V, budget: int, params: JacapParams = JacapParams()):
-    """Algorithm 1 for one unit; returns every intermediate the GPU exposes."""
+def oracle_unit(q_group, K, V, budget: int, params: JacapParams = JacapParams(), out_proj=None):
+    """Algorithm 1 for one unit; returns every intermediate the GPU exposes.
+
+    ``out_proj`` (d_o x d) gives the output directions u_i = W v_i (R15); by
+    default u_i = v_i. "A" is then d_o x d_o."""
     K64 = _f64(K)
     V64 = _f64(V)
+    U64 = V64 if out_proj is None else V64 @ _f64(out_proj).T
     q_group = _f64(q_group)
     G = q_group.shape[0]
     mus, lams, alphas = [], [], []
@@ -290,7 +300,7 @@ def oracle_unit(q_group, K, V, budget: int, params: JacapParams = JacapParams())
         lams.append(lam)  # the diagonal of Lambda_Q, also under R14
         alphas.append(pool_attention(K64, mu, params.tau))
     w = unit_weights(K64, q_group, params)
-    scores = jacap_scores(V64, w, params.ridge)
+    scores = jacap_scores(U64, w, params.ridge)
     idx, kept = select_topb(scores, budget)
     k_out, v_out = compact(K, V, idx, kept)
     return {
@@ -298,7 +308,7 @@ def oracle_unit(q_group, K, V, budget: int, params: JacapParams = JacapParams())
         "lam": np.stack(lams),
         "alpha": np.stack(alphas),
         "w": w,
-        "A": capacity_matrix(V64, w, params.ridge),
+        "A": capacity_matrix(U64, w, params.ridge),
         "scores": scores,
         "idx": idx,
         "kept": kept,

@@ -188,3 +188,48 @@ def test_full_covariance_unit_weight_composes_rho_and_logit_variance():
     w = J.unit_weights(K, q, J.JacapParams(tau=tau, full_covariance=True))
     np.testing.assert_allclose(w, ref, rtol=1e-11)
     assert FULL.full_covariance and not FULL.linear_weighting
+
+
+# -------------------------------------------------- R15 output directions ----
+def _unit(seed, n=60, d=16, G=2, wq=6):
+    r = rng(seed)
+    K = r.normal(size=(n, d)) * 2
+    V = r.normal(size=(n, d)) * r.lognormal(size=d)
+    q = r.normal(size=(G, wq, d))
+    return K, V, q
+
+
+def test_output_directions_reduce_to_a_d_by_d_problem():
+    # push-through identity: with W = Q R (Q orthonormal columns),
+    # u^T (I + sum w u u^T)^{-1} u = (R v)^T (I + R G R^T)^{-1} (R v), G = sum w v v^T,
+    # i.e. the d_o x d_o problem equals a d x d one -- checked against the
+    # oracle's explicit d_o-dimensional computation
+    K, V, q = _unit(13)
+    d, do = V.shape[1], 48
+    W = rng(14).normal(size=(do, d))
+    ora = J.oracle_unit(q, K, V, 8, out_proj=W)
+    w = J.unit_weights(K, q)
+    _, R = np.linalg.qr(W)
+    G = (V * w[:, None]).T @ V
+    M = np.eye(d) + R @ G @ R.T
+    Lm = np.linalg.cholesky(M)
+    Y = np.linalg.solve(Lm, R @ V.T)
+    np.testing.assert_allclose(ora["scores"], w * (Y * Y).sum(axis=0), rtol=1e-9)
+    assert ora["A"].shape == (do, do)
+
+
+def test_orthonormal_output_map_leaves_scores_unchanged():
+    # W with orthonormal columns (W^T W = I) is a rotation into a larger space:
+    # the scores equal those of the u = v proxy
+    K, V, q = _unit(15)
+    Q, _ = np.linalg.qr(rng(16).normal(size=(40, V.shape[1])))
+    np.testing.assert_allclose(J.oracle_unit(q, K, V, 8, out_proj=Q)["scores"],
+                               J.oracle_unit(q, K, V, 8)["scores"], rtol=1e-10)
+
+
+def test_scaled_identity_output_map_equals_scaled_values():
+    # W = c I: u = c v, so the scores equal those computed on c V
+    K, V, q = _unit(17)
+    c = 2.5
+    np.testing.assert_allclose(J.oracle_unit(q, K, V, 8, out_proj=c * np.eye(V.shape[1]))["scores"],
+                               J.oracle_unit(q, K, c * V, 8)["scores"], rtol=1e-11)
