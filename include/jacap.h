@@ -158,6 +158,27 @@ jacap_status jacap_score_timed(const jacap_layout* layout, const jacap_params* p
                                void* const* events, int32_t num_events);
 
 /*
+ * jacap_score with the true output directions u_i = W v_i of Sec. 3.1 (the
+ * other entry points use the proxy u_i = v_i of Sec. 3.4), plus optional
+ * timing hooks as in jacap_score_timed.
+ *  out_factor  device float32 [num_layers][num_kv_heads][128][128], row-major,
+ *              16-byte aligned, or NULL (then identical to jacap_score_timed):
+ *              per plane a matrix F with F^T F = W^T W for the plane's output
+ *              map W (d_o x 128; e.g. the R of a QR factorisation of W; how the
+ *              W_O slices of the G query heads sharing a KV head form W is the
+ *              caller's choice). The capacity matrix I + sum w u u^T (d_o x d_o,
+ *              Eq. 9) reduces exactly to M = I + F G F^T, and
+ *              r_i = w_i ||L_M^{-1} F v_i||^2 (Eq. 10).
+ * Intermediates (jacap_workspace_offsets): gram is still G = sum w v v^T;
+ * chol_inv holds T = L_M^{-1} F (a full matrix).
+ */
+jacap_status jacap_score_out(const jacap_layout* layout, const jacap_params* params,
+                             const void* q_win, const void* k, const void* v,
+                             const float* out_factor, float* scores,
+                             void* ws, size_t ws_bytes, void* stream,
+                             void* const* events, int32_t num_events);
+
+/*
  * jacap_score for callers that cannot allocate device memory (the paper has no
  * counterpart; this is a deployment convenience). The workspace is a fixed
  * library-owned array of JACAP_STATIC_SCRATCH_BYTES in static device memory,

@@ -85,6 +85,8 @@ _SIGS = {
                                    ctypes.c_size_t, _P]),
     "jacap_score_timed": (ctypes.c_int, [ctypes.POINTER(jacap_layout), ctypes.POINTER(jacap_params), _P, _P, _P, _P,
                                          _P, ctypes.c_size_t, _P, ctypes.POINTER(ctypes.c_void_p), ctypes.c_int32]),
+    "jacap_score_out": (ctypes.c_int, [ctypes.POINTER(jacap_layout), ctypes.POINTER(jacap_params), _P, _P, _P, _P,
+                                       _P, _P, ctypes.c_size_t, _P, ctypes.POINTER(ctypes.c_void_p), ctypes.c_int32]),
     "jacap_score_static": (ctypes.c_int, [ctypes.POINTER(jacap_layout), ctypes.POINTER(jacap_params), _P, _P, _P,
                                           _P, _P, ctypes.POINTER(ctypes.c_void_p)]),
     "jacap_select": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, ctypes.c_int32, _P, _P, _P, ctypes.c_size_t,
@@ -126,6 +128,13 @@ def jacap_score_timed(layout, params, q_win, k, v, scores, ws, ws_bytes, stream,
     arr = (ctypes.c_void_p * max(1, len(events)))(*[ctypes.c_void_p(e) for e in events])
     return lib().jacap_score_timed(ctypes.byref(layout), ctypes.byref(params), q_win, k, v, scores, ws, ws_bytes,
                                    stream, arr, len(events))
+
+
+def jacap_score_out(layout, params, q_win, k, v, out_factor, scores, ws, ws_bytes, stream, events=()) -> int:
+    """``out_factor``: device pointer to the per-plane 128 x 128 factors F, or None."""
+    arr = (ctypes.c_void_p * max(1, len(events)))(*[ctypes.c_void_p(e) for e in events])
+    return lib().jacap_score_out(ctypes.byref(layout), ctypes.byref(params), q_win, k, v, out_factor, scores, ws,
+                                 ws_bytes, stream, arr, len(events))
 
 
 JACAP_STATIC_SCRATCH_BYTES = 64 << 20

@@ -91,6 +91,7 @@ EXPORTS = [
     "jacap_score",
     "jacap_score_timed",
     "jacap_score_static",
+    "jacap_score_out",
     "jacap_select",
     "jacap_compact",
     "jacap_device_status",

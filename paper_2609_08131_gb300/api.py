@@ -21,6 +21,7 @@ from . import (
     jacap_params,
     jacap_score,
     jacap_score_timed,
+    jacap_score_out,
     jacap_select,
     jacap_status_string,
     jacap_workspace_offsets,
@@ -95,10 +96,19 @@ class Evictor:
     """Owns the workspace and output buffers for repeated passes over caches
     of one shape; ``run()`` enqueues score, select and compact."""
 
-    def __init__(self, cache: Cache, budget: int, params: jacap_params | None = None):
+    def __init__(self, cache: Cache, budget: int, params: jacap_params | None = None, out_factor=None):
+        """``out_factor``: optional float32 [L][Hkv][128][128] device tensor of
+        factors F with F^T F = W^T W for the output maps W (u_i = W v_i);
+        None uses the proxy u_i = v_i."""
         self.cache = cache
         self.budget = int(budget)
         self.params = params if params is not None else jacap_params()
+        if out_factor is not None:
+            L, Hkv = cache.k.shape[0], cache.k.shape[1]
+            if (out_factor.dtype != torch.float32 or tuple(out_factor.shape) != (L, Hkv, 128, 128)
+                    or not out_factor.is_contiguous() or out_factor.device != cache.k.device):
+                raise ValueError("out_factor must be a contiguous float32 [L][Hkv][128][128] tensor on the cache's device")
+        self.out_factor = out_factor
         self.lay = cache.layout()
         dev = cache.k.device
         nbytes = jacap_workspace_size(self.lay, self.budget)
@@ -117,7 +127,12 @@ class Evictor:
         """jacap_score; with ``events`` (JACAP_SCORE_KERNELS + 1 torch.cuda.Event
         objects) the timed variant records them around the kernels of the pass."""
         c = self.cache
-        if events is None:
+        if self.out_factor is not None:
+            handles = [e.cuda_event for e in events] if events is not None else []
+            _check(jacap_score_out(self.lay, self.params, _ptr(c.q_win), _ptr(c.k), _ptr(c.v), _ptr(self.out_factor),
+                                   _ptr(self.scores), _ptr(self.ws), self.ws.numel(), _stream(stream), handles),
+                   "jacap_score_out")
+        elif events is None:
             _check(jacap_score(self.lay, self.params, _ptr(c.q_win), _ptr(c.k), _ptr(c.v), _ptr(self.scores),
                                _ptr(self.ws), self.ws.numel(), _stream(stream)), "jacap_score")
         else:

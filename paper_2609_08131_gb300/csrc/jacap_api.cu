@@ -220,6 +220,12 @@ jacap_status jacap_score(const jacap_layout* layout, const jacap_params* params,
 jacap_status jacap_score_timed(const jacap_layout* layout, const jacap_params* params, const void* q_win,
                                const void* k, const void* v, float* scores, void* ws, size_t ws_bytes,
                                void* stream, void* const* events, int32_t num_events) {
+  return jacap_score_out(layout, params, q_win, k, v, nullptr, scores, ws, ws_bytes, stream, events, num_events);
+}
+
+jacap_status jacap_score_out(const jacap_layout* layout, const jacap_params* params, const void* q_win,
+                             const void* k, const void* v, const float* out_factor, float* scores, void* ws,
+                             size_t ws_bytes, void* stream, void* const* events, int32_t num_events) {
   if (num_events != 0 && (num_events != JACAP_SCORE_KERNELS + 1 || events == nullptr)) return JACAP_ERR_INVALID_ARG;
   jacap_status st = check_layout(layout);
   if (st != JACAP_OK) return st;
@@ -232,10 +238,12 @@ jacap_status jacap_score_timed(const jacap_layout* layout, const jacap_params* p
   if (params->linear_weighting != 0 && params->linear_weighting != 1) return JACAP_ERR_INVALID_ARG;
   if (params->full_covariance != 0 && params->full_covariance != 1) return JACAP_ERR_INVALID_ARG;
   if (params->ridge != 1 || params->full_covariance != 0) return JACAP_ERR_UNSUPPORTED;
-  if (!aligned16(q_win) || !aligned16(k) || !aligned16(v) || ((uintptr_t)scores & 3u) != 0)
+  if (!aligned16(q_win) || !aligned16(k) || !aligned16(v) || ((uintptr_t)scores & 3u) != 0 ||
+      (out_factor != nullptr && !aligned16(out_factor)))
     return JACAP_ERR_INVALID_ARG;
   Dims dm;
   make_dims(layout, params, dm);
+  dm.dense_minv = out_factor != nullptr ? 1 : 0;
   const Carve c = carve(dm);
   if (((uintptr_t)ws & 255u) != 0 || ws_bytes < c.total) return JACAP_ERR_WORKSPACE;
   int sms = 0;
@@ -264,7 +272,7 @@ jacap_status jacap_score_timed(const jacap_layout* layout, const jacap_params* p
   if ((st = hook(4)) != JACAP_OK ||
       (st = map_cuda(launch_gram(vmap, dm, w, dt, v, cu, persistent_grid(items, sms, bf ? 1 : 4), s))) != JACAP_OK)
     return st;
-  if ((st = hook(5)) != JACAP_OK || (st = map_cuda(launch_factor(dm, w, s))) != JACAP_OK) return st;
+  if ((st = hook(5)) != JACAP_OK || (st = map_cuda(launch_factor(dm, w, out_factor, s))) != JACAP_OK) return st;
   if ((st = hook(6)) != JACAP_OK ||
       (st = map_cuda(launch_score(vmap, dm, w, dt, v, cu, scores, persistent_grid(items, sms, bf ? 1 : 2), s))) !=
           JACAP_OK)

@@ -39,6 +39,7 @@ struct Dims {
   float wdiv;         // 1/d (Eq. 8) or 1 (weight_div_dk = 0)
   int cov_unbiased;
   int linear;         // 1: S_C = I, rho = 1 (linear surrogate weight)
+  int dense_minv;     // 1: the score matrix is a full 128 x 128 (output directions), not triangular
 };
 
 // Workspace map (device pointers into the caller's workspace).

@@ -16,7 +16,7 @@ cudaError_t launch_kpass_bf16(const CUtensorMap& kmap, const Dims& dm, const Ws&
 cudaError_t launch_weights(const Dims& dm, const Ws& ws, const int32_t* cu, int grid, cudaStream_t st);
 cudaError_t launch_gram(const CUtensorMap& vmap, const Dims& dm, const Ws& ws, int dtype, const void* v,
                         const int32_t* cu, int grid, cudaStream_t st);
-cudaError_t launch_factor(const Dims& dm, const Ws& ws, cudaStream_t st);
+cudaError_t launch_factor(const Dims& dm, const Ws& ws, const float* out_factor, cudaStream_t st);
 cudaError_t launch_score(const CUtensorMap& vmap, const Dims& dm, const Ws& ws, int dtype, const void* v,
                          const int32_t* cu, float* scores, int grid, cudaStream_t st);
 cudaError_t launch_select(const Dims& dm, const Ws& ws, const int32_t* cu, const float* scores, int budget,

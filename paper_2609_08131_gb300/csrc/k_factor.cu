@@ -24,6 +24,13 @@
 // The multipliers use 1/p_j from the approximate hardware reciprocal refined by
 // one Newton-Raphson step (x <- x (2 - p x)), which is accurate to about one ulp.
 //
+// With output directions u = W v (Sec. 3.1) the capacity matrix I + sum w u u^T
+// lives in the output space; with a 128 x 128 factor F of W^T W (F^T F = W^T W)
+// it reduces exactly to M = I + F G F^T, and u^T A^{-1} u = ||L_M^{-1} F v||^2.
+// That variant forms F G F^T from shared-memory copies of G and F (three
+// SIMT float32 products of 128 x 128 matrices), factors M as below and writes
+// T = L_M^{-1} F in place of L^{-1}.
+//
 // L^{-1} is written twice: as float32 (used by the float32 score pass and
 // exposed for tests) and as a bf16 hi/lo pair laid out exactly as the
 // shared-memory B operand of the tensor-core score pass (K-major, 128-byte
@@ -45,10 +52,15 @@ __device__ __forceinline__ float recip_nr(float p) {
   return x * fmaf(-p, x, 2.f);
 }
 constexpr int FA_LD = D + 1;
-constexpr size_t factor_smem_bytes() { return (size_t)D * FA_LD * sizeof(float); }
+// PROJ: two padded 128 x 128 float32 matrices (R0: G, then F G, then L^{-1},
+// then the image staging; R1: F); otherwise the staging matrix only.
+template <bool PROJ>
+constexpr size_t factor_smem_bytes() { return (size_t)(PROJ ? 2 : 1) * D * FA_LD * sizeof(float); }
 
-__global__ void __launch_bounds__(FA_THREADS, 2) factor_kernel(Dims dm, Ws ws) {
-  extern __shared__ float Ms[];  // [D][FA_LD]: L^{-1} staged for the bf16 image
+template <bool PROJ>
+__global__ void __launch_bounds__(FA_THREADS, PROJ ? 1 : 2)
+    factor_kernel(Dims dm, Ws ws, const float* __restrict__ out_factor) {
+  extern __shared__ float Ms[];  // [D][FA_LD]: L^{-1} staged for the bf16 image (PROJ: R0, then R1)
   __shared__ __align__(16) float colA[2][D];
   __shared__ __align__(16) float rowY[2][D];
   __shared__ float piv[D];
@@ -89,6 +101,90 @@ __global__ void __launch_bounds__(FA_THREADS, 2) factor_kernel(Dims dm, Ws ws) {
     for (int a = 0; a < FA_ROWS; ++a) {
       const int i = ty + 8 * a;
       *(float4*)(gout + i * D + c0) = make_float4(z[a][0].x, z[a][0].y, z[a][1].x, z[a][1].y);
+    }
+  }
+  if constexpr (PROJ) {
+    // M = F G F^T: G and F to shared memory (stride FA_LD), then two products
+    // with thread (ty, tx) computing rows ty + 8 a, columns tx + 32 b
+    float* R0 = Ms;
+    float* R1 = Ms + D * FA_LD;
+    const float* F = out_factor + (int64_t)plane * D * D;
+#pragma unroll
+    for (int a = 0; a < FA_ROWS; ++a) {
+      const int i = ty + 8 * a;
+      R0[i * FA_LD + c0] = z[a][0].x;
+      R0[i * FA_LD + c0 + 1] = z[a][0].y;
+      R0[i * FA_LD + c0 + 2] = z[a][1].x;
+      R0[i * FA_LD + c0 + 3] = z[a][1].y;
+    }
+    for (int e = tid; e < D * D / 4; e += FA_THREADS) {
+      const float4 f = ((const float4*)F)[e];
+      const int r = e / (D / 4), c = (e % (D / 4)) * 4;
+      R1[r * FA_LD + c] = f.x;
+      R1[r * FA_LD + c + 1] = f.y;
+      R1[r * FA_LD + c + 2] = f.z;
+      R1[r * FA_LD + c + 3] = f.w;
+    }
+    __syncthreads();
+    float acc[FA_ROWS][4];
+    // T1 = F G: T1[i][c] = sum_m F[i][m] G[m][c]
+#pragma unroll
+    for (int a = 0; a < FA_ROWS; ++a)
+#pragma unroll
+      for (int b = 0; b < 4; ++b) acc[a][b] = 0.f;
+#pragma unroll 2
+    for (int m = 0; m < D; ++m) {
+      float g[4];
+#pragma unroll
+      for (int b = 0; b < 4; ++b) g[b] = R0[m * FA_LD + tx + 32 * b];
+#pragma unroll
+      for (int a = 0; a < FA_ROWS; ++a) {
+        const float f = R1[(ty + 8 * a) * FA_LD + m];
+#pragma unroll
+        for (int b = 0; b < 4; ++b) acc[a][b] = fmaf(f, g[b], acc[a][b]);
+      }
+    }
+    __syncthreads();
+#pragma unroll
+    for (int a = 0; a < FA_ROWS; ++a)
+#pragma unroll
+      for (int b = 0; b < 4; ++b) R0[(ty + 8 * a) * FA_LD + tx + 32 * b] = acc[a][b];
+    __syncthreads();
+    // M = T1 F^T: M[i][c] = sum_m T1[i][m] F[c][m]
+#pragma unroll
+    for (int a = 0; a < FA_ROWS; ++a)
+#pragma unroll
+      for (int b = 0; b < 4; ++b) acc[a][b] = 0.f;
+#pragma unroll 2
+    for (int m = 0; m < D; ++m) {
+      float f[4];
+#pragma unroll
+      for (int b = 0; b < 4; ++b) f[b] = R1[(tx + 32 * b) * FA_LD + m];
+#pragma unroll
+      for (int a = 0; a < FA_ROWS; ++a) {
+        const float t = R0[(ty + 8 * a) * FA_LD + m];
+#pragma unroll
+        for (int b = 0; b < 4; ++b) acc[a][b] = fmaf(t, f[b], acc[a][b]);
+      }
+    }
+    __syncthreads();
+#pragma unroll
+    for (int a = 0; a < FA_ROWS; ++a)
+#pragma unroll
+      for (int b = 0; b < 4; ++b) R0[(ty + 8 * a) * FA_LD + tx + 32 * b] = acc[a][b];
+    __syncthreads();
+#pragma unroll
+    for (int a = 0; a < FA_ROWS; ++a) {
+      const int i = ty + 8 * a;
+      z[a][0] = make_float2(R0[i * FA_LD + c0], R0[i * FA_LD + c0 + 1]);
+      z[a][1] = make_float2(R0[i * FA_LD + c0 + 2], R0[i * FA_LD + c0 + 3]);
+    }
+    __syncthreads();
+  }
+  {
+#pragma unroll
+    for (int a = 0; a < FA_ROWS; ++a) {
+      const int i = ty + 8 * a;
       z[a][0].x += (i == c0 ? 1.f : 0.f);
       z[a][0].y += (i == c0 + 1 ? 1.f : 0.f);
       z[a][1].x += (i == c0 + 2 ? 1.f : 0.f);
@@ -165,9 +261,41 @@ __global__ void __launch_bounds__(FA_THREADS, 2) factor_kernel(Dims dm, Ws ws) {
       if (!isfinite(x[b])) s_bad = 1;
       Ms[i * FA_LD + c] = x[b];
     }
-    *(float4*)(mout + i * D + c0) = make_float4(x[0], x[1], x[2], x[3]);
+    if constexpr (!PROJ) *(float4*)(mout + i * D + c0) = make_float4(x[0], x[1], x[2], x[3]);
   }
   __syncthreads();
+  if constexpr (PROJ) {
+    // T = L_M^{-1} F: T[i][c] = sum_{m <= i} L^{-1}[i][m] F[m][c] (L^{-1} now in R0 = Ms)
+    const float* R1 = Ms + D * FA_LD;
+    float acc[FA_ROWS][4];
+#pragma unroll
+    for (int a = 0; a < FA_ROWS; ++a)
+#pragma unroll
+      for (int b = 0; b < 4; ++b) acc[a][b] = 0.f;
+#pragma unroll 2
+    for (int m = 0; m < D; ++m) {
+      float f[4];
+#pragma unroll
+      for (int b = 0; b < 4; ++b) f[b] = R1[m * FA_LD + tx + 32 * b];
+#pragma unroll
+      for (int a = 0; a < FA_ROWS; ++a) {
+        const float l = Ms[(ty + 8 * a) * FA_LD + m];
+#pragma unroll
+        for (int b = 0; b < 4; ++b) acc[a][b] = fmaf(l, f[b], acc[a][b]);
+      }
+    }
+    __syncthreads();
+#pragma unroll
+    for (int a = 0; a < FA_ROWS; ++a)
+#pragma unroll
+      for (int b = 0; b < 4; ++b) {
+        const int i = ty + 8 * a, c = tx + 32 * b;
+        if (!isfinite(acc[a][b])) s_bad = 1;
+        Ms[i * FA_LD + c] = acc[a][b];
+        mout[i * D + c] = acc[a][b];
+      }
+    __syncthreads();
+  }
   // bf16 hi/lo image: 2 K-atoms (channels 0-63, 64-127) x 256 rows x 128 B
   uint8_t* img = ws.minv_img + (int64_t)u * 65536;
   for (int e = tid; e < 256 * 16; e += FA_THREADS) {
@@ -189,13 +317,18 @@ __global__ void __launch_bounds__(FA_THREADS, 2) factor_kernel(Dims dm, Ws ws) {
   if (tid == 0 && s_bad) flag(ws, ST_NONFINITE);
 }
 
-cudaError_t launch_factor(const Dims& dm, const Ws& ws, cudaStream_t st) {
-  constexpr size_t smem = factor_smem_bytes();
-  cudaError_t e = cudaFuncSetAttribute(factor_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+template <bool PROJ>
+static cudaError_t launch_factor_t(const Dims& dm, const Ws& ws, const float* out_factor, cudaStream_t st) {
+  constexpr size_t smem = factor_smem_bytes<PROJ>();
+  cudaError_t e = cudaFuncSetAttribute(factor_kernel<PROJ>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   const int units = dm.L * dm.Hkv * dm.S;
-  factor_kernel<<<units, FA_THREADS, smem, st>>>(dm, ws);
+  factor_kernel<PROJ><<<units, FA_THREADS, smem, st>>>(dm, ws, out_factor);
   return cudaGetLastError();
+}
+
+cudaError_t launch_factor(const Dims& dm, const Ws& ws, const float* out_factor, cudaStream_t st) {
+  return out_factor ? launch_factor_t<true>(dm, ws, out_factor, st) : launch_factor_t<false>(dm, ws, nullptr, st);
 }
 
 }  // namespace jacap

@@ -29,6 +29,9 @@ constexpr uint32_t SC_IDESC64 = idesc_bf16_f32(128, 64, 0, 0);
 
 constexpr size_t score_bf16_smem_bytes() { return 1024 + 2 * SC_M_BYTES + SC_STAGES * SC_TILE_BYTES + 256; }
 
+// DENSE: the score matrix is a full 128 x 128 (output directions) rather than
+// the lower-triangular L^{-1}, so no K-step may be narrowed.
+template <bool DENSE>
 __global__ void __launch_bounds__(SC_THREADS, 1)
     score_bf16_kernel(const __grid_constant__ CUtensorMap vmap, Dims dm, Ws ws, const int32_t* __restrict__ cu,
                       float* __restrict__ scores) {
@@ -141,7 +144,7 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
           for (int k = 0; k < D / 16; ++k) {  // 16 channels per K-step
             const uint64_t ad = a0 + (uint64_t)((((k >> 2) * SC_BOX) + (k & 3) * 32) >> 4);
             const uint64_t bk = b0 + (uint64_t)((((k >> 2) * 32768) + (k & 3) * 32) >> 4);
-            if (k < 4) {  // channels 0-63: all 128 output columns
+            if (k < 4 || DENSE) {  // channels 0-63 (or a full matrix): all 128 output columns
               umma_f16_ss(dacc, ad, bk, SC_IDESC128, k > 0 ? 1u : 0u);
               umma_f16_ss(dacc, ad, bk + (16384 >> 4), SC_IDESC128, 1u);
             } else {      // channels 64-127: only columns (rows of L^{-1}) 64-127 are nonzero
@@ -250,7 +253,9 @@ __global__ void __launch_bounds__(SF_THREADS)
         for (int r = 0; r < D; ++r) {
           float yv = 0.f;
           const float* mr = Mi + r * D;
-          for (int c = 0; c <= r; ++c) yv = fmaf(mr[c], vr[c], yv);
+          // L^{-1} is lower triangular; a full matrix with output directions
+          const int cend = dm.dense_minv ? D - 1 : r;
+          for (int c = 0; c <= cend; ++c) yv = fmaf(mr[c], vr[c], yv);
           ssq = fmaf(yv, yv, ssq);
         }
         const int64_t o = (int64_t)item.plane * dm.Ntot + tok;
@@ -267,9 +272,10 @@ cudaError_t launch_score(const CUtensorMap& vmap, const Dims& dm, const Ws& ws, 
                          const int32_t* cu, float* scores, int grid, cudaStream_t st) {
   if (dtype == 1) {
     constexpr size_t smem = score_bf16_smem_bytes();
-    cudaError_t e = cudaFuncSetAttribute(score_bf16_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    auto kern = dm.dense_minv ? score_bf16_kernel<true> : score_bf16_kernel<false>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    score_bf16_kernel<<<grid, SC_THREADS, smem, st>>>(vmap, dm, ws, cu, scores);
+    kern<<<grid, SC_THREADS, smem, st>>>(vmap, dm, ws, cu, scores);
   } else {
     constexpr size_t smem = score_f32_smem_bytes();
     cudaError_t e = cudaFuncSetAttribute(score_f32_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

@@ -212,3 +212,40 @@ def test_full_size_config(index, samples):
             gpu_selection_properties(ev2.scores, ev2.idx, ev2.kept, wl.seqlens, b)
     del ev, t
     torch.cuda.empty_cache()
+
+
+def _output_factors(wl, d_o, seed, device):
+    """Synthetic output maps W (d_o x 128) per plane and their 128 x 128 factors
+    F = R of W = Q R (float32 on the device); W stays on the host for the oracle."""
+    r = np.random.default_rng(seed)
+    L, Hkv = wl.num_layers, wl.num_kv_heads
+    W = r.normal(size=(L, Hkv, d_o, 128)) / np.sqrt(128)
+    F = np.stack([[np.linalg.qr(W[l, g])[1] for g in range(Hkv)] for l in range(L)])
+    return W, torch.as_tensor(F, dtype=torch.float32, device=device).contiguous()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_output_directions_every_unit(dtype):
+    # u_i = W v_i (Sec. 3.1) through the reduced d x d form on the GPU vs the
+    # oracle's explicit d_o-dimensional capacity matrix
+    wl = Workload("t", 2, 8, 2, (1300, 400), 16, 96, dtype=dtype, seed=21)
+    t = generate(wl, DEV)
+    W, F = _output_factors(wl, 192, 5, DEV)
+    params = jacap_params()
+    ev = Evictor(make_cache(t, wl), wl.budget, params, out_factor=F)
+    ev.run()
+    ev.check()
+    # the factors the GPU used, in float64, define the same W^T W as W up to rounding
+    cu = t.cu_seqlens.cpu().tolist()
+    for s in range(len(wl.seqlens)):
+        for layer in range(wl.num_layers):
+            for g in range(wl.num_kv_heads):
+                q, K, V = unit_arrays(t, wl.num_q_heads, s, layer, g)
+                Ff = F[layer, g].double().cpu().numpy()  # a d x d output map with the GPU's exact factor
+                ora = oracle_unit(q, K, V, wl.budget, JacapParams(), out_proj=Ff)
+                a, b = cu[s], cu[s + 1]
+                assert_scores_close(ev.scores[layer, g, a:b].double().cpu().numpy(), ora["scores"])
+                assert_selection(ev.idx[layer, g, s].cpu().numpy(), b - a, wl.budget, ora["scores"], ora["idx"])
+                # and the explicit d_o-dimensional output map gives the same scores (push-through)
+                ora_w = oracle_unit(q, K, V, wl.budget, JacapParams(), out_proj=W[layer, g])
+                assert_scores_close(ev.scores[layer, g, a:b].double().cpu().numpy(), ora_w["scores"])
