@@ -44,6 +44,8 @@ def parse():
     p.add_argument("--budget", type=int, default=None)
     p.add_argument("--weighting", default="jacobian", choices=["jacobian", "linear"],
                    help="Eq. 8 softmax-aware weights (the method) or the linear S = I surrogate")
+    p.add_argument("--out-proj", type=int, default=0, metavar="D_O",
+                   help="use true output directions u = W v with synthetic W (D_O x 128) per plane")
     p.add_argument("--e2e-steps", type=int, default=10)
     p.add_argument("--cpu-seconds", type=float, default=15.0)
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -150,7 +152,7 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows), "power_w_max": max(pw) if pw else None}
 
 
-def workload_config(wl, budget, gpus, weighting="jacobian"):
+def workload_config(wl, budget, gpus, weighting="jacobian", out_proj=0):
     return {
         "workload": wl.name,
         "layers": wl.num_layers,
@@ -162,6 +164,7 @@ def workload_config(wl, budget, gpus, weighting="jacobian"):
         "budget": budget,
         "tau": 10.0,
         "weighting": weighting,
+        "output_directions": f"u = W v, synthetic W ({out_proj} x 128) per plane" if out_proj else "u = v (proxy)",
         "cache_dtype": wl.dtype,
         "l2": "inputs larger than L2: each step streams the whole cache (K and V alone are "
               f"{2 * wl.num_layers * wl.num_kv_heads * wl.total_tokens * wl.head_dim * (2 if wl.dtype == 'bf16' else 4) / 1e9:.2f} GB)",
@@ -170,7 +173,7 @@ def workload_config(wl, budget, gpus, weighting="jacobian"):
 
 
 # ------------------------------------------------------------------ oracle --
-def oracle_sample(wl, budget, seconds, device, tensors=None, weighting="jacobian"):
+def oracle_sample(wl, budget, seconds, device, tensors=None, weighting="jacobian", out_factor=None):
     """Time the float64 oracle on whole units of the workload for ~`seconds`.
 
     Returns (tokens_layers_per_s, sample_description, wall_s)."""
@@ -190,7 +193,8 @@ def oracle_sample(wl, budget, seconds, device, tensors=None, weighting="jacobian
             K = k.to(dt).double().numpy()
             V = v.to(dt).double().numpy()
         t0 = time.perf_counter()
-        oracle_unit(q, K, V, budget, JacapParams(linear_weighting=weighting == "linear"))
+        proj = None if out_factor is None else out_factor[l, g].double().cpu().numpy()
+        oracle_unit(q, K, V, budget, JacapParams(linear_weighting=weighting == "linear"), out_proj=proj)
         t_total += time.perf_counter() - t0
         done += 1
         tok += n
@@ -285,7 +289,15 @@ def run_ours(args):
     cache = Cache(t.q_win, t.k, t.v, t.cu_seqlens, t.seqlens, wl.num_q_heads)
     from paper_2609_08131_gb300 import jacap_params
 
-    ev = Evictor(cache, budget, jacap_params(linear_weighting=1 if args.weighting == "linear" else 0))
+    out_factor = None
+    if args.out_proj:
+        # synthetic output maps W (d_o x 128) per plane and their QR factors R
+        # (F^T F = W^T W); set-up only, outside every timed region
+        gen = torch.Generator(device=dev).manual_seed(7)
+        W = torch.randn(wl.num_layers * wl.num_kv_heads, args.out_proj, 128, generator=gen, device=dev) / 128 ** 0.5
+        out_factor = torch.linalg.qr(W, mode="r").R.reshape(wl.num_layers, wl.num_kv_heads, 128, 128).contiguous()
+    ev = Evictor(cache, budget, jacap_params(linear_weighting=1 if args.weighting == "linear" else 0),
+                 out_factor=out_factor)
     stream = torch.cuda.current_stream(dev)
 
     def barrier():
@@ -356,7 +368,8 @@ def run_ours(args):
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
-        v_cpu, desc, wall = oracle_sample(wl, budget, args.cpu_seconds, dev, tensors=t, weighting=args.weighting)
+        v_cpu, desc, wall = oracle_sample(wl, budget, args.cpu_seconds, dev, tensors=t, weighting=args.weighting,
+                                          out_factor=out_factor)
         cpu = {"value": v_cpu, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
                "sample": desc + f"; {wall:.1f} s of CPU work; numpy BLAS threads left at their default"}
 
@@ -378,7 +391,7 @@ def run_ours(args):
             "vs_baseline": None,
             "dtype": "bf16" if wl.dtype == "bf16" else "f32",
             "data": "synthetic",
-            "config": workload_config(wl, budget, world, args.weighting),
+            "config": workload_config(wl, budget, world, args.weighting, args.out_proj),
             "roofline": {
                 "bound": "hbm",
                 "kernel": dom,
