@@ -44,6 +44,9 @@ def parse():
     p.add_argument("--budget", type=int, default=None)
     p.add_argument("--weighting", default="jacobian", choices=["jacobian", "linear"],
                    help="Eq. 8 softmax-aware weights (the method) or the linear S = I surrogate")
+    p.add_argument("--covariance", default="diagonal", choices=["diagonal", "full"],
+                   help="query-response variance from the diagonal Lambda_Q (the method) or the full "
+                        "window covariance (App. B.2)")
     p.add_argument("--out-proj", type=int, default=0, metavar="D_O",
                    help="use true output directions u = W v with synthetic W (D_O x 128) per plane")
     p.add_argument("--e2e-steps", type=int, default=10)
@@ -152,7 +155,7 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows), "power_w_max": max(pw) if pw else None}
 
 
-def workload_config(wl, budget, gpus, weighting="jacobian", out_proj=0):
+def workload_config(wl, budget, gpus, weighting="jacobian", out_proj=0, covariance="diagonal"):
     return {
         "workload": wl.name,
         "layers": wl.num_layers,
@@ -164,6 +167,7 @@ def workload_config(wl, budget, gpus, weighting="jacobian", out_proj=0):
         "budget": budget,
         "tau": 10.0,
         "weighting": weighting,
+        "query_covariance": covariance,
         "output_directions": f"u = W v, synthetic W ({out_proj} x 128) per plane" if out_proj else "u = v (proxy)",
         "cache_dtype": wl.dtype,
         "l2": "inputs larger than L2: each step streams the whole cache (K and V alone are "
@@ -173,7 +177,8 @@ def workload_config(wl, budget, gpus, weighting="jacobian", out_proj=0):
 
 
 # ------------------------------------------------------------------ oracle --
-def oracle_sample(wl, budget, seconds, device, tensors=None, weighting="jacobian", out_factor=None):
+def oracle_sample(wl, budget, seconds, device, tensors=None, weighting="jacobian", out_factor=None,
+                  covariance="diagonal"):
     """Time the float64 oracle on whole units of the workload for ~`seconds`.
 
     Returns (tokens_layers_per_s, sample_description, wall_s)."""
@@ -194,7 +199,8 @@ def oracle_sample(wl, budget, seconds, device, tensors=None, weighting="jacobian
             V = v.to(dt).double().numpy()
         t0 = time.perf_counter()
         proj = None if out_factor is None else out_factor[l, g].double().cpu().numpy()
-        oracle_unit(q, K, V, budget, JacapParams(linear_weighting=weighting == "linear"), out_proj=proj)
+        oracle_unit(q, K, V, budget, JacapParams(linear_weighting=weighting == "linear",
+                                                 full_covariance=covariance == "full"), out_proj=proj)
         t_total += time.perf_counter() - t0
         done += 1
         tok += n
@@ -221,7 +227,7 @@ def run_reference(args):
     dt = wl.torch_dtype
     K64, V64, Q64 = k.to(dt).double().numpy(), v.to(dt).double().numpy(), q.to(dt).double().numpy()
     t0 = time.perf_counter()
-    P = JacapParams(linear_weighting=args.weighting == "linear")
+    P = JacapParams(linear_weighting=args.weighting == "linear", full_covariance=args.covariance == "full")
     oracle_unit(Q64, K64[:2048], V64[:2048], budget, P)
     per_tok = (time.perf_counter() - t0) / 2048
     target = 150.0 / max(1, args.steps + args.warmup)
@@ -251,7 +257,7 @@ def run_reference(args):
         "vs_baseline": None,
         "dtype": "f64",
         "data": "synthetic",
-        "config": workload_config(wl, budget, args.gpus, args.weighting),
+        "config": workload_config(wl, budget, args.gpus, args.weighting, covariance=args.covariance),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
@@ -296,7 +302,8 @@ def run_ours(args):
         gen = torch.Generator(device=dev).manual_seed(7)
         W = torch.randn(wl.num_layers * wl.num_kv_heads, args.out_proj, 128, generator=gen, device=dev) / 128 ** 0.5
         out_factor = torch.linalg.qr(W, mode="r").R.reshape(wl.num_layers, wl.num_kv_heads, 128, 128).contiguous()
-    ev = Evictor(cache, budget, jacap_params(linear_weighting=1 if args.weighting == "linear" else 0),
+    ev = Evictor(cache, budget, jacap_params(linear_weighting=1 if args.weighting == "linear" else 0,
+                                             full_covariance=1 if args.covariance == "full" else 0),
                  out_factor=out_factor)
     stream = torch.cuda.current_stream(dev)
 
@@ -369,7 +376,7 @@ def run_ours(args):
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         v_cpu, desc, wall = oracle_sample(wl, budget, args.cpu_seconds, dev, tensors=t, weighting=args.weighting,
-                                          out_factor=out_factor)
+                                          out_factor=out_factor, covariance=args.covariance)
         cpu = {"value": v_cpu, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
                "sample": desc + f"; {wall:.1f} s of CPU work; numpy BLAS threads left at their default"}
 
@@ -391,7 +398,7 @@ def run_ours(args):
             "vs_baseline": None,
             "dtype": "bf16" if wl.dtype == "bf16" else "f32",
             "data": "synthetic",
-            "config": workload_config(wl, budget, world, args.weighting, args.out_proj),
+            "config": workload_config(wl, budget, world, args.weighting, args.out_proj, args.covariance),
             "roofline": {
                 "bound": "hbm",
                 "kernel": dom,

@@ -108,8 +108,13 @@ typedef struct {
  *                 surrogate S_C = I that App. A contrasts Jacap with, i.e.
  *                 rho_i = 1 and w_i = (1/d) sum_h kappa_h,i (a CapKV-style
  *                 weight; the logits and softmax statistics are then unused).
- *  full_covariance  must be 0 (the diagonal Lambda_Q of App. B.2);
- *                 1 returns JACAP_ERR_UNSUPPORTED.
+ *  full_covariance  0: the diagonal Lambda_Q of App. B.2 (the method as the
+ *                 paper runs it); 1: the full covariance of the window queries,
+ *                 kappa_h,i = (1/w) sum_j ((q_h,j - mu_h) . k_i)^2 (1/(w-1) with
+ *                 cov_unbiased), the O(N d^2) variant of App. B.2. bf16 caches
+ *                 with window in {8, 16, 32, 64} and G * window <= 128 use the
+ *                 tensor cores; other shapes and float32 caches a much slower
+ *                 CUDA-core kernel. It adds a second read of K.
  * Callers that zero-initialise the two trailing fields get the method.
  */
 typedef struct {

@@ -19,7 +19,7 @@ constexpr size_t ALIGN = 1024;
 inline size_t align_up(size_t x) { return (x + ALIGN - 1) & ~(ALIGN - 1); }
 
 struct Carve {
-  size_t status, plan, chunks, counters, mu, lam, lk, cstats, w, wsplit, gpart, gram, minv, minv_img, total;
+  size_t status, plan, chunks, counters, mu, lam, qdev, lk, cstats, w, wsplit, gpart, gram, minv, minv_img, total;
 };
 
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
@@ -86,6 +86,7 @@ void make_dims(const jacap_layout* L, const jacap_params* P, Dims& dm) {
     dm.wdiv = P->weight_div_dk ? 1.0f / (float)D : 1.0f;
     dm.cov_unbiased = P->cov_unbiased;
     dm.linear = P->linear_weighting;
+    dm.full_cov = P->full_covariance;
   }
 }
 
@@ -100,6 +101,7 @@ Carve carve(const Dims& dm) {
   c.counters = o; o = align_up(o + units * 4);
   c.mu = o; o = align_up(o + (size_t)dm.S * dm.L * dm.Hq * D * 4);
   c.lam = o; o = align_up(o + (size_t)dm.S * dm.L * dm.Hq * D * 4);
+  c.qdev = o; o = align_up(o + (size_t)dm.S * dm.L * dm.Hq * dm.window * D * 4);
   c.lk = o; o = align_up(o + planes * (size_t)dm.Ntot * 2 * dm.G * 4);
   c.cstats = o; o = align_up(o + planes * (size_t)dm.c_cap * dm.G * 2 * 4);
   c.w = o; o = align_up(o + planes * (size_t)dm.Ntot * 4);
@@ -121,6 +123,7 @@ Ws make_ws(void* base, const Carve& c) {
   ws.counters = (int32_t*)(b + c.counters);
   ws.mu = (float*)(b + c.mu);
   ws.lam = (float*)(b + c.lam);
+  ws.qdev = (float*)(b + c.qdev);
   ws.lk = (float*)(b + c.lk);
   ws.cstats = (float*)(b + c.cstats);
   ws.w = (float*)(b + c.w);
@@ -237,7 +240,7 @@ jacap_status jacap_score_out(const jacap_layout* layout, const jacap_params* par
   if (params->cov_unbiased && layout->window < 2) return JACAP_ERR_INVALID_ARG;
   if (params->linear_weighting != 0 && params->linear_weighting != 1) return JACAP_ERR_INVALID_ARG;
   if (params->full_covariance != 0 && params->full_covariance != 1) return JACAP_ERR_INVALID_ARG;
-  if (params->ridge != 1 || params->full_covariance != 0) return JACAP_ERR_UNSUPPORTED;
+  if (params->ridge != 1) return JACAP_ERR_UNSUPPORTED;
   if (!aligned16(q_win) || !aligned16(k) || !aligned16(v) || ((uintptr_t)scores & 3u) != 0 ||
       (out_factor != nullptr && !aligned16(out_factor)))
     return JACAP_ERR_INVALID_ARG;
@@ -265,6 +268,11 @@ jacap_status jacap_score_out(const jacap_layout* layout, const jacap_params* par
   if ((st = hook(1)) != JACAP_OK || (st = map_cuda(launch_window_stats(dm, w, dt, q_win, s))) != JACAP_OK) return st;
   if ((st = hook(2)) != JACAP_OK ||
       (st = map_cuda(launch_kpass(kmap, dm, w, dt, cu, persistent_grid(items, sms, 1), s))) != JACAP_OK)
+    return st;
+  if (dm.full_cov &&  // overwrites the K pass's diagonal kappa; timed with the K pass
+      (st = map_cuda(launch_kfull(kmap, dm, w, dt, k,
+                                  persistent_grid(items, sms, kfull_uses_tensor_cores(dm, dt) ? 1 : 2), s))) !=
+          JACAP_OK)
     return st;
   if ((st = hook(3)) != JACAP_OK ||
       (st = map_cuda(launch_weights(dm, w, cu, persistent_grid(items, sms, 8), s))) != JACAP_OK)

@@ -40,6 +40,7 @@ struct Dims {
   int cov_unbiased;
   int linear;         // 1: S_C = I, rho = 1 (linear surrogate weight)
   int dense_minv;     // 1: the score matrix is a full 128 x 128 (output directions), not triangular
+  int full_cov;       // 1: kappa with the full window covariance of the queries (App. B.2)
 };
 
 // Workspace map (device pointers into the caller's workspace).
@@ -50,6 +51,7 @@ struct Ws {
   int32_t* counters;  // [units] per-unit completion counters (reserved)
   float* mu;          // [S][L][Hq][D]  mu / (tau sqrt d)
   float* lam;         // [S][L][Hq][D]  diagonal of Lambda_Q
+  float* qdev;        // [S][L][Hq][window][D]  centred window queries q_j - mu (full covariance only)
   float* lk;          // [L*Hkv][Ntot][2G]  logits then kappa per query head of the group
   float* cstats;      // [L*Hkv][c_cap][G][2]  per-chunk (max, sum exp(l - max))
   float* w;           // [L*Hkv][Ntot]  Eq. 8 weights summed over the group

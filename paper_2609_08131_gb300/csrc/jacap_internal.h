@@ -13,6 +13,9 @@ cudaError_t launch_kpass(const CUtensorMap& kmap, const Dims& dm, const Ws& ws, 
                          int grid, cudaStream_t st);
 cudaError_t launch_kpass_bf16(const CUtensorMap& kmap, const Dims& dm, const Ws& ws, const int32_t* cu, int grid,
                               cudaStream_t st);
+bool kfull_uses_tensor_cores(const Dims& dm, int dtype);
+cudaError_t launch_kfull(const CUtensorMap& kmap, const Dims& dm, const Ws& ws, int dtype, const void* k, int grid,
+                         cudaStream_t st);
 cudaError_t launch_weights(const Dims& dm, const Ws& ws, const int32_t* cu, int grid, cudaStream_t st);
 cudaError_t launch_gram(const CUtensorMap& vmap, const Dims& dm, const Ws& ws, int dtype, const void* v,
                         const int32_t* cu, int grid, cudaStream_t st);

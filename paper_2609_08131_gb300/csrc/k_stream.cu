@@ -80,6 +80,10 @@ __global__ void __launch_bounds__(D) window_stats_kernel(Dims dm, Ws ws, const T
   }
   const float lam = ss / (float)(dm.cov_unbiased ? dm.window - 1 : dm.window);
   const int64_t o = (((int64_t)s * dm.L + l) * dm.Hq + h) * D + c;
+  if (dm.full_cov) {  // the centred window queries for the full-covariance kappa
+    float* dst = ws.qdev + ((((int64_t)s * dm.L + l) * dm.Hq + h) * dm.window) * D + c;
+    for (int j = 0; j < dm.window; ++j) dst[(int64_t)j * D] = ld_elem(base + (int64_t)j * dm.q_sp) - mu;
+  }
   ws.mu[o] = mu * dm.inv_scale;
   ws.lam[o] = lam;
   if (!isfinite(mu) || !isfinite(lam)) flag(ws, ST_NONFINITE);

@@ -34,7 +34,8 @@ def check_unit(ev, t, wl, params, s, layer, g, check_w=True):
     q, K, V = unit_arrays(t, wl.num_q_heads, s, layer, g)
     ora = oracle_unit(q, K, V, ev.budget, JacapParams(tau=params.tau, weight_div_dk=bool(params.weight_div_dk),
                                                        cov_unbiased=bool(params.cov_unbiased),
-                                                       linear_weighting=bool(params.linear_weighting)))
+                                                       linear_weighting=bool(params.linear_weighting),
+                                                       full_covariance=bool(params.full_covariance)))
     cu = t.cu_seqlens.cpu().tolist()
     a, b = cu[s], cu[s + 1]
     n = b - a
@@ -68,6 +69,15 @@ SMALL = {
     "bf16_budget_exceeds_all": (Workload("t", 1, 4, 2, (100, 257), 8, 300, seed=18), jacap_params()),
     "bf16_gqa4_linear_weighting": (Workload("t", 2, 8, 2, (1500, 700), 16, 128, seed=19),
                                    jacap_params(linear_weighting=1)),
+    # full-covariance kappa (App. B.2): tensor-core kernel (w = 32, G = 4; w = 64, G = 2; w = 8, G = 8)
+    "bf16_gqa4_full_cov_w32": (Workload("t", 2, 8, 2, (1300, 300), 32, 96, seed=22), jacap_params(full_covariance=1)),
+    "bf16_gqa2_full_cov_w64_unbiased": (Workload("t", 1, 4, 2, (900, 129), 64, 64, seed=23),
+                                        jacap_params(full_covariance=1, cov_unbiased=1, tau=2.0)),
+    "bf16_gqa8_full_cov_w8": (Workload("t", 1, 8, 1, (700,), 8, 64, seed=24), jacap_params(full_covariance=1)),
+    # ... and the CUDA-core kernel (w = 24; float32)
+    "bf16_gqa4_full_cov_w24": (Workload("t", 1, 8, 2, (600, 200), 24, 64, seed=25), jacap_params(full_covariance=1)),
+    "f32_gqa2_full_cov": (Workload("t", 1, 4, 2, (500,), 16, 32, dtype="f32", seed=26),
+                          jacap_params(full_covariance=1)),
     "f32_mha_linear_weighting": (Workload("t", 1, 4, 4, (900,), 8, 64, dtype="f32", seed=20),
                                  jacap_params(linear_weighting=1, cov_unbiased=1)),
 }
