@@ -3,6 +3,7 @@
 // Validates arguments on the host before anything is enqueued, carves the
 // caller's workspace, encodes the TMA tensor maps of K and V, and enqueues the
 // kernels of the eviction pass on the caller's stream. Allocates nothing.
+#include <algorithm>
 #include <cudaTypedefs.h>
 #include <math.h>
 #include <string.h>
@@ -87,6 +88,7 @@ void make_dims(const jacap_layout* L, const jacap_params* P, Dims& dm) {
     dm.cov_unbiased = P->cov_unbiased;
     dm.linear = P->linear_weighting;
     dm.full_cov = P->full_covariance;
+    if (dm.full_cov && L->dtype == JACAP_BF16) dm.kf_rp = kfull_rows_padded(dm.G, dm.window);
   }
 }
 
@@ -101,7 +103,9 @@ Carve carve(const Dims& dm) {
   c.counters = o; o = align_up(o + units * 4);
   c.mu = o; o = align_up(o + (size_t)dm.S * dm.L * dm.Hq * D * 4);
   c.lam = o; o = align_up(o + (size_t)dm.S * dm.L * dm.Hq * D * 4);
-  c.qdev = o; o = align_up(o + (size_t)dm.S * dm.L * dm.Hq * dm.window * D * 4);
+  // centred window queries: fp32 rows, or the bf16 hi/lo image (512 bytes per padded row)
+  const size_t qrows = std::max((size_t)dm.G * dm.window, (size_t)kfull_rows_padded(dm.G, dm.window));
+  c.qdev = o; o = align_up(o + (size_t)dm.S * dm.L * dm.Hkv * qrows * 512);
   c.lk = o; o = align_up(o + planes * (size_t)dm.Ntot * 2 * dm.G * 4);
   c.cstats = o; o = align_up(o + planes * (size_t)dm.c_cap * dm.G * 2 * 4);
   c.w = o; o = align_up(o + planes * (size_t)dm.Ntot * 4);
@@ -124,6 +128,7 @@ Ws make_ws(void* base, const Carve& c) {
   ws.mu = (float*)(b + c.mu);
   ws.lam = (float*)(b + c.lam);
   ws.qdev = (float*)(b + c.qdev);
+  ws.qimg = b + c.qdev;
   ws.lk = (float*)(b + c.lk);
   ws.cstats = (float*)(b + c.cstats);
   ws.w = (float*)(b + c.w);

@@ -41,7 +41,17 @@ struct Dims {
   int linear;         // 1: S_C = I, rho = 1 (linear surrogate weight)
   int dense_minv;     // 1: the score matrix is a full 128 x 128 (output directions), not triangular
   int full_cov;       // 1: kappa with the full window covariance of the queries (App. B.2)
+  int kf_rp;          // full covariance on the tensor cores: rows per split part of the query image (else 0)
 };
+
+// Rows per split part of the full-covariance query image of one KV head's
+// group (G heads x W window queries, padded to 32, 64 or 128 rows); 0 where
+// the tensor-core kernel does not apply (window not in {8, 16, 32, 64} or more
+// than 128 centred queries per group).
+__host__ __device__ constexpr int kfull_rows_padded(int G, int W) {
+  return (W == 8 || W == 16 || W == 32 || W == 64) && G * W <= 128 ? (G * W <= 32 ? 32 : (G * W <= 64 ? 64 : 128))
+                                                                    : 0;
+}
 
 // Workspace map (device pointers into the caller's workspace).
 struct Ws {
@@ -51,7 +61,9 @@ struct Ws {
   int32_t* counters;  // [units] per-unit completion counters (reserved)
   float* mu;          // [S][L][Hq][D]  mu / (tau sqrt d)
   float* lam;         // [S][L][Hq][D]  diagonal of Lambda_Q
-  float* qdev;        // [S][L][Hq][window][D]  centred window queries q_j - mu (full covariance only)
+  float* qdev;        // [S][L][Hq][window][D]  centred window queries q_j - mu (full covariance, CUDA cores)
+  uint8_t* qimg;      // [S][L][Hkv][512 kf_rp]  the same as a bf16 hi/lo shared-memory image (tensor cores);
+                      // shares qdev's section
   float* lk;          // [L*Hkv][Ntot][2G]  logits then kappa per query head of the group
   float* cstats;      // [L*Hkv][c_cap][G][2]  per-chunk (max, sum exp(l - max))
   float* w;           // [L*Hkv][Ntot]  Eq. 8 weights summed over the group
@@ -355,6 +367,30 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Load two runs of 32 consecutive 32-bit columns of this thread's TMEM lane
+// (at ta and tb) and wait for both: one asm statement, so no use of the
+// registers can be scheduled before the wait.
+__device__ __forceinline__ void tmem_ld32x2(uint32_t ta, uint32_t tb, uint32_t* a, uint32_t* b) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%64];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,"
+      "%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%65];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(a[0]), "=r"(a[1]), "=r"(a[2]), "=r"(a[3]), "=r"(a[4]), "=r"(a[5]), "=r"(a[6]), "=r"(a[7]),
+        "=r"(a[8]), "=r"(a[9]), "=r"(a[10]), "=r"(a[11]), "=r"(a[12]), "=r"(a[13]), "=r"(a[14]), "=r"(a[15]),
+        "=r"(a[16]), "=r"(a[17]), "=r"(a[18]), "=r"(a[19]), "=r"(a[20]), "=r"(a[21]), "=r"(a[22]), "=r"(a[23]),
+        "=r"(a[24]), "=r"(a[25]), "=r"(a[26]), "=r"(a[27]), "=r"(a[28]), "=r"(a[29]), "=r"(a[30]), "=r"(a[31]),
+        "=r"(b[0]), "=r"(b[1]), "=r"(b[2]), "=r"(b[3]), "=r"(b[4]), "=r"(b[5]), "=r"(b[6]), "=r"(b[7]),
+        "=r"(b[8]), "=r"(b[9]), "=r"(b[10]), "=r"(b[11]), "=r"(b[12]), "=r"(b[13]), "=r"(b[14]), "=r"(b[15]),
+        "=r"(b[16]), "=r"(b[17]), "=r"(b[18]), "=r"(b[19]), "=r"(b[20]), "=r"(b[21]), "=r"(b[22]), "=r"(b[23]),
+        "=r"(b[24]), "=r"(b[25]), "=r"(b[26]), "=r"(b[27]), "=r"(b[28]), "=r"(b[29]), "=r"(b[30]), "=r"(b[31])
+      : "r"(ta), "r"(tb)
+      : "memory");
 }
 
 // Load 16 consecutive f32 columns of this thread's TMEM lane.

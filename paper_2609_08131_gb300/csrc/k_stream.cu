@@ -80,7 +80,28 @@ __global__ void __launch_bounds__(D) window_stats_kernel(Dims dm, Ws ws, const T
   }
   const float lam = ss / (float)(dm.cov_unbiased ? dm.window - 1 : dm.window);
   const int64_t o = (((int64_t)s * dm.L + l) * dm.Hq + h) * D + c;
-  if (dm.full_cov) {  // the centred window queries for the full-covariance kappa
+  if (dm.full_cov && dm.kf_rp) {
+    // centred window queries as the B operand image of the full-covariance
+    // MMA (K-major, 128-byte swizzle, two 64-channel atoms of 2 rp rows): row
+    // r = hh W + j holds the bf16 rounding hi of q_j - mu, row rp + r the
+    // bf16 rounding of the remainder, so hi + lo is within 2^-18 of q_j - mu
+    const int rp = dm.kf_rp, hh = h % dm.G;
+    uint8_t* img = ws.qimg + (((int64_t)s * dm.L + l) * dm.Hkv + h / dm.G) * (int64_t)(512 * rp);
+    img += (c >> 6) * (256 * rp) + (c & 7) * 2;
+    const uint32_t chunk = (c & 63) >> 3;
+    for (int j = 0; j < dm.window; ++j) {
+      const float e = ld_elem(base + (int64_t)j * dm.q_sp) - mu;
+      const __nv_bfloat16 hi = __float2bfloat16_rn(e);
+      const uint32_t r = (uint32_t)(hh * dm.window + j);
+      *(__nv_bfloat16*)(img + sw128_off(r, chunk)) = hi;
+      *(__nv_bfloat16*)(img + sw128_off(rp + r, chunk)) = __float2bfloat16_rn(e - __bfloat162float(hi));
+    }
+    if (hh == 0)  // padding rows of the group
+      for (int r = dm.G * dm.window; r < rp; ++r) {
+        *(__nv_bfloat16*)(img + sw128_off(r, chunk)) = __float2bfloat16_rn(0.f);
+        *(__nv_bfloat16*)(img + sw128_off(rp + r, chunk)) = __float2bfloat16_rn(0.f);
+      }
+  } else if (dm.full_cov) {  // fp32 centred window queries for the CUDA-core kernel
     float* dst = ws.qdev + ((((int64_t)s * dm.L + l) * dm.Hq + h) * dm.window) * D + c;
     for (int j = 0; j < dm.window; ++j) dst[(int64_t)j * D] = ld_elem(base + (int64_t)j * dm.q_sp) - mu;
   }

@@ -69,11 +69,15 @@ SMALL = {
     "bf16_budget_exceeds_all": (Workload("t", 1, 4, 2, (100, 257), 8, 300, seed=18), jacap_params()),
     "bf16_gqa4_linear_weighting": (Workload("t", 2, 8, 2, (1500, 700), 16, 128, seed=19),
                                    jacap_params(linear_weighting=1)),
-    # full-covariance kappa (App. B.2): tensor-core kernel (w = 32, G = 4; w = 64, G = 2; w = 8, G = 8)
+    # full-covariance kappa (App. B.2) on the tensor-core kernel
     "bf16_gqa4_full_cov_w32": (Workload("t", 2, 8, 2, (1300, 300), 32, 96, seed=22), jacap_params(full_covariance=1)),
     "bf16_gqa2_full_cov_w64_unbiased": (Workload("t", 1, 4, 2, (900, 129), 64, 64, seed=23),
                                         jacap_params(full_covariance=1, cov_unbiased=1, tau=2.0)),
     "bf16_gqa8_full_cov_w8": (Workload("t", 1, 8, 1, (700,), 8, 64, seed=24), jacap_params(full_covariance=1)),
+    "bf16_gqa8_full_cov_w16": (Workload("t", 1, 16, 2, (1100, 40), 16, 64, seed=27), jacap_params(full_covariance=1)),
+    # 8 centred queries per group: the image's zero padding rows
+    "bf16_mha_full_cov_w8_tau1": (Workload("t", 2, 4, 4, (650, 3), 8, 32, seed=28),
+                                  jacap_params(full_covariance=1, tau=1.0)),
     # ... and the CUDA-core kernel (w = 24; float32)
     "bf16_gqa4_full_cov_w24": (Workload("t", 1, 8, 2, (600, 200), 24, 64, seed=25), jacap_params(full_covariance=1)),
     "f32_gqa2_full_cov": (Workload("t", 1, 4, 2, (500,), 16, 32, dtype="f32", seed=26),
