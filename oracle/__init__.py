@@ -23,3 +23,4 @@ from .jacap_oracle import (  # noqa: F401
     oracle_pass,
     unit_views,
 )
+from .decode_oracle import decode_run  # noqa: F401,E402
