@@ -236,6 +236,63 @@ jacap_status jacap_compact(const jacap_layout* layout, const void* k, const void
                            const int32_t* idx, int32_t budget, void* k_out, void* v_out,
                            void* stream);
 
+/*
+ * Decoding-stage eviction (the paper's decoding experiments, Sec. 4; Sec. 3.4,
+ * last paragraph: during decoding mu_Q and Lambda_Q are estimated from the
+ * historical queries). Three calls on top of the ones above:
+ *
+ * jacap_stats_update merges new queries into running query statistics.
+ *  q_new   device, the layout's Q_win strides and dtype; `window` (>= 1) is
+ *          the number of new queries per (request, layer, query head).
+ *  stats   device float32 [num_seqs][num_layers][num_q_heads][2][128],
+ *          16-byte aligned: per channel the mean of every query merged so far
+ *          and M2, the sum of their squared deviations from that mean.
+ *  counts  device int32 [num_seqs][num_layers][num_q_heads]: how many queries
+ *          have been merged (a negative count is read as 0).
+ *  reset   1: discard the previous statistics and start from q_new;
+ *          0: merge (Chan-Golub-LeVeque pairwise update, float32).
+ * The caller owns both arrays. Only the layout's sizes, dtype and Q strides
+ * are used (it must still pass the checks of jacap_score).
+ */
+jacap_status jacap_stats_update(const jacap_layout* layout, const void* q_new, int32_t reset,
+                                float* stats, int32_t* counts, void* stream);
+
+/*
+ * jacap_score_timed with the query statistics taken from running statistics
+ * (as kept by jacap_stats_update) instead of a query window: per query head
+ * mu = mean and lambda = M2 / n (M2 / (n - 1) with cov_unbiased), n = counts.
+ * q strides are unused and `window` only sizes the workspace (1 suffices).
+ * A count below 1 (below 2 with cov_unbiased) records JACAP_ERR_INVALID_ARG in
+ * the status word. full_covariance must be 0 (no running d x d covariance is
+ * kept): 1 returns JACAP_ERR_UNSUPPORTED. The outputs and the other arguments
+ * are those of jacap_score_timed.
+ */
+jacap_status jacap_score_stats(const jacap_layout* layout, const jacap_params* params,
+                               const float* stats, const int32_t* counts,
+                               const void* k, const void* v, float* scores,
+                               void* ws, size_t ws_bytes, void* stream,
+                               void* const* events, int32_t num_events);
+
+/*
+ * The retained cache in place: for every unit the rows idx[0 .. kept - 1]
+ * (relative to cu[s], as produced by jacap_select) of K and V move, bit for
+ * bit, to rows 0 .. kept - 1 of the request's token range; rows from kept on
+ * are left as they were (free for the next tokens). kept = min(n_s, budget).
+ *  k, v  device, the layout; written in place.
+ *  pos   device int32 [num_layers][num_kv_heads][total_tokens] or NULL: a
+ *        per-token tag (e.g. the original position) moved with the rows.
+ *  ws    the workspace of jacap_score for this layout (status word).
+ * The kept positions of every unit must ascend strictly within [0, n_s) (as
+ * jacap_select emits them); a unit where they do not is left untouched and
+ * JACAP_ERR_INVALID_ARG is recorded in the status word. Units run
+ * concurrently; each moves its rows in chunks that are read whole before any
+ * row of the chunk is written, which cannot overwrite a row still to be read
+ * because idx[r] >= r.
+ */
+jacap_status jacap_compact_inplace(const jacap_layout* layout, void* k, void* v, int32_t* pos,
+                                   const int32_t* idx, int32_t budget, void* ws, size_t ws_bytes,
+                                   void* stream);
+
 /* Synchronises `stream`, then reads the workspace status word: JACAP_OK or the
  * first device-side error recorded since the last jacap_score on `ws`. */
 jacap_status jacap_device_status(const void* ws, void* stream);

@@ -92,6 +92,12 @@ _SIGS = {
     "jacap_select": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, ctypes.c_int32, _P, _P, _P, ctypes.c_size_t,
                                     _P]),
     "jacap_compact": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, _P, _P, ctypes.c_int32, _P, _P, _P]),
+    "jacap_score_stats": (ctypes.c_int, [ctypes.POINTER(jacap_layout), ctypes.POINTER(jacap_params), _P, _P, _P,
+                                         _P, _P, _P, ctypes.c_size_t, _P, ctypes.POINTER(ctypes.c_void_p),
+                                         ctypes.c_int32]),
+    "jacap_stats_update": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, ctypes.c_int32, _P, _P, _P]),
+    "jacap_compact_inplace": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, _P, _P, _P, ctypes.c_int32, _P,
+                                             ctypes.c_size_t, _P]),
     "jacap_device_status": (ctypes.c_int, [_P, _P]),
     "jacap_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "jacap_workspace_offsets": (ctypes.c_int, [ctypes.POINTER(jacap_layout), ctypes.c_int32,
@@ -135,6 +141,21 @@ def jacap_score_out(layout, params, q_win, k, v, out_factor, scores, ws, ws_byte
     arr = (ctypes.c_void_p * max(1, len(events)))(*[ctypes.c_void_p(e) for e in events])
     return lib().jacap_score_out(ctypes.byref(layout), ctypes.byref(params), q_win, k, v, out_factor, scores, ws,
                                  ws_bytes, stream, arr, len(events))
+
+
+def jacap_score_stats(layout, params, stats, counts, k, v, scores, ws, ws_bytes, stream, events=()) -> int:
+    """Scoring pass with running query statistics (``stats``, ``counts``: device pointers)."""
+    arr = (ctypes.c_void_p * max(1, len(events)))(*[ctypes.c_void_p(e) for e in events])
+    return lib().jacap_score_stats(ctypes.byref(layout), ctypes.byref(params), stats, counts, k, v, scores, ws,
+                                   ws_bytes, stream, arr, len(events))
+
+
+def jacap_stats_update(layout, q_new, reset, stats, counts, stream) -> int:
+    return lib().jacap_stats_update(ctypes.byref(layout), q_new, int(reset), stats, counts, stream)
+
+
+def jacap_compact_inplace(layout, k, v, pos, idx, budget, ws, ws_bytes, stream) -> int:
+    return lib().jacap_compact_inplace(ctypes.byref(layout), k, v, pos, idx, budget, ws, ws_bytes, stream)
 
 
 JACAP_STATIC_SCRATCH_BYTES = 64 << 20

@@ -23,7 +23,7 @@ BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libjacap.so")
 
 SOURCES = ["jacap_api.cu", "k_stream.cu", "k_kpass.cu", "k_gram.cu", "k_factor.cu", "k_score.cu", "k_select.cu",
-           "jacap_static.cu", "k_kfull.cu"]
+           "jacap_static.cu", "k_kfull.cu", "k_decode.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
           "-I" + INCLUDE, "-I" + CSRC]
@@ -92,6 +92,9 @@ EXPORTS = [
     "jacap_score_timed",
     "jacap_score_static",
     "jacap_score_out",
+    "jacap_score_stats",
+    "jacap_stats_update",
+    "jacap_compact_inplace",
     "jacap_select",
     "jacap_compact",
     "jacap_device_status",

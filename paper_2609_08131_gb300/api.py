@@ -16,13 +16,16 @@ from . import (
     JACAP_F32,
     JACAP_OK,
     jacap_compact,
+    jacap_compact_inplace,
     jacap_device_status,
     jacap_layout,
     jacap_params,
     jacap_score,
     jacap_score_timed,
     jacap_score_out,
+    jacap_score_stats,
     jacap_select,
+    jacap_stats_update,
     jacap_status_string,
     jacap_workspace_offsets,
     jacap_workspace_size,
@@ -193,3 +196,139 @@ def evict(cache: Cache, budget: int, params: jacap_params | None = None, check: 
     if check:
         ev.check()
     return ev
+
+
+class DecodeEvictor:
+    """Decoding-stage eviction (Sec. 3.4: statistics from the queries seen so
+    far; the decoding experiments of Sec. 4): one cache slot of
+    ``budget + interval`` tokens per request and running query statistics.
+    Whenever a request's cache reaches budget + interval tokens it is scored
+    with those statistics and compacted in place back to ``budget`` tokens.
+
+    Buffers (device):
+      k, v    [S, L, Hkv, cap, 128], cap = budget + interval; request s holds
+              its ``lengths[s]`` tokens in rows 0 .. lengths[s] - 1
+      pos     int32 [S, L, Hkv, cap]: the id of every cached token (the
+              prefill tokens are 0 .. n0 - 1, decode step t of a request adds
+              n0 + t); it moves with the rows
+      stats   float32 [S, L, Hq, 2, 128] (mean, M2), counts int32 [S, L, Hq]
+    Writing a decode step's k, v into the slot is the model's cache write (a
+    plain copy here); the statistics, the scoring pass, the selection and the
+    compaction run in libjacap's kernels.
+    """
+
+    def __init__(self, num_seqs: int, num_layers: int, num_q_heads: int, num_kv_heads: int, budget: int,
+                 interval: int, dtype=torch.bfloat16, params: jacap_params | None = None, device="cuda"):
+        if budget < 1 or interval < 1:
+            raise ValueError("budget and interval must be >= 1")
+        if dtype not in (torch.bfloat16, torch.float32):
+            raise ValueError("dtype must be bfloat16 or float32")
+        self.S, self.L, self.Hq, self.Hkv = num_seqs, num_layers, num_q_heads, num_kv_heads
+        self.budget, self.interval = int(budget), int(interval)
+        self.cap = self.budget + self.interval
+        self.dtype = dtype
+        self.params = params if params is not None else jacap_params()
+        dev = torch.device(device)
+        S, L, Hq, Hkv, cap, d = self.S, self.L, self.Hq, self.Hkv, self.cap, 128
+        self.k = torch.zeros((S, L, Hkv, cap, d), dtype=dtype, device=dev)
+        self.v = torch.zeros_like(self.k)
+        self.pos = torch.full((S, L, Hkv, cap), -1, dtype=torch.int32, device=dev)
+        self.stats = torch.zeros((S, L, Hq, 2, d), dtype=torch.float32, device=dev)
+        self.counts = torch.zeros((S, L, Hq), dtype=torch.int32, device=dev)
+        self.lengths = [0] * S
+        self.next_id = [0] * S
+        self.events = 0
+        self.cu = torch.tensor([0, cap], dtype=torch.int32, device=dev)
+        # one request's slot as a cache of cap tokens
+        self.slot = self._layout(1, window=1, q_strides=(d, d, d, d))
+        nbytes = jacap_workspace_size(self.slot, self.budget)
+        if nbytes == 0:
+            raise JacapError(1, "jacap_workspace_size")
+        self.ws = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+        self.scores = torch.empty((L, Hkv, cap), dtype=torch.float32, device=dev)
+        self.idx = torch.empty((L, Hkv, 1, self.budget), dtype=torch.int32, device=dev)
+        self.kept = torch.empty((1,), dtype=torch.int32, device=dev)
+
+    def _layout(self, num_seqs, window, q_strides) -> jacap_layout:
+        lay = jacap_layout()
+        lay.num_seqs = num_seqs
+        lay.cu_seqlens = self.cu.data_ptr()
+        lay.max_seqlen = self.cap
+        lay.total_tokens = self.cap
+        lay.num_layers, lay.num_q_heads, lay.num_kv_heads, lay.head_dim = self.L, self.Hq, self.Hkv, 128
+        lay.window = window
+        lay.dtype = JACAP_BF16 if self.dtype == torch.bfloat16 else JACAP_F32
+        st = self.k.stride()
+        lay.kv_stride_layer, lay.kv_stride_head, lay.kv_stride_token = st[1], st[2], st[3]
+        lay.q_stride_seq, lay.q_stride_layer, lay.q_stride_head, lay.q_stride_pos = q_strides
+        return lay
+
+    def _merge(self, q, reset: bool, stream=None):
+        """q: [S, L, Hq, m, 128] queries (the slot dtype, channel contiguous)."""
+        if q.dtype != self.dtype or q.stride(-1) != 1 or tuple(q.shape[:3]) != (self.S, self.L, self.Hq):
+            raise ValueError("queries must be [S, L, Hq, m, 128] in the cache dtype")
+        lay = self._layout(self.S, q.shape[3], (q.stride(0), q.stride(1), q.stride(2), q.stride(3)))
+        _check(jacap_stats_update(lay, _ptr(q), 1 if reset else 0, _ptr(self.stats), _ptr(self.counts),
+                                  _stream(stream)), "jacap_stats_update")
+
+    def start(self, k0, v0, q_win, lengths, stream=None):
+        """Load the prefill caches (k0, v0: [S, L, Hkv, n, 128], request s using
+        its first lengths[s] < cap rows) and start the statistics from the
+        prefill window queries q_win [S, L, Hq, w, 128]."""
+        if any(n < 0 or n >= self.cap for n in lengths):
+            raise ValueError("a prefill cache must hold fewer than budget + interval tokens; evict it first")
+        n = k0.shape[3]
+        self.k[:, :, :, :n].copy_(k0)
+        self.v[:, :, :, :n].copy_(v0)
+        ar = torch.arange(self.cap, dtype=torch.int32, device=self.pos.device)
+        self.pos.copy_(torch.where(ar < torch.tensor(lengths, device=ar.device)[:, None], ar, -1)[:, None, None, :]
+                       .expand_as(self.pos))
+        self.lengths = list(lengths)
+        self.next_id = list(lengths)
+        self._merge(q_win, reset=True, stream=stream)
+
+    def append(self, k_new, v_new, q_new, stream=None):
+        """One decode step for every request: k_new, v_new [S, L, Hkv, 128],
+        q_new [S, L, Hq, 128]. Returns the requests whose cache is now full
+        (each must be evicted before its next append)."""
+        for s in range(self.S):
+            if self.lengths[s] >= self.cap:
+                raise RuntimeError(f"request {s} is full; evict it first")
+            t = self.lengths[s]
+            self.k[s, :, :, t].copy_(k_new[s])
+            self.v[s, :, :, t].copy_(v_new[s])
+            self.pos[s, :, :, t] = self.next_id[s]
+            self.lengths[s] += 1
+            self.next_id[s] += 1
+        self._merge(q_new.unsqueeze(3), reset=False, stream=stream)
+        return [s for s in range(self.S) if self.lengths[s] >= self.cap]
+
+    def evict(self, s: int, stream=None):
+        """Score request s's full slot with the running statistics, select the
+        budget best tokens and compact them in place to rows 0 .. budget - 1."""
+        if self.lengths[s] != self.cap:
+            raise RuntimeError("only a full slot is evicted")
+        lay, st = self.slot, _stream(stream)
+        off_stats = s * self.L * self.Hq * 2 * 128 * 4
+        off_counts = s * self.L * self.Hq * 4
+        stats = ctypes.c_void_p(self.stats.data_ptr() + off_stats)
+        counts = ctypes.c_void_p(self.counts.data_ptr() + off_counts)
+        k, v, pos = _ptr(self.k[s]), _ptr(self.v[s]), _ptr(self.pos[s])
+        _check(jacap_score_stats(lay, self.params, stats, counts, k, v, _ptr(self.scores), _ptr(self.ws),
+                                 self.ws.numel(), st), "jacap_score_stats")
+        _check(jacap_select(lay, _ptr(self.scores), self.budget, _ptr(self.idx), _ptr(self.kept), _ptr(self.ws),
+                            self.ws.numel(), st), "jacap_select")
+        _check(jacap_compact_inplace(lay, k, v, pos, _ptr(self.idx), self.budget, _ptr(self.ws), self.ws.numel(),
+                                     st), "jacap_compact_inplace")
+        self.lengths[s] = self.budget
+        self.events += 1
+
+    def step(self, k_new, v_new, q_new, stream=None):
+        """append() then evict() every request that became full."""
+        full = self.append(k_new, v_new, q_new, stream)
+        for s in full:
+            self.evict(s, stream)
+        return full
+
+    def check(self, stream=None):
+        _check(jacap_device_status(_ptr(self.ws), _stream(stream)), "device status")

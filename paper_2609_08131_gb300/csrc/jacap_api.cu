@@ -231,23 +231,32 @@ jacap_status jacap_score_timed(const jacap_layout* layout, const jacap_params* p
   return jacap_score_out(layout, params, q_win, k, v, nullptr, scores, ws, ws_bytes, stream, events, num_events);
 }
 
-jacap_status jacap_score_out(const jacap_layout* layout, const jacap_params* params, const void* q_win,
-                             const void* k, const void* v, const float* out_factor, float* scores, void* ws,
-                             size_t ws_bytes, void* stream, void* const* events, int32_t num_events) {
+}  // extern "C"
+
+namespace {
+
+// The scoring pass behind jacap_score_out (query statistics from q_win) and
+// jacap_score_stats (from running statistics: stats != NULL, q_win unused).
+jacap_status score_pass(const jacap_layout* layout, const jacap_params* params, const void* q_win,
+                        const float* stats, const int32_t* counts, const void* k, const void* v,
+                        const float* out_factor, float* scores, void* ws, size_t ws_bytes, void* stream,
+                        void* const* events, int32_t num_events) {
   if (num_events != 0 && (num_events != JACAP_SCORE_KERNELS + 1 || events == nullptr)) return JACAP_ERR_INVALID_ARG;
   jacap_status st = check_layout(layout);
   if (st != JACAP_OK) return st;
-  if (params == nullptr || q_win == nullptr || k == nullptr || v == nullptr || scores == nullptr || ws == nullptr)
+  const bool running = stats != nullptr;
+  if (params == nullptr || (!running && q_win == nullptr) || (running && counts == nullptr) || k == nullptr ||
+      v == nullptr || scores == nullptr || ws == nullptr)
     return JACAP_ERR_INVALID_ARG;
   if (!(params->tau > 0.f) || !isfinite(params->tau)) return JACAP_ERR_INVALID_ARG;
   if (params->weight_div_dk != 0 && params->weight_div_dk != 1) return JACAP_ERR_INVALID_ARG;
   if (params->cov_unbiased != 0 && params->cov_unbiased != 1) return JACAP_ERR_INVALID_ARG;
-  if (params->cov_unbiased && layout->window < 2) return JACAP_ERR_INVALID_ARG;
+  if (!running && params->cov_unbiased && layout->window < 2) return JACAP_ERR_INVALID_ARG;
   if (params->linear_weighting != 0 && params->linear_weighting != 1) return JACAP_ERR_INVALID_ARG;
   if (params->full_covariance != 0 && params->full_covariance != 1) return JACAP_ERR_INVALID_ARG;
-  if (params->ridge != 1) return JACAP_ERR_UNSUPPORTED;
-  if (!aligned16(q_win) || !aligned16(k) || !aligned16(v) || ((uintptr_t)scores & 3u) != 0 ||
-      (out_factor != nullptr && !aligned16(out_factor)))
+  if (params->ridge != 1 || (running && params->full_covariance != 0)) return JACAP_ERR_UNSUPPORTED;
+  if ((!running && !aligned16(q_win)) || !aligned16(k) || !aligned16(v) || ((uintptr_t)scores & 3u) != 0 ||
+      (out_factor != nullptr && !aligned16(out_factor)) || (running && (!aligned16(stats) || ((uintptr_t)counts & 3u))))
     return JACAP_ERR_INVALID_ARG;
   Dims dm;
   make_dims(layout, params, dm);
@@ -270,7 +279,10 @@ jacap_status jacap_score_out(const jacap_layout* layout, const jacap_params* par
   };
   if ((st = map_cuda(cudaMemsetAsync(w.status, 0, 64, s))) != JACAP_OK) return st;
   if ((st = hook(0)) != JACAP_OK || (st = map_cuda(launch_plan(dm, w, cu, s))) != JACAP_OK) return st;
-  if ((st = hook(1)) != JACAP_OK || (st = map_cuda(launch_window_stats(dm, w, dt, q_win, s))) != JACAP_OK) return st;
+  if ((st = hook(1)) != JACAP_OK ||
+      (st = map_cuda(running ? launch_stats_moments(dm, w, stats, counts, s)
+                             : launch_window_stats(dm, w, dt, q_win, s))) != JACAP_OK)
+    return st;
   if ((st = hook(2)) != JACAP_OK ||
       (st = map_cuda(launch_kpass(kmap, dm, w, dt, cu, persistent_grid(items, sms, 1), s))) != JACAP_OK)
     return st;
@@ -292,6 +304,59 @@ jacap_status jacap_score_out(const jacap_layout* layout, const jacap_params* par
     return st;
   if ((st = hook(7)) != JACAP_OK) return st;
   return JACAP_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+jacap_status jacap_score_out(const jacap_layout* layout, const jacap_params* params, const void* q_win,
+                             const void* k, const void* v, const float* out_factor, float* scores, void* ws,
+                             size_t ws_bytes, void* stream, void* const* events, int32_t num_events) {
+  return score_pass(layout, params, q_win, nullptr, nullptr, k, v, out_factor, scores, ws, ws_bytes, stream, events,
+                    num_events);
+}
+
+jacap_status jacap_score_stats(const jacap_layout* layout, const jacap_params* params, const float* stats,
+                               const int32_t* counts, const void* k, const void* v, float* scores, void* ws,
+                               size_t ws_bytes, void* stream, void* const* events, int32_t num_events) {
+  if (stats == nullptr) return JACAP_ERR_INVALID_ARG;
+  return score_pass(layout, params, nullptr, stats, counts, k, v, nullptr, scores, ws, ws_bytes, stream, events,
+                    num_events);
+}
+
+jacap_status jacap_stats_update(const jacap_layout* layout, const void* q_new, int32_t reset, float* stats,
+                                int32_t* counts, void* stream) {
+  jacap_status st = check_layout(layout);
+  if (st != JACAP_OK) return st;
+  if (q_new == nullptr || stats == nullptr || counts == nullptr || (reset != 0 && reset != 1))
+    return JACAP_ERR_INVALID_ARG;
+  if (!aligned16(q_new) || !aligned16(stats) || ((uintptr_t)counts & 3u) != 0) return JACAP_ERR_INVALID_ARG;
+  int sms = 0;
+  if ((st = check_device(&sms)) != JACAP_OK) return st;
+  Dims dm;
+  make_dims(layout, nullptr, dm);
+  return map_cuda(launch_stats_update(dm, layout->dtype == JACAP_BF16 ? 1 : 0, q_new, stats, counts, reset,
+                                      (cudaStream_t)stream));
+}
+
+jacap_status jacap_compact_inplace(const jacap_layout* layout, void* k, void* v, int32_t* pos, const int32_t* idx,
+                                   int32_t budget, void* ws, size_t ws_bytes, void* stream) {
+  jacap_status st = check_layout(layout);
+  if (st != JACAP_OK) return st;
+  if (k == nullptr || v == nullptr || idx == nullptr || ws == nullptr || budget < 1) return JACAP_ERR_INVALID_ARG;
+  if (!aligned16(k) || !aligned16(v) || ((uintptr_t)idx & 3u) != 0 || ((uintptr_t)pos & 3u) != 0)
+    return JACAP_ERR_INVALID_ARG;
+  if ((int64_t)layout->num_layers * layout->num_kv_heads * layout->num_seqs >= ((int64_t)1 << 31))
+    return JACAP_ERR_INVALID_ARG;
+  Dims dm;
+  make_dims(layout, nullptr, dm);
+  const Carve c = carve(dm);
+  if (((uintptr_t)ws & 255u) != 0 || ws_bytes < c.total) return JACAP_ERR_WORKSPACE;
+  int sms = 0;
+  if ((st = check_device(&sms)) != JACAP_OK) return st;
+  return map_cuda(launch_compact_inplace(dm, make_ws(ws, c), layout->dtype == JACAP_BF16 ? 1 : 0,
+                                         layout->cu_seqlens, k, v, pos, idx, budget, (cudaStream_t)stream));
 }
 
 jacap_status jacap_select(const jacap_layout* layout, const float* scores, int32_t budget, int32_t* idx,

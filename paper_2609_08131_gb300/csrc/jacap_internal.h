@@ -26,5 +26,11 @@ cudaError_t launch_select(const Dims& dm, const Ws& ws, const int32_t* cu, const
                           int32_t* idx, int32_t* kept, int grid, cudaStream_t st);
 cudaError_t launch_compact(const Dims& dm, int dtype, const int32_t* cu, const void* k, const void* v,
                            const int32_t* idx, int budget, void* k_out, void* v_out, cudaStream_t st);
+cudaError_t launch_stats_update(const Dims& dm, int dtype, const void* q, float* stats, int32_t* counts, int reset,
+                                cudaStream_t st);
+cudaError_t launch_stats_moments(const Dims& dm, const Ws& ws, const float* stats, const int32_t* counts,
+                                 cudaStream_t st);
+cudaError_t launch_compact_inplace(const Dims& dm, const Ws& ws, int dtype, const int32_t* cu, void* k, void* v,
+                                   int32_t* pos, const int32_t* idx, int budget, cudaStream_t st);
 
 }  // namespace jacap

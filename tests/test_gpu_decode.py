@@ -1,0 +1,125 @@
+"""GPU parity of decoding-stage eviction (reading R16) against the oracle.
+
+A synthetic decode stream: the workload generator's cache rows n0 .. n0+T-1
+of a request are the tokens its decode steps append, and its window queries
+w .. w+T-1 are their queries (the first w are the prefill window). At every
+eviction the slot is read back before the library touches it; the GPU's
+scores and kept set are compared with ``oracle_unit`` on that exact cache
+with the whole query history (so a near tie settled differently earlier
+cannot make later comparisons fail), the in-place compaction bit for bit, the
+running statistics with numpy moments of the history, and the eviction steps
+with ``decode_run``'s schedule.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import JacapParams, oracle_unit
+from oracle.decode_oracle import decode_run
+from paper_2609_08131_gb300 import jacap_params
+from paper_2609_08131_gb300.api import DecodeEvictor
+from paper_2609_08131_gb300.workloads import Workload, generate
+
+from parity import assert_rows_bitwise, assert_scores_close, assert_selection
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda:0"
+
+CASES = {
+    # name: (layers, Hq, Hkv, prefill lengths, window, steps, budget, interval, dtype, params, seed)
+    "bf16_gqa4": (2, 8, 2, (40, 63), 8, 70, 48, 16, "bf16", jacap_params(), 31),
+    "bf16_gqa2_interval1": (1, 4, 2, (30,), 4, 12, 32, 1, "bf16", jacap_params(tau=2.0), 32),
+    "f32_mha_unbiased": (1, 4, 4, (10, 24), 4, 30, 20, 5, "f32", jacap_params(cov_unbiased=1, tau=3.0), 33),
+    "bf16_gqa8_long_slot": (1, 8, 1, (700,), 16, 40, 512, 200, "bf16", jacap_params(), 34),
+}
+
+
+def _oracle_params(p):
+    return JacapParams(tau=p.tau, weight_div_dk=bool(p.weight_div_dk), cov_unbiased=bool(p.cov_unbiased),
+                       linear_weighting=bool(p.linear_weighting))
+
+
+@pytest.mark.parametrize("name", list(CASES))
+def test_decode_evictions_match_the_oracle_event_by_event(name):
+    L, Hq, Hkv, n0s, w, T, B, D, dtype, params, seed = CASES[name]
+    S, G, cap = len(n0s), Hq // Hkv, B + D
+    wl = Workload("decode stream", L, Hq, Hkv, tuple(n + T for n in n0s), w + T, B, dtype=dtype, seed=seed)
+    t = generate(wl, DEV)
+    cu = t.cu_seqlens.cpu().tolist()
+    tdt = t.k.dtype
+    k0 = torch.zeros((S, L, Hkv, max(n0s), 128), dtype=tdt, device=DEV)
+    v0 = torch.zeros_like(k0)
+    for s, n in enumerate(n0s):
+        k0[s, :, :, :n] = t.k[:, :, cu[s]:cu[s] + n]
+        v0[s, :, :, :n] = t.v[:, :, cu[s]:cu[s] + n]
+    ev = DecodeEvictor(S, L, Hq, Hkv, B, D, dtype=tdt, params=params, device=DEV)
+    ev.start(k0, v0, t.q_win[:, :, :, :w].contiguous(), list(n0s))
+    q_all = t.q_win.double().cpu().numpy()  # [S, L, Hq, w + T, d]
+    P = _oracle_params(params)
+    event_steps = {s: [] for s in range(S)}
+    for step in range(T):
+        rows = [cu[s] + n0s[s] + step for s in range(S)]
+        k_new = torch.stack([t.k[:, :, r] for r in rows])
+        v_new = torch.stack([t.v[:, :, r] for r in rows])
+        q_new = t.q_win[:, :, :, w + step].contiguous()
+        for s in ev.append(k_new, v_new, q_new):
+            event_steps[s].append(step)
+            kb, vb, pb = ev.k[s].clone(), ev.v[s].clone(), ev.pos[s].cpu().numpy()
+            nq = w + step + 1
+            # running statistics = moments of the whole history
+            stats = ev.stats[s].double().cpu().numpy()
+            assert (ev.counts[s].cpu().numpy() == nq).all()
+            hist = q_all[s, :, :, :nq]
+            scale = np.abs(hist).max()
+            np.testing.assert_allclose(stats[:, :, 0], hist.mean(axis=2), rtol=1e-4, atol=1e-5 * scale)
+            np.testing.assert_allclose(stats[:, :, 1] / nq, hist.var(axis=2), rtol=1e-4, atol=1e-6 * scale * scale)
+            ev.evict(s)
+            ev.check()
+            for layer in range(L):
+                for g in range(Hkv):
+                    K = kb[layer, g].double().cpu().numpy()
+                    V = vb[layer, g].double().cpu().numpy()
+                    ora = oracle_unit(hist[layer, g * G:(g + 1) * G], K, V, B, P)
+                    assert_scores_close(ev.scores[layer, g].double().cpu().numpy(), ora["scores"],
+                                        f"event {step} request {s} unit ({layer}, {g})")
+                    gidx = ev.idx[layer, g, 0].cpu().numpy()
+                    assert_selection(gidx, cap, B, ora["scores"], ora["idx"])
+                    sel = torch.as_tensor(gidx[:B], dtype=torch.long, device=DEV)
+                    after_k, after_v = ev.k[s, layer, g], ev.v[s, layer, g]
+                    assert_rows_bitwise(kb[layer, g][sel], after_k[:B])
+                    assert_rows_bitwise(vb[layer, g][sel], after_v[:B])
+                    assert_rows_bitwise(kb[layer, g][B:], after_k[B:])  # the free rows are left alone
+                    assert_rows_bitwise(vb[layer, g][B:], after_v[B:])
+                    np.testing.assert_array_equal(ev.pos[s, layer, g, :B].cpu().numpy(), pb[layer, g][gidx[:B]])
+    # the schedule of every request is decode_run's (it does not depend on scores)
+    for s in range(S):
+        r = cu[s]
+        Kr = t.k[0, 0, r:r + n0s[s] + T].double().cpu().numpy()
+        Vr = t.v[0, 0, r:r + n0s[s] + T].double().cpu().numpy()
+        steps = [(q_all[s, 0, :G, w + j], Kr[n0s[s] + j], Vr[n0s[s] + j]) for j in range(T)]
+        events, ids, _, _ = decode_run(q_all[s, 0, :G, :w], Kr[:n0s[s]], Vr[:n0s[s]], steps, B, D, P)
+        assert [e["step"] for e in events] == event_steps[s]
+        assert ev.lengths[s] == len(ids)
+    assert ev.events == sum(len(v) for v in event_steps.values()) > 0
+
+
+def test_compaction_refuses_positions_that_do_not_ascend():
+    # a hand-made index list with a repeat: the unit is left untouched and the
+    # status word says invalid argument (no out-of-range access is possible:
+    # the positions are checked before any row moves)
+    from paper_2609_08131_gb300 import JACAP_ERR_INVALID_ARG, jacap_compact_inplace, jacap_device_status
+    from paper_2609_08131_gb300.api import _ptr, _stream
+
+    ev = DecodeEvictor(1, 1, 2, 2, 4, 4, dtype=torch.bfloat16, device=DEV)
+    ev.k.normal_()
+    ev.v.normal_()
+    before = ev.k.clone()
+    ev.idx[:] = torch.tensor([0, 2, 2, 5], dtype=torch.int32, device=DEV)
+    ev.ws.zero_()
+    st = jacap_compact_inplace(ev.slot, _ptr(ev.k[0]), _ptr(ev.v[0]), _ptr(ev.pos[0]), _ptr(ev.idx), 4, _ptr(ev.ws),
+                               ev.ws.numel(), _stream())
+    assert st == 0
+    assert jacap_device_status(_ptr(ev.ws), _stream()) == JACAP_ERR_INVALID_ARG
+    assert torch.equal(ev.k, before)
