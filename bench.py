@@ -49,6 +49,12 @@ def parse():
                         "window covariance (App. B.2)")
     p.add_argument("--out-proj", type=int, default=0, metavar="D_O",
                    help="use true output directions u = W v with synthetic W (D_O x 128) per plane")
+    p.add_argument("--decode", type=int, default=0, metavar="B",
+                   help="measure decoding-stage eviction instead: one Llama-3-8B-shaped request whose cache slot "
+                        "of B + interval tokens is scored with running query statistics and compacted to B")
+    p.add_argument("--interval", type=int, default=128, help="decoding-stage eviction interval (tokens)")
+    p.add_argument("--preserve-order", action="store_true",
+                   help="decoding-stage eviction: compact to ascending slot order instead of filling the holes")
     p.add_argument("--e2e-steps", type=int, default=10)
     p.add_argument("--cpu-seconds", type=float, default=15.0)
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -474,10 +480,103 @@ def run_e2e(args, ev, t, stream, world, dist):
             "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": n}
 
 
+def run_decode(args):
+    """Decoding-stage eviction events (reading R16) on one GPU.
+
+    One request of the Llama-3-8B shape (32 layers, 32 query / 8 KV heads)
+    with a full slot of B + interval tokens; each timed step is one eviction
+    event: the scoring pass with running statistics, TOP-B and the in-place
+    compaction. After an event the slot is marked full again (its free rows
+    still hold earlier tokens), so every event scores B + interval tokens."""
+    import torch
+
+    from paper_2609_08131_gb300 import SCORE_KERNEL_NAMES, jacap_params
+    from paper_2609_08131_gb300.api import DecodeEvictor
+    from paper_2609_08131_gb300.workloads import Workload, generate
+
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", "0")))
+    torch.cuda.set_device(dev)
+    B, D = args.decode, args.interval
+    cap = B + D
+    L, Hq, Hkv, w = 32, 32, 8, 32
+    wl = Workload(f"decoding-stage eviction, Llama-3-8B-shaped, reserved tokens B={B}, interval {D}", L, Hq, Hkv,
+                  (cap,), w + 1, B, seed=40)
+    t = generate(wl, dev)
+    ev = DecodeEvictor(1, L, Hq, Hkv, B, D, dtype=t.k.dtype, params=jacap_params(), device=dev,
+                       preserve_order=args.preserve_order)
+    ev.start(t.k[:, :, :cap - 1].unsqueeze(0), t.v[:, :, :cap - 1].unsqueeze(0),
+             t.q_win[:, :, :, :w].contiguous(), [cap - 1])
+    q_new = t.q_win[:, :, :, w].contiguous()
+    ev.append(t.k[:, :, cap - 1].unsqueeze(0), t.v[:, :, cap - 1].unsqueeze(0), q_new)
+    stream = torch.cuda.current_stream(dev)
+    for _ in range(max(3, args.warmup)):
+        ev.lengths[0] = cap
+        ev.evict(0)
+    ev.check()
+    K = args.steps
+    nk = len(SCORE_KERNEL_NAMES)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(nk + 3)] for _ in range(K)]
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    for e in [x for row in evs for x in row] + [start, stop]:
+        e.record(stream)
+    torch.cuda.synchronize()
+    sampler = ClockSampler(dev.index)
+    sampler.start()
+    start.record(stream)
+    for i in range(K):
+        ev.lengths[0] = cap
+        ev.evict(0, events=evs[i][:nk + 1], tail=evs[i][nk + 1:])
+    stop.record(stream)
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    ev.check()
+    t_ms = start.elapsed_time(stop) / K
+    kern = {name: sum(evs[i][j].elapsed_time(evs[i][j + 1]) for i in range(K)) / K
+            for j, name in enumerate(SCORE_KERNEL_NAMES)}
+    kern["select"] = sum(evs[i][nk].elapsed_time(evs[i][nk + 1]) for i in range(K)) / K
+    kern["compact_inplace"] = sum(evs[i][nk + 1].elapsed_time(evs[i][nk + 2]) for i in range(K)) / K
+    # one decode step's statistics update (one query per layer and head)
+    M = 200
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(M):
+        ev.merge_queries(q_new)
+    b.record(stream)
+    torch.cuda.synchronize()
+    upd_us = a.elapsed_time(b) / M * 1e3
+    kv_bytes = 2 * L * Hkv * cap * 128 * t.k.element_size()
+    line = {
+        "mode": "decode",
+        "metric": "decoding-stage eviction: cached tokens x layers scored per second (1 GB300)",
+        "value": cap * L / (t_ms * 1e-3),
+        "unit": "tokens/s",
+        "ms_per_event": t_ms,
+        "n_gpus": 1,
+        "steps": K,
+        "warmup": args.warmup,
+        "higher_is_better": True,
+        "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": wl.name, "layers": L, "q_heads": Hq, "kv_heads": Hkv, "head_dim": 128,
+                   "slot_tokens": cap, "budget": B, "interval": D, "statistics": "running, all queries seen",
+                   "compaction": "ascending order" if args.preserve_order else "hole filling",
+                   "l2": f"inputs larger than L2: each event reads K and V of the slot ({kv_bytes / 1e6:.0f} MB)"},
+        "kernel_ms": kern,
+        "stats_update_us_per_decode_step": upd_us,
+        "event_hbm_fraction": {"kv_bytes": kv_bytes, "of_8tbs": kv_bytes / (t_ms * 1e-3) / 8e12},
+        "clocks": clocks,
+        "gpu_launches_per_event": nk + 3,  # plan is two launches; select, in-place compaction
+    }
+    print(json.dumps(line))
+    return 0
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         return run_reference(args)
+    if args.decode:
+        return run_decode(args)
     return run_ours(args)
 
 

@@ -274,24 +274,32 @@ jacap_status jacap_score_stats(const jacap_layout* layout, const jacap_params* p
                                void* const* events, int32_t num_events);
 
 /*
- * The retained cache in place: for every unit the rows idx[0 .. kept - 1]
- * (relative to cu[s], as produced by jacap_select) of K and V move, bit for
- * bit, to rows 0 .. kept - 1 of the request's token range; rows from kept on
+ * The retained cache in place: for every unit the kept rows idx[0 .. kept - 1]
+ * (relative to cu[s], as produced by jacap_select) of K and V end up, bit for
+ * bit, in rows 0 .. kept - 1 of the request's token range; rows from kept on
  * are left as they were (free for the next tokens). kept = min(n_s, budget).
  *  k, v  device, the layout; written in place.
  *  pos   device int32 [num_layers][num_kv_heads][total_tokens] or NULL: a
  *        per-token tag (e.g. the original position) moved with the rows.
+ *  preserve_order
+ *        1: row r receives idx[r] (ascending order, as jacap_compact); up to
+ *           `kept` rows move, in chunks that are read whole before any row of
+ *           the chunk is written, which cannot overwrite a row still to be
+ *           read because idx[r] >= r.
+ *        0: hole filling: kept rows below `kept` stay in place and the kept
+ *           rows at or above `kept` move, in ascending order, into the evicted
+ *           rows below `kept`, in ascending order; at most n_s - kept rows
+ *           move (the order of a cache does not matter to attention once the
+ *           positions are encoded in the keys; `pos` keeps them).
  *  ws    the workspace of jacap_score for this layout (status word).
  * The kept positions of every unit must ascend strictly within [0, n_s) (as
  * jacap_select emits them); a unit where they do not is left untouched and
  * JACAP_ERR_INVALID_ARG is recorded in the status word. Units run
- * concurrently; each moves its rows in chunks that are read whole before any
- * row of the chunk is written, which cannot overwrite a row still to be read
- * because idx[r] >= r.
+ * concurrently.
  */
 jacap_status jacap_compact_inplace(const jacap_layout* layout, void* k, void* v, int32_t* pos,
-                                   const int32_t* idx, int32_t budget, void* ws, size_t ws_bytes,
-                                   void* stream);
+                                   const int32_t* idx, int32_t budget, int32_t preserve_order,
+                                   void* ws, size_t ws_bytes, void* stream);
 
 /* Synchronises `stream`, then reads the workspace status word: JACAP_OK or the
  * first device-side error recorded since the last jacap_score on `ws`. */

@@ -96,8 +96,8 @@ _SIGS = {
                                          _P, _P, _P, ctypes.c_size_t, _P, ctypes.POINTER(ctypes.c_void_p),
                                          ctypes.c_int32]),
     "jacap_stats_update": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, ctypes.c_int32, _P, _P, _P]),
-    "jacap_compact_inplace": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, _P, _P, _P, ctypes.c_int32, _P,
-                                             ctypes.c_size_t, _P]),
+    "jacap_compact_inplace": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, _P, _P, _P, ctypes.c_int32,
+                                             ctypes.c_int32, _P, ctypes.c_size_t, _P]),
     "jacap_device_status": (ctypes.c_int, [_P, _P]),
     "jacap_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "jacap_workspace_offsets": (ctypes.c_int, [ctypes.POINTER(jacap_layout), ctypes.c_int32,
@@ -154,8 +154,9 @@ def jacap_stats_update(layout, q_new, reset, stats, counts, stream) -> int:
     return lib().jacap_stats_update(ctypes.byref(layout), q_new, int(reset), stats, counts, stream)
 
 
-def jacap_compact_inplace(layout, k, v, pos, idx, budget, ws, ws_bytes, stream) -> int:
-    return lib().jacap_compact_inplace(ctypes.byref(layout), k, v, pos, idx, budget, ws, ws_bytes, stream)
+def jacap_compact_inplace(layout, k, v, pos, idx, budget, preserve_order, ws, ws_bytes, stream) -> int:
+    return lib().jacap_compact_inplace(ctypes.byref(layout), k, v, pos, idx, budget, int(preserve_order), ws,
+                                       ws_bytes, stream)
 
 
 JACAP_STATIC_SCRATCH_BYTES = 64 << 20

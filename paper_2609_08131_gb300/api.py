@@ -203,7 +203,9 @@ class DecodeEvictor:
     far; the decoding experiments of Sec. 4): one cache slot of
     ``budget + interval`` tokens per request and running query statistics.
     Whenever a request's cache reaches budget + interval tokens it is scored
-    with those statistics and compacted in place back to ``budget`` tokens.
+    with those statistics and compacted in place back to ``budget`` tokens
+    (by default by moving the kept rows from past the budget into the evicted
+    rows, so the slot order is not the token order; ``pos`` records it).
 
     Buffers (device):
       k, v    [S, L, Hkv, cap, 128], cap = budget + interval; request s holds
@@ -218,7 +220,12 @@ class DecodeEvictor:
     """
 
     def __init__(self, num_seqs: int, num_layers: int, num_q_heads: int, num_kv_heads: int, budget: int,
-                 interval: int, dtype=torch.bfloat16, params: jacap_params | None = None, device="cuda"):
+                 interval: int, dtype=torch.bfloat16, params: jacap_params | None = None, device="cuda",
+                 preserve_order: bool = False):
+        """``preserve_order``: keep the retained rows in ascending slot order
+        (moves up to ``budget`` rows per eviction) instead of filling the
+        evicted rows with the kept rows from past the budget (moves at most
+        ``interval`` rows)."""
         if budget < 1 or interval < 1:
             raise ValueError("budget and interval must be >= 1")
         if dtype not in (torch.bfloat16, torch.float32):
@@ -228,6 +235,7 @@ class DecodeEvictor:
         self.cap = self.budget + self.interval
         self.dtype = dtype
         self.params = params if params is not None else jacap_params()
+        self.preserve_order = bool(preserve_order)
         dev = torch.device(device)
         S, L, Hq, Hkv, cap, d = self.S, self.L, self.Hq, self.Hkv, self.cap, 128
         self.k = torch.zeros((S, L, Hkv, cap, d), dtype=dtype, device=dev)
@@ -241,6 +249,8 @@ class DecodeEvictor:
         self.cu = torch.tensor([0, cap], dtype=torch.int32, device=dev)
         # one request's slot as a cache of cap tokens
         self.slot = self._layout(1, window=1, q_strides=(d, d, d, d))
+        # one query per (request, layer, head), [S, L, Hq, 128] contiguous
+        self.step_layout = self._layout(S, window=1, q_strides=(L * Hq * d, Hq * d, d, d))
         nbytes = jacap_workspace_size(self.slot, self.budget)
         if nbytes == 0:
             raise JacapError(1, "jacap_workspace_size")
@@ -300,26 +310,42 @@ class DecodeEvictor:
             self.pos[s, :, :, t] = self.next_id[s]
             self.lengths[s] += 1
             self.next_id[s] += 1
-        self._merge(q_new.unsqueeze(3), reset=False, stream=stream)
+        self.merge_queries(q_new, stream)
         return [s for s in range(self.S) if self.lengths[s] >= self.cap]
 
-    def evict(self, s: int, stream=None):
+    def merge_queries(self, q_new, stream=None):
+        """Merge one decode step's queries [S, L, Hq, 128] into the running statistics."""
+        if q_new.is_contiguous() and q_new.dtype == self.dtype and tuple(q_new.shape) == (self.S, self.L, self.Hq, 128):
+            _check(jacap_stats_update(self.step_layout, _ptr(q_new), 0, _ptr(self.stats), _ptr(self.counts),
+                                      _stream(stream)), "jacap_stats_update")
+        else:
+            self._merge(q_new.unsqueeze(3), reset=False, stream=stream)
+
+    def evict(self, s: int, stream=None, events=None, tail=None):
         """Score request s's full slot with the running statistics, select the
-        budget best tokens and compact them in place to rows 0 .. budget - 1."""
+        budget best tokens and compact them in place to rows 0 .. budget - 1.
+        ``events``: JACAP_SCORE_KERNELS + 1 torch.cuda.Event recorded around
+        the scoring kernels; ``tail``: two more, recorded after the selection
+        and after the compaction."""
         if self.lengths[s] != self.cap:
             raise RuntimeError("only a full slot is evicted")
         lay, st = self.slot, _stream(stream)
+        handles = [e.cuda_event for e in events] if events is not None else []
         off_stats = s * self.L * self.Hq * 2 * 128 * 4
         off_counts = s * self.L * self.Hq * 4
         stats = ctypes.c_void_p(self.stats.data_ptr() + off_stats)
         counts = ctypes.c_void_p(self.counts.data_ptr() + off_counts)
         k, v, pos = _ptr(self.k[s]), _ptr(self.v[s]), _ptr(self.pos[s])
         _check(jacap_score_stats(lay, self.params, stats, counts, k, v, _ptr(self.scores), _ptr(self.ws),
-                                 self.ws.numel(), st), "jacap_score_stats")
+                                 self.ws.numel(), st, handles), "jacap_score_stats")
         _check(jacap_select(lay, _ptr(self.scores), self.budget, _ptr(self.idx), _ptr(self.kept), _ptr(self.ws),
                             self.ws.numel(), st), "jacap_select")
-        _check(jacap_compact_inplace(lay, k, v, pos, _ptr(self.idx), self.budget, _ptr(self.ws), self.ws.numel(),
-                                     st), "jacap_compact_inplace")
+        if tail is not None:
+            tail[0].record(stream)
+        _check(jacap_compact_inplace(lay, k, v, pos, _ptr(self.idx), self.budget, self.preserve_order, _ptr(self.ws),
+                                     self.ws.numel(), st), "jacap_compact_inplace")
+        if tail is not None:
+            tail[1].record(stream)
         self.lengths[s] = self.budget
         self.events += 1
 

@@ -341,10 +341,12 @@ jacap_status jacap_stats_update(const jacap_layout* layout, const void* q_new, i
 }
 
 jacap_status jacap_compact_inplace(const jacap_layout* layout, void* k, void* v, int32_t* pos, const int32_t* idx,
-                                   int32_t budget, void* ws, size_t ws_bytes, void* stream) {
+                                   int32_t budget, int32_t preserve_order, void* ws, size_t ws_bytes, void* stream) {
   jacap_status st = check_layout(layout);
   if (st != JACAP_OK) return st;
-  if (k == nullptr || v == nullptr || idx == nullptr || ws == nullptr || budget < 1) return JACAP_ERR_INVALID_ARG;
+  if (k == nullptr || v == nullptr || idx == nullptr || ws == nullptr || budget < 1 ||
+      (preserve_order != 0 && preserve_order != 1))
+    return JACAP_ERR_INVALID_ARG;
   if (!aligned16(k) || !aligned16(v) || ((uintptr_t)idx & 3u) != 0 || ((uintptr_t)pos & 3u) != 0)
     return JACAP_ERR_INVALID_ARG;
   if ((int64_t)layout->num_layers * layout->num_kv_heads * layout->num_seqs >= ((int64_t)1 << 31))
@@ -356,7 +358,8 @@ jacap_status jacap_compact_inplace(const jacap_layout* layout, void* k, void* v,
   int sms = 0;
   if ((st = check_device(&sms)) != JACAP_OK) return st;
   return map_cuda(launch_compact_inplace(dm, make_ws(ws, c), layout->dtype == JACAP_BF16 ? 1 : 0,
-                                         layout->cu_seqlens, k, v, pos, idx, budget, (cudaStream_t)stream));
+                                         layout->cu_seqlens, k, v, pos, idx, budget, preserve_order,
+                                         (cudaStream_t)stream));
 }
 
 jacap_status jacap_select(const jacap_layout* layout, const float* scores, int32_t budget, int32_t* idx,

@@ -31,6 +31,7 @@ cudaError_t launch_stats_update(const Dims& dm, int dtype, const void* q, float*
 cudaError_t launch_stats_moments(const Dims& dm, const Ws& ws, const float* stats, const int32_t* counts,
                                  cudaStream_t st);
 cudaError_t launch_compact_inplace(const Dims& dm, const Ws& ws, int dtype, const int32_t* cu, void* k, void* v,
-                                   int32_t* pos, const int32_t* idx, int budget, cudaStream_t st);
+                                   int32_t* pos, const int32_t* idx, int budget, int preserve_order,
+                                   cudaStream_t st);
 
 }  // namespace jacap

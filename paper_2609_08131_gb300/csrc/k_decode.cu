@@ -13,12 +13,22 @@
 // scoring pass reads mu = m and lambda = M2 / n (or M2 / (n - 1)) instead of
 // window statistics.
 //
-// After the TOP-B selection the cache of a request is compacted in place: the
-// kept rows move to the front of the request's token range. One CTA owns one
-// unit and moves its rows in chunks; every chunk is read completely before any
-// of it is written (a barrier in between). Because the kept positions ascend
-// strictly from 0, idx[r] >= r, so a chunk's writes (rows c0 .. c0 + CH - 1)
-// never touch a row that a later chunk still has to read (rows >= c0 + CH).
+// After the TOP-B selection the cache of a request is compacted in place so
+// that the kept rows occupy rows 0 .. kept - 1 of the request's range, in one
+// of two ways (one CTA per unit in both):
+//  - ascending order (the order of jacap_compact): every kept row moves to
+//    its rank. The rows move in chunks; every chunk is read completely before
+//    any of it is written (a barrier in between). Because the kept positions
+//    ascend strictly from 0, idx[r] >= r, so a chunk's writes (rows c0 ..
+//    c0 + CH - 1) never touch a row that a later chunk still has to read
+//    (rows >= c0 + CH). Up to `kept` rows move.
+//  - hole filling: kept rows below `kept` stay where they are; the kept rows
+//    at or above `kept` move, in ascending order, into the evicted rows below
+//    `kept`, in ascending order. Sources and destinations are disjoint, so all
+//    copies run at once, and at most n - kept rows move (the eviction interval
+//    during decoding, instead of the whole budget). If f kept positions lie
+//    below `kept`, the evicted row r between the (i-1)-th and i-th of them is
+//    hole number r - i and receives row idx[f + r - i].
 #include "jacap_dev.cuh"
 #include "jacap_internal.h"
 
@@ -149,6 +159,59 @@ __global__ void __launch_bounds__(CI_THREADS)
   }
 }
 
+// Hole filling (see the header comment). c(p) = idx[p] - p counts the evicted
+// rows below kept position p and does not decrease, so hole j lies after the
+// i = #{p < f : c(p) <= j} kept positions below it, at row j + i. One warp per
+// hole (lanes over the 16-byte pieces of the row); the holes are independent.
+template <typename T>
+__global__ void __launch_bounds__(CI_THREADS)
+    fill_holes_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu, T* k, T* v, int32_t* pos,
+                      const int32_t* __restrict__ idx, int budget) {
+  constexpr int RB = D * (int)sizeof(T) / 16;
+  __shared__ int s_f;
+  if (status_failed(ws)) return;
+  const int u = blockIdx.x;
+  const int s = u % dm.S, plane = u / dm.S;
+  const int l = plane / dm.Hkv, g = plane % dm.Hkv;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t t0 = cu[s];
+  const int64_t n = (int64_t)cu[s + 1] - t0;
+  const int kept = (int)(n < (int64_t)budget ? n : (int64_t)budget);
+  const int32_t* ix = idx + (int64_t)u * budget;
+  if (tid == 0) s_f = 0;
+  __syncthreads();
+  int bad = 0;
+  for (int r = tid; r < kept; r += CI_THREADS) {
+    const int32_t x = ix[r];
+    bad |= x < 0 || (int64_t)x >= n || (r > 0 && x <= ix[r - 1]);
+    // f = the number of kept positions below `kept`
+    if (x < kept && (r + 1 == kept || ix[r + 1] >= kept)) s_f = r + 1;
+  }
+  if (__syncthreads_or(bad)) {
+    if (tid == 0) flag(ws, ST_INVALID);
+    return;
+  }
+  const int f = s_f, holes = kept - f;
+  const int64_t rowoff = (int64_t)l * dm.kv_sl + (int64_t)g * dm.kv_sh;
+  uint4* kb = (uint4*)(k + rowoff);
+  uint4* vb = (uint4*)(v + rowoff);
+  const int64_t st16 = dm.kv_st * (int64_t)sizeof(T) / 16;
+  int32_t* pb = pos != nullptr ? pos + (int64_t)plane * dm.Ntot : nullptr;
+  for (int j = warp; j < holes; j += CI_THREADS / 32) {
+    int lo = 0, hi = f;  // first p in [0, f) with c(p) > j (f if none)
+    while (lo < hi) {
+      const int mid = (lo + hi) >> 1;
+      if (ix[mid] - mid <= j) lo = mid + 1; else hi = mid;
+    }
+    const int64_t dst = t0 + j + lo, src = t0 + ix[f + j];
+    for (int piece = lane; piece < RB; piece += 32) {
+      kb[dst * st16 + piece] = kb[src * st16 + piece];
+      vb[dst * st16 + piece] = vb[src * st16 + piece];
+    }
+    if (pb != nullptr && lane == 0) pb[dst] = pb[src];
+  }
+}
+
 template <typename T>
 static cudaError_t launch_stats_update_t(const Dims& dm, const void* q, float* stats, int32_t* counts, int reset,
                                          cudaStream_t st) {
@@ -169,8 +232,17 @@ cudaError_t launch_stats_moments(const Dims& dm, const Ws& ws, const float* stat
 }
 
 cudaError_t launch_compact_inplace(const Dims& dm, const Ws& ws, int dtype, const int32_t* cu, void* k, void* v,
-                                   int32_t* pos, const int32_t* idx, int budget, cudaStream_t st) {
+                                   int32_t* pos, const int32_t* idx, int budget, int preserve_order,
+                                   cudaStream_t st) {
   const int units = dm.L * dm.Hkv * dm.S;
+  if (!preserve_order) {
+    if (dtype == 1)
+      fill_holes_kernel<__nv_bfloat16><<<units, CI_THREADS, 0, st>>>(dm, ws, cu, (__nv_bfloat16*)k,
+                                                                     (__nv_bfloat16*)v, pos, idx, budget);
+    else
+      fill_holes_kernel<float><<<units, CI_THREADS, 0, st>>>(dm, ws, cu, (float*)k, (float*)v, pos, idx, budget);
+    return cudaGetLastError();
+  }
   if (dtype == 1)
     compact_inplace_kernel<__nv_bfloat16><<<units, CI_THREADS, 0, st>>>(
         dm, ws, cu, (__nv_bfloat16*)k, (__nv_bfloat16*)v, pos, idx, budget);

@@ -28,12 +28,31 @@ pytestmark = pytest.mark.gpu
 DEV = "cuda:0"
 
 CASES = {
-    # name: (layers, Hq, Hkv, prefill lengths, window, steps, budget, interval, dtype, params, seed)
-    "bf16_gqa4": (2, 8, 2, (40, 63), 8, 70, 48, 16, "bf16", jacap_params(), 31),
-    "bf16_gqa2_interval1": (1, 4, 2, (30,), 4, 12, 32, 1, "bf16", jacap_params(tau=2.0), 32),
-    "f32_mha_unbiased": (1, 4, 4, (10, 24), 4, 30, 20, 5, "f32", jacap_params(cov_unbiased=1, tau=3.0), 33),
-    "bf16_gqa8_long_slot": (1, 8, 1, (700,), 16, 40, 512, 200, "bf16", jacap_params(), 34),
+    # name: (layers, Hq, Hkv, prefill lengths, window, steps, budget, interval, dtype, params, seed, preserve_order)
+    "bf16_gqa4": (2, 8, 2, (40, 63), 8, 70, 48, 16, "bf16", jacap_params(), 31, False),
+    "bf16_gqa4_ordered": (2, 8, 2, (40, 63), 8, 70, 48, 16, "bf16", jacap_params(), 31, True),
+    "bf16_gqa2_interval1": (1, 4, 2, (30,), 4, 12, 32, 1, "bf16", jacap_params(tau=2.0), 32, False),
+    "f32_mha_unbiased": (1, 4, 4, (10, 24), 4, 30, 20, 5, "f32", jacap_params(cov_unbiased=1, tau=3.0), 33, False),
+    "f32_mha_unbiased_ordered": (1, 4, 4, (10, 24), 4, 30, 20, 5, "f32", jacap_params(cov_unbiased=1, tau=3.0), 33,
+                                 True),
+    "bf16_gqa8_long_slot": (1, 8, 1, (700,), 16, 40, 512, 200, "bf16", jacap_params(), 34, False),
+    "bf16_gqa8_long_slot_ordered": (1, 8, 1, (700,), 16, 40, 512, 200, "bf16", jacap_params(), 34, True),
 }
+
+
+def _arrangement(gidx, B, preserve_order):
+    """Slot row r after the compaction holds pre-compaction row out[r]."""
+    kept = [int(x) for x in gidx[:B]]
+    if preserve_order:
+        return kept
+    out = list(range(B))
+    front = {x for x in kept if x < B}
+    holes = [r for r in range(B) if r not in front]
+    back = [x for x in kept if x >= B]
+    assert len(holes) == len(back)
+    for r, x in zip(holes, back):
+        out[r] = x
+    return out
 
 
 def _oracle_params(p):
@@ -43,7 +62,7 @@ def _oracle_params(p):
 
 @pytest.mark.parametrize("name", list(CASES))
 def test_decode_evictions_match_the_oracle_event_by_event(name):
-    L, Hq, Hkv, n0s, w, T, B, D, dtype, params, seed = CASES[name]
+    L, Hq, Hkv, n0s, w, T, B, D, dtype, params, seed, ordered = CASES[name]
     S, G, cap = len(n0s), Hq // Hkv, B + D
     wl = Workload("decode stream", L, Hq, Hkv, tuple(n + T for n in n0s), w + T, B, dtype=dtype, seed=seed)
     t = generate(wl, DEV)
@@ -54,7 +73,7 @@ def test_decode_evictions_match_the_oracle_event_by_event(name):
     for s, n in enumerate(n0s):
         k0[s, :, :, :n] = t.k[:, :, cu[s]:cu[s] + n]
         v0[s, :, :, :n] = t.v[:, :, cu[s]:cu[s] + n]
-    ev = DecodeEvictor(S, L, Hq, Hkv, B, D, dtype=tdt, params=params, device=DEV)
+    ev = DecodeEvictor(S, L, Hq, Hkv, B, D, dtype=tdt, params=params, device=DEV, preserve_order=ordered)
     ev.start(k0, v0, t.q_win[:, :, :, :w].contiguous(), list(n0s))
     q_all = t.q_win.double().cpu().numpy()  # [S, L, Hq, w + T, d]
     P = _oracle_params(params)
@@ -86,13 +105,14 @@ def test_decode_evictions_match_the_oracle_event_by_event(name):
                                         f"event {step} request {s} unit ({layer}, {g})")
                     gidx = ev.idx[layer, g, 0].cpu().numpy()
                     assert_selection(gidx, cap, B, ora["scores"], ora["idx"])
-                    sel = torch.as_tensor(gidx[:B], dtype=torch.long, device=DEV)
+                    sel = torch.as_tensor(_arrangement(gidx, B, ordered), dtype=torch.long, device=DEV)
                     after_k, after_v = ev.k[s, layer, g], ev.v[s, layer, g]
                     assert_rows_bitwise(kb[layer, g][sel], after_k[:B])
                     assert_rows_bitwise(vb[layer, g][sel], after_v[:B])
                     assert_rows_bitwise(kb[layer, g][B:], after_k[B:])  # the free rows are left alone
                     assert_rows_bitwise(vb[layer, g][B:], after_v[B:])
-                    np.testing.assert_array_equal(ev.pos[s, layer, g, :B].cpu().numpy(), pb[layer, g][gidx[:B]])
+                    np.testing.assert_array_equal(ev.pos[s, layer, g, :B].cpu().numpy(), pb[layer, g][sel.cpu().numpy()])
+                    assert sorted(sel.tolist()) == [int(x) for x in gidx[:B]]
     # the schedule of every request is decode_run's (it does not depend on scores)
     for s in range(S):
         r = cu[s]
@@ -117,9 +137,10 @@ def test_compaction_refuses_positions_that_do_not_ascend():
     ev.v.normal_()
     before = ev.k.clone()
     ev.idx[:] = torch.tensor([0, 2, 2, 5], dtype=torch.int32, device=DEV)
-    ev.ws.zero_()
-    st = jacap_compact_inplace(ev.slot, _ptr(ev.k[0]), _ptr(ev.v[0]), _ptr(ev.pos[0]), _ptr(ev.idx), 4, _ptr(ev.ws),
-                               ev.ws.numel(), _stream())
-    assert st == 0
-    assert jacap_device_status(_ptr(ev.ws), _stream()) == JACAP_ERR_INVALID_ARG
-    assert torch.equal(ev.k, before)
+    for ordered in (0, 1):
+        ev.ws.zero_()
+        st = jacap_compact_inplace(ev.slot, _ptr(ev.k[0]), _ptr(ev.v[0]), _ptr(ev.pos[0]), _ptr(ev.idx), 4, ordered,
+                                   _ptr(ev.ws), ev.ws.numel(), _stream())
+        assert st == 0
+        assert jacap_device_status(_ptr(ev.ws), _stream()) == JACAP_ERR_INVALID_ARG
+        assert torch.equal(ev.k, before)
