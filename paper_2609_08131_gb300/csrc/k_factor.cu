@@ -86,10 +86,12 @@ __global__ void __launch_bounds__(FA_THREADS, PROJ ? 1 : 2)
 #pragma unroll
     for (int a = 0; a < FA_ROWS; ++a) z[a][0] = z[a][1] = make_float2(0.f, 0.f);
     for (int ch = ch0; ch < ch1; ++ch) {  // 16 independent 16-byte loads in flight per chunk
-      // partial layout: (m, n) at ((n / 32) D + m) 32 + n % 32
+      // partial layout: (m, n) at ((n / 32) D + m) 32 + n % 32; only the
+      // lower 32 x 32 blocks are stored (rows ty + 8 a lie in block a / 4)
       const float* src = gp + (int64_t)ch * D * D + (c0 >> 5) * D * 32 + (c0 & 31);
 #pragma unroll
       for (int a = 0; a < FA_ROWS; ++a) {
+        if (a / 4 < (c0 >> 5)) continue;
         const float4 v = *(const float4*)(src + (ty + 8 * a) * 32);
         z[a][0].x += v.x;
         z[a][0].y += v.y;
@@ -97,11 +99,26 @@ __global__ void __launch_bounds__(FA_THREADS, PROJ ? 1 : 2)
         z[a][1].y += v.w;
       }
     }
+    // the upper blocks by symmetry, through the staging matrix
 #pragma unroll
     for (int a = 0; a < FA_ROWS; ++a) {
       const int i = ty + 8 * a;
+      if (a / 4 < (c0 >> 5)) continue;
+      Ms[i * FA_LD + c0] = z[a][0].x;
+      Ms[i * FA_LD + c0 + 1] = z[a][0].y;
+      Ms[i * FA_LD + c0 + 2] = z[a][1].x;
+      Ms[i * FA_LD + c0 + 3] = z[a][1].y;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int a = 0; a < FA_ROWS; ++a) {
+      const int i = ty + 8 * a;
+      if (a / 4 < (c0 >> 5))
+        z[a][0] = make_float2(Ms[c0 * FA_LD + i], Ms[(c0 + 1) * FA_LD + i]),
+        z[a][1] = make_float2(Ms[(c0 + 2) * FA_LD + i], Ms[(c0 + 3) * FA_LD + i]);
       *(float4*)(gout + i * D + c0) = make_float4(z[a][0].x, z[a][0].y, z[a][1].x, z[a][1].y);
     }
+    __syncthreads();
   }
   if constexpr (PROJ) {
     // M = F G F^T: G and F to shared memory (stride FA_LD), then two products
@@ -317,6 +334,329 @@ __global__ void __launch_bounds__(FA_THREADS, PROJ ? 1 : 2)
   if (tid == 0 && s_bad) flag(ws, ST_NONFINITE);
 }
 
+// ------------------------------------------------------------ blocked ------
+// The proxy path (u = v) factors A with a blocked right-looking Cholesky on
+// 32 x 32 blocks (I, J = 0..3) and inverts the factor blockwise, so the
+// sequential part is four 32-step eliminations inside one warp instead of
+// 128 block-wide steps:
+//  for K = 0..3:
+//    T_KK = L_KK^{-1}   one warp: the forward elimination above on the 32 x 32
+//                       block A_KK (its lower triangle), X_KK -> T_KK
+//    L_IK = A_IK T_KK^T                 I > K
+//    A_IJ -= L_IK L_JK^T                K < J <= I
+//  X = L^{-1}:  X_II = T_II,  X_IJ = -T_II sum_{M=J}^{I-1} L_IM X_MJ   (I > J,
+//  by increasing I - J).
+// Every product is a 32 x 32 block of "rows times rows" (P Q^T) read from
+// shared memory with row stride FB_LD; the inverse is built transposed
+// (XT_JI = X_IJ^T) so its products have that form too. Thread t owns the
+// outputs (a + 16 p, b + 16 q), a = t / 16, b = t % 16, p, q in {0, 1}.
+constexpr int FB_THREADS = 256;
+constexpr int FB_LD = 36;             // row stride of a 32 x 32 block (floats); 16-byte rows
+constexpr int FB_BLK = 32 * FB_LD;    // floats per block
+// 10 lower blocks of A (then L_IJ, and T_II on the diagonal), 10 blocks of
+// XT (XT_JI at tri(I, J)), 3 scratch blocks
+constexpr size_t FB_SMEM = (size_t)23 * FB_BLK * sizeof(float);
+
+__device__ __forceinline__ int tri(int i, int j) { return i * (i + 1) / 2 + j; }  // block (i, j), j <= i
+// a partial Gram's lower blocks staged in shared memory: column block nb,
+// rows 32 nb .. 127, 32 floats per row, after the segments of blocks < nb
+__host__ __device__ constexpr int fb_seg(int nb) { return 32 * (128 * nb - 16 * nb * (nb - 1)); }
+constexpr int FB_STAGE = fb_seg(4);  // floats per stage (10 blocks of 32 x 32)
+static_assert(2 * FB_STAGE <= 20 * FB_BLK, "the staging ring fits in the A and XT blocks");
+
+// acc[p][q] += sum_m P[a + 16 p][m] Q[b + 16 q][m]
+__device__ __forceinline__ void nt_block(float (&acc)[2][2], const float* P, const float* Q, int a, int b) {
+#pragma unroll
+  for (int m = 0; m < 32; m += 4) {
+    const float4 p0 = *(const float4*)(P + a * FB_LD + m);
+    const float4 p1 = *(const float4*)(P + (a + 16) * FB_LD + m);
+    const float4 q0 = *(const float4*)(Q + b * FB_LD + m);
+    const float4 q1 = *(const float4*)(Q + (b + 16) * FB_LD + m);
+    const float4 pv[2] = {p0, p1}, qv[2] = {q0, q1};
+#pragma unroll
+    for (int i = 0; i < 2; ++i)
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        float t = acc[i][j];
+        t = fmaf(pv[i].x, qv[j].x, t);
+        t = fmaf(pv[i].y, qv[j].y, t);
+        t = fmaf(pv[i].z, qv[j].z, t);
+        t = fmaf(pv[i].w, qv[j].w, t);
+        acc[i][j] = t;
+      }
+  }
+}
+
+// T = L^{-1} of one 32 x 32 diagonal block by the elimination described at the
+// top of the file, in one warp: lane r holds row r in registers and the pivot
+// row comes by shuffles -- its scaled inverse part (columns < k) from lane k,
+// its A part (columns > k) from column k of the rows below, which keeps to the
+// lower triangle of A. Writes T row-major into `blk` and T^T into `tblk`.
+__device__ __forceinline__ void diag_inverse(float* blk, float* tblk, int lane, bool& bad) {
+  float z[32], pk[32];
+#pragma unroll
+  for (int c = 0; c < 32; c += 4) {
+    const float4 v = *(const float4*)(blk + lane * FB_LD + c);
+    z[c] = v.x;
+    z[c + 1] = v.y;
+    z[c + 2] = v.z;
+    z[c + 3] = v.w;
+  }
+#pragma unroll
+  for (int k = 0; k < 32; ++k) {
+    const float p = __shfl_sync(0xffffffffu, z[k], k);
+    pk[k] = p;
+    const float m = lane > k ? z[k] * recip_nr(p) : 0.f;
+#pragma unroll
+    for (int c = 0; c < 32; ++c) {
+      if (c == k) continue;
+      const float r = c < k ? __shfl_sync(0xffffffffu, z[c], k) : __shfl_sync(0xffffffffu, z[k], c);
+      z[c] = fmaf(-m, r, z[c]);
+    }
+  }
+  // T_rc = X_rc / sqrt(p_r), X_rc = -z_c / p_c (c < r), X_rr = 1
+  float pr = 0.f;
+#pragma unroll
+  for (int c = 0; c < 32; ++c) pr = lane == c ? pk[c] : pr;
+  if (!(pr > 0.f) || !isfinite(pr)) bad = true;
+  const float sc = rsqrtf(fmaxf(pr, 1e-30f));
+  float t[32];
+#pragma unroll
+  for (int c = 0; c < 32; ++c) {
+    const float x = c < lane ? -z[c] * recip_nr(pk[c]) : (c == lane ? 1.f : 0.f);
+    t[c] = x * sc;
+    if (!isfinite(t[c])) bad = true;
+  }
+#pragma unroll
+  for (int c = 0; c < 32; c += 4) *(float4*)(blk + lane * FB_LD + c) = make_float4(t[c], t[c + 1], t[c + 2], t[c + 3]);
+#pragma unroll
+  for (int c = 0; c < 32; ++c) tblk[c * FB_LD + lane] = t[c];
+}
+
+// The trailing update of block step K: block i of the pairs K < J <= I < 4 in
+// the order (I, J) = (K+1, K+1), (K+2, K+1), (K+2, K+2), ...
+__device__ __forceinline__ void trailing_pair(int K, int i, int& I, int& J) {
+  I = K + 1;
+  J = K + 1;
+  for (int n = 0; n < i; ++n) {
+    if (J < I) {
+      ++J;
+    } else {
+      ++I;
+      J = K + 1;
+    }
+  }
+}
+
+// A_IJ -= L_IK L_JK^T for the trailing pairs i0 .. i1 - 1 of step K, by
+// `nthr` threads (thread index vt), each taking a thread's share of one block
+__device__ __forceinline__ void trailing_update(float* As, int K, int i0, int i1, int vt, int nthr) {
+  for (int w = vt; w < (i1 - i0) * FB_THREADS; w += nthr) {
+    int I, J;
+    trailing_pair(K, i0 + w / FB_THREADS, I, J);
+    const int t = w % FB_THREADS, a = t >> 4, b = t & 15;
+    float d[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
+    nt_block(d, As + tri(I, K) * FB_BLK, As + tri(J, K) * FB_BLK, a, b);
+    float* o = As + tri(I, J) * FB_BLK;
+#pragma unroll
+    for (int p = 0; p < 2; ++p)
+#pragma unroll
+      for (int q = 0; q < 2; ++q) o[(a + 16 * p) * FB_LD + b + 16 * q] -= d[p][q];
+  }
+}
+
+__global__ void __launch_bounds__(FB_THREADS, 2) factor_blocked_kernel(Dims dm, Ws ws) {
+  extern __shared__ __align__(16) float fsm[];
+  float* As = fsm;                // tri(I, J): A_IJ, then L_IJ (I > J) / T_II (I == J)
+  float* XT = fsm + 10 * FB_BLK;  // tri(I, J): XT_JI = (L^{-1})_IJ^T
+  float* Sc = fsm + 20 * FB_BLK;  // scratch
+  __shared__ __align__(8) uint64_t s_full[2];
+  __shared__ int s_skip, s_bad;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  if (tid == 0) {
+    s_skip = status_failed(ws) ? 1 : 0;
+    s_bad = 0;
+  }
+  __syncthreads();
+  if (s_skip) return;
+  const int u = blockIdx.x;
+  const int plane = u / dm.S, s = u % dm.S;
+  const int ch0 = ws.plan[1 + s], ch1 = ws.plan[2 + s];
+  const float* gp = ws.gpart + ((int64_t)plane * dm.c_cap) * D * D;
+  bool bad = false;
+
+  // A = I + sum of partial Grams (chunk order) over the lower 32 x 32 blocks
+  // (the partials hold only those); G to the workspace and the lower blocks of
+  // A to shared memory. The partials stream through a two-stage ring of bulk
+  // copies (the 4 lower segments of one partial per stage: rows 32 nb .. 127
+  // of column block nb, contiguous in the partial layout) while the threads
+  // add the previous stage. Thread (ty, tx) sums rows ty + 8 a, columns
+  // 4 tx .. 4 tx + 3; rows ty + 8 a lie in block a / 4.
+  float* gout = ws.gram + (int64_t)u * D * D;
+  {
+    if (tid == 0) {
+      for (int i = 0; i < 2; ++i) mbar_init(smem_u32(&s_full[i]), 1);
+      fence_mbar_init();
+    }
+    __syncthreads();
+    auto issue = [&](int ch, int st) {  // one partial into stage st
+      uint8_t* dst = (uint8_t*)(fsm + st * FB_STAGE);
+      const float* src = gp + (int64_t)ch * D * D;
+      mbar_arrive_expect_tx(smem_u32(&s_full[st]), FB_STAGE * 4);
+#pragma unroll
+      for (int nb = 0; nb < 4; ++nb)
+        bulk_g2s(smem_u32(dst + fb_seg(nb) * 4), src + (nb * D + 32 * nb) * 32, (D - 32 * nb) * 32 * 4,
+                 smem_u32(&s_full[st]));
+    };
+    if (tid == 0) {
+      if (ch0 < ch1) issue(ch0, 0);
+      if (ch0 + 1 < ch1) issue(ch0 + 1, 1);
+    }
+    const int ty = tid >> 5, tx = tid & 31, c0 = 4 * tx;
+    const int J = c0 >> 5, c = c0 & 31;
+    float4 z[FA_ROWS];
+#pragma unroll
+    for (int a = 0; a < FA_ROWS; ++a) z[a] = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int ch = ch0; ch < ch1; ++ch) {
+      const int st = (ch - ch0) & 1;
+      if (!mbar_wait(smem_u32(&s_full[st]), ((ch - ch0) >> 1) & 1, ws, nullptr)) bad = true;
+      const float* sb = fsm + st * FB_STAGE + fb_seg(J) + c;
+#pragma unroll
+      for (int a = 0; a < FA_ROWS; ++a) {
+        if (a / 4 < J) continue;  // upper block
+        const float4 v = *(const float4*)(sb + (ty + 8 * a - 32 * J) * 32);
+        z[a].x += v.x;
+        z[a].y += v.y;
+        z[a].z += v.z;
+        z[a].w += v.w;
+      }
+      __syncthreads();  // stage st is read; it may be refilled
+      if (tid == 0 && ch + 2 < ch1) {
+        fence_proxy_async_smem();
+        issue(ch + 2, st);
+      }
+    }
+#pragma unroll
+    for (int a = 0; a < FA_ROWS; ++a) {
+      const int i = ty + 8 * a, I = a / 4;
+      if (I < J) continue;
+      *(float4*)(gout + i * D + c0) = z[a];
+      float4 v = z[a];
+      v.x += i == c0 ? 1.f : 0.f;
+      v.y += i == c0 + 1 ? 1.f : 0.f;
+      v.z += i == c0 + 2 ? 1.f : 0.f;
+      v.w += i == c0 + 3 ? 1.f : 0.f;
+      *(float4*)(As + tri(I, J) * FB_BLK + (i & 31) * FB_LD + c) = v;
+    }
+  }
+  __syncthreads();
+  // the upper blocks of G by symmetry: G_IJ = A_JI^T (I < J), 4 x 4 tiles
+  // transposed in registers
+  for (int e = tid; e < 6 * 64; e += FB_THREADS) {
+    const int ub = e >> 6, si = e & 7, sj = (e >> 3) & 7;
+    const int I = ub < 3 ? 0 : (ub < 5 ? 1 : 2), J = ub < 3 ? ub + 1 : (ub < 5 ? ub - 1 : 3);
+    const float* src = As + tri(J, I) * FB_BLK + (4 * sj) * FB_LD + 4 * si;
+    float4 r[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) r[k] = *(const float4*)(src + k * FB_LD);
+    float* dst = gout + (32 * I + 4 * si) * D + 32 * J + 4 * sj;
+    *(float4*)(dst) = make_float4(r[0].x, r[1].x, r[2].x, r[3].x);
+    *(float4*)(dst + D) = make_float4(r[0].y, r[1].y, r[2].y, r[3].y);
+    *(float4*)(dst + 2 * D) = make_float4(r[0].z, r[1].z, r[2].z, r[3].z);
+    *(float4*)(dst + 3 * D) = make_float4(r[0].w, r[1].w, r[2].w, r[3].w);
+  }
+
+  const int a = tid >> 4, b = tid & 15;
+#pragma unroll 1
+  for (int K = 0; K < 4; ++K) {
+    // (the warp's elimination runs alone: next to multiply-add-heavy warps on
+    // its sub-partition it would get a fraction of the issue slots)
+    if (warp == 0) diag_inverse(As + tri(K, K) * FB_BLK, XT + tri(K, K) * FB_BLK, lane, bad);
+    __syncthreads();
+    // L_IK = A_IK T_KK^T for I > K
+    float acc[3][2][2];
+#pragma unroll
+    for (int q = 0; q < 3; ++q) {
+      acc[q][0][0] = acc[q][0][1] = acc[q][1][0] = acc[q][1][1] = 0.f;
+      if (K + 1 + q < 4) nt_block(acc[q], As + tri(K + 1 + q, K) * FB_BLK, As + tri(K, K) * FB_BLK, a, b);
+    }
+    __syncthreads();
+#pragma unroll
+    for (int q = 0; q < 3; ++q)
+      if (K + 1 + q < 4) {
+        float* L = As + tri(K + 1 + q, K) * FB_BLK;
+#pragma unroll
+        for (int i = 0; i < 2; ++i)
+#pragma unroll
+          for (int j = 0; j < 2; ++j) L[(a + 16 * i) * FB_LD + b + 16 * j] = acc[q][i][j];
+      }
+    __syncthreads();
+    if (K == 3) break;
+    // A_IJ -= L_IK L_JK^T for K < J <= I
+    trailing_update(As, K, 0, (3 - K) * (4 - K) / 2, tid, FB_THREADS);
+    __syncthreads();
+  }
+
+  // XT_JI = -(T_II sum_{M=J}^{I-1} L_IM X_MJ)^T, by level I - J
+#pragma unroll 1
+  for (int lev = 1; lev < 4; ++lev) {
+#pragma unroll 1
+    for (int J = 0; J + lev < 4; ++J) {
+      const int I = J + lev;
+      float acc[2][2] = {{0.f, 0.f}, {0.f, 0.f}};  // S^T = sum_M XT_JM L_IM^T
+#pragma unroll 1
+      for (int M = J; M < I; ++M) nt_block(acc, XT + tri(M, J) * FB_BLK, As + tri(I, M) * FB_BLK, a, b);
+      float* St = Sc + J * FB_BLK;
+#pragma unroll
+      for (int i = 0; i < 2; ++i)
+#pragma unroll
+        for (int j = 0; j < 2; ++j) St[(a + 16 * i) * FB_LD + b + 16 * j] = acc[i][j];
+    }
+    __syncthreads();
+#pragma unroll 1
+    for (int J = 0; J + lev < 4; ++J) {
+      const int I = J + lev;
+      float acc[2][2] = {{0.f, 0.f}, {0.f, 0.f}};  // XT_JI = -S^T T_II^T
+      nt_block(acc, Sc + J * FB_BLK, As + tri(I, I) * FB_BLK, a, b);
+      float* X = XT + tri(I, J) * FB_BLK;
+#pragma unroll
+      for (int i = 0; i < 2; ++i)
+#pragma unroll
+        for (int j = 0; j < 2; ++j) X[(a + 16 * i) * FB_LD + b + 16 * j] = -acc[i][j];
+    }
+    __syncthreads();
+  }
+  if (bad) s_bad = 1;
+
+  // L^{-1}[n][c] = XT(tri(n / 32, c / 32))[c % 32][n % 32] for n >= c, 0 above:
+  // float32 rows and the bf16 hi/lo image (as in the elimination kernel). A
+  // warp takes 32 consecutive rows n of one 8-channel chunk, so its transposed
+  // shared-memory reads are consecutive.
+  float* mout = ws.minv + (int64_t)u * D * D;
+  uint8_t* img = ws.minv_img + (int64_t)u * 65536;
+  for (int e = tid; e < D * 16; e += FB_THREADS) {
+    const int n = e & (D - 1), cc = e >> 7;  // row n, 8-channel chunk cc
+    float x[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const int c = cc * 8 + q;
+      x[q] = c <= n ? XT[tri(n >> 5, c >> 5) * FB_BLK + (c & 31) * FB_LD + (n & 31)] : 0.f;
+    }
+    *(float4*)(mout + n * D + cc * 8) = make_float4(x[0], x[1], x[2], x[3]);
+    *(float4*)(mout + n * D + cc * 8 + 4) = make_float4(x[4], x[5], x[6], x[7]);
+    uint32_t hi[4], lo[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      hi[q] = pack_bf16x2(x[2 * q], x[2 * q + 1]);
+      lo[q] = pack_bf16x2(x[2 * q] - bf16lo(hi[q]), x[2 * q + 1] - bf16hi(hi[q]));
+    }
+    *(uint4*)(img + (cc >> 3) * 32768 + sw128_off(n, cc & 7)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+    *(uint4*)(img + (cc >> 3) * 32768 + sw128_off(n + 128, cc & 7)) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+  }
+  __syncthreads();
+  if (tid == 0 && s_bad) flag(ws, ST_NONFINITE);
+}
+
 template <bool PROJ>
 static cudaError_t launch_factor_t(const Dims& dm, const Ws& ws, const float* out_factor, cudaStream_t st) {
   constexpr size_t smem = factor_smem_bytes<PROJ>();
@@ -328,7 +668,12 @@ static cudaError_t launch_factor_t(const Dims& dm, const Ws& ws, const float* ou
 }
 
 cudaError_t launch_factor(const Dims& dm, const Ws& ws, const float* out_factor, cudaStream_t st) {
-  return out_factor ? launch_factor_t<true>(dm, ws, out_factor, st) : launch_factor_t<false>(dm, ws, nullptr, st);
+  if (out_factor != nullptr) return launch_factor_t<true>(dm, ws, out_factor, st);
+  cudaError_t e = cudaFuncSetAttribute(factor_blocked_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)FB_SMEM);
+  if (e != cudaSuccess) return e;
+  factor_blocked_kernel<<<dm.L * dm.Hkv * dm.S, FB_THREADS, FB_SMEM, st>>>(dm, ws);
+  return cudaGetLastError();
 }
 
 }  // namespace jacap

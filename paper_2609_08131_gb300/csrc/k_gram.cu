@@ -336,7 +336,9 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
     // ------------------------------------------------------ epilogue ------
     // D is a chunk's partial Gram; warp (quarter q) copies rows 32 q .. +31,
     // each lane its row: 32 consecutive floats per column block, so a lane
-    // writes 128 contiguous bytes per block.
+    // writes 128 contiguous bytes per block. The Gram is symmetric and its
+    // consumers read the lower triangle only, so only the column blocks
+    // cb <= q (the lower 32 x 32 blocks) are written.
     const int quarter = warp & 3;
     const int m = quarter * 32 + lane;
     uint32_t nitem = 0;
@@ -348,7 +350,7 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
       const uint32_t trow = tmem + (db ? GR_DCOL1 : 0u) + ((uint32_t)(quarter * 32) << 16);
       float* dst = ws.gpart + ((int64_t)item.plane * dm.c_cap + item.cidx) * D * D + (int64_t)m * 32;
 #pragma unroll 1
-      for (int cb = 0; cb < D / 32; ++cb) {
+      for (int cb = 0; cb <= quarter; ++cb) {
         float a[32];
         tmem_ld32(trow + cb * 32, a);
 #pragma unroll
@@ -428,6 +430,7 @@ __global__ void __launch_bounds__(GF_THREADS)
       __syncthreads();
     }
     float* dst = ws.gpart + ((int64_t)item.plane * dm.c_cap + item.cidx) * D * D;
+    if ((rb * 8) >> 5 < (cb * 8) >> 5) continue;  // upper 32 x 32 blocks: not read (symmetry)
 #pragma unroll
     for (int p = 0; p < 8; ++p) {
       // (m, n) at ((n / 32) D + m) 32 + n % 32; the 8 columns share one block
