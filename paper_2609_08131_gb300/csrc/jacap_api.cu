@@ -378,7 +378,7 @@ jacap_status jacap_select(const jacap_layout* layout, const float* scores, int32
   if ((st = check_device(&sms)) != JACAP_OK) return st;
   const Ws w = make_ws(ws, c);
   const int64_t units = (int64_t)dm.L * dm.Hkv * dm.S;
-  return map_cuda(launch_select(dm, w, layout->cu_seqlens, scores, budget, idx, kept,
+  return map_cuda(launch_select(dm, w, layout->cu_seqlens, scores, budget, idx, kept, layout->max_seqlen,
                                 persistent_grid(units, sms, 2), (cudaStream_t)stream));
 }
 

@@ -6,10 +6,11 @@
 // Three radix passes (digits of 11, 11 and 10 bits, most significant first,
 // shared-memory histograms; a pass counts only keys that match the digits
 // found so far) find the B-th largest key T and how many keys equal to T are
-// still needed. The keys are read in slabs of 32768 into registers (32 per
-// lane, all loads in flight together); a request of up to 32768 tokens is
+// still needed. The keys are read in slabs of 1024 KPT into registers (KPT
+// per lane, all loads in flight together; KPT = 4, 8, 16 or 32, the smallest
+// that holds the longest request in one slab); a request that fits one slab is
 // read once and every pass works on registers. Emission walks the slabs in
-// order; in a slab each warp owns 1024 consecutive positions, counts its keys
+// order; in a slab each warp owns 32 KPT consecutive positions, counts its keys
 // > T and == T with ballots, and the warp totals give where its kept
 // positions go and which of its keys == T are among the first `need` by
 // position (ties go to the lower position); kept positions come out in
@@ -26,24 +27,28 @@ namespace jacap {
 constexpr int SE_THREADS = 1024;
 
 constexpr int SE_BINS = 2048;
-constexpr int SE_KPT = 32;                       // keys per lane of a slab
-constexpr int SE_SLAB = SE_THREADS * SE_KPT;     // 32768 keys: warp w holds positions 1024 w .. +1023
 
 // Keys of slab `sl` into registers: lane's register j holds position
-// sl * SE_SLAB + 1024 w + 32 j + lane (coalesced; all loads in flight at once).
+// sl * 1024 KPT + 32 KPT w + 32 j + lane (coalesced; all loads in flight at
+// once). KPT keys per lane (4 .. 32) is chosen from the longest request, so a
+// short cache does not carry empty register slots through every pass.
+template <int KPT>
 __device__ __forceinline__ void load_slab(const uint32_t* key, int n, int sl, int warp, int lane,
-                                          uint32_t (&kr)[SE_KPT]) {
-  const int base = sl * SE_SLAB + warp * (32 * SE_KPT) + lane;
+                                          uint32_t (&kr)[KPT]) {
+  const int base = sl * SE_THREADS * KPT + warp * (32 * KPT) + lane;
 #pragma unroll
-  for (int j = 0; j < SE_KPT; ++j) {
+  for (int j = 0; j < KPT; ++j) {
     const int i = base + 32 * j;
     kr[j] = i < n ? __ldg(key + i) : 0u;
   }
 }
 
+template <int KPT>
 __global__ void __launch_bounds__(SE_THREADS)
     select_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu, const float* __restrict__ scores, int B,
                   int32_t* __restrict__ idx, int32_t* __restrict__ kept) {
+  constexpr int SE_KPT = KPT;
+  constexpr int SE_SLAB = SE_THREADS * KPT;  // warp w holds positions 32 KPT w .. + 32 KPT - 1 of a slab
   __shared__ uint32_t hist[SE_BINS];
   __shared__ uint32_t s_digit, s_need;
   __shared__ int s_skip;
@@ -75,7 +80,7 @@ __global__ void __launch_bounds__(SE_THREADS)
     }
     const int nslab = (n + SE_SLAB - 1) / SE_SLAB;
     uint32_t kr[SE_KPT];
-    if (nslab == 1) load_slab(key, n, 0, warp, lane, kr);  // register-resident for all passes
+    if (nslab == 1) load_slab<KPT>(key, n, 0, warp, lane, kr);  // register-resident for all passes
     // ---- radix select of the B-th largest key: digits [31:21], [20:10], [9:0] ----
     uint32_t prefix = 0, mask = 0, need = (uint32_t)B;
 #pragma unroll 1
@@ -86,7 +91,7 @@ __global__ void __launch_bounds__(SE_THREADS)
       __syncthreads();
 #pragma unroll 1
       for (int sl = 0; sl < nslab; ++sl) {
-        if (nslab > 1) load_slab(key, n, sl, warp, lane, kr);
+        if (nslab > 1) load_slab<KPT>(key, n, sl, warp, lane, kr);
         const int base = sl * SE_SLAB + warp * (32 * SE_KPT) + lane;
 #pragma unroll
         for (int j = 0; j < SE_KPT; ++j)
@@ -123,11 +128,11 @@ __global__ void __launch_bounds__(SE_THREADS)
       __syncthreads();
     }
     const uint32_t T = prefix;  // the B-th largest key; the first `need` keys == T are kept
-    // ---- emission, slab by slab; in a slab warp w owns positions 1024 w .. +1023 ----
+    // ---- emission, slab by slab; in a slab warp w owns positions 32 KPT w .. ----
     uint32_t gt_run = 0, eq_run = 0;  // kept-greater and equal keys before this slab
 #pragma unroll 1
     for (int sl = 0; sl < nslab; ++sl) {
-      if (nslab > 1) load_slab(key, n, sl, warp, lane, kr);
+      if (nslab > 1) load_slab<KPT>(key, n, sl, warp, lane, kr);
       const int base = sl * SE_SLAB + warp * (32 * SE_KPT) + lane;
       uint32_t gt = 0, eq = 0;
 #pragma unroll
@@ -202,8 +207,15 @@ __global__ void __launch_bounds__(256)
 }
 
 cudaError_t launch_select(const Dims& dm, const Ws& ws, const int32_t* cu, const float* scores, int budget,
-                          int32_t* idx, int32_t* kept, int grid, cudaStream_t st) {
-  select_kernel<<<grid, SE_THREADS, 0, st>>>(dm, ws, cu, scores, budget, idx, kept);
+                          int32_t* idx, int32_t* kept, int max_seqlen, int grid, cudaStream_t st) {
+  if (max_seqlen <= SE_THREADS * 4)
+    select_kernel<4><<<grid, SE_THREADS, 0, st>>>(dm, ws, cu, scores, budget, idx, kept);
+  else if (max_seqlen <= SE_THREADS * 8)
+    select_kernel<8><<<grid, SE_THREADS, 0, st>>>(dm, ws, cu, scores, budget, idx, kept);
+  else if (max_seqlen <= SE_THREADS * 16)
+    select_kernel<16><<<grid, SE_THREADS, 0, st>>>(dm, ws, cu, scores, budget, idx, kept);
+  else
+    select_kernel<32><<<grid, SE_THREADS, 0, st>>>(dm, ws, cu, scores, budget, idx, kept);
   return cudaGetLastError();
 }
 
