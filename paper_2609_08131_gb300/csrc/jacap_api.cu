@@ -20,7 +20,8 @@ constexpr size_t ALIGN = 1024;
 inline size_t align_up(size_t x) { return (x + ALIGN - 1) & ~(ALIGN - 1); }
 
 struct Carve {
-  size_t status, plan, chunks, counters, mu, lam, qdev, lk, cstats, w, wsplit, gpart, gram, minv, minv_img, total;
+  size_t status, plan, chunks, counters, mu, lam, qdev, lk, cstats, w, wsplit, gpart, pflag, gram, minv, minv_img,
+      total;
 };
 
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
@@ -51,15 +52,17 @@ jacap_status check_layout(const jacap_layout* L) {
   return JACAP_OK;
 }
 
-// Tokens per work item: the largest of 16384..128 that still yields enough
-// items to fill the GPU several times over (independent of the device so the
-// workspace size is a pure function of the layout). Larger items mean fewer
-// partial Grams to write and re-read and fewer item boundaries.
+// Tokens per work item: the largest of 16384..128 that still yields 4096
+// items (independent of the device so the workspace size is a pure function
+// of the layout). Each CTA takes a contiguous range of items, so the counts
+// per CTA differ by one item at most: with ~27 items per CTA on 152 SMs the
+// last item costs under 4 % of a pass. Items of one unit that follow each
+// other in a CTA's range share one partial Gram and one factor image.
 int pick_chunk(const jacap_layout* L) {
   const int64_t planes = (int64_t)L->num_layers * L->num_kv_heads;
   for (int c = 16384; c > TILE; c >>= 1) {
     const int64_t items = planes * (L->total_tokens / c + L->num_seqs);
-    if (items >= 1024) return c;
+    if (items >= 4096) return c;
   }
   return TILE;
 }
@@ -111,6 +114,7 @@ Carve carve(const Dims& dm) {
   c.w = o; o = align_up(o + planes * (size_t)dm.Ntot * 4);
   c.wsplit = o; o = align_up(o + planes * (size_t)dm.Ntot * 4 + 64);  // + tail read by 16-byte rounded copies
   c.gpart = o; o = align_up(o + planes * (size_t)dm.c_cap * D * D * 4);
+  c.pflag = o; o = align_up(o + planes * (size_t)dm.c_cap * 4);
   c.gram = o; o = align_up(o + units * D * D * 4);
   c.minv = o; o = align_up(o + units * D * D * 4);
   c.minv_img = o; o = align_up(o + units * 65536);
@@ -134,6 +138,7 @@ Ws make_ws(void* base, const Carve& c) {
   ws.w = (float*)(b + c.w);
   ws.wsplit = (uint32_t*)(b + c.wsplit);
   ws.gpart = (float*)(b + c.gpart);
+  ws.pflag = (int32_t*)(b + c.pflag);
   ws.gram = (float*)(b + c.gram);
   ws.minv = (float*)(b + c.minv);
   ws.minv_img = b + c.minv_img;
@@ -188,10 +193,21 @@ bool encode_kv_map(CUtensorMap* map, const jacap_layout* L, const void* base) {
 
 jacap_status map_cuda(cudaError_t e) { return e == cudaSuccess ? JACAP_OK : JACAP_ERR_CUDA; }
 
+// CTAs for `items` work items with at most per_sm CTAs per SM: each CTA takes
+// a contiguous range, so the grid is chosen to split the items as evenly as
+// the cap allows (ceil(items / cap) items for every CTA but the last few).
 int persistent_grid(int64_t items, int sms, int per_sm) {
   const int64_t cap = (int64_t)sms * per_sm;
-  const int64_t g = items < cap ? items : cap;
-  return g < 1 ? 1 : (int)g;
+  if (items <= cap) return items < 1 ? 1 : (int)items;
+  const int64_t per = (items + cap - 1) / cap;
+  return (int)((items + per - 1) / per);
+}
+
+// Work items of the pass (plane x chunk): exact for one request, otherwise the
+// capacity bound (the device computes the exact count from cu_seqlens).
+int64_t pass_items(const jacap_layout* L, const Dims& dm) {
+  const int64_t per_plane = L->num_seqs == 1 ? (L->total_tokens + dm.chunk - 1) / dm.chunk : dm.c_cap;
+  return (int64_t)dm.L * dm.Hkv * per_plane;
 }
 
 }  // namespace
@@ -270,7 +286,7 @@ jacap_status score_pass(const jacap_layout* layout, const jacap_params* params, 
   CUtensorMap kmap, vmap;
   const bool bf = layout->dtype == JACAP_BF16;
   if (!encode_kv_map(&kmap, layout, k) || !encode_kv_map(&vmap, layout, v)) return JACAP_ERR_CUDA;
-  const int64_t items = (int64_t)dm.L * dm.Hkv * dm.c_cap;
+  const int64_t items = pass_items(layout, dm);
   const int dt = bf ? 1 : 0;
   const int32_t* cu = layout->cu_seqlens;
   auto hook = [&](int i) -> jacap_status {

@@ -68,7 +68,10 @@ struct Ws {
   float* cstats;      // [L*Hkv][c_cap][G][2]  per-chunk (max, sum exp(l - max))
   float* w;           // [L*Hkv][Ntot]  Eq. 8 weights summed over the group
   uint32_t* wsplit;   // [L*Hkv][Ntot]  w as bf16 hi (low half) + bf16 lo = w - hi (high half)
-  float* gpart;       // [L*Hkv][c_cap][D/32][D][32]  per-chunk partial Grams: (m, n) at ((n/32) D + m) 32 + n%32
+  float* gpart;       // [L*Hkv][c_cap][D/32][D][32]  partial Grams: (m, n) at ((n/32) D + m) 32 + n%32,
+                      // lower 32 x 32 blocks only; one per run of a CTA's consecutive chunks of a unit,
+                      // stored at the run's first chunk
+  int32_t* pflag;     // [L*Hkv][c_cap]  1 where gpart holds a partial (a run's first chunk), else 0
   float* gram;        // [units][D][D]  sum_i w_i v_i v_i^T
   float* minv;        // [units][D][D]  L^{-1} (float32, lower triangular)
   uint8_t* minv_img;  // [units][65536]  L^{-1} as bf16 hi/lo, shared-memory image for the score MMA
@@ -87,26 +90,37 @@ struct Item {
 // next item is loaded while the current one is processed, so an item
 // boundary costs no dependent global loads.
 struct ItemStream {
+  // CTA `part` of `parts` walks the contiguous item range [part T / parts,
+  // (part + 1) T / parts) of the T = L Hkv C_tot items (plane-major, chunks of
+  // a plane in request order), so the counts differ by at most one item and
+  // consecutive items mostly belong to one unit (accumulators and images
+  // carry over between them).
   const int4* tab;
-  int64_t total, i, step;
+  int64_t i, end;
   int ctot;
   int4 rec;
-  __device__ __forceinline__ ItemStream(const Dims& dm, const Ws& ws, int64_t start, int64_t stride)
-      : tab(ws.chunks), i(start), step(stride) {
+  __device__ __forceinline__ ItemStream(const Dims& dm, const Ws& ws, int64_t part, int64_t parts) : tab(ws.chunks) {
     ctot = ws.plan[0];
-    total = (int64_t)dm.L * dm.Hkv * ctot;
-    if (i < total) rec = tab[i % ctot];
+    const int64_t total = (int64_t)dm.L * dm.Hkv * ctot;
+    i = part * total / parts;
+    end = (part + 1) * total / parts;
+    if (i < end) rec = tab[i % ctot];
   }
   __device__ __forceinline__ bool next(Item& it) {
-    if (i >= total) return false;
+    if (i >= end) return false;
     it.plane = (int)(i / ctot);
     it.t0 = rec.x;
     it.t1 = rec.y;
     it.seq = rec.z;
     it.cidx = rec.w;
-    i += step;
-    if (i < total) rec = tab[i % ctot];
+    ++i;
+    if (i < end) rec = tab[i % ctot];
     return true;
+  }
+  // whether this CTA's next item exists and belongs to the same unit as `cur`
+  // (the item last returned by next())
+  __device__ __forceinline__ bool next_same_unit(const Item& cur) const {
+    return i < end && (int)(i / ctot) == cur.plane && rec.z == cur.seq;
   }
 };
 

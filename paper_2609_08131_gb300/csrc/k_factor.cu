@@ -85,7 +85,9 @@ __global__ void __launch_bounds__(FA_THREADS, PROJ ? 1 : 2)
     float* gout = ws.gram + (int64_t)u * D * D;
 #pragma unroll
     for (int a = 0; a < FA_ROWS; ++a) z[a][0] = z[a][1] = make_float2(0.f, 0.f);
+    const int32_t* pf = ws.pflag + (int64_t)plane * dm.c_cap;
     for (int ch = ch0; ch < ch1; ++ch) {  // 16 independent 16-byte loads in flight per chunk
+      if (!pf[ch]) continue;  // no partial at this chunk (it continued a run)
       // partial layout: (m, n) at ((n / 32) D + m) 32 + n % 32; only the
       // lower 32 x 32 blocks are stored (rows ty + 8 a lie in block a / 4)
       const float* src = gp + (int64_t)ch * D * D + (c0 >> 5) * D * 32 + (c0 & 31);
@@ -471,7 +473,7 @@ __global__ void __launch_bounds__(FB_THREADS, 2) factor_blocked_kernel(Dims dm, 
   float* XT = fsm + 10 * FB_BLK;  // tri(I, J): XT_JI = (L^{-1})_IJ^T
   float* Sc = fsm + 20 * FB_BLK;  // scratch
   __shared__ __align__(8) uint64_t s_full[2];
-  __shared__ int s_skip, s_bad;
+  __shared__ int s_skip, s_bad, s_np;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) {
     s_skip = status_failed(ws) ? 1 : 0;
@@ -485,8 +487,8 @@ __global__ void __launch_bounds__(FB_THREADS, 2) factor_blocked_kernel(Dims dm, 
   const float* gp = ws.gpart + ((int64_t)plane * dm.c_cap) * D * D;
   bool bad = false;
 
-  // A = I + sum of partial Grams (chunk order) over the lower 32 x 32 blocks
-  // (the partials hold only those); G to the workspace and the lower blocks of
+  // A = I + sum of the unit's partial Grams (chunk order) over the lower
+  // 32 x 32 blocks (the partials hold only those); G to the workspace and the lower blocks of
   // A to shared memory. The partials stream through a two-stage ring of bulk
   // copies (the 4 lower segments of one partial per stage: rows 32 nb .. 127
   // of column block nb, contiguous in the partial layout) while the threads
@@ -494,11 +496,22 @@ __global__ void __launch_bounds__(FB_THREADS, 2) factor_blocked_kernel(Dims dm, 
   // 4 tx .. 4 tx + 3; rows ty + 8 a lie in block a / 4.
   float* gout = ws.gram + (int64_t)u * D * D;
   {
+    // the chunks that hold partials (the first chunk of every run)
+    const int32_t* pf = ws.pflag + (int64_t)plane * dm.c_cap;
     if (tid == 0) {
       for (int i = 0; i < 2; ++i) mbar_init(smem_u32(&s_full[i]), 1);
       fence_mbar_init();
+      int np = 0;
+      for (int ch = ch0; ch < ch1; ++ch) np += pf[ch] != 0;
+      s_np = np;
     }
     __syncthreads();
+    const int np = s_np;
+    int cursor = ch0;  // (thread 0) next chunk to look at for a partial
+    auto next_partial = [&]() {
+      while (cursor < ch1 && !pf[cursor]) ++cursor;
+      return cursor++;
+    };
     auto issue = [&](int ch, int st) {  // one partial into stage st
       uint8_t* dst = (uint8_t*)(fsm + st * FB_STAGE);
       const float* src = gp + (int64_t)ch * D * D;
@@ -509,17 +522,17 @@ __global__ void __launch_bounds__(FB_THREADS, 2) factor_blocked_kernel(Dims dm, 
                  smem_u32(&s_full[st]));
     };
     if (tid == 0) {
-      if (ch0 < ch1) issue(ch0, 0);
-      if (ch0 + 1 < ch1) issue(ch0 + 1, 1);
+      if (np > 0) issue(next_partial(), 0);
+      if (np > 1) issue(next_partial(), 1);
     }
     const int ty = tid >> 5, tx = tid & 31, c0 = 4 * tx;
     const int J = c0 >> 5, c = c0 & 31;
     float4 z[FA_ROWS];
 #pragma unroll
     for (int a = 0; a < FA_ROWS; ++a) z[a] = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int ch = ch0; ch < ch1; ++ch) {
-      const int st = (ch - ch0) & 1;
-      if (!mbar_wait(smem_u32(&s_full[st]), ((ch - ch0) >> 1) & 1, ws, nullptr)) bad = true;
+    for (int k = 0; k < np; ++k) {
+      const int st = k & 1;
+      if (!mbar_wait(smem_u32(&s_full[st]), (k >> 1) & 1, ws, nullptr)) bad = true;
       const float* sb = fsm + st * FB_STAGE + fb_seg(J) + c;
 #pragma unroll
       for (int a = 0; a < FA_ROWS; ++a) {
@@ -531,9 +544,9 @@ __global__ void __launch_bounds__(FB_THREADS, 2) factor_blocked_kernel(Dims dm, 
         z[a].w += v.w;
       }
       __syncthreads();  // stage st is read; it may be refilled
-      if (tid == 0 && ch + 2 < ch1) {
+      if (tid == 0 && k + 2 < np) {
         fence_proxy_async_smem();
-        issue(ch + 2, st);
+        issue(next_partial(), st);
       }
     }
 #pragma unroll

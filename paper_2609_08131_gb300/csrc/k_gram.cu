@@ -57,54 +57,67 @@ __global__ void __launch_bounds__(WT_THREADS) weight_kernel(Dims dm, Ws ws, cons
   if (tid == 0) s_skip = status_failed(ws) ? 1 : 0;
   __syncthreads();
   if (s_skip) return;
-  bool bad = false;
+  bool bad = false, cont = false;
+  float u[2 * G];
   Item item;
   for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
-    __syncthreads();
-    if (warp < G) {
-      float M, Z;
-      unit_softmax_stats_warp<G>(dm, ws, item.plane, item.seq, warp, M, Z);
-      if (lane == 0) {
-        us[warp] = M;
-        us[G + warp] = 1.f / Z;
+    if (!cont) {  // a new unit: its (M_h, Z_h); consecutive items of the unit reuse them
+      __syncthreads();
+      if (warp < G) {
+        float M, Z;
+        unit_softmax_stats_warp<G>(dm, ws, item.plane, item.seq, warp, M, Z);
+        if (lane == 0) {
+          us[warp] = M;
+          us[G + warp] = 1.f / Z;
+        }
       }
+      __syncthreads();
+#pragma unroll
+      for (int e = 0; e < 2 * G; ++e) u[e] = us[e];
     }
-    __syncthreads();
-    float u[2 * G];
-#pragma unroll
-    for (int e = 0; e < 2 * G; ++e) u[e] = us[e];
+    cont = is.next_same_unit(item);
     const int64_t base = (int64_t)item.plane * dm.Ntot;
-    for (int64_t tok = item.t0 + tid; tok < item.t1; tok += WT_THREADS) {
-      const float* src = ws.lk + (base + tok) * (2 * G);
-      float lk[2 * G];
-      if constexpr ((2 * G) % 4 == 0) {
+    // four tokens per thread per round, their loads issued together
+    for (int64_t t4 = item.t0 + tid; t4 < item.t1; t4 += 4 * WT_THREADS) {
+      float lk[4][2 * G];
 #pragma unroll
-        for (int e = 0; e < 2 * G; e += 4) {
-          const float4 q4 = *(const float4*)(src + e);
-          lk[e] = q4.x; lk[e + 1] = q4.y; lk[e + 2] = q4.z; lk[e + 3] = q4.w;
-        }
-      } else {
-        const float2 q2 = *(const float2*)src;
-        lk[0] = q2.x;
-        lk[1] = q2.y;
-      }
-      float wt = 0.f;
-      if (dm.linear) {  // S_C = I: rho = 1
+      for (int q = 0; q < 4; ++q) {
+        const int64_t tok = t4 + q * WT_THREADS;
+        const float* src = ws.lk + (base + (tok < item.t1 ? tok : t4)) * (2 * G);
+        if constexpr ((2 * G) % 4 == 0) {
 #pragma unroll
-        for (int h = 0; h < G; ++h) wt += lk[G + h];
-      } else {
-#pragma unroll
-        for (int h = 0; h < G; ++h) {
-          const float a = expf(lk[h] - u[h]) * u[G + h];  // alpha_bar
-          const float rho = a * (1.f - a);                 // diagonal of the softmax Jacobian
-          wt = fmaf(rho * rho, lk[G + h], wt);             // rho^2 kappa
+          for (int e = 0; e < 2 * G; e += 4) {
+            const float4 q4 = *(const float4*)(src + e);
+            lk[q][e] = q4.x; lk[q][e + 1] = q4.y; lk[q][e + 2] = q4.z; lk[q][e + 3] = q4.w;
+          }
+        } else {
+          const float2 q2 = *(const float2*)src;
+          lk[q][0] = q2.x;
+          lk[q][1] = q2.y;
         }
       }
-      wt *= dm.wdiv;
-      bad |= !isfinite(wt);
-      ws.w[base + tok] = wt;
-      // hi = RN(w), lo = RN(w - hi) (w - hi is exact in float32)
-      ws.wsplit[base + tok] = pack_bf16x2(wt, wt - bf16lo(pack_bf16x2(wt, 0.f)));
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int64_t tok = t4 + q * WT_THREADS;
+        if (tok >= item.t1) break;
+        float wt = 0.f;
+        if (dm.linear) {  // S_C = I: rho = 1
+#pragma unroll
+          for (int h = 0; h < G; ++h) wt += lk[q][G + h];
+        } else {
+#pragma unroll
+          for (int h = 0; h < G; ++h) {
+            const float a = expf(lk[q][h] - u[h]) * u[G + h];  // alpha_bar
+            const float rho = a * (1.f - a);                    // diagonal of the softmax Jacobian
+            wt = fmaf(rho * rho, lk[q][G + h], wt);             // rho^2 kappa
+          }
+        }
+        wt *= dm.wdiv;
+        bad |= !isfinite(wt);
+        ws.w[base + tok] = wt;
+        // hi = RN(w), lo = RN(w - hi) (w - hi is exact in float32)
+        ws.wsplit[base + tok] = pack_bf16x2(wt, wt - bf16lo(pack_bf16x2(wt, 0.f)));
+      }
     }
   }
   if (bad) flag(ws, ST_NONFINITE);
@@ -118,10 +131,12 @@ __global__ void __launch_bounds__(WT_THREADS) weight_kernel(Dims dm, Ws ws, cons
 // hi + lo from the weight pass). The scaling warps read V transposed with
 // ldmatrix, form w_i v_i = hi + lo with packed bf16 arithmetic and store hi
 // and lo as two A operands; two MMAs per 16 tokens accumulate v (hi + lo)^T.
-// The scaling warps share nothing but the mbarriers of the pipeline; four
-// epilogue warps copy each finished chunk Gram out of tensor memory while the
-// next chunk accumulates in the other buffer.
+// The scaling warps share nothing but the mbarriers of the pipeline. A run of
+// consecutive chunks of one unit in a CTA's item range accumulates in one
+// tensor-memory buffer; four epilogue warps copy each finished run's Gram out
+// while the next run accumulates in the other buffer.
 constexpr int GR_THREADS = 448;   // warp 0: TMA, warp 1: MMA, warps 2-9: scale, warps 10-13: epilogue
+constexpr int GR_EPI0 = 10;       // first epilogue warp
 constexpr int GR_SCALERS = 256;
 constexpr int GR_VST = 6;          // V tiles in flight
 constexpr int GR_BOX = 16384;      // {64 channels, 128 tokens} bf16, 128-byte swizzle
@@ -230,16 +245,20 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer ----------
     if (lane == 0) {
-      uint32_t it = 0, nitem = 0;
-      bool ok = true;
+      uint32_t it = 0, nrun = 0;
+      bool ok = true, cont = false, first = true;
+      int db = 0;
       Item item;
       for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); ok && is.next(item);) {
-        // accumulator of this item; its previous item's epilogue must be done
-        const int db = nitem & 1;
+        // one accumulator per run of consecutive chunks of a unit; a new run
+        // takes the other buffer once its previous run's epilogue is done
+        if (!cont) {
+          db = nrun & 1;
+          if (nrun >= 2 && !mbar_wait(smem_u32(&accempty[db]), ((nrun >> 1) & 1) ^ 1, ws, abort)) break;
+          tc_fence_after();
+          first = true;
+        }
         const uint32_t dacc = tmem + (db ? GR_DCOL1 : 0u);
-        if (nitem >= 2 && !mbar_wait(smem_u32(&accempty[db]), ((nitem >> 1) & 1) ^ 1, ws, abort)) break;
-        tc_fence_after();
-        bool first = true;
         for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
           const int vs = it % GR_VST, ab = it & 1;
           // the scaling warps arrive on afull only after the tile's V landed
@@ -262,8 +281,11 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
           umma_commit(smem_u32(&aempty[ab]));
         }
         if (!ok) break;
-        umma_commit(smem_u32(&accfull[db]));
-        ++nitem;
+        cont = is.next_same_unit(item);
+        if (!cont) {
+          umma_commit(smem_u32(&accfull[db]));
+          ++nrun;
+        }
       }
       if (it > 0) mbar_wait(smem_u32(&aempty[(it - 1) & 1]), ((it - 1) >> 1) & 1, ws, nullptr);
     }
@@ -341,14 +363,22 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
     // cb <= q (the lower 32 x 32 blocks) are written.
     const int quarter = warp & 3;
     const int m = quarter * 32 + lane;
-    uint32_t nitem = 0;
+    uint32_t nrun = 0;
+    bool cont = false;
+    int run_cidx = 0;
     Item item;
     for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
-      const int db = nitem & 1;
-      if (!mbar_wait(smem_u32(&accfull[db]), (nitem >> 1) & 1, ws, abort)) break;
+      // the partial of a run goes to its first chunk; pflag marks which
+      // chunks hold one
+      if (!cont) run_cidx = item.cidx;
+      if (warp == GR_EPI0 && lane == 0) ws.pflag[(int64_t)item.plane * dm.c_cap + item.cidx] = cont ? 0 : 1;
+      cont = is.next_same_unit(item);
+      if (cont) continue;
+      const int db = nrun & 1;
+      if (!mbar_wait(smem_u32(&accfull[db]), (nrun >> 1) & 1, ws, abort)) break;
       tc_fence_after();
       const uint32_t trow = tmem + (db ? GR_DCOL1 : 0u) + ((uint32_t)(quarter * 32) << 16);
-      float* dst = ws.gpart + ((int64_t)item.plane * dm.c_cap + item.cidx) * D * D + (int64_t)m * 32;
+      float* dst = ws.gpart + ((int64_t)item.plane * dm.c_cap + run_cidx) * D * D + (int64_t)m * 32;
 #pragma unroll 1
       for (int cb = 0; cb <= quarter; ++cb) {
         float a[32];
@@ -360,7 +390,7 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&accempty[db]));
-      ++nitem;
+      ++nrun;
     }
   }
   tc_fence_before();
@@ -430,6 +460,7 @@ __global__ void __launch_bounds__(GF_THREADS)
       __syncthreads();
     }
     float* dst = ws.gpart + ((int64_t)item.plane * dm.c_cap + item.cidx) * D * D;
+    if (tid == 0) ws.pflag[(int64_t)item.plane * dm.c_cap + item.cidx] = 1;  // a partial per chunk here
     if ((rb * 8) >> 5 < (cb * 8) >> 5) continue;  // upper 32 x 32 blocks: not read (symmetry)
 #pragma unroll
     for (int p = 0; p < 8; ++p) {

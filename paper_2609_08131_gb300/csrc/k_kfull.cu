@@ -15,8 +15,8 @@
 // logits carry about 17 significant bits of delta before fp32 accumulation
 // instead of the 8 that one bf16 rounding would leave). The query-statistics
 // kernel writes that B operand straight into the workspace in shared-memory
-// image form; here it is one bulk copy per item, issued one item ahead into
-// a double buffer. One MMA job of N = 2 rp columns per 128-token tile, the
+// image form; here it is one bulk copy per unit (a CTA's consecutive items
+// of one unit share it), issued one item ahead into a double buffer. One MMA job of N = 2 rp columns per 128-token tile, the
 // accumulator double-buffered in tensor memory, so one tile's readout overlaps
 // the next tile's MMAs. Eight readout warps (two per tensor-memory lane
 // quarter, alternating tiles) add the two parts, square and sum per head.
@@ -124,12 +124,15 @@ __global__ void __launch_bounds__(KF_THREADS, 1)
           ++it;
         }
         if (!ok) break;
-        // the next item's image goes to the buffer of item n - 1, whose MMAs
-        // were all issued before this item's first tile
+        // a next item of another unit needs its image: it goes to the buffer
+        // of the run before this one, whose MMAs were all issued before this
+        // run's first tile
         have = is.next(nxt);
         if (have) {
-          if (nimg >= 2 && !mbar_wait(smem_u32(&imgfree[nimg & 1]), ((nimg - 2) >> 1) & 1, ws, abort)) break;
-          issue_image(nxt, nimg++);
+          if (nxt.plane != cur.plane || nxt.seq != cur.seq) {
+            if (nimg >= 2 && !mbar_wait(smem_u32(&imgfree[nimg & 1]), ((nimg - 2) >> 1) & 1, ws, abort)) break;
+            issue_image(nxt, nimg++);
+          }
           cur = nxt;
         }
       }
@@ -142,13 +145,16 @@ __global__ void __launch_bounds__(KF_THREADS, 1)
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer ----------
     if (lane == 0) {
-      uint32_t it = 0, n = 0;
-      bool ok = true;
+      uint32_t it = 0, n = 0;  // n: runs (units) started
+      bool ok = true, cont = false;
+      int p = 0;
       Item item;
-      for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); ok && is.next(item); ++n) {
-        const int p = n & 1;
-        if (!mbar_wait(smem_u32(&imgfull[p]), (n >> 1) & 1, ws, abort)) break;
-        tc_fence_after();
+      for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); ok && is.next(item);) {
+        if (!cont) {
+          p = n & 1;
+          if (!mbar_wait(smem_u32(&imgfull[p]), (n >> 1) & 1, ws, abort)) break;
+          tc_fence_after();
+        }
         const uint64_t b0 = smem_desc_sw128(smem_u32(img + p * C::IMG_BYTES), 16, 1024);
         for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
           const int st = it % KF_STAGES, slot = it & 1;
@@ -170,7 +176,11 @@ __global__ void __launch_bounds__(KF_THREADS, 1)
           umma_commit(smem_u32(&empty[st]));
         }
         if (!ok) break;
-        umma_commit(smem_u32(&imgfree[p]));
+        cont = is.next_same_unit(item);
+        if (!cont) {
+          umma_commit(smem_u32(&imgfree[p]));
+          ++n;
+        }
       }
       // every MMA issued here completes before the CTA tears down tensor memory
       if (it > 0) mbar_wait(smem_u32(&accfull[(it - 1) & 1]), ((it - 1) >> 1) & 1, ws, nullptr);

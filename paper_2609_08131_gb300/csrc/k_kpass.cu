@@ -17,7 +17,8 @@
 // packed fp32x2 multiply-adds.
 //
 // Warp roles: 0 TMA producer; 1 issues the logits MMAs; 14 builds the mu'
-// image and lambda of each item (double-buffered, one item ahead); 2-9 kappa (two groups of four warps alternate
+// image and lambda of each unit a CTA reaches (double-buffered, one run of the
+// unit's consecutive items ahead); 2-9 kappa (two groups of four warps alternate
 // tiles; in a group each warp takes one quarter of the channels for all 128
 // tokens, four per lane, so every lambda value read from shared memory serves
 // four tokens; the quarters are reduce-scattered through shared memory);
@@ -212,13 +213,16 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
   } else if (warp == 1) {
     // ------------------------------------------------ logits MMA issuer ---
     if (lane == 0) {
-      uint32_t it = 0, nitem = 0;
-      bool ok = true;
+      uint32_t it = 0, nrun = 0;  // nrun: runs of consecutive items of one unit started
+      bool ok = true, cont = false;
+      int p = 0;
       Item item;
       for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); ok && is.next(item);) {
-        const int p = nitem & 1;
-        if (!mbar_wait(smem_u32(&imgready[p]), (nitem >> 1) & 1, ws, abort)) break;
-        tc_fence_after();
+        if (!cont) {
+          p = nrun & 1;
+          if (!mbar_wait(smem_u32(&imgready[p]), (nrun >> 1) & 1, ws, abort)) break;
+          tc_fence_after();
+        }
         const uint64_t b0 = smem_desc_sw128(smem_u32(img + p * C::IMG_BYTES), 16, 1024);
         for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
           const int st = it % KB_STAGES;
@@ -242,20 +246,28 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
           umma_commit(smem_u32(&empty[st]));
           umma_commit(smem_u32(&accfull[ab]));
         }
-        if (ok) umma_commit(smem_u32(&imgfree[p]));
-        ++nitem;
+        if (!ok) break;
+        cont = is.next_same_unit(item);
+        if (!cont) {
+          umma_commit(smem_u32(&imgfree[p]));
+          ++nrun;
+        }
       }
       // every MMA issued here completes before the CTA tears down tensor memory
       if (it > 0) mbar_wait(smem_u32(&accfull[(it - 1) % KB_NACC]), ((it - 1) / KB_NACC) & 1, ws, nullptr);
     }
   } else if (warp == KB_BUILD_WARP) {
-    // ---------------------------------- mu' image and lambda, one item ahead
-    uint32_t nitem = 0;
+    // ------------------ mu' image and lambda, once per run, one run ahead
+    uint32_t nrun = 0;
+    bool cont = false;
     Item item;
     for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
+      const bool same = cont;
+      cont = is.next_same_unit(item);
+      if (same) continue;  // the run's image is in place
       const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
-      const int p = nitem & 1;
-      if (nitem >= 2 && !mbar_wait(smem_u32(&imgfree[p]), ((nitem >> 1) - 1) & 1, ws, abort)) break;
+      const int p = nrun & 1;
+      if (nrun >= 2 && !mbar_wait(smem_u32(&imgfree[p]), ((nrun >> 1) - 1) & 1, ws, abort)) break;
       const int64_t qb = (((int64_t)item.seq * dm.L + l) * dm.Hq + (int64_t)g * G) * D;
       build_split_image<G>(img + p * C::IMG_BYTES, ws.mu + qb, lane);
       float* lam_s = lams + p * G * D;
@@ -263,7 +275,7 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&imgready[p]));
-      ++nitem;
+      ++nrun;
     }
   } else if (warp >= KB_KAPPA_WARP0 && warp < KB_READ_WARP0) {
     // ------------------------------------------------------ kappa ---------
@@ -272,16 +284,21 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
     const int cq = kw & 3;                    // channel quarter; also the token subset finished here
     const int bar_id = 2 + grp;               // the four warps of the group
     float* slot = kred + grp * (4 * 4 * G * 32);
-    uint32_t it = 0, nitem = 0;
-    bool bad = false;
+    uint32_t it = 0, nrun = 0;
+    bool bad = false, cont = false;
+    int p = 0;
     Item item;
     // A failed wait (which means the abort flag is set) still arrives at the
     // group's named barriers, and the four warps leave together after them.
+    // All four see the same runs (the same item stream), so they meet at the
+    // same barriers.
     for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
-      const int p = nitem & 1;
-      mbar_wait(smem_u32(&imgready[p]), (nitem >> 1) & 1, ws, abort);
-      named_barrier_sync(bar_id, 128);
-      if (*abort) goto kappa_done;
+      if (!cont) {
+        p = nrun & 1;
+        mbar_wait(smem_u32(&imgready[p]), (nrun >> 1) & 1, ws, abort);
+        named_barrier_sync(bar_id, 128);
+        if (*abort) goto kappa_done;
+      }
       {
         const uint32_t lam_s = smem_u32(lams + p * G * D);
         float* lkp = ws.lk + (int64_t)item.plane * dm.Ntot * (2 * G) + G;
@@ -325,9 +342,12 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
           if (tok < item.t1) store_part<G>(lkp + tok * (2 * G), kap);
         }
       }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&imgfree[p]));
-      ++nitem;
+      cont = is.next_same_unit(item);
+      if (!cont) {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&imgfree[p]));
+        ++nrun;
+      }
     }
   kappa_done:
     if (bad) flag(ws, ST_NONFINITE);
@@ -338,14 +358,16 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
     const uint32_t lanes = (uint32_t)(quarter * 32) << 16;
     const int rw = warp - KB_READ_WARP0;
     uint32_t it = 0;
-    bool bad = false;
+    bool bad = false, cont = false;
+    float run_m[G], run_s[G];
     Item item;
     for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
-      float run_m[G], run_s[G];
+      if (!cont) {  // a new run of the unit's consecutive chunks: fresh statistics
 #pragma unroll
-      for (int h = 0; h < G; ++h) {
-        run_m[h] = -INFINITY;
-        run_s[h] = 0.f;
+        for (int h = 0; h < G; ++h) {
+          run_m[h] = -INFINITY;
+          run_s[h] = 0.f;
+        }
       }
       float* lkp = ws.lk + (int64_t)item.plane * dm.Ntot * (2 * G);
       for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
@@ -373,7 +395,17 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
           store_part<G>(lkp + tok * (2 * G), lg);
         }
       }
-      // ---- per-item softmax statistics: warp butterflies, then 4 warps ----
+      // ---- softmax statistics of a run, at its last chunk; the run's other
+      // chunks get empty statistics (m = -inf, s = 0), which merge as nothing
+      cont = is.next_same_unit(item);
+      if (cont) {
+        if (rw == 0 && lane < G) {
+          float* cs = ws.cstats + (((int64_t)item.plane * dm.c_cap + item.cidx) * G + lane) * 2;
+          cs[0] = -INFINITY;
+          cs[1] = 0.f;
+        }
+        continue;
+      }
 #pragma unroll
       for (int h = 0; h < G; ++h) {
         softmax_warp_merge(run_m[h], run_s[h]);

@@ -9,8 +9,9 @@
 // Each epilogue thread owns one token (one TMEM lane) and reduces
 // ||y||^2 = sum_j D[j]^2 in fp32, then multiplies by w_i. The tensor-memory accumulator
 // is double-buffered so the epilogue of tile i overlaps the MMAs of tile i+1,
-// and so is the L^{-1} image, so the next item's image streams in while the
-// current item's tiles run.
+// and so is the L^{-1} image: it is loaded once per run of consecutive items
+// of one unit, and the next unit's image streams in while the current run's
+// tiles go through.
 // float32 caches: SIMT forward products with L^{-1} held in shared memory.
 #include "jacap_dev.cuh"
 #include "jacap_internal.h"
@@ -37,7 +38,7 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
                       float* __restrict__ scores) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint8_t* mimg = smem;                       // [2][SC_M_BYTES], by item parity
+  uint8_t* mimg = smem;                       // [2][SC_M_BYTES], by run parity
   uint8_t* stages = smem + 2 * SC_M_BYTES;
   uint64_t* vfull = (uint64_t*)(stages + SC_STAGES * SC_TILE_BYTES);
   uint64_t* vempty = vfull + SC_STAGES;
@@ -83,17 +84,21 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
   if (warp == 0) {
     if (lane == 0) {
       prefetch_tmap(&vmap);
-      uint32_t it = 0, nitem = 0;
-      bool ok = true;
+      uint32_t it = 0, nrun = 0;
+      bool ok = true, cont = false;
       Item item;
       for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); ok && is.next(item);) {
         const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
         const int64_t u = (int64_t)item.plane * dm.S + item.seq;
-        const int mp = nitem & 1;
-        if (nitem >= 2 && !mbar_wait(smem_u32(&mempty[mp]), ((nitem >> 1) & 1) ^ 1, ws, abort)) break;
-        mbar_arrive_expect_tx(smem_u32(&mfull[mp]), SC_M_BYTES);
-        bulk_g2s(smem_u32(mimg + mp * SC_M_BYTES), ws.minv_img + u * SC_M_BYTES, SC_M_BYTES, smem_u32(&mfull[mp]));
-        ++nitem;
+        if (!cont) {  // a new unit: its image, into the buffer of the run before last
+          const int mp = nrun & 1;
+          if (nrun >= 2 && !mbar_wait(smem_u32(&mempty[mp]), ((nrun >> 1) & 1) ^ 1, ws, abort)) break;
+          mbar_arrive_expect_tx(smem_u32(&mfull[mp]), SC_M_BYTES);
+          bulk_g2s(smem_u32(mimg + mp * SC_M_BYTES), ws.minv_img + u * SC_M_BYTES, SC_M_BYTES,
+                   smem_u32(&mfull[mp]));
+          ++nrun;
+        }
+        cont = is.next_same_unit(item);
         for (int64_t t = item.t0; t < item.t1; t += TILE) {
           const int st = it % SC_STAGES;
           if (it >= (uint32_t)SC_STAGES &&
@@ -110,18 +115,21 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
       }
       for (uint32_t k = (it > (uint32_t)SC_STAGES ? it - SC_STAGES : 0); k < it; ++k)
         mbar_wait(smem_u32(&vfull[k % SC_STAGES]), (k / SC_STAGES) & 1, ws, nullptr);
-      for (uint32_t k = (nitem > 2 ? nitem - 2 : 0); k < nitem; ++k)
+      for (uint32_t k = (nrun > 2 ? nrun - 2 : 0); k < nrun; ++k)
         mbar_wait(smem_u32(&mfull[k & 1]), (k >> 1) & 1, ws, nullptr);
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      uint32_t it = 0, nitem = 0;
-      bool ok = true;
+      uint32_t it = 0, nrun = 0;
+      bool ok = true, cont = false;
+      int mp = 0;
       Item item;
       for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); ok && is.next(item);) {
-        const int mp = nitem & 1;
-        if (!mbar_wait(smem_u32(&mfull[mp]), (nitem >> 1) & 1, ws, abort)) break;
-        tc_fence_after();
+        if (!cont) {
+          mp = nrun & 1;
+          if (!mbar_wait(smem_u32(&mfull[mp]), (nrun >> 1) & 1, ws, abort)) break;
+          tc_fence_after();
+        }
         const uint32_t ma = smem_u32(mimg + mp * SC_M_BYTES);
         for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
           const int st = it % SC_STAGES;
@@ -156,8 +164,11 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
           umma_commit(smem_u32(&accfull[ab]));
         }
         if (!ok) break;
-        umma_commit(smem_u32(&mempty[mp]));
-        ++nitem;
+        cont = is.next_same_unit(item);
+        if (!cont) {  // the run's last MMAs read the image: release it after them
+          umma_commit(smem_u32(&mempty[mp]));
+          ++nrun;
+        }
       }
       // every MMA issued by this thread has completed before teardown
       umma_commit(smem_u32(mdone));
