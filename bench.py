@@ -365,14 +365,17 @@ def run_ours(args):
     kv_bytes = L * Hkv * N * d * es
     kept_rows = L * Hkv * sum(min(n, budget) for n in t.seqlens)
     G = wl.num_q_heads // wl.num_kv_heads
+    fused_weights = wl.dtype == "bf16"  # the tensor-core Gram computes the Eq. 8 weights itself
     alg_kernel = {
         "k_pass": kv_bytes,                       # K read once
-        "weights": L * Hkv * N * (8 * G + 8),     # logits + kappa read, w and its bf16 split written
-        "gram": kv_bytes,                         # V read once
+        # V read once; with the weights folded in also the logits + kappa rows read and w written
+        "gram": kv_bytes + (L * Hkv * N * (8 * G + 4) if fused_weights else 0),
         "scores": kv_bytes + L * Hkv * N * 4,     # V read, scores written
         "select": L * Hkv * N * 4,                # scores read
         "compact": 4 * kept_rows * d * es,        # retained K, V read and written
     }
+    if not fused_weights:
+        alg_kernel["weights"] = L * Hkv * N * (8 * G + 4)  # logits + kappa read, w written
     dom = max(alg_kernel, key=lambda k: kern[k])
     hbm, src = peaks()
     achieved = alg_kernel[dom] / (kern[dom] * 1e-3) / 1e9

@@ -140,9 +140,10 @@ size_t jacap_workspace_size(const jacap_layout* layout, int32_t budget);
  *               score of token t of plane (l, g); r_i of Eq. 10.
  *  ws, ws_bytes device workspace of at least jacap_workspace_size() bytes.
  * Resets the status word, then enqueues: query statistics, a streaming pass
- * over K (logits, kappa, softmax statistics), the Eq. 8 weights, the
- * weighted-Gram pass over V (tensor cores for bf16), the Cholesky factor and
- * inverse of A, and the quadratic forms.
+ * over K (logits, kappa, softmax statistics), the Eq. 8 weights (inside the
+ * weighted-Gram pass for bf16 caches), the weighted-Gram pass over V (tensor
+ * cores for bf16), the Cholesky factor and inverse of A, and the quadratic
+ * forms.
  */
 jacap_status jacap_score(const jacap_layout* layout, const jacap_params* params,
                          const void* q_win, const void* k, const void* v, float* scores,
@@ -154,7 +155,9 @@ jacap_status jacap_score(const jacap_layout* layout, const jacap_params* params,
  * events[num_events - 1] after the last one. `events` holds cudaEvent_t
  * handles (as void*) created by the caller; num_events must be 0 (no hooks)
  * or JACAP_SCORE_KERNELS + 1. Kernel order: plan, query statistics, K pass,
- * weights, Gram, factor, scores.
+ * weights, Gram, factor, scores. With bf16 caches the Gram kernel computes the
+ * Eq. 8 weights itself and the weights slot is empty (its two events are
+ * recorded back to back).
  */
 #define JACAP_SCORE_KERNELS 7
 jacap_status jacap_score_timed(const jacap_layout* layout, const jacap_params* params,

@@ -20,7 +20,7 @@ constexpr size_t ALIGN = 1024;
 inline size_t align_up(size_t x) { return (x + ALIGN - 1) & ~(ALIGN - 1); }
 
 struct Carve {
-  size_t status, plan, chunks, counters, mu, lam, qdev, lk, cstats, w, wsplit, gpart, pflag, gram, minv, minv_img,
+  size_t status, plan, chunks, counters, mu, lam, qdev, lk, cstats, w, gpart, pflag, gram, minv, minv_img,
       total;
 };
 
@@ -109,10 +109,9 @@ Carve carve(const Dims& dm) {
   // centred window queries: fp32 rows, or the bf16 hi/lo image (512 bytes per padded row)
   const size_t qrows = std::max((size_t)dm.G * dm.window, (size_t)kfull_rows_padded(dm.G, dm.window));
   c.qdev = o; o = align_up(o + (size_t)dm.S * dm.L * dm.Hkv * qrows * 512);
-  c.lk = o; o = align_up(o + planes * (size_t)dm.Ntot * 2 * dm.G * 4);
+  c.lk = o; o = align_up(o + planes * (size_t)dm.Ntot * 2 * dm.G * 4 + 16);  // + tail of 16-byte rounded copies
   c.cstats = o; o = align_up(o + planes * (size_t)dm.c_cap * dm.G * 2 * 4);
   c.w = o; o = align_up(o + planes * (size_t)dm.Ntot * 4);
-  c.wsplit = o; o = align_up(o + planes * (size_t)dm.Ntot * 4 + 64);  // + tail read by 16-byte rounded copies
   c.gpart = o; o = align_up(o + planes * (size_t)dm.c_cap * D * D * 4);
   c.pflag = o; o = align_up(o + planes * (size_t)dm.c_cap * 4);
   c.gram = o; o = align_up(o + units * D * D * 4);
@@ -136,7 +135,6 @@ Ws make_ws(void* base, const Carve& c) {
   ws.lk = (float*)(b + c.lk);
   ws.cstats = (float*)(b + c.cstats);
   ws.w = (float*)(b + c.w);
-  ws.wsplit = (uint32_t*)(b + c.wsplit);
   ws.gpart = (float*)(b + c.gpart);
   ws.pflag = (int32_t*)(b + c.pflag);
   ws.gram = (float*)(b + c.gram);
@@ -307,8 +305,9 @@ jacap_status score_pass(const jacap_layout* layout, const jacap_params* params, 
                                   persistent_grid(items, sms, kfull_uses_tensor_cores(dm, dt) ? 1 : 2), s))) !=
           JACAP_OK)
     return st;
+  // (bf16 caches: the Gram kernel computes the weights from the K pass's rows)
   if ((st = hook(3)) != JACAP_OK ||
-      (st = map_cuda(launch_weights(dm, w, cu, persistent_grid(items, sms, 8), s))) != JACAP_OK)
+      (!bf && (st = map_cuda(launch_weights(dm, w, cu, persistent_grid(items, sms, 8), s))) != JACAP_OK))
     return st;
   if ((st = hook(4)) != JACAP_OK ||
       (st = map_cuda(launch_gram(vmap, dm, w, dt, v, cu, persistent_grid(items, sms, bf ? 1 : 4), s))) != JACAP_OK)

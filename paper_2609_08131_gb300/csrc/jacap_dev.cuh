@@ -67,7 +67,6 @@ struct Ws {
   float* lk;          // [L*Hkv][Ntot][2G]  logits then kappa per query head of the group
   float* cstats;      // [L*Hkv][c_cap][G][2]  per-chunk (max, sum exp(l - max))
   float* w;           // [L*Hkv][Ntot]  Eq. 8 weights summed over the group
-  uint32_t* wsplit;   // [L*Hkv][Ntot]  w as bf16 hi (low half) + bf16 lo = w - hi (high half)
   float* gpart;       // [L*Hkv][c_cap][D/32][D][32]  partial Grams: (m, n) at ((n/32) D + m) 32 + n%32,
                       // lower 32 x 32 blocks only; one per run of a CTA's consecutive chunks of a unit,
                       // stored at the run's first chunk

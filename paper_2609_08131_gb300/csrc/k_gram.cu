@@ -45,8 +45,8 @@ __device__ __forceinline__ void unit_softmax_stats_warp(const Dims& dm, const Ws
 // weights): w_i = wdiv * sum_h [alpha_bar (1 - alpha_bar)]^2 kappa_h,i with
 // alpha_bar = exp(l_h,i - M_h) / Z_h; with the linear surrogate (S_C = I)
 // rho = 1 and w_i = wdiv * sum_h kappa_h,i. One streaming pass over the K pass's
-// logits/kappa rows; writes w (float32, for the score pass) and w as a bf16
-// pair hi + lo (for the tensor-core Gram, whose scaling is done in bf16).
+// logits/kappa rows that writes w, for float32 caches (with bf16 caches the
+// tensor-core Gram computes the same weights itself).
 constexpr int WT_THREADS = 256;
 
 template <int G>
@@ -115,8 +115,6 @@ __global__ void __launch_bounds__(WT_THREADS) weight_kernel(Dims dm, Ws ws, cons
         wt *= dm.wdiv;
         bad |= !isfinite(wt);
         ws.w[base + tok] = wt;
-        // hi = RN(w), lo = RN(w - hi) (w - hi is exact in float32)
-        ws.wsplit[base + tok] = pack_bf16x2(wt, wt - bf16lo(pack_bf16x2(wt, 0.f)));
       }
     }
   }
@@ -127,56 +125,72 @@ __global__ void __launch_bounds__(WT_THREADS) weight_kernel(Dims dm, Ws ws, cons
 // G = sum_i v_i (w_i v_i)^T on the tensor cores with the scaled operand in
 // tensor memory: D (128 x 128, fp32) += A (128 channels x 16 tokens, TMEM)
 // * B (16 tokens x 128 channels, the TMA-staged V tile, MN-major). The TMA
-// warp stages each V tile together with the tile's weights (bf16 pairs
-// hi + lo from the weight pass). The scaling warps read V transposed with
-// ldmatrix, form w_i v_i = hi + lo with packed bf16 arithmetic and store hi
-// and lo as two A operands; two MMAs per 16 tokens accumulate v (hi + lo)^T.
+// warp stages each V tile together with the tile's logits/kappa rows from the
+// K pass (2G floats per token). The weight warp turns them into the Eq. 8
+// weights (the same arithmetic as weight_kernel, with the unit's softmax
+// statistics merged once per run), writes w for the score pass and leaves w
+// as a bf16 pair hi + lo in the stage for the scaling warps. The scaling warps
+// read V transposed with ldmatrix, form w_i v_i = hi + lo with packed bf16
+// arithmetic and store hi and lo as two A operands; two MMAs per 16 tokens
+// accumulate v (hi + lo)^T.
 // The scaling warps share nothing but the mbarriers of the pipeline. A run of
 // consecutive chunks of one unit in a CTA's item range accumulates in one
 // tensor-memory buffer; four epilogue warps copy each finished run's Gram out
 // while the next run accumulates in the other buffer.
-constexpr int GR_THREADS = 448;   // warp 0: TMA, warp 1: MMA, warps 2-9: scale, warps 10-13: epilogue
+constexpr int GR_THREADS = 480;   // warp 0: TMA, 1: MMA, 2-9: scale, 10-13: epilogue, 14: weights
 constexpr int GR_EPI0 = 10;       // first epilogue warp
+constexpr int GR_WEIGHT_WARP = 14;
 constexpr int GR_SCALERS = 256;
-constexpr int GR_VST = 6;          // V tiles in flight
 constexpr int GR_BOX = 16384;      // {64 channels, 128 tokens} bf16, 128-byte swizzle
 constexpr int GR_V_BYTES = 2 * GR_BOX;
-constexpr int GR_W_BYTES = 640;    // weight words of a tile: <= 3 + 128, rounded to 16-byte copies
+constexpr int GR_W_BYTES = 512;    // the tile's weights as bf16 pairs, one word per token
 constexpr uint32_t GR_TMEM_COLS = 512;
 constexpr uint32_t GR_ACOL = 128;  // A buffers: [128 + 128 ab, +64) hi, [+64, +128) lo
 constexpr uint32_t GR_DCOL1 = 384; // accumulators: columns [0, 128) and [384, 512), alternating by item
 // M = 128 (channels), N = 128 (channels), A in TMEM (K-major), B MN-major.
 constexpr uint32_t GR_IDESC = idesc_bf16_f32(128, 128, 0, 1);
 
-constexpr size_t gram_bf16_smem_bytes() { return 1024 + GR_VST * (GR_V_BYTES + GR_W_BYTES) + 256; }
+template <int G>
+struct GrCfg {
+  static constexpr int LK_BYTES = TILE * 2 * G * 4 + 16;  // a tile's logits/kappa rows (+ alignment slack)
+  static constexpr int VST = G == 8 ? 5 : 6;              // stages in flight
+  static constexpr size_t SMEM = 1024 + (size_t)VST * (GR_V_BYTES + GR_W_BYTES + LK_BYTES) + 256;
+  static_assert(SMEM <= 232448, "shared memory");
+};
 
-// Weight words of the tile starting at token t of the plane: the copy starts
-// at the 16-byte boundary at or below the tile's first word (`off` words
-// before it) and covers the tile's `nvalid` tokens, rounded up to 16 bytes.
-struct WTile {
-  int64_t word0;  // first copied word (multiple of 4)
+// The tile's logits/kappa rows (2G floats per token): the copy starts at the
+// 16-byte boundary at or below the tile's first float (`off` floats before
+// it) and covers the tile's `nvalid` tokens, rounded up to 16 bytes.
+struct LkTile {
+  int64_t f0;  // first copied float (multiple of 4)
   int off, nvalid;
   uint32_t bytes;
 };
-__device__ __forceinline__ WTile weight_tile(const Dims& dm, const Item& item, int64_t t) {
-  WTile w;
-  const int64_t a = (int64_t)item.plane * dm.Ntot + t;
-  w.word0 = a & ~(int64_t)3;
-  w.off = (int)(a - w.word0);
-  w.nvalid = (int)(item.t1 - t < TILE ? item.t1 - t : TILE);
-  w.bytes = (uint32_t)(((w.off + w.nvalid + 3) & ~3) * 4);
-  return w;
+template <int G>
+__device__ __forceinline__ LkTile lk_tile(const Dims& dm, const Item& item, int64_t t) {
+  LkTile r;
+  const int64_t a = ((int64_t)item.plane * dm.Ntot + t) * (2 * G);
+  r.f0 = a & ~(int64_t)3;
+  r.off = (int)(a - r.f0);
+  r.nvalid = (int)(item.t1 - t < TILE ? item.t1 - t : TILE);
+  r.bytes = (uint32_t)(((r.off + r.nvalid * 2 * G + 3) & ~3) * 4);
+  return r;
 }
 
+template <int G>
 __global__ void __launch_bounds__(GR_THREADS, 1)
     gram_bf16_kernel(const __grid_constant__ CUtensorMap vmap, Dims dm, Ws ws, const int32_t* __restrict__ cu) {
+  using C = GrCfg<G>;
+  constexpr int GR_VST = C::VST;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t* vring = smem;                                   // [GR_VST][GR_V_BYTES]
   uint8_t* wring = vring + GR_VST * GR_V_BYTES;            // [GR_VST][GR_W_BYTES] weight words
-  uint64_t* vfull = (uint64_t*)(wring + GR_VST * GR_W_BYTES);
+  uint8_t* lkring = wring + GR_VST * GR_W_BYTES;           // [GR_VST][LK_BYTES] logits/kappa rows
+  uint64_t* vfull = (uint64_t*)(lkring + GR_VST * C::LK_BYTES);
   uint64_t* vempty = vfull + GR_VST;
-  uint64_t* afull = vempty + GR_VST;
+  uint64_t* wready = vempty + GR_VST;  // the weight warp has written the tile's weights
+  uint64_t* afull = wready + GR_VST;
   uint64_t* aempty = afull + 2;
   uint64_t* accfull = aempty + 2;   // [2]
   uint64_t* accempty = accfull + 2; // [2]
@@ -190,6 +204,7 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
     for (int i = 0; i < GR_VST; ++i) {
       mbar_init(smem_u32(&vfull[i]), 1);
       mbar_init(smem_u32(&vempty[i]), 1);
+      mbar_init(smem_u32(&wready[i]), 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&afull[i]), GR_SCALERS / 32);
@@ -230,12 +245,12 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
             break;
           }
           uint8_t* vt = vring + st * GR_V_BYTES;
-          const WTile wt = weight_tile(dm, item, t);
+          const LkTile lt = lk_tile<G>(dm, item, t);
           const uint32_t bar = smem_u32(&vfull[st]);
-          mbar_arrive_expect_tx(bar, GR_V_BYTES + wt.bytes);
+          mbar_arrive_expect_tx(bar, GR_V_BYTES + lt.bytes);
           tma_load_4d(smem_u32(vt), &vmap, 0, (int)t, g, l, bar);
           tma_load_4d(smem_u32(vt + GR_BOX), &vmap, 64, (int)t, g, l, bar);
-          bulk_g2s(smem_u32(wring + st * GR_W_BYTES), ws.wsplit + wt.word0, wt.bytes, bar);
+          bulk_g2s(smem_u32(lkring + st * C::LK_BYTES), ws.lk + lt.f0, lt.bytes, bar);
           ++it;
         }
       }
@@ -300,19 +315,21 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
     for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
       for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
         const int vs = it % GR_VST, ab = it & 1;
-        if (!mbar_wait(smem_u32(&vfull[vs]), (it / GR_VST) & 1, ws, abort)) goto scale_done;
+        if (!mbar_wait(smem_u32(&vfull[vs]), (it / GR_VST) & 1, ws, abort) ||
+            !mbar_wait(smem_u32(&wready[vs]), (it / GR_VST) & 1, ws, abort))
+          goto scale_done;
         // weights of this lane's token pairs (rows 2(l%4), 2(l%4)+1 of each
         // 8-token half of its 4 blocks) as bf16 pairs; tokens past the item
         // weigh zero
         uint32_t wph[8], wpl[8];
         {
-          const WTile wt = weight_tile(dm, item, t);
-          const uint32_t wsl = smem_u32(wring + vs * GR_W_BYTES) + 4 * wt.off;
+          const int nvalid = (int)(item.t1 - t < TILE ? item.t1 - t : TILE);
+          const uint32_t wsl = smem_u32(wring + vs * GR_W_BYTES);
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
             const int i0 = 16 * (4 * th + (e >> 1)) + 8 * (e & 1) + 2 * (lane & 3);
-            const uint32_t x0 = i0 < wt.nvalid ? lds_u32(wsl + 4 * i0) : 0u;
-            const uint32_t x1 = i0 + 1 < wt.nvalid ? lds_u32(wsl + 4 * i0 + 4) : 0u;
+            const uint32_t x0 = i0 < nvalid ? lds_u32(wsl + 4 * i0) : 0u;
+            const uint32_t x1 = i0 + 1 < nvalid ? lds_u32(wsl + 4 * i0 + 4) : 0u;
             wph[e] = __byte_perm(x0, x1, 0x5410);  // (hi of token i0, hi of i0 + 1)
             wpl[e] = __byte_perm(x0, x1, 0x7632);  // (lo, lo)
           }
@@ -354,6 +371,68 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
       }
     }
   scale_done:;
+  } else if (warp == GR_WEIGHT_WARP) {
+    // ------------------------------------------------------ weights -------
+    // Eq. 8 for the tile's tokens (four per lane) from the staged logits and
+    // kappa: w = wdiv sum_h rho_h^2 kappa_h, rho = alpha_bar (1 - alpha_bar),
+    // alpha_bar = exp(l_h - M_h) / Z_h (rho = 1 for the linear surrogate);
+    // (M_h, Z_h) merged from the unit's chunk statistics once per run.
+    uint32_t it = 0;
+    bool bad = false, cont = false;
+    float u[2 * G];  // M_h, then 1 / Z_h
+#pragma unroll
+    for (int e = 0; e < 2 * G; ++e) u[e] = 0.f;
+    Item item;
+    for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
+      if (!cont && !dm.linear) {
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+          float M, Z;
+          unit_softmax_stats_warp<G>(dm, ws, item.plane, item.seq, h, M, Z);
+          u[h] = M;
+          u[G + h] = 1.f / Z;
+        }
+      }
+      cont = is.next_same_unit(item);
+      const int64_t base = (int64_t)item.plane * dm.Ntot;
+      for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
+        const int vs = it % GR_VST;
+        if (!mbar_wait(smem_u32(&vfull[vs]), (it / GR_VST) & 1, ws, abort)) goto weights_done;
+        const LkTile lt = lk_tile<G>(dm, item, t);
+        const float* rows = (const float*)(lkring + vs * C::LK_BYTES) + lt.off;
+        uint32_t* wout = (uint32_t*)(wring + vs * GR_W_BYTES);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int i = lane + 32 * q;
+          uint32_t word = 0u;
+          if (i < lt.nvalid) {
+            const float* r = rows + i * 2 * G;
+            float wt = 0.f;
+            if (dm.linear) {
+#pragma unroll
+              for (int h = 0; h < G; ++h) wt += r[G + h];
+            } else {
+#pragma unroll
+              for (int h = 0; h < G; ++h) {
+                const float a = expf(r[h] - u[h]) * u[G + h];  // alpha_bar
+                const float rho = a * (1.f - a);                // diagonal of the softmax Jacobian
+                wt = fmaf(rho * rho, r[G + h], wt);             // rho^2 kappa
+              }
+            }
+            wt *= dm.wdiv;
+            bad |= !isfinite(wt);
+            ws.w[base + t + i] = wt;
+            // hi = RN(w), lo = RN(w - hi) (w - hi is exact in float32)
+            word = pack_bf16x2(wt, wt - bf16lo(pack_bf16x2(wt, 0.f)));
+          }
+          wout[i] = word;
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&wready[vs]));
+      }
+    }
+  weights_done:
+    if (bad) flag(ws, ST_NONFINITE);
   } else {
     // ------------------------------------------------------ epilogue ------
     // D is a chunk's partial Gram; warp (quarter q) copies rows 32 q .. +31,
@@ -490,13 +569,26 @@ cudaError_t launch_weights(const Dims& dm, const Ws& ws, const int32_t* cu, int 
   }
 }
 
+template <int G>
+static cudaError_t launch_gram_bf16(const CUtensorMap& vmap, const Dims& dm, const Ws& ws, const int32_t* cu,
+                                   int grid, cudaStream_t st) {
+  constexpr size_t smem = GrCfg<G>::SMEM;
+  cudaError_t e = cudaFuncSetAttribute(gram_bf16_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  gram_bf16_kernel<G><<<grid, GR_THREADS, smem, st>>>(vmap, dm, ws, cu);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_gram(const CUtensorMap& vmap, const Dims& dm, const Ws& ws, int dtype, const void* v,
                         const int32_t* cu, int grid, cudaStream_t st) {
   if (dtype == 1) {
-    constexpr size_t smem = gram_bf16_smem_bytes();
-    cudaError_t e = cudaFuncSetAttribute(gram_bf16_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    gram_bf16_kernel<<<grid, GR_THREADS, smem, st>>>(vmap, dm, ws, cu);
+    switch (dm.G) {
+      case 1: return launch_gram_bf16<1>(vmap, dm, ws, cu, grid, st);
+      case 2: return launch_gram_bf16<2>(vmap, dm, ws, cu, grid, st);
+      case 4: return launch_gram_bf16<4>(vmap, dm, ws, cu, grid, st);
+      case 8: return launch_gram_bf16<8>(vmap, dm, ws, cu, grid, st);
+      default: return cudaErrorInvalidValue;
+    }
   } else {
     gram_f32_kernel<<<grid, GF_THREADS, 0, st>>>(dm, ws, cu, (const float*)v);
   }
