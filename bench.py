@@ -365,11 +365,14 @@ def run_ours(args):
     kv_bytes = L * Hkv * N * d * es
     kept_rows = L * Hkv * sum(min(n, budget) for n in t.seqlens)
     G = wl.num_q_heads // wl.num_kv_heads
-    fused_weights = wl.dtype == "bf16"  # the tensor-core Gram computes the Eq. 8 weights itself
+    # Algorithmic bytes count the K, V, window and retained-row traffic only; the
+    # logits/kappa round trip, the second read of V and the partials are extra
+    # traffic (visible in `traffic`). With bf16 caches the Gram computes the
+    # Eq. 8 weights itself (it also reads the logits/kappa rows).
+    fused_weights = wl.dtype == "bf16"
     alg_kernel = {
         "k_pass": kv_bytes,                       # K read once
-        # V read once; with the weights folded in also the logits + kappa rows read and w written
-        "gram": kv_bytes + (L * Hkv * N * (8 * G + 4) if fused_weights else 0),
+        "gram": kv_bytes,                         # V read once
         "scores": kv_bytes + L * Hkv * N * 4,     # V read, scores written
         "select": L * Hkv * N * 4,                # scores read
         "compact": 4 * kept_rows * d * es,        # retained K, V read and written
