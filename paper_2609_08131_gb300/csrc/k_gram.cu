@@ -137,9 +137,9 @@ __global__ void __launch_bounds__(WT_THREADS) weight_kernel(Dims dm, Ws ws, cons
 // consecutive chunks of one unit in a CTA's item range accumulates in one
 // tensor-memory buffer; four epilogue warps copy each finished run's Gram out
 // while the next run accumulates in the other buffer.
-constexpr int GR_THREADS = 480;   // warp 0: TMA, 1: MMA, 2-9: scale, 10-13: epilogue, 14: weights
+constexpr int GR_THREADS = 512;   // warp 0: TMA, 1: MMA, 2-9: scale, 10-13: epilogue, 14-15: weights
 constexpr int GR_EPI0 = 10;       // first epilogue warp
-constexpr int GR_WEIGHT_WARP = 14;
+constexpr int GR_WEIGHT_WARP = 14;  // 14 and 15, 64 tokens of each tile each
 constexpr int GR_SCALERS = 256;
 constexpr int GR_BOX = 16384;      // {64 channels, 128 tokens} bf16, 128-byte swizzle
 constexpr int GR_V_BYTES = 2 * GR_BOX;
@@ -204,7 +204,7 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
     for (int i = 0; i < GR_VST; ++i) {
       mbar_init(smem_u32(&vfull[i]), 1);
       mbar_init(smem_u32(&vempty[i]), 1);
-      mbar_init(smem_u32(&wready[i]), 1);
+      mbar_init(smem_u32(&wready[i]), 2);  // the two weight warps
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&afull[i]), GR_SCALERS / 32);
@@ -371,9 +371,9 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
       }
     }
   scale_done:;
-  } else if (warp == GR_WEIGHT_WARP) {
+  } else if (warp >= GR_WEIGHT_WARP) {
     // ------------------------------------------------------ weights -------
-    // Eq. 8 for the tile's tokens (four per lane) from the staged logits and
+    // Eq. 8 for the tile's tokens (two per lane of each of the two warps) from the staged logits and
     // kappa: w = wdiv sum_h rho_h^2 kappa_h, rho = alpha_bar (1 - alpha_bar),
     // alpha_bar = exp(l_h - M_h) / Z_h (rho = 1 for the linear surrogate);
     // (M_h, Z_h) merged from the unit's chunk statistics once per run.
@@ -402,11 +402,22 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
         const float* rows = (const float*)(lkring + vs * C::LK_BYTES) + lt.off;
         uint32_t* wout = (uint32_t*)(wring + vs * GR_W_BYTES);
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const int i = lane + 32 * q;
+        for (int q = 0; q < 2; ++q) {
+          const int i = 64 * (warp - GR_WEIGHT_WARP) + lane + 32 * q;
           uint32_t word = 0u;
           if (i < lt.nvalid) {
-            const float* r = rows + i * 2 * G;
+            float r[2 * G];
+            if constexpr ((2 * G) % 4 == 0) {  // 16-byte aligned rows (off = 0 for G >= 2)
+#pragma unroll
+              for (int e = 0; e < 2 * G; e += 4) {
+                const float4 x = *(const float4*)(rows + i * 2 * G + e);
+                r[e] = x.x; r[e + 1] = x.y; r[e + 2] = x.z; r[e + 3] = x.w;
+              }
+            } else {
+              const float2 x = *(const float2*)(rows + i * 2 * G);
+              r[0] = x.x;
+              r[1] = x.y;
+            }
             float wt = 0.f;
             if (dm.linear) {
 #pragma unroll
