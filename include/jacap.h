@@ -139,7 +139,8 @@ size_t jacap_workspace_size(const jacap_layout* layout, int32_t budget);
  *  scores       device float32 [num_layers][num_kv_heads][total_tokens]:
  *               score of token t of plane (l, g); r_i of Eq. 10.
  *  ws, ws_bytes device workspace of at least jacap_workspace_size() bytes.
- * Resets the status word, then enqueues: query statistics, a streaming pass
+ * Enqueues: a planning kernel (which also resets the status word), query
+ * statistics, a streaming pass
  * over K (logits, kappa, softmax statistics), the Eq. 8 weights (inside the
  * weighted-Gram pass for bf16 caches), the weighted-Gram pass over V (tensor
  * cores for bf16), the Cholesky factor and inverse of A, and the quadratic

@@ -291,7 +291,6 @@ jacap_status score_pass(const jacap_layout* layout, const jacap_params* params, 
     if (num_events == 0) return JACAP_OK;
     return map_cuda(cudaEventRecord((cudaEvent_t)events[i], s));
   };
-  if ((st = map_cuda(cudaMemsetAsync(w.status, 0, 64, s))) != JACAP_OK) return st;
   if ((st = hook(0)) != JACAP_OK || (st = map_cuda(launch_plan(dm, w, cu, s))) != JACAP_OK) return st;
   if ((st = hook(1)) != JACAP_OK ||
       (st = map_cuda(running ? launch_stats_moments(dm, w, stats, counts, s)

@@ -53,9 +53,9 @@ jacap_status jacap_score_static(const jacap_layout* layout, const jacap_params* 
   void* ws = scratch_for_current_device();
   if (ws == nullptr) return JACAP_ERR_CUDA;
   if (scratch_out != nullptr) *scratch_out = ws;
-  // jacap_score clears the status word (the only state that must start at
-  // zero) on the stream before its first kernel; every other section of the
-  // workspace is written before it is read within one pass.
+  // jacap_score's first kernel clears the status word (the only state that
+  // must start at zero); every other section of the workspace is written
+  // before it is read within one pass.
   return jacap_score(layout, params, q_win, k, v, scores, ws, (size_t)JACAP_STATIC_SCRATCH_BYTES, stream);
 }
 

@@ -1,7 +1,8 @@
 // k_stream.cu - work plan, query-window statistics and the streaming K pass.
 //
-//  plan_kernel          validates cu_seqlens and lays out the work items
-//                       (chunks of `chunk` tokens that never straddle requests).
+//  plan_kernel          clears the status word, validates cu_seqlens and lays
+//                       out the work items (chunks of `chunk` tokens that never
+//                       straddle requests) in the chunk table.
 //  window_stats_kernel  mu_h and the diagonal of Lambda_Q from the last w queries
 //                       of each query head (Sec. 3.4 last paragraph; App. B.2).
 //  kpass_kernel         (float32 caches; bf16 caches use k_kpass.cu) one
@@ -16,39 +17,43 @@
 
 namespace jacap {
 
-__global__ void plan_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu) {
-  if (threadIdx.x != 0) return;
-  bool ok = (cu[0] == 0) && ((int64_t)cu[dm.S] == dm.Ntot);
-  int32_t acc = 0;
-  ws.plan[1] = 0;
-  for (int s = 0; s < dm.S; ++s) {
-    const int32_t n = cu[s + 1] - cu[s];
-    if (n < 0) ok = false;
-    const int32_t c = n > 0 ? (n + dm.chunk - 1) / dm.chunk : 0;
-    acc += c;
-    ws.plan[2 + s] = acc;
+// The pass's first kernel, one block: clears the status word, validates
+// cu_seqlens and lays out the chunks (thread 0), then writes the chunk table:
+// record r = {t0, t1, request, r} for the C_tot chunks of a plane.
+__global__ void __launch_bounds__(256) plan_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu) {
+  __shared__ int s_ctot;
+  if (threadIdx.x < 16) ws.status[threadIdx.x] = 0u;
+  if (threadIdx.x == 0) {
+    bool ok = (cu[0] == 0) && ((int64_t)cu[dm.S] == dm.Ntot);
+    int32_t acc = 0;
+    ws.plan[1] = 0;
+    for (int s = 0; s < dm.S; ++s) {
+      const int32_t n = cu[s + 1] - cu[s];
+      if (n < 0) ok = false;
+      const int32_t c = n > 0 ? (n + dm.chunk - 1) / dm.chunk : 0;
+      acc += c;
+      ws.plan[2 + s] = acc;
+    }
+    if (!ok || acc > dm.c_cap) {
+      atomicOr(ws.status, ST_INVALID);
+      acc = 0;
+    }
+    ws.plan[0] = acc;
+    s_ctot = acc;
   }
-  if (!ok || acc > dm.c_cap) {
-    atomicOr(ws.status, ST_INVALID);
-    acc = 0;
+  __syncthreads();
+  const int ctot = s_ctot;
+  for (int r = threadIdx.x; r < ctot; r += blockDim.x) {
+    // largest s with prefix[s] <= r (prefix is plan[1 .. S+1], nondecreasing)
+    int lo = 0, hi = dm.S - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (ws.plan[1 + mid] <= r) lo = mid; else hi = mid - 1;
+    }
+    const int64_t t0 = (int64_t)cu[lo] + (int64_t)(r - ws.plan[1 + lo]) * dm.chunk;
+    const int64_t t1 = min((int64_t)cu[lo + 1], t0 + (int64_t)dm.chunk);
+    ws.chunks[r] = make_int4((int)t0, (int)t1, lo, r);
   }
-  ws.plan[0] = acc;
-}
-
-// Chunk table: record r = {t0, t1, request, r} for the C_tot chunks of a plane.
-__global__ void chunk_table_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu) {
-  const int ctot = ws.plan[0];
-  const int r = blockIdx.x * blockDim.x + threadIdx.x;
-  if (r >= ctot) return;
-  // largest s with prefix[s] <= r (prefix is plan[1 .. S+1], nondecreasing)
-  int lo = 0, hi = dm.S - 1;
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (ws.plan[1 + mid] <= r) lo = mid; else hi = mid - 1;
-  }
-  const int64_t t0 = (int64_t)cu[lo] + (int64_t)(r - ws.plan[1 + lo]) * dm.chunk;
-  const int64_t t1 = min((int64_t)cu[lo + 1], t0 + (int64_t)dm.chunk);
-  ws.chunks[r] = make_int4((int)t0, (int)t1, lo, r);
 }
 
 template <typename T>
@@ -319,10 +324,7 @@ static cudaError_t launch_window_stats_t(const Dims& dm, const Ws& ws, const voi
 }
 
 cudaError_t launch_plan(const Dims& dm, const Ws& ws, const int32_t* cu, cudaStream_t st) {
-  plan_kernel<<<1, 32, 0, st>>>(dm, ws, cu);
-  const cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  chunk_table_kernel<<<(unsigned)((dm.c_cap + 255) / 256), 256, 0, st>>>(dm, ws, cu);
+  plan_kernel<<<1, 256, 0, st>>>(dm, ws, cu);
   return cudaGetLastError();
 }
 
