@@ -69,6 +69,7 @@ int pick_chunk(const jacap_layout* L) {
 
 void make_dims(const jacap_layout* L, const jacap_params* P, Dims& dm) {
   memset(&dm, 0, sizeof(dm));
+  dm.pdl = 1;
   dm.S = L->num_seqs;
   dm.L = L->num_layers;
   dm.Hq = L->num_q_heads;
@@ -275,6 +276,7 @@ jacap_status score_pass(const jacap_layout* layout, const jacap_params* params, 
   Dims dm;
   make_dims(layout, params, dm);
   dm.dense_minv = out_factor != nullptr ? 1 : 0;
+  dm.pdl = num_events == 0 ? 1 : 0;  // timing events between kernels serialise them anyway
   const Carve c = carve(dm);
   if (((uintptr_t)ws & 255u) != 0 || ws_bytes < c.total) return JACAP_ERR_WORKSPACE;
   int sms = 0;

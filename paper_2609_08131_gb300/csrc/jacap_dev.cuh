@@ -42,6 +42,7 @@ struct Dims {
   int dense_minv;     // 1: the score matrix is a full 128 x 128 (output directions), not triangular
   int full_cov;       // 1: kappa with the full window covariance of the queries (App. B.2)
   int kf_rp;          // full covariance on the tensor cores: rows per split part of the query image (else 0)
+  int pdl;            // 1: launch with programmatic stream serialization (0 when timing events sit between kernels)
 };
 
 // Rows per split part of the full-covariance query image of one KV head's
@@ -122,6 +123,15 @@ struct ItemStream {
     return i < end && (int)(i / ctot) == cur.plane && rec.z == cur.seq;
   }
 };
+
+// Programmatic dependent launch. A kernel launched with the programmatic
+// stream-serialization attribute is set up while the previous kernel of the
+// stream still runs and is scheduled as its CTAs exit (no kernel here triggers
+// its dependents early: measured, an early trigger made the pass slower). Every
+// kernel starts with pdl_wait(), which blocks until the previous kernel has
+// completed with its memory visible (a no-op for a normal launch). Nothing
+// before pdl_wait() may touch global memory.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
 __device__ __forceinline__ bool status_failed(const Ws& ws) {
   return *((volatile uint32_t*)ws.status) != 0u;

@@ -7,6 +7,32 @@
 
 namespace jacap {
 
+// Returns a failed CUDA call's error from the enclosing launcher.
+#define JACAP_TRY(call)                     \
+  do {                                      \
+    const cudaError_t e_ = (call);          \
+    if (e_ != cudaSuccess) return e_;       \
+  } while (0)
+
+// Launch `kernel`, with programmatic stream serialization when `pdl` (see
+// pdl_wait()): the launch is prepared while the previous kernel of the stream
+// runs and the kernel waits for it inside. Returns the launch error.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(bool pdl, void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                       Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = pdl ? attr : nullptr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 cudaError_t launch_plan(const Dims& dm, const Ws& ws, const int32_t* cu, cudaStream_t st);
 cudaError_t launch_window_stats(const Dims& dm, const Ws& ws, int dtype, const void* q, cudaStream_t st);
 cudaError_t launch_kpass(const CUtensorMap& kmap, const Dims& dm, const Ws& ws, int dtype, const int32_t* cu,

@@ -46,6 +46,7 @@ __device__ __forceinline__ float q_elem<__nv_bfloat16>(const __nv_bfloat16* p) {
 template <typename T>
 __global__ void __launch_bounds__(D)
     stats_update_kernel(Dims dm, const T* __restrict__ q, float* stats, int32_t* counts, int reset) {
+  pdl_wait();
   const int b = blockIdx.x;
   const int h = b % dm.Hq;
   const int l = (b / dm.Hq) % dm.L;
@@ -81,6 +82,7 @@ __global__ void __launch_bounds__(D)
 // outputs as the window statistics (mu / (tau sqrt d) and lambda).
 __global__ void __launch_bounds__(D)
     stats_moments_kernel(Dims dm, Ws ws, const float* __restrict__ stats, const int32_t* __restrict__ counts) {
+  pdl_wait();
   if (status_failed(ws)) return;
   const int b = blockIdx.x, c = threadIdx.x;
   const int n = counts[b];
@@ -103,6 +105,7 @@ template <typename T>
 __global__ void __launch_bounds__(CI_THREADS)
     compact_inplace_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu, T* k, T* v, int32_t* pos,
                            const int32_t* __restrict__ idx, int budget) {
+  pdl_wait();
   constexpr int RB = D * (int)sizeof(T) / 16;  // 16-byte pieces per row
   constexpr int CH = CI_CHUNK_BYTES / (D * (int)sizeof(T));
   constexpr int PER = CH * RB / CI_THREADS;    // pieces per thread and tensor
@@ -167,6 +170,7 @@ template <typename T>
 __global__ void __launch_bounds__(CI_THREADS)
     fill_holes_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu, T* k, T* v, int32_t* pos,
                       const int32_t* __restrict__ idx, int budget) {
+  pdl_wait();
   constexpr int RB = D * (int)sizeof(T) / 16;
   __shared__ int s_f;
   if (status_failed(ws)) return;
@@ -215,7 +219,8 @@ __global__ void __launch_bounds__(CI_THREADS)
 template <typename T>
 static cudaError_t launch_stats_update_t(const Dims& dm, const void* q, float* stats, int32_t* counts, int reset,
                                          cudaStream_t st) {
-  stats_update_kernel<T><<<dm.S * dm.L * dm.Hq, D, 0, st>>>(dm, (const T*)q, stats, counts, reset);
+  JACAP_TRY(launch_pdl(dm.pdl != 0, stats_update_kernel<T>, dm.S * dm.L * dm.Hq, D, 0, st, dm, (const T*)q, stats,
+                       counts, reset));
   return cudaGetLastError();
 }
 
@@ -227,7 +232,7 @@ cudaError_t launch_stats_update(const Dims& dm, int dtype, const void* q, float*
 
 cudaError_t launch_stats_moments(const Dims& dm, const Ws& ws, const float* stats, const int32_t* counts,
                                  cudaStream_t st) {
-  stats_moments_kernel<<<dm.S * dm.L * dm.Hq, D, 0, st>>>(dm, ws, stats, counts);
+  JACAP_TRY(launch_pdl(dm.pdl != 0, stats_moments_kernel, dm.S * dm.L * dm.Hq, D, 0, st, dm, ws, stats, counts));
   return cudaGetLastError();
 }
 
@@ -237,17 +242,19 @@ cudaError_t launch_compact_inplace(const Dims& dm, const Ws& ws, int dtype, cons
   const int units = dm.L * dm.Hkv * dm.S;
   if (!preserve_order) {
     if (dtype == 1)
-      fill_holes_kernel<__nv_bfloat16><<<units, CI_THREADS, 0, st>>>(dm, ws, cu, (__nv_bfloat16*)k,
-                                                                     (__nv_bfloat16*)v, pos, idx, budget);
+      JACAP_TRY(launch_pdl(dm.pdl != 0, fill_holes_kernel<__nv_bfloat16>, units, CI_THREADS, 0, st, dm, ws, cu,
+                           (__nv_bfloat16*)k, (__nv_bfloat16*)v, pos, idx, budget));
     else
-      fill_holes_kernel<float><<<units, CI_THREADS, 0, st>>>(dm, ws, cu, (float*)k, (float*)v, pos, idx, budget);
+      JACAP_TRY(launch_pdl(dm.pdl != 0, fill_holes_kernel<float>, units, CI_THREADS, 0, st, dm, ws, cu, (float*)k,
+                           (float*)v, pos, idx, budget));
     return cudaGetLastError();
   }
   if (dtype == 1)
-    compact_inplace_kernel<__nv_bfloat16><<<units, CI_THREADS, 0, st>>>(
-        dm, ws, cu, (__nv_bfloat16*)k, (__nv_bfloat16*)v, pos, idx, budget);
+    JACAP_TRY(launch_pdl(dm.pdl != 0, compact_inplace_kernel<__nv_bfloat16>, units, CI_THREADS, 0, st, dm, ws, cu,
+                         (__nv_bfloat16*)k, (__nv_bfloat16*)v, pos, idx, budget));
   else
-    compact_inplace_kernel<float><<<units, CI_THREADS, 0, st>>>(dm, ws, cu, (float*)k, (float*)v, pos, idx, budget);
+    JACAP_TRY(launch_pdl(dm.pdl != 0, compact_inplace_kernel<float>, units, CI_THREADS, 0, st, dm, ws, cu, (float*)k,
+                         (float*)v, pos, idx, budget));
   return cudaGetLastError();
 }
 

@@ -60,6 +60,7 @@ constexpr size_t factor_smem_bytes() { return (size_t)(PROJ ? 2 : 1) * D * FA_LD
 template <bool PROJ>
 __global__ void __launch_bounds__(FA_THREADS, PROJ ? 1 : 2)
     factor_kernel(Dims dm, Ws ws, const float* __restrict__ out_factor) {
+  pdl_wait();
   extern __shared__ float Ms[];  // [D][FA_LD]: L^{-1} staged for the bf16 image (PROJ: R0, then R1)
   __shared__ __align__(16) float colA[2][D];
   __shared__ __align__(16) float rowY[2][D];
@@ -468,6 +469,7 @@ __device__ __forceinline__ void trailing_update(float* As, int K, int i0, int i1
 }
 
 __global__ void __launch_bounds__(FB_THREADS, 2) factor_blocked_kernel(Dims dm, Ws ws) {
+  pdl_wait();
   extern __shared__ __align__(16) float fsm[];
   float* As = fsm;                // tri(I, J): A_IJ, then L_IJ (I > J) / T_II (I == J)
   float* XT = fsm + 10 * FB_BLK;  // tri(I, J): XT_JI = (L^{-1})_IJ^T
@@ -676,7 +678,7 @@ static cudaError_t launch_factor_t(const Dims& dm, const Ws& ws, const float* ou
   cudaError_t e = cudaFuncSetAttribute(factor_kernel<PROJ>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   const int units = dm.L * dm.Hkv * dm.S;
-  factor_kernel<PROJ><<<units, FA_THREADS, smem, st>>>(dm, ws, out_factor);
+  JACAP_TRY(launch_pdl(dm.pdl != 0, factor_kernel<PROJ>, units, FA_THREADS, smem, st, dm, ws, out_factor));
   return cudaGetLastError();
 }
 
@@ -685,7 +687,7 @@ cudaError_t launch_factor(const Dims& dm, const Ws& ws, const float* out_factor,
   cudaError_t e = cudaFuncSetAttribute(factor_blocked_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)FB_SMEM);
   if (e != cudaSuccess) return e;
-  factor_blocked_kernel<<<dm.L * dm.Hkv * dm.S, FB_THREADS, FB_SMEM, st>>>(dm, ws);
+  JACAP_TRY(launch_pdl(dm.pdl != 0, factor_blocked_kernel, dm.L * dm.Hkv * dm.S, FB_THREADS, FB_SMEM, st, dm, ws));
   return cudaGetLastError();
 }
 

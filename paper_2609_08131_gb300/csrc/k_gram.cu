@@ -51,6 +51,7 @@ constexpr int WT_THREADS = 256;
 
 template <int G>
 __global__ void __launch_bounds__(WT_THREADS) weight_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu) {
+  pdl_wait();
   __shared__ float us[2 * G];  // M_h, then 1 / Z_h
   __shared__ int s_skip;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -180,6 +181,7 @@ __device__ __forceinline__ LkTile lk_tile(const Dims& dm, const Item& item, int6
 template <int G>
 __global__ void __launch_bounds__(GR_THREADS, 1)
     gram_bf16_kernel(const __grid_constant__ CUtensorMap vmap, Dims dm, Ws ws, const int32_t* __restrict__ cu) {
+  pdl_wait();
   using C = GrCfg<G>;
   constexpr int GR_VST = C::VST;
   extern __shared__ uint8_t smem_raw[];
@@ -500,6 +502,7 @@ constexpr int GF_LD = D + 4;
 
 __global__ void __launch_bounds__(GF_THREADS)
     gram_f32_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu, const float* __restrict__ v) {
+  pdl_wait();
   __shared__ float xs[GF_SLAB][GF_LD];  // w_i v_i
   __shared__ float vs[GF_SLAB][GF_LD];  // v_i
   __shared__ float wsl[GF_SLAB];
@@ -566,7 +569,7 @@ __global__ void __launch_bounds__(GF_THREADS)
 // ------------------------------------------------------------ launchers ----
 template <int G>
 static cudaError_t launch_weights_g(const Dims& dm, const Ws& ws, const int32_t* cu, int grid, cudaStream_t st) {
-  weight_kernel<G><<<grid, WT_THREADS, 0, st>>>(dm, ws, cu);
+  JACAP_TRY(launch_pdl(dm.pdl != 0, weight_kernel<G>, grid, WT_THREADS, 0, st, dm, ws, cu));
   return cudaGetLastError();
 }
 
@@ -586,7 +589,7 @@ static cudaError_t launch_gram_bf16(const CUtensorMap& vmap, const Dims& dm, con
   constexpr size_t smem = GrCfg<G>::SMEM;
   cudaError_t e = cudaFuncSetAttribute(gram_bf16_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  gram_bf16_kernel<G><<<grid, GR_THREADS, smem, st>>>(vmap, dm, ws, cu);
+  JACAP_TRY(launch_pdl(dm.pdl != 0, gram_bf16_kernel<G>, grid, GR_THREADS, smem, st, vmap, dm, ws, cu));
   return cudaGetLastError();
 }
 
@@ -601,7 +604,7 @@ cudaError_t launch_gram(const CUtensorMap& vmap, const Dims& dm, const Ws& ws, i
       default: return cudaErrorInvalidValue;
     }
   } else {
-    gram_f32_kernel<<<grid, GF_THREADS, 0, st>>>(dm, ws, cu, (const float*)v);
+    JACAP_TRY(launch_pdl(dm.pdl != 0, gram_f32_kernel, grid, GF_THREADS, 0, st, dm, ws, cu, (const float*)v));
   }
   return cudaGetLastError();
 }

@@ -16,8 +16,9 @@
 // instead of the 8 that one bf16 rounding would leave). The query-statistics
 // kernel writes that B operand straight into the workspace in shared-memory
 // image form; here it is one bulk copy per unit (a CTA's consecutive items
-// of one unit share it), issued one item ahead into a double buffer. One MMA job of N = 2 rp columns per 128-token tile, the
-// accumulator double-buffered in tensor memory, so one tile's readout overlaps
+// of one unit share it), issued one item ahead into a double buffer. One MMA
+// job of N = 2 rp columns per 128-token tile, the accumulator
+// double-buffered in tensor memory, so one tile's readout overlaps
 // the next tile's MMAs. Eight readout warps (two per tensor-memory lane
 // quarter, alternating tiles) add the two parts, square and sum per head.
 //
@@ -49,6 +50,7 @@ struct KfCfg {
 template <int G, int W>
 __global__ void __launch_bounds__(KF_THREADS, 1)
     kfull_bf16_kernel(const __grid_constant__ CUtensorMap kmap, Dims dm, Ws ws) {
+  pdl_wait();
   using C = KfCfg<G, W>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -252,6 +254,7 @@ constexpr int KS_WMAX = 64;  // window queries staged per round
 template <typename T>
 __global__ void __launch_bounds__(KS_THREADS)
     kfull_simt_kernel(Dims dm, Ws ws, const T* __restrict__ k) {
+  pdl_wait();
   extern __shared__ float ksm[];
   float* Ks = ksm;                    // [TILE][KS_LD] the tile's keys
   float* Qs = ksm + TILE * KS_LD;     // [KS_WMAX][D] centred queries of one head
@@ -308,7 +311,7 @@ static cudaError_t launch_kfull_tc(const CUtensorMap& kmap, const Dims& dm, cons
   cudaError_t e =
       cudaFuncSetAttribute(kfull_bf16_kernel<G, W>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
   if (e != cudaSuccess) return e;
-  kfull_bf16_kernel<G, W><<<grid, KF_THREADS, C::SMEM, st>>>(kmap, dm, ws);
+  JACAP_TRY(launch_pdl(dm.pdl != 0, kfull_bf16_kernel<G, W>, grid, KF_THREADS, C::SMEM, st, kmap, dm, ws));
   return cudaGetLastError();
 }
 
@@ -350,12 +353,13 @@ cudaError_t launch_kfull(const CUtensorMap& kmap, const Dims& dm, const Ws& ws, 
     cudaError_t e = cudaFuncSetAttribute(kfull_simt_kernel<__nv_bfloat16>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    kfull_simt_kernel<__nv_bfloat16><<<grid, KS_THREADS, smem, st>>>(dm, ws, (const __nv_bfloat16*)k);
+    JACAP_TRY(launch_pdl(dm.pdl != 0, kfull_simt_kernel<__nv_bfloat16>, grid, KS_THREADS, smem, st, dm, ws,
+                         (const __nv_bfloat16*)k));
   } else {
     cudaError_t e =
         cudaFuncSetAttribute(kfull_simt_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    kfull_simt_kernel<float><<<grid, KS_THREADS, smem, st>>>(dm, ws, (const float*)k);
+    JACAP_TRY(launch_pdl(dm.pdl != 0, kfull_simt_kernel<float>, grid, KS_THREADS, smem, st, dm, ws, (const float*)k));
   }
   return cudaGetLastError();
 }

@@ -136,6 +136,7 @@ __device__ __forceinline__ void store_part(float* dst, const float (&v)[G]) {
 template <int G>
 __global__ void __launch_bounds__(KB_THREADS, 1)
     kpass_bf16_kernel(const __grid_constant__ CUtensorMap kmap, Dims dm, Ws ws, const int32_t* __restrict__ cu) {
+  pdl_wait();
   using C = KbCfg<G>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -445,7 +446,7 @@ static cudaError_t launch_g(const CUtensorMap& kmap, const Dims& dm, const Ws& w
   static_assert(smem <= 232448, "shared memory budget");
   cudaError_t e = cudaFuncSetAttribute(kpass_bf16_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  kpass_bf16_kernel<G><<<grid, KB_THREADS, smem, st>>>(kmap, dm, ws, cu);
+  JACAP_TRY(launch_pdl(dm.pdl != 0, kpass_bf16_kernel<G>, grid, KB_THREADS, smem, st, kmap, dm, ws, cu));
   return cudaGetLastError();
 }
 

@@ -36,6 +36,7 @@ template <bool DENSE>
 __global__ void __launch_bounds__(SC_THREADS, 1)
     score_bf16_kernel(const __grid_constant__ CUtensorMap vmap, Dims dm, Ws ws, const int32_t* __restrict__ cu,
                       float* __restrict__ scores) {
+  pdl_wait();
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t* mimg = smem;                       // [2][SC_M_BYTES], by run parity
@@ -226,6 +227,7 @@ constexpr size_t score_f32_smem_bytes() { return (size_t)(D * D + TILE * SF_LD) 
 __global__ void __launch_bounds__(SF_THREADS)
     score_f32_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu, const float* __restrict__ v,
                      float* __restrict__ scores) {
+  pdl_wait();
   extern __shared__ float ssm[];
   float* Mi = ssm;               // [D][D] L^{-1}
   float* vt = ssm + D * D;       // [TILE][SF_LD]
@@ -286,12 +288,13 @@ cudaError_t launch_score(const CUtensorMap& vmap, const Dims& dm, const Ws& ws, 
     auto kern = dm.dense_minv ? score_bf16_kernel<true> : score_bf16_kernel<false>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    kern<<<grid, SC_THREADS, smem, st>>>(vmap, dm, ws, cu, scores);
+    JACAP_TRY(launch_pdl(dm.pdl != 0, kern, grid, SC_THREADS, smem, st, vmap, dm, ws, cu, scores));
   } else {
     constexpr size_t smem = score_f32_smem_bytes();
     cudaError_t e = cudaFuncSetAttribute(score_f32_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    score_f32_kernel<<<grid, SF_THREADS, smem, st>>>(dm, ws, cu, (const float*)v, scores);
+    JACAP_TRY(launch_pdl(dm.pdl != 0, score_f32_kernel, grid, SF_THREADS, smem, st, dm, ws, cu, (const float*)v,
+                         scores));
   }
   return cudaGetLastError();
 }

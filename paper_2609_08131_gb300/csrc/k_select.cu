@@ -47,6 +47,7 @@ template <int KPT>
 __global__ void __launch_bounds__(SE_THREADS)
     select_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu, const float* __restrict__ scores, int B,
                   int32_t* __restrict__ idx, int32_t* __restrict__ kept) {
+  pdl_wait();
   constexpr int SE_KPT = KPT;
   constexpr int SE_SLAB = SE_THREADS * KPT;  // warp w holds positions 32 KPT w .. + 32 KPT - 1 of a slab
   __shared__ uint32_t hist[SE_BINS];
@@ -183,6 +184,7 @@ template <typename T>
 __global__ void __launch_bounds__(256)
     compact_kernel(Dims dm, const int32_t* __restrict__ cu, const T* __restrict__ k, const T* __restrict__ v,
                    const int32_t* __restrict__ idx, int B, T* __restrict__ k_out, T* __restrict__ v_out) {
+  pdl_wait();
   constexpr int CH = D * (int)sizeof(T) / 16;  // 16-byte chunks per row
   const int64_t rows = (int64_t)dm.L * dm.Hkv * dm.S * B;
   const int64_t total = rows * CH;
@@ -209,13 +211,17 @@ __global__ void __launch_bounds__(256)
 cudaError_t launch_select(const Dims& dm, const Ws& ws, const int32_t* cu, const float* scores, int budget,
                           int32_t* idx, int32_t* kept, int max_seqlen, int grid, cudaStream_t st) {
   if (max_seqlen <= SE_THREADS * 4)
-    select_kernel<4><<<grid, SE_THREADS, 0, st>>>(dm, ws, cu, scores, budget, idx, kept);
+    JACAP_TRY(launch_pdl(dm.pdl != 0, select_kernel<4>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget, idx,
+                         kept));
   else if (max_seqlen <= SE_THREADS * 8)
-    select_kernel<8><<<grid, SE_THREADS, 0, st>>>(dm, ws, cu, scores, budget, idx, kept);
+    JACAP_TRY(launch_pdl(dm.pdl != 0, select_kernel<8>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget, idx,
+                         kept));
   else if (max_seqlen <= SE_THREADS * 16)
-    select_kernel<16><<<grid, SE_THREADS, 0, st>>>(dm, ws, cu, scores, budget, idx, kept);
+    JACAP_TRY(launch_pdl(dm.pdl != 0, select_kernel<16>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget, idx,
+                         kept));
   else
-    select_kernel<32><<<grid, SE_THREADS, 0, st>>>(dm, ws, cu, scores, budget, idx, kept);
+    JACAP_TRY(launch_pdl(dm.pdl != 0, select_kernel<32>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget, idx,
+                         kept));
   return cudaGetLastError();
 }
 
@@ -228,11 +234,12 @@ cudaError_t launch_compact(const Dims& dm, int dtype, const int32_t* cu, const v
   const int blocks = (int)(blocks64 < 65535 * 16 ? blocks64 : 65535 * 16);
   if (blocks <= 0) return cudaSuccess;
   if (dtype == 1)
-    compact_kernel<__nv_bfloat16><<<blocks, 256, 0, st>>>(dm, cu, (const __nv_bfloat16*)k, (const __nv_bfloat16*)v,
-                                                          idx, budget, (__nv_bfloat16*)k_out, (__nv_bfloat16*)v_out);
+    JACAP_TRY(launch_pdl(dm.pdl != 0, compact_kernel<__nv_bfloat16>, blocks, 256, 0, st, dm, cu,
+                         (const __nv_bfloat16*)k, (const __nv_bfloat16*)v, idx, budget, (__nv_bfloat16*)k_out,
+                         (__nv_bfloat16*)v_out));
   else
-    compact_kernel<float><<<blocks, 256, 0, st>>>(dm, cu, (const float*)k, (const float*)v, idx, budget,
-                                                  (float*)k_out, (float*)v_out);
+    JACAP_TRY(launch_pdl(dm.pdl != 0, compact_kernel<float>, blocks, 256, 0, st, dm, cu, (const float*)k,
+                         (const float*)v, idx, budget, (float*)k_out, (float*)v_out));
   return cudaGetLastError();
 }
 

@@ -21,6 +21,7 @@ namespace jacap {
 // cu_seqlens and lays out the chunks (thread 0), then writes the chunk table:
 // record r = {t0, t1, request, r} for the C_tot chunks of a plane.
 __global__ void __launch_bounds__(256) plan_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu) {
+  pdl_wait();
   __shared__ int s_ctot;
   if (threadIdx.x < 16) ws.status[threadIdx.x] = 0u;
   if (threadIdx.x == 0) {
@@ -68,6 +69,7 @@ __device__ __forceinline__ float ld_elem<__nv_bfloat16>(const __nv_bfloat16* p) 
 // One block per (request, layer, query head); thread c owns channel c.
 template <typename T>
 __global__ void __launch_bounds__(D) window_stats_kernel(Dims dm, Ws ws, const T* __restrict__ q) {
+  pdl_wait();
   if (status_failed(ws)) return;
   const int b = blockIdx.x;
   const int h = b % dm.Hq;
@@ -138,6 +140,7 @@ constexpr size_t kpass_smem_bytes() {
 template <typename T, int G>
 __global__ void __launch_bounds__(KP_THREADS, 1)
     kpass_kernel(const __grid_constant__ CUtensorMap kmap, Dims dm, Ws ws, const int32_t* __restrict__ cu) {
+  pdl_wait();
   using C = KpCfg<T>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -283,7 +286,8 @@ __global__ void __launch_bounds__(KP_THREADS, 1)
         float* dst = ws.lk + ((int64_t)item.plane * dm.Ntot + tok) * (2 * G);
         if constexpr ((2 * G) % 4 == 0) {
 #pragma unroll
-          for (int e = 0; e < 2 * G; e += 4) *(float4*)(dst + e) = make_float4(out[e], out[e + 1], out[e + 2], out[e + 3]);
+          for (int e = 0; e < 2 * G; e += 4)
+            *(float4*)(dst + e) = make_float4(out[e], out[e + 1], out[e + 2], out[e + 3]);
         } else {
 #pragma unroll
           for (int e = 0; e < 2 * G; ++e) dst[e] = out[e];
@@ -319,12 +323,12 @@ compute_done:
 template <typename T>
 static cudaError_t launch_window_stats_t(const Dims& dm, const Ws& ws, const void* q, cudaStream_t st) {
   const int blocks = dm.S * dm.L * dm.Hq;
-  window_stats_kernel<T><<<blocks, D, 0, st>>>(dm, ws, (const T*)q);
+  JACAP_TRY(launch_pdl(dm.pdl != 0, window_stats_kernel<T>, blocks, D, 0, st, dm, ws, (const T*)q));
   return cudaGetLastError();
 }
 
 cudaError_t launch_plan(const Dims& dm, const Ws& ws, const int32_t* cu, cudaStream_t st) {
-  plan_kernel<<<1, 256, 0, st>>>(dm, ws, cu);
+  JACAP_TRY(launch_pdl(dm.pdl != 0, plan_kernel, 1, 256, 0, st, dm, ws, cu));
   return cudaGetLastError();
 }
 
@@ -339,7 +343,7 @@ static cudaError_t launch_kpass_tg(const CUtensorMap& kmap, const Dims& dm, cons
   constexpr size_t smem = kpass_smem_bytes<T, G>();
   cudaError_t e = cudaFuncSetAttribute(kpass_kernel<T, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  kpass_kernel<T, G><<<grid, KP_THREADS, smem, st>>>(kmap, dm, ws, cu);
+  JACAP_TRY(launch_pdl(dm.pdl != 0, kpass_kernel<T, G>, grid, KP_THREADS, smem, st, kmap, dm, ws, cu));
   return cudaGetLastError();
 }
 
