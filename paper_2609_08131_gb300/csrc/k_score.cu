@@ -20,6 +20,7 @@ namespace jacap {
 
 constexpr int SC_THREADS = 192;  // warp 0: TMA, warp 1: MMA, warps 2-5: epilogue
 constexpr int SC_STAGES = 3;
+constexpr int SC_IMGS = 2;  // L^{-1} image buffers
 constexpr int SC_BOX = 16384;
 constexpr int SC_TILE_BYTES = 2 * SC_BOX;
 constexpr int SC_M_BYTES = 65536;
@@ -28,7 +29,7 @@ constexpr uint32_t SC_TMEM_COLS = 256;  // two 128-column accumulators
 constexpr uint32_t SC_IDESC128 = idesc_bf16_f32(128, 128, 0, 0);
 constexpr uint32_t SC_IDESC64 = idesc_bf16_f32(128, 64, 0, 0);
 
-constexpr size_t score_bf16_smem_bytes() { return 1024 + 2 * SC_M_BYTES + SC_STAGES * SC_TILE_BYTES + 256; }
+constexpr size_t score_bf16_smem_bytes() { return 1024 + SC_IMGS * SC_M_BYTES + SC_STAGES * SC_TILE_BYTES + 256; }
 
 // DENSE: the score matrix is a full 128 x 128 (output directions) rather than
 // the lower-triangular L^{-1}, so no K-step may be narrowed.
@@ -39,8 +40,8 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
   pdl_wait();
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint8_t* mimg = smem;                       // [2][SC_M_BYTES], by run parity
-  uint8_t* stages = smem + 2 * SC_M_BYTES;
+  uint8_t* mimg = smem;                       // [SC_IMGS][SC_M_BYTES], by run
+  uint8_t* stages = smem + SC_IMGS * SC_M_BYTES;
   uint64_t* vfull = (uint64_t*)(stages + SC_STAGES * SC_TILE_BYTES);
   uint64_t* vempty = vfull + SC_STAGES;
   uint64_t* accfull = vempty + SC_STAGES;
@@ -91,9 +92,9 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
       for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); ok && is.next(item);) {
         const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
         const int64_t u = (int64_t)item.plane * dm.S + item.seq;
-        if (!cont) {  // a new unit: its image, into the buffer of the run before last
-          const int mp = nrun & 1;
-          if (nrun >= 2 && !mbar_wait(smem_u32(&mempty[mp]), ((nrun >> 1) & 1) ^ 1, ws, abort)) break;
+        if (!cont) {  // a new unit: its image, into the buffer of the run SC_IMGS runs back
+          const int mp = nrun % SC_IMGS;
+          if (nrun >= SC_IMGS && !mbar_wait(smem_u32(&mempty[mp]), ((nrun / SC_IMGS) & 1) ^ 1, ws, abort)) break;
           mbar_arrive_expect_tx(smem_u32(&mfull[mp]), SC_M_BYTES);
           bulk_g2s(smem_u32(mimg + mp * SC_M_BYTES), ws.minv_img + u * SC_M_BYTES, SC_M_BYTES,
                    smem_u32(&mfull[mp]));
@@ -116,8 +117,8 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
       }
       for (uint32_t k = (it > (uint32_t)SC_STAGES ? it - SC_STAGES : 0); k < it; ++k)
         mbar_wait(smem_u32(&vfull[k % SC_STAGES]), (k / SC_STAGES) & 1, ws, nullptr);
-      for (uint32_t k = (nrun > 2 ? nrun - 2 : 0); k < nrun; ++k)
-        mbar_wait(smem_u32(&mfull[k & 1]), (k >> 1) & 1, ws, nullptr);
+      for (uint32_t k = (nrun > SC_IMGS ? nrun - SC_IMGS : 0); k < nrun; ++k)
+        mbar_wait(smem_u32(&mfull[k % SC_IMGS]), (k / SC_IMGS) & 1, ws, nullptr);
     }
   } else if (warp == 1) {
     if (lane == 0) {
@@ -127,8 +128,8 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
       Item item;
       for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); ok && is.next(item);) {
         if (!cont) {
-          mp = nrun & 1;
-          if (!mbar_wait(smem_u32(&mfull[mp]), (nrun >> 1) & 1, ws, abort)) break;
+          mp = nrun % SC_IMGS;
+          if (!mbar_wait(smem_u32(&mfull[mp]), (nrun / SC_IMGS) & 1, ws, abort)) break;
           tc_fence_after();
         }
         const uint32_t ma = smem_u32(mimg + mp * SC_M_BYTES);
