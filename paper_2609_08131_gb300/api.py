@@ -126,6 +126,17 @@ class Evictor:
         self.k_out = torch.empty((L, Hkv, S, self.budget, d), dtype=cache.k.dtype, device=dev)
         self.v_out = torch.empty_like(self.k_out)
 
+    def bind_outputs(self, idx, kept, k_out, v_out):
+        """Write the results into caller-owned device tensors (views into a
+        larger buffer, for instance) of the shapes and dtypes of ``idx``,
+        ``kept``, ``k_out`` and ``v_out``; each must be contiguous."""
+        for name, t in (("idx", idx), ("kept", kept), ("k_out", k_out), ("v_out", v_out)):
+            ref = getattr(self, name)
+            if t.shape != ref.shape or t.dtype != ref.dtype or t.device != ref.device or not t.is_contiguous():
+                raise ValueError(f"{name} must be a contiguous {ref.dtype} tensor of shape {tuple(ref.shape)} "
+                                 f"on {ref.device}")
+        self.idx, self.kept, self.k_out, self.v_out = idx, kept, k_out, v_out
+
     def score(self, stream=None, events=None):
         """jacap_score; with ``events`` (JACAP_SCORE_KERNELS + 1 torch.cuda.Event
         objects) the timed variant records them around the kernels of the pass."""
@@ -358,3 +369,118 @@ class DecodeEvictor:
 
     def check(self, stream=None):
         _check(jacap_device_status(_ptr(self.ws), _stream(stream)), "device status")
+
+
+class HostEvictor:
+    """Eviction of a cache held in pinned host memory (an offloaded cache).
+
+    The layers go to the device in groups of ``group_layers`` through two
+    device buffers: while group g is scored, selected and compacted on the
+    compute stream, group g + 1 is copied on a copy stream, so the device never
+    holds more than two groups and the pass overlaps the host->device copies.
+    A buffer is refilled once the pass over its previous group has finished,
+    which lets the next ``run()``'s first copies overlap this one's last pass.
+
+    q_win_h [S, L, Hq, w, 128], k_h and v_h [L, Hkv, N, 128]: pinned host
+    tensors (contiguous); cu_seqlens: int32 [S + 1] (host or device), fixed
+    with ``seqlens`` at construction like the layout; ``out_factor``: optional
+    float32 [L][Hkv][128][128] device tensor, as for ``Evictor``. The host
+    tensors are read while the copies execute: leave them unchanged until the
+    stream has been synchronised. After ``run()`` the device tensors
+    idx [L, Hkv, S, B], kept [S] and k_out, v_out [L, Hkv, S, B, 128] hold the
+    result and ``idx_h`` / ``kept_h`` (pinned host) the kept positions once the
+    stream is synchronised.
+    """
+
+    def __init__(self, q_win_h, k_h, v_h, cu_seqlens, seqlens, num_q_heads: int, budget: int,
+                 params: jacap_params | None = None, group_layers: int = 8, device="cuda", out_factor=None):
+        dev = torch.device(device)
+        for name, t in (("q_win_h", q_win_h), ("k_h", k_h), ("v_h", v_h)):
+            if t.device.type != "cpu" or not t.is_pinned() or not t.is_contiguous():
+                raise ValueError(f"{name} must be a contiguous tensor in pinned host memory")
+        L, Hkv, N, d = k_h.shape
+        S = len(seqlens)
+        if v_h.shape != k_h.shape or q_win_h.shape[:2] != (S, L):
+            raise ValueError("k_h and v_h must be [L, Hkv, N, 128] and q_win_h [S, L, Hq, w, 128]")
+        if out_factor is not None and (out_factor.dtype != torch.float32 or tuple(out_factor.shape) != (L, Hkv, d, d)
+                                       or not out_factor.is_contiguous() or out_factor.device != dev):
+            raise ValueError("out_factor must be a contiguous float32 [L][Hkv][128][128] tensor on the device")
+        self.out_factor = out_factor
+        self.L, self.S, self.gl = L, S, max(1, min(int(group_layers), L))
+        self.q_h, self.k_h, self.v_h = q_win_h, k_h, v_h
+        self.budget = int(budget)
+        self.params = params
+        self.num_q_heads = num_q_heads
+        self.seqlens = list(seqlens)
+        self.cu = torch.as_tensor(cu_seqlens, dtype=torch.int32).to(dev)
+        gl = self.gl
+        self.kb = [torch.empty((gl, Hkv, N, d), dtype=k_h.dtype, device=dev) for _ in range(2)]
+        self.vb = [torch.empty_like(self.kb[0]) for _ in range(2)]
+        self._qrow = tuple(q_win_h.shape[2:])
+        self.qb = [torch.empty(S * gl * q_win_h[0, 0].numel(), dtype=q_win_h.dtype, device=dev) for _ in range(2)]
+        self._ev = {}  # one Evictor per buffer and group size (the last group may be shorter)
+        self.idx = torch.empty((L, Hkv, S, self.budget), dtype=torch.int32, device=dev)
+        self.kept = torch.empty((S,), dtype=torch.int32, device=dev)
+        self.k_out = torch.empty((L, Hkv, S, self.budget, d), dtype=k_h.dtype, device=dev)
+        self.v_out = torch.empty_like(self.k_out)
+        self.idx_h = torch.empty(self.idx.shape, dtype=torch.int32).pin_memory()
+        self.kept_h = torch.empty(self.kept.shape, dtype=torch.int32).pin_memory()
+        self.copy_stream = torch.cuda.Stream(device=dev)
+        self._done = [torch.cuda.Event(), torch.cuda.Event()]
+        self._copied = [torch.cuda.Event(), torch.cuda.Event()]
+        self._used = [False, False]
+
+    def _qview(self, b, n):
+        per = 1
+        for x in self._qrow:
+            per *= x
+        return self.qb[b][:self.S * n * per].view(self.S, n, *self._qrow)
+
+    def _evictor(self, b, n):
+        key = (b, n)
+        if key not in self._ev:
+            c = Cache(self._qview(b, n), self.kb[b][:n], self.vb[b][:n], self.cu, self.seqlens, self.num_q_heads)
+            of = None if self.out_factor is None else self.out_factor[:n]
+            self._ev[key] = Evictor(c, self.budget, self.params, out_factor=of)
+        return self._ev[key]
+
+    @property
+    def h2d_bytes(self) -> int:
+        """Bytes one ``run()`` copies host->device."""
+        return sum(t.numel() * t.element_size() for t in (self.q_h, self.k_h, self.v_h))
+
+    @property
+    def d2h_bytes(self) -> int:
+        """Bytes one ``run()`` copies device->host."""
+        return (self.idx_h.numel() + self.kept_h.numel()) * 4
+
+    def run(self, stream=None):
+        comp = stream if stream is not None else torch.cuda.current_stream()
+        cs = self.copy_stream
+        for g, l0 in enumerate(range(0, self.L, self.gl)):
+            n = min(self.gl, self.L - l0)
+            b = g & 1
+            with torch.cuda.stream(cs):
+                if self._used[b]:
+                    cs.wait_event(self._done[b])  # the pass over the buffer's previous group is finished
+                self.kb[b][:n].copy_(self.k_h[l0:l0 + n], non_blocking=True)
+                self.vb[b][:n].copy_(self.v_h[l0:l0 + n], non_blocking=True)
+                qv = self._qview(b, n)
+                for s in range(self.S):
+                    qv[s].copy_(self.q_h[s, l0:l0 + n], non_blocking=True)
+                self._copied[b].record(cs)
+            comp.wait_event(self._copied[b])
+            ev = self._evictor(b, n)
+            ev.bind_outputs(self.idx[l0:l0 + n], self.kept, self.k_out[l0:l0 + n], self.v_out[l0:l0 + n])
+            if self.out_factor is not None:
+                ev.out_factor = self.out_factor[l0:l0 + n]
+            ev.run(comp)
+            self._done[b].record(comp)
+            self._used[b] = True
+        with torch.cuda.stream(comp):
+            self.idx_h.copy_(self.idx, non_blocking=True)
+            self.kept_h.copy_(self.kept, non_blocking=True)
+
+    def check(self, stream=None):
+        for ev in self._ev.values():
+            ev.check(stream)

@@ -144,3 +144,35 @@ def test_compaction_refuses_positions_that_do_not_ascend():
         assert st == 0
         assert jacap_device_status(_ptr(ev.ws), _stream()) == JACAP_ERR_INVALID_ARG
         assert torch.equal(ev.k, before)
+
+
+def test_host_evictor_matches_the_oracle():
+    # a cache in pinned host memory, evicted in layer groups of 2 through two
+    # device buffers (the groups' copies overlap the previous group's pass)
+    from oracle import JacapParams as JP
+    from paper_2609_08131_gb300.api import HostEvictor
+    from paper_2609_08131_gb300.workloads import unit_arrays
+
+    wl = Workload("host cache", 5, 8, 2, (900, 333), 16, 64, seed=41)
+    t = generate(wl, DEV)
+    he = HostEvictor(t.q_win.cpu().pin_memory(), t.k.cpu().pin_memory(), t.v.cpu().pin_memory(),
+                     t.cu_seqlens, list(wl.seqlens), wl.num_q_heads, wl.budget, jacap_params(),
+                     group_layers=2, device=DEV)
+    for _ in range(2):  # the second run reuses the buffers
+        he.run()
+        torch.cuda.synchronize()
+        he.check()
+    cu = t.cu_seqlens.cpu().tolist()
+    assert he.kept_h.tolist() == [min(n, wl.budget) for n in wl.seqlens]
+    assert torch.equal(he.idx_h, he.idx.cpu())
+    for layer in range(wl.num_layers):
+        for g in range(wl.num_kv_heads):
+            for s in range(len(wl.seqlens)):
+                q, K, V = unit_arrays(t, wl.num_q_heads, s, layer, g)
+                ora = oracle_unit(q, K, V, wl.budget, JP())
+                gidx = he.idx_h[layer, g, s].numpy()
+                assert_selection(gidx, cu[s + 1] - cu[s], wl.budget, ora["scores"], ora["idx"])
+                kept = min(cu[s + 1] - cu[s], wl.budget)
+                sel = torch.as_tensor(gidx[:kept], dtype=torch.long, device=DEV)
+                assert_rows_bitwise(t.k[layer, g, cu[s]:cu[s + 1]][sel], he.k_out[layer, g, s, :kept])
+                assert_rows_bitwise(t.v[layer, g, cu[s]:cu[s + 1]][sel], he.v_out[layer, g, s, :kept])
