@@ -1,8 +1,8 @@
 #!/usr/bin/env python
 """Throughput of Jacap's prefill eviction pass on GB300; prints ONE JSON line.
 
-A step is one whole pass (jacap_score + jacap_select + jacap_compact: every
-row of the hot path) over one synthetic Llama-3-8B-shaped cache (32 layers,
+A step is one whole pass (jacap_score + jacap_select_compact, i.e. the
+selection and the compaction in one launch: every row of the hot path) over one synthetic Llama-3-8B-shaped cache (32 layers,
 32 query / 8 KV heads, head_dim 128, n = 32768, w = 32, B = 512, bf16), with
 the inputs resident in HBM. The metric is evicted-cache tokens per second per
 layer-pass, sum_s n_s * L / t_step, summed over ranks.
@@ -349,10 +349,8 @@ def run_ours(args):
     kb0.record(stream)
     for i in range(KB):
         ev.score(events=ev_score[i])
-        ev.select()
+        ev.select_compact()
         ev_tail[i][0].record(stream)
-        ev.compact()
-        ev_tail[i][1].record(stream)
     kb1.record(stream)
     torch.cuda.synchronize()
     clocks = sampler.stop()
@@ -364,13 +362,11 @@ def run_ours(args):
 
     # per-kernel average durations inside the timed region
     kern = {name: 0.0 for name in SCORE_KERNEL_NAMES}
-    kern["select"] = 0.0
-    kern["compact"] = 0.0
+    kern["select_compact"] = 0.0
     for i in range(KB):
         for j, name in enumerate(SCORE_KERNEL_NAMES):
             kern[name] += ev_score[i][j].elapsed_time(ev_score[i][j + 1])
-        kern["select"] += ev_score[i][nk].elapsed_time(ev_tail[i][0])
-        kern["compact"] += ev_tail[i][0].elapsed_time(ev_tail[i][1])
+        kern["select_compact"] += ev_score[i][nk].elapsed_time(ev_tail[i][0])
     kern = {k: v / KB for k, v in kern.items()}
 
     L, Hkv, N, d = t.k.shape
@@ -387,8 +383,8 @@ def run_ours(args):
         "k_pass": kv_bytes,                       # K read once
         "gram": kv_bytes,                         # V read once
         "scores": kv_bytes + L * Hkv * N * 4,     # V read, scores written
-        "select": L * Hkv * N * 4,                # scores read
-        "compact": 4 * kept_rows * d * es,        # retained K, V read and written
+        # scores read; retained K, V rows read and written
+        "select_compact": L * Hkv * N * 4 + 4 * kept_rows * d * es,
     }
     if not fused_weights:
         alg_kernel["weights"] = L * Hkv * N * (8 * G + 4)  # logits + kappa read, w written
@@ -443,8 +439,8 @@ def run_ours(args):
             "kernel_ms": kern,
             "ms_per_step_with_kernel_events": t_ms_events,
             # plan, query statistics, K pass, [full covariance], [weights: float32 only], Gram,
-            # factor, scores, select, compact
-            "gpu_launches": K * (8 + (1 if args.covariance == "full" else 0) + (0 if fused_weights else 1)),
+            # factor, scores, selection + compaction
+            "gpu_launches": K * (7 + (1 if args.covariance == "full" else 0) + (0 if fused_weights else 1)),
             "clocks": clocks,
             "cpu_baseline": cpu,
             "e2e": e2e,
@@ -471,9 +467,17 @@ def run_e2e(args, ev, t, stream, world, dist):
     for _ in range(2):
         he.run(stream)
     torch.cuda.synchronize()
+    # the host link on its own: one layer group's K copied host -> device
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    grp = he.k_h[:he.gl]
+    a.record(stream)
+    for _ in range(3):
+        he.kb[0].copy_(grp, non_blocking=True)
+    b.record(stream)
+    torch.cuda.synchronize()
+    link_gbs = 3 * grp.numel() * grp.element_size() / (a.elapsed_time(b) * 1e-3) / 1e9
     if dist is not None:
         dist.barrier()
-    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     a.record(stream)
     n = max(1, args.e2e_steps)
     for _ in range(n):
@@ -499,7 +503,8 @@ def run_e2e(args, ev, t, stream, world, dist):
     L = c.k.shape[0]
     return {"value": sum(t.seqlens) * L * world / (ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": he.h2d_bytes,
             "d2h_bytes_per_step": he.d2h_bytes, "ms_per_step": ms, "steps": n, "group_layers": he.gl,
-            "idx_differ_vs_resident": differ}
+            "idx_differ_vs_resident": differ, "h2d_link_gbs": link_gbs,
+            "h2d_bound_ms": he.h2d_bytes / (link_gbs * 1e9) * 1e3}
 
 
 def run_decode(args):
@@ -587,7 +592,9 @@ def run_decode(args):
         "stats_update_us_per_decode_step": upd_us,
         "event_hbm_fraction": {"kv_bytes": kv_bytes, "of_8tbs": kv_bytes / (t_ms * 1e-3) / 8e12},
         "clocks": clocks,
-        "gpu_launches_per_event": nk + 3,  # plan is two launches; select, in-place compaction
+        # plan, query statistics, K pass, Gram (with the weights), factor, scores,
+        # select, in-place compaction
+        "gpu_launches_per_event": 8,
     }
     print(json.dumps(line))
     return 0

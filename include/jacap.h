@@ -241,6 +241,19 @@ jacap_status jacap_compact(const jacap_layout* layout, const void* k, const void
                            void* stream);
 
 /*
+ * jacap_select followed by jacap_compact in one launch (Algorithm 1 step 5 and
+ * the retained cache Z_C of Sec. 3.1): each unit's kept rows are copied as
+ * soon as its positions are known. Arguments, layouts, results and error
+ * behaviour are those of the two calls: idx and kept as from jacap_select,
+ * k_out and v_out as from jacap_compact with that idx (zero rows where idx is
+ * -1). k, v, k_out and v_out must be 16-byte aligned and k_out, v_out must
+ * overlap neither k, v, scores nor idx.
+ */
+jacap_status jacap_select_compact(const jacap_layout* layout, const float* scores, int32_t budget,
+                                  int32_t* idx, int32_t* kept, const void* k, const void* v,
+                                  void* k_out, void* v_out, void* ws, size_t ws_bytes, void* stream);
+
+/*
  * Decoding-stage eviction (the paper's decoding experiments, Sec. 4; Sec. 3.4,
  * last paragraph: during decoding mu_Q and Lambda_Q are estimated from the
  * historical queries). Three calls on top of the ones above:

@@ -92,6 +92,8 @@ _SIGS = {
     "jacap_select": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, ctypes.c_int32, _P, _P, _P, ctypes.c_size_t,
                                     _P]),
     "jacap_compact": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, _P, _P, ctypes.c_int32, _P, _P, _P]),
+    "jacap_select_compact": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, ctypes.c_int32, _P, _P, _P, _P, _P,
+                                            _P, _P, ctypes.c_size_t, _P]),
     "jacap_score_stats": (ctypes.c_int, [ctypes.POINTER(jacap_layout), ctypes.POINTER(jacap_params), _P, _P, _P,
                                          _P, _P, _P, ctypes.c_size_t, _P, ctypes.POINTER(ctypes.c_void_p),
                                          ctypes.c_int32]),
@@ -173,6 +175,11 @@ def jacap_score_static(layout, params, q_win, k, v, scores, stream):
 
 def jacap_select(layout, scores, budget, idx, kept, ws, ws_bytes, stream) -> int:
     return lib().jacap_select(ctypes.byref(layout), scores, budget, idx, kept, ws, ws_bytes, stream)
+
+
+def jacap_select_compact(layout, scores, budget, idx, kept, k, v, k_out, v_out, ws, ws_bytes, stream) -> int:
+    return lib().jacap_select_compact(ctypes.byref(layout), scores, budget, idx, kept, k, v, k_out, v_out, ws,
+                                      ws_bytes, stream)
 
 
 def jacap_compact(layout, k, v, idx, budget, k_out, v_out, stream) -> int:

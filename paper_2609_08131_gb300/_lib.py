@@ -96,6 +96,7 @@ EXPORTS = [
     "jacap_stats_update",
     "jacap_compact_inplace",
     "jacap_select",
+    "jacap_select_compact",
     "jacap_compact",
     "jacap_device_status",
     "jacap_status_string",

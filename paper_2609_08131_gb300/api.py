@@ -25,6 +25,7 @@ from . import (
     jacap_score_out,
     jacap_score_stats,
     jacap_select,
+    jacap_select_compact,
     jacap_stats_update,
     jacap_status_string,
     jacap_workspace_offsets,
@@ -163,10 +164,16 @@ class Evictor:
         _check(jacap_compact(self.lay, _ptr(c.k), _ptr(c.v), _ptr(self.idx), self.budget, _ptr(self.k_out),
                              _ptr(self.v_out), _stream(stream)), "jacap_compact")
 
+    def select_compact(self, stream=None):
+        """jacap_select and jacap_compact in one launch."""
+        c = self.cache
+        _check(jacap_select_compact(self.lay, _ptr(self.scores), self.budget, _ptr(self.idx), _ptr(self.kept),
+                                    _ptr(c.k), _ptr(c.v), _ptr(self.k_out), _ptr(self.v_out), _ptr(self.ws),
+                                    self.ws.numel(), _stream(stream)), "jacap_select_compact")
+
     def run(self, stream=None):
         self.score(stream)
-        self.select(stream)
-        self.compact(stream)
+        self.select_compact(stream)
 
     def device_status(self, stream=None) -> int:
         return jacap_device_status(_ptr(self.ws), _stream(stream))

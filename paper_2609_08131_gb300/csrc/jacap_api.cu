@@ -398,6 +398,30 @@ jacap_status jacap_select(const jacap_layout* layout, const float* scores, int32
                                 persistent_grid(units, sms, 2), (cudaStream_t)stream));
 }
 
+jacap_status jacap_select_compact(const jacap_layout* layout, const float* scores, int32_t budget, int32_t* idx,
+                                  int32_t* kept, const void* k, const void* v, void* k_out, void* v_out, void* ws,
+                                  size_t ws_bytes, void* stream) {
+  jacap_status st = check_layout(layout);
+  if (st != JACAP_OK) return st;
+  if (scores == nullptr || idx == nullptr || kept == nullptr || ws == nullptr || budget < 1 || k == nullptr ||
+      v == nullptr || k_out == nullptr || v_out == nullptr)
+    return JACAP_ERR_INVALID_ARG;
+  if (((uintptr_t)scores & 3u) != 0 || ((uintptr_t)idx & 3u) != 0 || ((uintptr_t)kept & 3u) != 0)
+    return JACAP_ERR_INVALID_ARG;
+  if (!aligned16(k) || !aligned16(v) || !aligned16(k_out) || !aligned16(v_out)) return JACAP_ERR_INVALID_ARG;
+  Dims dm;
+  make_dims(layout, nullptr, dm);
+  const Carve c = carve(dm);
+  if (((uintptr_t)ws & 255u) != 0 || ws_bytes < c.total) return JACAP_ERR_WORKSPACE;
+  int sms = 0;
+  if ((st = check_device(&sms)) != JACAP_OK) return st;
+  const Ws w = make_ws(ws, c);
+  const int64_t units = (int64_t)dm.L * dm.Hkv * dm.S;
+  return map_cuda(launch_select(dm, w, layout->cu_seqlens, scores, budget, idx, kept, layout->max_seqlen,
+                                persistent_grid(units, sms, 2), (cudaStream_t)stream,
+                                layout->dtype == JACAP_BF16 ? 1 : 0, k, v, k_out, v_out));
+}
+
 jacap_status jacap_compact(const jacap_layout* layout, const void* k, const void* v, const int32_t* idx,
                            int32_t budget, void* k_out, void* v_out, void* stream) {
   jacap_status st = check_layout(layout);

@@ -5,7 +5,9 @@
 // by the factor kernel) accumulate into the same 128 fp32 columns, so
 // y = V (hi + lo)^T. L^{-1} is lower triangular, so output columns 0-63 need
 // only channels 0-63: the first four K-steps are N = 128 MMAs, the last four
-// N = 64 MMAs into columns 64-127. V comes straight from the TMA-staged tile.
+// N = 64 MMAs into columns 64-127. The image's zero quarter (rows 0-63 of
+// channels 64-127) is not copied into shared memory, which leaves room for a
+// fourth V stage. V comes straight from the TMA-staged tile.
 // Each epilogue thread owns one token (one TMEM lane) and reduces
 // ||y||^2 = sum_j D[j]^2 in fp32, then multiplies by w_i. The tensor-memory accumulator
 // is double-buffered so the epilogue of tile i overlaps the MMAs of tile i+1,
@@ -19,7 +21,7 @@
 namespace jacap {
 
 constexpr int SC_THREADS = 192;  // warp 0: TMA, warp 1: MMA, warps 2-5: epilogue
-constexpr int SC_STAGES = 3;
+template <bool DENSE> __host__ __device__ constexpr int sc_stages() { return DENSE ? 3 : 4; }  // V tiles in flight
 constexpr int SC_IMGS = 2;  // L^{-1} image buffers
 constexpr int SC_BOX = 16384;
 constexpr int SC_TILE_BYTES = 2 * SC_BOX;
@@ -29,7 +31,14 @@ constexpr uint32_t SC_TMEM_COLS = 256;  // two 128-column accumulators
 constexpr uint32_t SC_IDESC128 = idesc_bf16_f32(128, 128, 0, 0);
 constexpr uint32_t SC_IDESC64 = idesc_bf16_f32(128, 64, 0, 0);
 
-constexpr size_t score_bf16_smem_bytes() { return 1024 + SC_IMGS * SC_M_BYTES + SC_STAGES * SC_TILE_BYTES + 256; }
+// the lower-triangular image without its zero quarter: channel atom 0 whole
+// (32 KB), then rows 64-127 of atom 1 for hi (8 KB) and for lo (8 KB)
+constexpr int SC_MT_BYTES = 49152;
+template <bool DENSE> __host__ __device__ constexpr int sc_img_bytes() { return DENSE ? SC_M_BYTES : SC_MT_BYTES; }
+template <bool DENSE>
+constexpr size_t score_bf16_smem_bytes() {
+  return 1024 + SC_IMGS * sc_img_bytes<DENSE>() + sc_stages<DENSE>() * SC_TILE_BYTES + 256;
+}
 
 // DENSE: the score matrix is a full 128 x 128 (output directions) rather than
 // the lower-triangular L^{-1}, so no K-step may be narrowed.
@@ -38,10 +47,12 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
     score_bf16_kernel(const __grid_constant__ CUtensorMap vmap, Dims dm, Ws ws, const int32_t* __restrict__ cu,
                       float* __restrict__ scores) {
   pdl_wait();
+  constexpr int SC_STAGES = sc_stages<DENSE>();
+  constexpr int IMG = sc_img_bytes<DENSE>();
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint8_t* mimg = smem;                       // [SC_IMGS][SC_M_BYTES], by run
-  uint8_t* stages = smem + SC_IMGS * SC_M_BYTES;
+  uint8_t* mimg = smem;                       // [SC_IMGS][IMG], by run
+  uint8_t* stages = smem + SC_IMGS * IMG;
   uint64_t* vfull = (uint64_t*)(stages + SC_STAGES * SC_TILE_BYTES);
   uint64_t* vempty = vfull + SC_STAGES;
   uint64_t* accfull = vempty + SC_STAGES;
@@ -95,9 +106,16 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
         if (!cont) {  // a new unit: its image, into the buffer of the run SC_IMGS runs back
           const int mp = nrun % SC_IMGS;
           if (nrun >= SC_IMGS && !mbar_wait(smem_u32(&mempty[mp]), ((nrun / SC_IMGS) & 1) ^ 1, ws, abort)) break;
-          mbar_arrive_expect_tx(smem_u32(&mfull[mp]), SC_M_BYTES);
-          bulk_g2s(smem_u32(mimg + mp * SC_M_BYTES), ws.minv_img + u * SC_M_BYTES, SC_M_BYTES,
-                   smem_u32(&mfull[mp]));
+          mbar_arrive_expect_tx(smem_u32(&mfull[mp]), IMG);
+          const uint8_t* src = ws.minv_img + u * SC_M_BYTES;
+          uint8_t* dst = mimg + mp * IMG;
+          if (DENSE) {
+            bulk_g2s(smem_u32(dst), src, SC_M_BYTES, smem_u32(&mfull[mp]));
+          } else {
+            bulk_g2s(smem_u32(dst), src, 32768, smem_u32(&mfull[mp]));
+            bulk_g2s(smem_u32(dst + 32768), src + 32768 + 8192, 8192, smem_u32(&mfull[mp]));
+            bulk_g2s(smem_u32(dst + 40960), src + 32768 + 24576, 8192, smem_u32(&mfull[mp]));
+          }
           ++nrun;
         }
         cont = is.next_same_unit(item);
@@ -132,7 +150,7 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
           if (!mbar_wait(smem_u32(&mfull[mp]), (nrun / SC_IMGS) & 1, ws, abort)) break;
           tc_fence_after();
         }
-        const uint32_t ma = smem_u32(mimg + mp * SC_M_BYTES);
+        const uint32_t ma = smem_u32(mimg + mp * IMG);
         for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
           const int st = it % SC_STAGES;
           const int ab = it & 1;
@@ -158,8 +176,9 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
               umma_f16_ss(dacc, ad, bk, SC_IDESC128, k > 0 ? 1u : 0u);
               umma_f16_ss(dacc, ad, bk + (16384 >> 4), SC_IDESC128, 1u);
             } else {      // channels 64-127: only columns (rows of L^{-1}) 64-127 are nonzero
-              umma_f16_ss(dacc + 64, ad, bk + (8192 >> 4), SC_IDESC64, 1u);
-              umma_f16_ss(dacc + 64, ad, bk + (24576 >> 4), SC_IDESC64, 1u);
+              const uint64_t bt = b0 + (uint64_t)((32768 + (k & 3) * 32) >> 4);
+              umma_f16_ss(dacc + 64, ad, bt, SC_IDESC64, 1u);
+              umma_f16_ss(dacc + 64, ad, bt + (8192 >> 4), SC_IDESC64, 1u);
             }
           }
           umma_commit(smem_u32(&vempty[st]));
@@ -285,7 +304,8 @@ __global__ void __launch_bounds__(SF_THREADS)
 cudaError_t launch_score(const CUtensorMap& vmap, const Dims& dm, const Ws& ws, int dtype, const void* v,
                          const int32_t* cu, float* scores, int grid, cudaStream_t st) {
   if (dtype == 1) {
-    constexpr size_t smem = score_bf16_smem_bytes();
+    const size_t smem = dm.dense_minv ? score_bf16_smem_bytes<true>() : score_bf16_smem_bytes<false>();
+    static_assert(score_bf16_smem_bytes<true>() <= 232448 && score_bf16_smem_bytes<false>() <= 232448, "smem");
     auto kern = dm.dense_minv ? score_bf16_kernel<true> : score_bf16_kernel<false>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;

@@ -19,6 +19,11 @@
 // compact_kernel: 16-byte vector copies of the kept K and V rows into the
 // dense [L][Hkv][S][B][d] output; rows of -1 (or of a position outside the
 // request) are zero-filled, so no index value can make it read out of bounds.
+//
+// With GATHER, select_kernel does that copy itself for each unit as soon as
+// the unit's positions are emitted (same rows, same zero fill), so the
+// retained rows stream while other CTAs are still selecting and the pass
+// needs no separate compaction launch.
 #include "jacap_dev.cuh"
 #include "jacap_internal.h"
 
@@ -43,10 +48,40 @@ __device__ __forceinline__ void load_slab(const uint32_t* key, int n, int sl, in
   }
 }
 
-template <int KPT>
+// Rows out[0 .. B) of unit u (positions relative to the request start, as
+// emitted) from K and V into k_out, v_out; -1 or a position outside the
+// request gives a zero row. All threads of the CTA; out was written by them
+// before the barrier that precedes this call.
+template <typename T>
+__device__ __forceinline__ void gather_unit(const Dims& dm, int plane, int64_t start, int64_t end, bool valid,
+                                            const T* __restrict__ k, const T* __restrict__ v,
+                                            const int32_t* out, int B, int64_t u, T* __restrict__ k_out,
+                                            T* __restrict__ v_out) {
+  constexpr int CH = D * (int)sizeof(T) / 16;  // 16-byte chunks per row
+  const int l = plane / dm.Hkv, g = plane % dm.Hkv;
+  const int64_t base = (int64_t)l * dm.kv_sl + (int64_t)g * dm.kv_sh;
+  uint4* ko = (uint4*)(k_out + u * B * D);
+  uint4* vo = (uint4*)(v_out + u * B * D);
+#pragma unroll 2
+  for (int e = threadIdx.x; e < B * CH; e += SE_THREADS) {
+    const int r = e / CH, c = e % CH;
+    const int32_t src = out[r];
+    uint4 kk = make_uint4(0, 0, 0, 0), vv = make_uint4(0, 0, 0, 0);
+    if (valid && src >= 0 && start + src < end) {
+      const int64_t off = base + (start + src) * dm.kv_st;
+      kk = *((const uint4*)(k + off) + c);
+      vv = *((const uint4*)(v + off) + c);
+    }
+    ko[e] = kk;
+    vo[e] = vv;
+  }
+}
+
+template <int KPT, typename E, bool GATHER>
 __global__ void __launch_bounds__(SE_THREADS)
     select_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu, const float* __restrict__ scores, int B,
-                  int32_t* __restrict__ idx, int32_t* __restrict__ kept) {
+                  int32_t* __restrict__ idx, int32_t* __restrict__ kept, const E* __restrict__ k,
+                  const E* __restrict__ v, E* __restrict__ k_out, E* __restrict__ v_out) {
   pdl_wait();
   constexpr int SE_KPT = KPT;
   constexpr int SE_SLAB = SE_THREADS * KPT;  // warp w holds positions 32 KPT w .. + 32 KPT - 1 of a slab
@@ -64,11 +99,16 @@ __global__ void __launch_bounds__(SE_THREADS)
     const int64_t start = cu[s];
     const int64_t end = cu[s + 1];
     int32_t* out = idx + (int64_t)u * B;
-    if (start < 0 || end < start || end > dm.Ntot) {  // malformed cu_seqlens: no reads
+    const bool valid = !(start < 0 || end < start || end > dm.Ntot);
+    if (!valid) {  // malformed cu_seqlens: no reads
       for (int r = tid; r < B; r += SE_THREADS) out[r] = -1;
       if (tid == 0) {
         flag(ws, ST_INVALID);
         if (plane == 0) kept[s] = 0;
+      }
+      if constexpr (GATHER) {
+        __syncthreads();
+        gather_unit<E>(dm, plane, start, end, false, k, v, out, B, u, k_out, v_out);
       }
       continue;
     }
@@ -77,6 +117,10 @@ __global__ void __launch_bounds__(SE_THREADS)
     if (plane == 0 && tid == 0) kept[s] = min(n, B);
     if (n <= B) {
       for (int r = tid; r < B; r += SE_THREADS) out[r] = r < n ? r : -1;
+      if constexpr (GATHER) {
+        __syncthreads();
+        gather_unit<E>(dm, plane, start, end, true, k, v, out, B, u, k_out, v_out);
+      }
       continue;
     }
     const int nslab = (n + SE_SLAB - 1) / SE_SLAB;
@@ -177,6 +221,9 @@ __global__ void __launch_bounds__(SE_THREADS)
       eq_run += eq_all;
       __syncthreads();  // the totals in hist are read before the next slab rewrites them
     }
+    // (the barrier that ends the last slab also orders the emitted positions
+    // before the gather reads them)
+    if constexpr (GATHER) gather_unit<E>(dm, plane, start, end, true, k, v, out, B, u, k_out, v_out);
   }
 }
 
@@ -208,20 +255,32 @@ __global__ void __launch_bounds__(256)
   }
 }
 
+template <int KPT>
+static cudaError_t launch_select_kpt(const Dims& dm, const Ws& ws, const int32_t* cu, const float* scores, int budget,
+                                     int32_t* idx, int32_t* kept, int dtype, const void* k, const void* v,
+                                     void* k_out, void* v_out, int grid, cudaStream_t st) {
+  using bf = __nv_bfloat16;
+  if (k == nullptr)
+    return launch_pdl(dm.pdl != 0, select_kernel<KPT, bf, false>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget,
+                      idx, kept, (const bf*)nullptr, (const bf*)nullptr, (bf*)nullptr, (bf*)nullptr);
+  if (dtype == 1)
+    return launch_pdl(dm.pdl != 0, select_kernel<KPT, bf, true>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget,
+                      idx, kept, (const bf*)k, (const bf*)v, (bf*)k_out, (bf*)v_out);
+  return launch_pdl(dm.pdl != 0, select_kernel<KPT, float, true>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget,
+                    idx, kept, (const float*)k, (const float*)v, (float*)k_out, (float*)v_out);
+}
+
 cudaError_t launch_select(const Dims& dm, const Ws& ws, const int32_t* cu, const float* scores, int budget,
-                          int32_t* idx, int32_t* kept, int max_seqlen, int grid, cudaStream_t st) {
+                          int32_t* idx, int32_t* kept, int max_seqlen, int grid, cudaStream_t st, int dtype,
+                          const void* k, const void* v, void* k_out, void* v_out) {
   if (max_seqlen <= SE_THREADS * 4)
-    JACAP_TRY(launch_pdl(dm.pdl != 0, select_kernel<4>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget, idx,
-                         kept));
+    JACAP_TRY(launch_select_kpt<4>(dm, ws, cu, scores, budget, idx, kept, dtype, k, v, k_out, v_out, grid, st));
   else if (max_seqlen <= SE_THREADS * 8)
-    JACAP_TRY(launch_pdl(dm.pdl != 0, select_kernel<8>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget, idx,
-                         kept));
+    JACAP_TRY(launch_select_kpt<8>(dm, ws, cu, scores, budget, idx, kept, dtype, k, v, k_out, v_out, grid, st));
   else if (max_seqlen <= SE_THREADS * 16)
-    JACAP_TRY(launch_pdl(dm.pdl != 0, select_kernel<16>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget, idx,
-                         kept));
+    JACAP_TRY(launch_select_kpt<16>(dm, ws, cu, scores, budget, idx, kept, dtype, k, v, k_out, v_out, grid, st));
   else
-    JACAP_TRY(launch_pdl(dm.pdl != 0, select_kernel<32>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget, idx,
-                         kept));
+    JACAP_TRY(launch_select_kpt<32>(dm, ws, cu, scores, budget, idx, kept, dtype, k, v, k_out, v_out, grid, st));
   return cudaGetLastError();
 }
 

@@ -162,6 +162,49 @@ def test_strided_cache_views():
     check_unit(ev, t2, wl, jacap_params(), 1, 1, 1)
 
 
+@pytest.mark.parametrize("name", ["bf16_gqa4_ragged_tails", "bf16_gqa2_peaky_tiny_seq", "f32_gqa4_peaky",
+                                  "bf16_budget_exceeds_all"])
+def test_fused_select_compact_equals_the_two_calls(name):
+    # jacap_select_compact (one launch) against jacap_select + jacap_compact on
+    # the same scores: positions, kept counts and rows bit for bit
+    wl, params = SMALL[name]
+    t = generate(wl, DEV)
+    ev = evict(make_cache(t, wl), wl.budget, params)  # the fused call
+    sep = Evictor(make_cache(t, wl), wl.budget, params)
+    sep.scores.copy_(ev.scores)
+    sep.ws[:64].zero_()
+    sep.k_out.fill_(7)  # the zero rows must be written, not left over
+    sep.v_out.fill_(7)
+    sep.select()
+    sep.compact()
+    sep.check()
+    assert torch.equal(ev.idx, sep.idx) and torch.equal(ev.kept, sep.kept)
+    assert_rows_bitwise(sep.k_out, ev.k_out)
+    assert_rows_bitwise(sep.v_out, ev.v_out)
+
+
+def test_fused_select_compact_zero_fills_a_malformed_request():
+    # request 1 claims tokens 300 .. 599 of a 500-token cache: it is refused
+    # (positions -1, zero rows, status invalid argument) and request 0 is served
+    wl = Workload("t", 1, 4, 2, (300, 200), 8, 32, seed=25)
+    t = generate(wl, DEV)
+    bad = torch.tensor([0, 300, 600], dtype=torch.int32, device=DEV)
+    ev = Evictor(Cache(t.q_win, t.k, t.v, bad, [300, 300], wl.num_q_heads), wl.budget)
+    ev.scores.fill_(1.0)  # all equal: the first B positions are kept
+    ev.k_out.fill_(7)
+    ev.v_out.fill_(7)
+    ev.ws[:64].zero_()
+    ev.select_compact()
+    assert ev.device_status() == 1  # JACAP_ERR_INVALID_ARG
+    assert ev.kept.cpu().tolist() == [wl.budget, 0]
+    assert bool((ev.idx[:, :, 1] == -1).all())
+    assert bool((ev.k_out[:, :, 1] == 0).all()) and bool((ev.v_out[:, :, 1] == 0).all())
+    assert ev.idx[0, 0, 0].cpu().tolist() == list(range(wl.budget))
+    for g in range(wl.num_kv_heads):
+        assert_rows_bitwise(t.k[0, g, :wl.budget], ev.k_out[0, g, 0])
+        assert_rows_bitwise(t.v[0, g, :wl.budget], ev.v_out[0, g, 0])
+
+
 def test_window_of_one_gives_zero_scores_and_first_positions():
     wl = Workload("t", 1, 4, 2, (600,), 1, 40, seed=24)
     t = generate(wl, DEV)
@@ -224,6 +267,11 @@ def test_full_size_config(index, samples):
             ev2.select()
             ev2.compact()
             gpu_selection_properties(ev2.scores, ev2.idx, ev2.kept, wl.seqlens, b)
+            k2, v2 = ev2.k_out.clone(), ev2.v_out.clone()
+            ev2.select_compact()
+            assert_rows_bitwise(k2, ev2.k_out)
+            assert_rows_bitwise(v2, ev2.v_out)
+            del k2, v2
     del ev, t
     torch.cuda.empty_cache()
 
