@@ -379,6 +379,9 @@ def run_ours(args):
     # traffic (visible in `traffic`). With bf16 caches the Gram computes the
     # Eq. 8 weights itself (it also reads the logits/kappa rows).
     fused_weights = wl.dtype == "bf16"
+    # full covariance on the tensor cores runs inside the K pass (one kernel)
+    full_cov_fused = (wl.dtype == "bf16" and wl.window in (8, 16, 32, 64)
+                      and (wl.num_q_heads // wl.num_kv_heads) * wl.window <= 128)
     alg_kernel = {
         "k_pass": kv_bytes,                       # K read once
         "gram": kv_bytes,                         # V read once
@@ -438,9 +441,11 @@ def run_ours(args):
             },
             "kernel_ms": kern,
             "ms_per_step_with_kernel_events": t_ms_events,
-            # plan, query statistics, K pass, [full covariance], [weights: float32 only], Gram,
-            # factor, scores, selection + compaction
-            "gpu_launches": K * (7 + (1 if args.covariance == "full" else 0) + (0 if fused_weights else 1)),
+            # plan, query statistics, K pass (with the full-covariance kappa when that
+            # runs on the tensor cores), [full covariance on the CUDA cores],
+            # [weights: float32 only], Gram, factor, scores, selection + compaction
+            "gpu_launches": K * (7 + (1 if args.covariance == "full" and not full_cov_fused else 0)
+                                 + (0 if fused_weights else 1)),
             "clocks": clocks,
             "cpu_baseline": cpu,
             "e2e": e2e,

@@ -298,13 +298,14 @@ jacap_status score_pass(const jacap_layout* layout, const jacap_params* params, 
       (st = map_cuda(running ? launch_stats_moments(dm, w, stats, counts, s)
                              : launch_window_stats(dm, w, dt, q_win, s))) != JACAP_OK)
     return st;
+  // full covariance on the tensor cores: one kernel does the K pass with that kappa
+  const bool fused_full = dm.full_cov && kfull_uses_tensor_cores(dm, dt);
   if ((st = hook(2)) != JACAP_OK ||
-      (st = map_cuda(launch_kpass(kmap, dm, w, dt, cu, persistent_grid(items, sms, 1), s))) != JACAP_OK)
+      (st = map_cuda(fused_full ? launch_kpass_full(kmap, dm, w, persistent_grid(items, sms, 1), s)
+                                : launch_kpass(kmap, dm, w, dt, cu, persistent_grid(items, sms, 1), s))) != JACAP_OK)
     return st;
-  if (dm.full_cov &&  // overwrites the K pass's diagonal kappa; timed with the K pass
-      (st = map_cuda(launch_kfull(kmap, dm, w, dt, k,
-                                  persistent_grid(items, sms, kfull_uses_tensor_cores(dm, dt) ? 1 : 2), s))) !=
-          JACAP_OK)
+  if (dm.full_cov && !fused_full &&  // overwrites the K pass's diagonal kappa; timed with the K pass
+      (st = map_cuda(launch_kfull(kmap, dm, w, dt, k, persistent_grid(items, sms, 2), s))) != JACAP_OK)
     return st;
   // (bf16 caches: the Gram kernel computes the weights from the K pass's rows)
   if ((st = hook(3)) != JACAP_OK ||

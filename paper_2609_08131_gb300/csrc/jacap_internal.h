@@ -39,7 +39,12 @@ cudaError_t launch_kpass(const CUtensorMap& kmap, const Dims& dm, const Ws& ws, 
                          int grid, cudaStream_t st);
 cudaError_t launch_kpass_bf16(const CUtensorMap& kmap, const Dims& dm, const Ws& ws, const int32_t* cu, int grid,
                               cudaStream_t st);
+// Full covariance (App. B.2): with a bf16 cache and a supported window shape
+// (kfull_uses_tensor_cores) launch_kpass_full replaces the K pass (logits,
+// full-covariance kappa and softmax statistics in one read of K); otherwise
+// the K pass runs and launch_kfull (CUDA cores) overwrites its diagonal kappa.
 bool kfull_uses_tensor_cores(const Dims& dm, int dtype);
+cudaError_t launch_kpass_full(const CUtensorMap& kmap, const Dims& dm, const Ws& ws, int grid, cudaStream_t st);
 cudaError_t launch_kfull(const CUtensorMap& kmap, const Dims& dm, const Ws& ws, int dtype, const void* k, int grid,
                          cudaStream_t st);
 cudaError_t launch_weights(const Dims& dm, const Ws& ws, const int32_t* cu, int grid, cudaStream_t st);

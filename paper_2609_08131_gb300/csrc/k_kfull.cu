@@ -9,18 +9,25 @@
 // squares. These kernels run after the K pass (which supplies the logits and
 // the softmax statistics) and overwrite its diagonal kappa.
 //
-// bf16 caches (w in {8, 16, 32, 64}, G w <= 128): tcgen05. A = the TMA-staged K
-// tile (K-major), B = the group's G w centred queries, each split into a bf16
-// hi and lo part (hi + lo is within 2^-18 relative of delta, so the centred
-// logits carry about 17 significant bits of delta before fp32 accumulation
-// instead of the 8 that one bf16 rounding would leave). The query-statistics
-// kernel writes that B operand straight into the workspace in shared-memory
-// image form; here it is one bulk copy per unit (a CTA's consecutive items
-// of one unit share it), issued one item ahead into a double buffer. One MMA
-// job of N = 2 rp columns per 128-token tile, the accumulator
-// double-buffered in tensor memory, so one tile's readout overlaps
-// the next tile's MMAs. Eight readout warps (two per tensor-memory lane
-// quarter, alternating tiles) add the two parts, square and sum per head.
+// bf16 caches (w in {8, 16, 32, 64}, G w <= 128): one tcgen05 kernel does the
+// whole K pass in this mode, so K is read once: the pool-softmax logits
+// l_h = k . mu'_h (mu' = mu / (tau sqrt d)), this kappa and the per-chunk
+// softmax statistics. A = the TMA-staged K tile (K-major); B = a per-unit
+// image with, per 64-channel atom, two sections of N = rp + nb rows:
+//   section 0: rows 0 .. rp-1   hi(delta_j), the bf16 rounding of q_j - mu,
+//              rows rp .. rp+nb-1  mu' split exactly into three bf16 parts;
+//   section 1: rows 0 .. rp-1   lo(delta_j), the bf16 rounding of the rest,
+//              rows rp .. rp+nb-1  zero.
+// Two MMAs of N columns per 16 channels accumulate both sections into one
+// accumulator, so column j < rp holds delta_j . k with hi + lo within 2^-18
+// relative of delta (about 17 significant bits before fp32 accumulation
+// instead of the 8 that one bf16 rounding would leave), and column rp + n
+// part n of mu' . k. The query-statistics kernel writes the delta rows in
+// image form into the workspace; here they arrive by bulk copies, once per
+// run of a CTA's consecutive items of one unit, and a builder warp adds the
+// mu' rows. Four readout warps (one per tensor-memory lane quarter) square and
+// sum the delta columns per head, add the three logit parts, keep the online
+// (max, sum exp) and write the token's logits/kappa row in one piece.
 //
 // Other shapes and float32 caches: a SIMT kernel (one thread per token, the
 // tile's keys and one head's centred queries staged in shared memory).
@@ -29,39 +36,74 @@
 
 namespace jacap {
 
-constexpr int KF_STAGES = 3;
-constexpr int KF_BOX = 16384;  // {64 channels, 128 tokens} bf16
-constexpr int KF_TILE_BYTES = 2 * KF_BOX;
-constexpr int KF_THREADS = 320;  // warp 0: TMA, warp 1: MMA, warps 2-9: readout
-constexpr int KF_READ0 = 2;
-constexpr uint32_t KF_TMEM_COLS = 512;
+constexpr int KX_STAGES = 4;
+constexpr int KX_BOX = 16384;  // {64 channels, 128 tokens} bf16
+constexpr int KX_TILE_BYTES = 2 * KX_BOX;
+constexpr int KX_THREADS = 256;  // warp 0: TMA, 1: MMA, 2: image builder, 3: idle, 4-7: readout
+constexpr int KX_READ0 = 4;
+constexpr uint32_t KX_TMEM_COLS = 512;
 
 template <int G, int W>
-struct KfCfg {
-  static constexpr int RP = kfull_rows_padded(G, W);  // padded rows per split part
-  static constexpr int N = 2 * RP;                     // MMA N
-  static constexpr int IMG_ATOM = N * 128;             // one 64-channel atom of the image
-  static constexpr int IMG_BYTES = 2 * IMG_ATOM;       // = 512 RP, as written by the query statistics
+struct KxCfg {
+  static constexpr int RP = kfull_rows_padded(G, W);  // delta rows (G w, padded)
+  static constexpr int NB = (3 * G <= 16) ? 16 : 32;   // mu' rows (3 G parts, padded)
+  static constexpr int N = RP + NB;                    // MMA N
+  static constexpr int SEC = N * 128;                  // bytes of one section of one atom
+  static constexpr int ATOM = 2 * SEC;
+  static constexpr int IMG_BYTES = 2 * ATOM;
+  static constexpr int QIMG_BYTES = 512 * RP;          // the delta image as the query statistics write it
+  static constexpr uint32_t ACC = N <= 128 ? 128 : 256;  // tensor-memory columns per accumulator
   static constexpr uint32_t IDESC = idesc_bf16_f32(128, N, 0, 0);
-  static_assert(RP > 0 && N <= 256, "tensor-core shape");
-  static constexpr size_t SMEM = 1024 + (size_t)KF_STAGES * KF_TILE_BYTES + 2 * (size_t)IMG_BYTES + 256;
+  static_assert(RP > 0 && N <= 256 && N % 16 == 0 && 2 * ACC <= KX_TMEM_COLS, "tensor-core shape");
+  static_assert(SEC % 1024 == 0, "sections start on a swizzle-pattern boundary");
+  static constexpr size_t SMEM = 1024 + (size_t)KX_STAGES * KX_TILE_BYTES + IMG_BYTES + 4 * 2 * G * 4 + 256;
 };
 
+// Rows rp .. rp + nb - 1 of section 0 of both atoms: row rp + part G + h holds
+// part (0 hi, 1 mid, 2 lo) of mu'_h with hi + mid + lo = mu'_h to about 24
+// bits; rows past 3 G are zero. One warp.
 template <int G, int W>
-__global__ void __launch_bounds__(KF_THREADS, 1)
-    kfull_bf16_kernel(const __grid_constant__ CUtensorMap kmap, Dims dm, Ws ws) {
+__device__ __forceinline__ void write_mu_rows(uint8_t* img, const float* mu, int lane) {
+  using C = KxCfg<G, W>;
+  for (int e = lane; e < C::NB * 16; e += 32) {
+    const int n = e >> 4, cc = e & 15;  // row, 8-channel chunk
+    uint32_t wv[4] = {0u, 0u, 0u, 0u};
+    if (n < 3 * G) {
+      const int part = n / G, h = n % G;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        float x[2];
+#pragma unroll
+        for (int z = 0; z < 2; ++z) {
+          const float v = mu[h * D + cc * 8 + 2 * q + z];
+          const float hi = __bfloat162float(__float2bfloat16_rn(v));
+          const float r1 = v - hi;
+          const float mid = __bfloat162float(__float2bfloat16_rn(r1));
+          x[z] = part == 0 ? hi : (part == 1 ? mid : r1 - mid);
+        }
+        wv[q] = pack_bf16x2(x[0], x[1]);
+      }
+    }
+    *(uint4*)(img + (cc >> 3) * C::ATOM + sw128_off(C::RP + n, cc & 7)) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+  }
+}
+
+template <int G, int W>
+__global__ void __launch_bounds__(KX_THREADS, 1)
+    kpass_full_bf16_kernel(const __grid_constant__ CUtensorMap kmap, Dims dm, Ws ws) {
   pdl_wait();
-  using C = KfCfg<G, W>;
+  using C = KxCfg<G, W>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t* tiles = smem;
-  uint8_t* img = tiles + KF_STAGES * KF_TILE_BYTES;  // [2][IMG_BYTES]
-  uint64_t* full = (uint64_t*)(img + 2 * C::IMG_BYTES);
-  uint64_t* empty = full + KF_STAGES;
-  uint64_t* accfull = empty + KF_STAGES;  // [2]
+  uint8_t* img = tiles + KX_STAGES * KX_TILE_BYTES;     // one image, refilled per run
+  float* red = (float*)(img + C::IMG_BYTES);             // [4 readout warps][2G]
+  uint64_t* full = (uint64_t*)(red + 4 * 2 * G);
+  uint64_t* empty = full + KX_STAGES;
+  uint64_t* accfull = empty + KX_STAGES;  // [2]
   uint64_t* accempty = accfull + 2;       // [2]
-  uint64_t* imgfull = accempty + 2;       // [2]
-  uint64_t* imgfree = imgfull + 2;        // [2]
+  uint64_t* imgfull = accempty + 2;
+  uint64_t* imgfree = imgfull + 1;
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort, s_skip;
 
@@ -69,22 +111,22 @@ __global__ void __launch_bounds__(KF_THREADS, 1)
   if (tid == 0) {
     s_abort = 0;
     s_skip = status_failed(ws) ? 1 : 0;
-    for (int i = 0; i < KF_STAGES; ++i) {
+    for (int i = 0; i < KX_STAGES; ++i) {
       mbar_init(smem_u32(&full[i]), 1);
       mbar_init(smem_u32(&empty[i]), 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&accfull[i]), 1);
       mbar_init(smem_u32(&accempty[i]), 4);
-      mbar_init(smem_u32(&imgfull[i]), 1);
-      mbar_init(smem_u32(&imgfree[i]), 1);
     }
+    mbar_init(smem_u32(imgfull), 2);  // the bulk copies' arrival + the builder's mu' rows
+    mbar_init(smem_u32(imgfree), 1);
     fence_mbar_init();
   }
   __syncthreads();
   if (s_skip) return;
   if (warp == 1) {
-    tmem_alloc(smem_u32(&s_tmem), KF_TMEM_COLS);
+    tmem_alloc(smem_u32(&s_tmem), KX_TMEM_COLS);
     tmem_relinquish();
   }
   tc_fence_before();
@@ -94,85 +136,97 @@ __global__ void __launch_bounds__(KF_THREADS, 1)
   volatile int* abort = &s_abort;
 
   if (warp == 0) {
-    // ------------------------------------ TMA: key tiles and query images --
+    // ------------------------------------------------ TMA: key tiles ------
     if (lane == 0) {
       prefetch_tmap(&kmap);
-      auto issue_image = [&](const Item& item, uint32_t n) {
-        const int p = n & 1;
-        const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
-        const uint8_t* src = ws.qimg + (((int64_t)item.seq * dm.L + l) * dm.Hkv + g) * (int64_t)C::IMG_BYTES;
-        mbar_arrive_expect_tx(smem_u32(&imgfull[p]), C::IMG_BYTES);
-        bulk_g2s(smem_u32(img + p * C::IMG_BYTES), src, C::IMG_BYTES, smem_u32(&imgfull[p]));
-      };
-      uint32_t it = 0, nimg = 0;
+      uint32_t it = 0;
       bool ok = true;
-      ItemStream is(dm, ws, blockIdx.x, gridDim.x);
-      Item cur, nxt;
-      bool have = is.next(cur);
-      if (have) issue_image(cur, nimg++);
-      while (ok && have) {
-        const int l = cur.plane / dm.Hkv, g = cur.plane % dm.Hkv;
-        for (int64_t t = cur.t0; t < cur.t1; t += TILE) {
-          const int st = it % KF_STAGES;
-          if (it >= (uint32_t)KF_STAGES &&
-              !mbar_wait(smem_u32(&empty[st]), ((it / KF_STAGES) & 1) ^ 1, ws, abort)) {
+      Item item;
+      for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); ok && is.next(item);) {
+        const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
+        for (int64_t t = item.t0; t < item.t1; t += TILE) {
+          const int st = it % KX_STAGES;
+          if (it >= (uint32_t)KX_STAGES &&
+              !mbar_wait(smem_u32(&empty[st]), ((it / KX_STAGES) & 1) ^ 1, ws, abort)) {
             ok = false;
             break;
           }
-          uint8_t* kt = tiles + st * KF_TILE_BYTES;
-          mbar_arrive_expect_tx(smem_u32(&full[st]), KF_TILE_BYTES);
+          uint8_t* kt = tiles + st * KX_TILE_BYTES;
+          mbar_arrive_expect_tx(smem_u32(&full[st]), KX_TILE_BYTES);
           tma_load_4d(smem_u32(kt), &kmap, 0, (int)t, g, l, smem_u32(&full[st]));
-          tma_load_4d(smem_u32(kt + KF_BOX), &kmap, 64, (int)t, g, l, smem_u32(&full[st]));
+          tma_load_4d(smem_u32(kt + KX_BOX), &kmap, 64, (int)t, g, l, smem_u32(&full[st]));
           ++it;
-        }
-        if (!ok) break;
-        // a next item of another unit needs its image: it goes to the buffer
-        // of the run before this one, whose MMAs were all issued before this
-        // run's first tile
-        have = is.next(nxt);
-        if (have) {
-          if (nxt.plane != cur.plane || nxt.seq != cur.seq) {
-            if (nimg >= 2 && !mbar_wait(smem_u32(&imgfree[nimg & 1]), ((nimg - 2) >> 1) & 1, ws, abort)) break;
-            issue_image(nxt, nimg++);
-          }
-          cur = nxt;
         }
       }
       // no copy may still be landing when the CTA exits
-      for (uint32_t k = (it > (uint32_t)KF_STAGES ? it - KF_STAGES : 0); k < it; ++k)
-        mbar_wait(smem_u32(&full[k % KF_STAGES]), (k / KF_STAGES) & 1, ws, nullptr);
-      for (uint32_t k = (nimg > 2u ? nimg - 2 : 0); k < nimg; ++k)
-        mbar_wait(smem_u32(&imgfull[k & 1]), (k >> 1) & 1, ws, nullptr);
+      for (uint32_t k = (it > (uint32_t)KX_STAGES ? it - KX_STAGES : 0); k < it; ++k)
+        mbar_wait(smem_u32(&full[k % KX_STAGES]), (k / KX_STAGES) & 1, ws, nullptr);
     }
+  } else if (warp == 2) {
+    // ------------------------- the unit's image, once per run ------------
+    // single buffer: a run's image is written once the previous run's MMAs
+    // have all completed (imgfree)
+    uint32_t n = 0;
+    bool cont = false;
+    Item item;
+    for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
+      const bool same = cont;
+      cont = is.next_same_unit(item);
+      if (same) continue;
+      if (n >= 1 && !mbar_wait(smem_u32(imgfree), (n - 1) & 1, ws, abort)) break;
+      const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
+      if (lane == 0) {
+        const uint8_t* src = ws.qimg + (((int64_t)item.seq * dm.L + l) * dm.Hkv + g) * (int64_t)C::QIMG_BYTES;
+        mbar_arrive_expect_tx(smem_u32(imgfull), 4 * C::RP * 128);
+#pragma unroll
+        for (int a = 0; a < 2; ++a) {
+          const uint8_t* sa = src + a * (256 * C::RP);
+          bulk_g2s(smem_u32(img + a * C::ATOM), sa, C::RP * 128, smem_u32(imgfull));
+          bulk_g2s(smem_u32(img + a * C::ATOM + C::SEC), sa + C::RP * 128, C::RP * 128, smem_u32(imgfull));
+        }
+      }
+      const int64_t qb = (((int64_t)item.seq * dm.L + l) * dm.Hq + (int64_t)g * G) * D;
+      write_mu_rows<G, W>(img, ws.mu + qb, lane);
+      if (n == 0)  // the zero rows of section 1 (never rewritten)
+        for (int e = lane; e < 2 * C::NB * 8; e += 32) {
+          const int a = e / (C::NB * 8), r = (e / 8) % C::NB, cc = e % 8;
+          *(uint4*)(img + a * C::ATOM + C::SEC + sw128_off(C::RP + r, cc)) = make_uint4(0u, 0u, 0u, 0u);
+        }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(imgfull));
+      ++n;
+    }
+    // no image copy may still be landing when the CTA exits
+    if (lane == 0 && n > 0) mbar_wait(smem_u32(imgfull), (n - 1) & 1, ws, nullptr);
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer ----------
     if (lane == 0) {
-      uint32_t it = 0, n = 0;  // n: runs (units) started
+      uint32_t it = 0, n = 0;  // n: runs started
       bool ok = true, cont = false;
-      int p = 0;
       Item item;
+      const uint64_t b0 = smem_desc_sw128(smem_u32(img), 16, 1024);
       for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); ok && is.next(item);) {
         if (!cont) {
-          p = n & 1;
-          if (!mbar_wait(smem_u32(&imgfull[p]), (n >> 1) & 1, ws, abort)) break;
+          if (!mbar_wait(smem_u32(imgfull), n & 1, ws, abort)) break;
           tc_fence_after();
         }
-        const uint64_t b0 = smem_desc_sw128(smem_u32(img + p * C::IMG_BYTES), 16, 1024);
         for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
-          const int st = it % KF_STAGES, slot = it & 1;
-          if (!mbar_wait(smem_u32(&full[st]), (it / KF_STAGES) & 1, ws, abort) ||
+          const int st = it % KX_STAGES, slot = it & 1;
+          if (!mbar_wait(smem_u32(&full[st]), (it / KX_STAGES) & 1, ws, abort) ||
               (it >= 2 && !mbar_wait(smem_u32(&accempty[slot]), ((it >> 1) & 1) ^ 1, ws, abort))) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint64_t a0 = smem_desc_sw128(smem_u32(tiles + st * KF_TILE_BYTES), 16, 1024);
-          const uint32_t dacc = tmem + slot * 256;
+          const uint64_t a0 = smem_desc_sw128(smem_u32(tiles + st * KX_TILE_BYTES), 16, 1024);
+          const uint32_t dacc = tmem + slot * C::ACC;
 #pragma unroll
           for (int k = 0; k < D / 16; ++k) {  // descriptors advance by (byte offset >> 4)
-            const uint64_t ad = a0 + (uint64_t)((((k >> 2) * KF_BOX) + (k & 3) * 32) >> 4);
-            const uint64_t bd = b0 + (uint64_t)((((k >> 2) * C::IMG_ATOM) + (k & 3) * 32) >> 4);
-            umma_f16_ss(dacc, ad, bd, C::IDESC, k > 0 ? 1u : 0u);
+            const uint64_t ad = a0 + (uint64_t)((((k >> 2) * KX_BOX) + (k & 3) * 32) >> 4);
+            const uint64_t bh = b0 + (uint64_t)((((k >> 2) * C::ATOM) + (k & 3) * 32) >> 4);
+            umma_f16_ss(dacc, ad, bh, C::IDESC, k > 0 ? 1u : 0u);
+            umma_f16_ss(dacc, ad, bh + (uint64_t)(C::SEC >> 4), C::IDESC, 1u);
           }
           umma_commit(smem_u32(&accfull[slot]));
           umma_commit(smem_u32(&empty[st]));
@@ -180,60 +234,129 @@ __global__ void __launch_bounds__(KF_THREADS, 1)
         if (!ok) break;
         cont = is.next_same_unit(item);
         if (!cont) {
-          umma_commit(smem_u32(&imgfree[p]));
+          umma_commit(smem_u32(imgfree));
           ++n;
         }
       }
       // every MMA issued here completes before the CTA tears down tensor memory
       if (it > 0) mbar_wait(smem_u32(&accfull[(it - 1) & 1]), ((it - 1) >> 1) & 1, ws, nullptr);
     }
-  } else {
+  } else if (warp >= KX_READ0) {
     // ------------------------------------------------ readout -------------
-    const int set = (warp - KF_READ0) >> 2;  // tiles with it % 2 == set
     const int quarter = warp & 3;
-    const int y = quarter * 32 + lane;        // token row of the tile (tensor-memory lane)
+    const int rw = warp - KX_READ0;
+    const int y = quarter * 32 + lane;  // token row of the tile (tensor-memory lane)
     const uint32_t lanes = (uint32_t)(quarter * 32) << 16;
     const float invw = 1.f / (float)(dm.cov_unbiased ? dm.window - 1 : dm.window);
     uint32_t it = 0;
-    bool bad = false;
+    bool bad = false, cont = false;
+    float run_m[G], run_s[G];
     Item item;
     for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
-      float* lkp = ws.lk + (int64_t)item.plane * dm.Ntot * (2 * G) + G;
+      if (!cont) {  // a new run of the unit's consecutive chunks: fresh statistics
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+          run_m[h] = -INFINITY;
+          run_s[h] = 0.f;
+        }
+      }
+      float* lkp = ws.lk + (int64_t)item.plane * dm.Ntot * (2 * G);
       for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
-        if ((int)(it & 1) != set) continue;
-        if (!mbar_wait(smem_u32(&accfull[set]), (it >> 1) & 1, ws, abort)) goto read_done;
+        const int slot = it & 1;
+        if (!mbar_wait(smem_u32(&accfull[slot]), (it >> 1) & 1, ws, abort)) break;  // abort: see below
         tc_fence_after();
+        const uint32_t ta = tmem + slot * C::ACC + lanes;
         float kap[G];
 #pragma unroll
-        for (int hh = 0; hh < G; ++hh) kap[hh] = 0.f;
-        const uint32_t ta = tmem + set * 256 + lanes;
+        for (int h = 0; h < G; ++h) kap[h] = 0.f;
 #pragma unroll
-        for (int b = 0; b < C::RP / 32; ++b) {
-          uint32_t hi[32], lo[32];  // the two parts of 32 centred logits delta_j . k
-          tmem_ld32x2(ta + b * 32, ta + C::RP + b * 32, hi, lo);
+        for (int b = 0; b < C::RP / 32; b += 2) {
+          uint32_t xa[32], xb[32];
+          if (b + 1 < C::RP / 32) {
+            tmem_ld32x2(ta + b * 32, ta + (b + 1) * 32, xa, xb);
+          } else {
+            tmem_ld32(ta + b * 32, (float*)xa);
+          }
 #pragma unroll
           for (int jj = 0; jj < 32; ++jj) {
             const int r = b * 32 + jj;
             if (r < G * W) {
-              const float c = __uint_as_float(hi[jj]) + __uint_as_float(lo[jj]);
+              const float c = __uint_as_float(xa[jj]);
               kap[r / W] = fmaf(c, c, kap[r / W]);
             }
           }
+          if (b + 1 < C::RP / 32) {
+#pragma unroll
+            for (int jj = 0; jj < 32; ++jj) {
+              const int r = (b + 1) * 32 + jj;
+              if (r < G * W) {
+                const float c = __uint_as_float(xb[jj]);
+                kap[r / W] = fmaf(c, c, kap[r / W]);
+              }
+            }
+          }
         }
+        float dv[C::NB];
+        if constexpr (C::NB == 16) tmem_ld16(ta + C::RP, dv);
+        else tmem_ld32(ta + C::RP, dv);
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(smem_u32(&accempty[set]));
+        if (lane == 0) mbar_arrive(smem_u32(&accempty[slot]));
         const int64_t tok = t + y;
         if (tok < item.t1) {
-          float* dst = lkp + tok * (2 * G);
+          float row[2 * G];
 #pragma unroll
-          for (int hh = 0; hh < G; ++hh) {
-            const float v = kap[hh] * invw;
-            bad |= !isfinite(v);
-            dst[hh] = v;
+          for (int h = 0; h < G; ++h) {
+            const float lg = dv[h] + dv[G + h] + dv[2 * G + h];
+            bad |= !isfinite(lg);
+            // branch-free online update: one of the two exponentials is exp(0)
+            const float mn = fmaxf(run_m[h], lg);
+            run_s[h] = run_s[h] * expf(run_m[h] - mn) + expf(lg - mn);
+            run_m[h] = mn;
+            row[h] = lg;
+            row[G + h] = kap[h] * invw;
+            bad |= !isfinite(row[G + h]);
+          }
+          float* dst = lkp + tok * (2 * G);
+          if constexpr (G >= 2) {
+#pragma unroll
+            for (int e = 0; e < 2 * G; e += 4) *(float4*)(dst + e) = make_float4(row[e], row[e + 1], row[e + 2], row[e + 3]);
+          } else {
+            *(float2*)dst = make_float2(row[0], row[1]);
           }
         }
       }
+      // ---- softmax statistics of a run, at its last chunk; the run's other
+      // chunks get empty statistics (m = -inf, s = 0), which merge as nothing
+      cont = is.next_same_unit(item);
+      if (cont) {
+        if (rw == 0 && lane < G) {
+          float* cs = ws.cstats + (((int64_t)item.plane * dm.c_cap + item.cidx) * G + lane) * 2;
+          cs[0] = -INFINITY;
+          cs[1] = 0.f;
+        }
+        continue;
+      }
+#pragma unroll
+      for (int h = 0; h < G; ++h) {
+        softmax_warp_merge(run_m[h], run_s[h]);
+        if (lane == 0) {
+          red[rw * 2 * G + h] = run_m[h];
+          red[rw * 2 * G + G + h] = run_s[h];
+        }
+      }
+      // a warp that met an abort still arrives here; all four leave together
+      named_barrier_sync(1, 128);
+      if (*abort) goto read_done;
+      if (rw == 0 && lane < G) {
+        const int h = lane;
+        float m = -INFINITY, ssum = 0.f;
+        for (int j = 0; j < 4; ++j) softmax_merge(m, ssum, red[j * 2 * G + h], red[j * 2 * G + G + h]);
+        float* cs = ws.cstats + (((int64_t)item.plane * dm.c_cap + item.cidx) * G + h) * 2;
+        cs[0] = m;
+        cs[1] = ssum;
+      }
+      named_barrier_sync(1, 128);
     }
   read_done:
     if (bad) flag(ws, ST_NONFINITE);
@@ -242,7 +365,7 @@ __global__ void __launch_bounds__(KF_THREADS, 1)
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, KF_TMEM_COLS);
+    tmem_dealloc(tmem, KX_TMEM_COLS);
   }
 }
 
@@ -305,29 +428,36 @@ __global__ void __launch_bounds__(KS_THREADS)
 
 // ------------------------------------------------------------ launchers ----
 template <int G, int W>
-static cudaError_t launch_kfull_tc(const CUtensorMap& kmap, const Dims& dm, const Ws& ws, int grid, cudaStream_t st) {
-  using C = KfCfg<G, W>;
+static cudaError_t launch_kpf(const CUtensorMap& kmap, const Dims& dm, const Ws& ws, int grid, cudaStream_t st) {
+  using C = KxCfg<G, W>;
   static_assert(C::SMEM <= 232448, "shared memory budget");
   cudaError_t e =
-      cudaFuncSetAttribute(kfull_bf16_kernel<G, W>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
+      cudaFuncSetAttribute(kpass_full_bf16_kernel<G, W>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
   if (e != cudaSuccess) return e;
-  JACAP_TRY(launch_pdl(dm.pdl != 0, kfull_bf16_kernel<G, W>, grid, KF_THREADS, C::SMEM, st, kmap, dm, ws));
+  JACAP_TRY(launch_pdl(dm.pdl != 0, kpass_full_bf16_kernel<G, W>, grid, KX_THREADS, C::SMEM, st, kmap, dm, ws));
   return cudaGetLastError();
 }
 
 template <int G>
-static cudaError_t launch_kfull_g(const CUtensorMap& kmap, const Dims& dm, const Ws& ws, int grid, cudaStream_t st,
-                                  bool* done) {
-  *done = true;
+static cudaError_t launch_kpf_g(const CUtensorMap& kmap, const Dims& dm, const Ws& ws, int grid, cudaStream_t st) {
   switch (dm.window) {
-    case 8: if constexpr (kfull_rows_padded(G, 8) > 0) return launch_kfull_tc<G, 8>(kmap, dm, ws, grid, st); break;
-    case 16: if constexpr (kfull_rows_padded(G, 16) > 0) return launch_kfull_tc<G, 16>(kmap, dm, ws, grid, st); break;
-    case 32: if constexpr (kfull_rows_padded(G, 32) > 0) return launch_kfull_tc<G, 32>(kmap, dm, ws, grid, st); break;
-    case 64: if constexpr (kfull_rows_padded(G, 64) > 0) return launch_kfull_tc<G, 64>(kmap, dm, ws, grid, st); break;
+    case 8: if constexpr (kfull_rows_padded(G, 8) > 0) return launch_kpf<G, 8>(kmap, dm, ws, grid, st); break;
+    case 16: if constexpr (kfull_rows_padded(G, 16) > 0) return launch_kpf<G, 16>(kmap, dm, ws, grid, st); break;
+    case 32: if constexpr (kfull_rows_padded(G, 32) > 0) return launch_kpf<G, 32>(kmap, dm, ws, grid, st); break;
+    case 64: if constexpr (kfull_rows_padded(G, 64) > 0) return launch_kpf<G, 64>(kmap, dm, ws, grid, st); break;
     default: break;
   }
-  *done = false;
-  return cudaSuccess;
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_kpass_full(const CUtensorMap& kmap, const Dims& dm, const Ws& ws, int grid, cudaStream_t st) {
+  switch (dm.G) {
+    case 1: return launch_kpf_g<1>(kmap, dm, ws, grid, st);
+    case 2: return launch_kpf_g<2>(kmap, dm, ws, grid, st);
+    case 4: return launch_kpf_g<4>(kmap, dm, ws, grid, st);
+    case 8: return launch_kpf_g<8>(kmap, dm, ws, grid, st);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 // The tensor-core kernel reads the image that the query statistics wrote
@@ -336,18 +466,7 @@ bool kfull_uses_tensor_cores(const Dims& dm, int dtype) { return dtype == 1 && d
 
 cudaError_t launch_kfull(const CUtensorMap& kmap, const Dims& dm, const Ws& ws, int dtype, const void* k, int grid,
                          cudaStream_t st) {
-  if (kfull_uses_tensor_cores(dm, dtype)) {
-    bool done = false;
-    cudaError_t e = cudaSuccess;
-    switch (dm.G) {
-      case 1: e = launch_kfull_g<1>(kmap, dm, ws, grid, st, &done); break;
-      case 2: e = launch_kfull_g<2>(kmap, dm, ws, grid, st, &done); break;
-      case 4: e = launch_kfull_g<4>(kmap, dm, ws, grid, st, &done); break;
-      case 8: e = launch_kfull_g<8>(kmap, dm, ws, grid, st, &done); break;
-      default: break;
-    }
-    if (done) return e;
-  }
+  (void)kmap;
   constexpr size_t smem = (size_t)(TILE * KS_LD + KS_WMAX * D) * sizeof(float);
   if (dtype == 1) {
     cudaError_t e = cudaFuncSetAttribute(kfull_simt_kernel<__nv_bfloat16>,
