@@ -347,8 +347,12 @@ __global__ void __launch_bounds__(FA_THREADS, PROJ ? 1 : 2)
 //                       block A_KK (its lower triangle), X_KK -> T_KK
 //    L_IK = A_IK T_KK^T                 I > K
 //    A_IJ -= L_IK L_JK^T                K < J <= I
-//  X = L^{-1}:  X_II = T_II,  X_IJ = -T_II sum_{M=J}^{I-1} L_IM X_MJ   (I > J,
-//  by increasing I - J).
+//  X = L^{-1}:  X_II = T_II,  X_IJ = -T_II S_IJ,  S_IJ = sum_{M=J}^{I-1} L_IM X_MJ
+//  (I > J). Phase P of the inverse (P = 0 .. 3) forms X_PJ = -T_PP S_PJ for
+//  J < P and adds the terms M = P, S_IJ += L_IP X_PJ (I > P, J <= P); it needs
+//  only blocks of step P and earlier, so phases 0-2 run on six warps while
+//  warp 0 eliminates the next diagonal block, and only X_3J follows the last
+//  elimination.
 // Every product is a 32 x 32 block of "rows times rows" (P Q^T) read from
 // shared memory with row stride FB_LD; the inverse is built transposed
 // (XT_JI = X_IJ^T) so its products have that form too. Thread t owns the
@@ -356,9 +360,9 @@ __global__ void __launch_bounds__(FA_THREADS, PROJ ? 1 : 2)
 constexpr int FB_THREADS = 256;
 constexpr int FB_LD = 36;             // row stride of a 32 x 32 block (floats); 16-byte rows
 constexpr int FB_BLK = 32 * FB_LD;    // floats per block
-// 10 lower blocks of A (then L_IJ, and T_II on the diagonal), 10 blocks of
-// XT (XT_JI at tri(I, J)), 3 scratch blocks
-constexpr size_t FB_SMEM = (size_t)23 * FB_BLK * sizeof(float);
+// 10 lower blocks of A (then L_IJ, and T_II on the diagonal) and 10 blocks of
+// XT (XT_JI at tri(I, J); S_IJ^T there until X_IJ replaces it)
+constexpr size_t FB_SMEM = (size_t)20 * FB_BLK * sizeof(float);
 
 __device__ __forceinline__ int tri(int i, int j) { return i * (i + 1) / 2 + j; }  // block (i, j), j <= i
 // a partial Gram's lower blocks staged in shared memory: column block nb,
@@ -468,12 +472,68 @@ __device__ __forceinline__ void trailing_update(float* As, int K, int i0, int i1
   }
 }
 
+// Threads vt = 0 .. nthr - 1 (nthr = 192 or 256) meet at barrier `bar` (0:
+// the whole CTA).
+__device__ __forceinline__ void fb_sync(int bar, int nthr) {
+  if (bar == 0) __syncthreads();
+  else named_barrier_sync(bar, nthr);
+}
+
+// Inverse phase P, first half: X_PJ = -T_PP S_PJ for J < P, in place over
+// S_PJ^T (XT(tri(P, J))). At most three 32 x 32 blocks' thread shares per thread.
+__device__ __forceinline__ void inv_rows(float* As, float* XT, int P, int vt, int nthr, int bar) {
+  float acc[3][2][2];
+  const int items = P * FB_THREADS;
+#pragma unroll
+  for (int q = 0; q < 3; ++q) {
+    acc[q][0][0] = acc[q][0][1] = acc[q][1][0] = acc[q][1][1] = 0.f;
+    const int w = vt + q * nthr;
+    if (w < items) {
+      const int J = w / FB_THREADS, t = w % FB_THREADS;
+      nt_block(acc[q], XT + tri(P, J) * FB_BLK, As + tri(P, P) * FB_BLK, t >> 4, t & 15);  // (T S)^T
+    }
+  }
+  fb_sync(bar, nthr);  // every S_PJ is read before any X_PJ overwrites it
+#pragma unroll
+  for (int q = 0; q < 3; ++q) {
+    const int w = vt + q * nthr;
+    if (w < items) {
+      const int J = w / FB_THREADS, t = w % FB_THREADS, a = t >> 4, b = t & 15;
+      float* X = XT + tri(P, J) * FB_BLK;
+#pragma unroll
+      for (int i = 0; i < 2; ++i)
+#pragma unroll
+        for (int j = 0; j < 2; ++j) X[(a + 16 * i) * FB_LD + b + 16 * j] = -acc[q][i][j];
+    }
+  }
+  fb_sync(bar, nthr);
+}
+
+// Inverse phase P, second half: S_IJ += L_IP X_PJ for I > P, J <= P (X_PP =
+// T_PP); the first term of S_IJ (P == J) overwrites.
+__device__ __forceinline__ void inv_accumulate(float* As, float* XT, int P, int vt, int nthr) {
+  const int nj = P + 1;
+  for (int w = vt; w < (3 - P) * nj * FB_THREADS; w += nthr) {
+    const int blk = w / FB_THREADS, t = w % FB_THREADS, a = t >> 4, b = t & 15;
+    const int I = P + 1 + blk / nj, J = blk % nj;
+    float d[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
+    nt_block(d, XT + tri(P, J) * FB_BLK, As + tri(I, P) * FB_BLK, a, b);  // (L_IP X_PJ)^T
+    float* S = XT + tri(I, J) * FB_BLK;
+#pragma unroll
+    for (int i = 0; i < 2; ++i)
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        float* e = S + (a + 16 * i) * FB_LD + b + 16 * j;
+        *e = (J == P) ? d[i][j] : *e + d[i][j];
+      }
+  }
+}
+
 __global__ void __launch_bounds__(FB_THREADS, 2) factor_blocked_kernel(Dims dm, Ws ws) {
   pdl_wait();
   extern __shared__ __align__(16) float fsm[];
   float* As = fsm;                // tri(I, J): A_IJ, then L_IJ (I > J) / T_II (I == J)
   float* XT = fsm + 10 * FB_BLK;  // tri(I, J): XT_JI = (L^{-1})_IJ^T
-  float* Sc = fsm + 20 * FB_BLK;  // scratch
   __shared__ __align__(8) uint64_t s_full[2];
   __shared__ int s_skip, s_bad, s_np;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -582,11 +642,17 @@ __global__ void __launch_bounds__(FB_THREADS, 2) factor_blocked_kernel(Dims dm, 
   }
 
   const int a = tid >> 4, b = tid & 15;
+  // the six warps off warp 0's sub-partition (1-3, 5-7) run inverse phases
+  // next to the elimination, so it keeps its issue slots
+  const int vt = (warp < 4 ? warp - 1 : warp - 2) * 32 + lane;
 #pragma unroll 1
   for (int K = 0; K < 4; ++K) {
-    // (the warp's elimination runs alone: next to multiply-add-heavy warps on
-    // its sub-partition it would get a fraction of the issue slots)
-    if (warp == 0) diag_inverse(As + tri(K, K) * FB_BLK, XT + tri(K, K) * FB_BLK, lane, bad);
+    if (warp == 0) {
+      diag_inverse(As + tri(K, K) * FB_BLK, XT + tri(K, K) * FB_BLK, lane, bad);
+    } else if (warp != 4 && K >= 1) {  // inverse phase K - 1
+      inv_rows(As, XT, K - 1, vt, 192, 2);
+      inv_accumulate(As, XT, K - 1, vt, 192);
+    }
     __syncthreads();
     // L_IK = A_IK T_KK^T for I > K
     float acc[3][2][2];
@@ -612,35 +678,8 @@ __global__ void __launch_bounds__(FB_THREADS, 2) factor_blocked_kernel(Dims dm, 
     __syncthreads();
   }
 
-  // XT_JI = -(T_II sum_{M=J}^{I-1} L_IM X_MJ)^T, by level I - J
-#pragma unroll 1
-  for (int lev = 1; lev < 4; ++lev) {
-#pragma unroll 1
-    for (int J = 0; J + lev < 4; ++J) {
-      const int I = J + lev;
-      float acc[2][2] = {{0.f, 0.f}, {0.f, 0.f}};  // S^T = sum_M XT_JM L_IM^T
-#pragma unroll 1
-      for (int M = J; M < I; ++M) nt_block(acc, XT + tri(M, J) * FB_BLK, As + tri(I, M) * FB_BLK, a, b);
-      float* St = Sc + J * FB_BLK;
-#pragma unroll
-      for (int i = 0; i < 2; ++i)
-#pragma unroll
-        for (int j = 0; j < 2; ++j) St[(a + 16 * i) * FB_LD + b + 16 * j] = acc[i][j];
-    }
-    __syncthreads();
-#pragma unroll 1
-    for (int J = 0; J + lev < 4; ++J) {
-      const int I = J + lev;
-      float acc[2][2] = {{0.f, 0.f}, {0.f, 0.f}};  // XT_JI = -S^T T_II^T
-      nt_block(acc, Sc + J * FB_BLK, As + tri(I, I) * FB_BLK, a, b);
-      float* X = XT + tri(I, J) * FB_BLK;
-#pragma unroll
-      for (int i = 0; i < 2; ++i)
-#pragma unroll
-        for (int j = 0; j < 2; ++j) X[(a + 16 * i) * FB_LD + b + 16 * j] = -acc[i][j];
-    }
-    __syncthreads();
-  }
+  // inverse phase 3: X_3J = -T_33 S_3J (all threads)
+  inv_rows(As, XT, 3, tid, FB_THREADS, 0);
   if (bad) s_bad = 1;
 
   // L^{-1}[n][c] = XT(tri(n / 32, c / 32))[c % 32][n % 32] for n >= c, 0 above:
