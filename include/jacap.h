@@ -318,6 +318,20 @@ jacap_status jacap_compact_inplace(const jacap_layout* layout, void* k, void* v,
                                    const int32_t* idx, int32_t budget, int32_t preserve_order,
                                    void* ws, size_t ws_bytes, void* stream);
 
+/*
+ * jacap_select followed by jacap_compact_inplace in one launch: each unit's
+ * kept rows are moved in place as soon as its positions are selected.
+ * Arguments, layouts, results and error behaviour are those of the two calls
+ * (idx and kept as from jacap_select; k, v and pos as after
+ * jacap_compact_inplace with that idx and preserve_order). The positions
+ * come from the selection itself, so no unit is refused for them. Hole filling
+ * (preserve_order = 0) runs inside the selection kernel; the ascending-order
+ * compaction, which moves every kept row, is enqueued as a second launch.
+ */
+jacap_status jacap_select_compact_inplace(const jacap_layout* layout, const float* scores, int32_t budget,
+                                          int32_t* idx, int32_t* kept, void* k, void* v, int32_t* pos,
+                                          int32_t preserve_order, void* ws, size_t ws_bytes, void* stream);
+
 /* Synchronises `stream`, then reads the workspace status word: JACAP_OK or the
  * first device-side error recorded since the last jacap_score on `ws`. */
 jacap_status jacap_device_status(const void* ws, void* stream);

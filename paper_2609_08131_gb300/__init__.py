@@ -100,6 +100,8 @@ _SIGS = {
     "jacap_stats_update": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, ctypes.c_int32, _P, _P, _P]),
     "jacap_compact_inplace": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, _P, _P, _P, ctypes.c_int32,
                                              ctypes.c_int32, _P, ctypes.c_size_t, _P]),
+    "jacap_select_compact_inplace": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, ctypes.c_int32, _P, _P, _P, _P,
+                                                    _P, ctypes.c_int32, _P, ctypes.c_size_t, _P]),
     "jacap_device_status": (ctypes.c_int, [_P, _P]),
     "jacap_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "jacap_workspace_offsets": (ctypes.c_int, [ctypes.POINTER(jacap_layout), ctypes.c_int32,
@@ -154,6 +156,12 @@ def jacap_score_stats(layout, params, stats, counts, k, v, scores, ws, ws_bytes,
 
 def jacap_stats_update(layout, q_new, reset, stats, counts, stream) -> int:
     return lib().jacap_stats_update(ctypes.byref(layout), q_new, int(reset), stats, counts, stream)
+
+
+def jacap_select_compact_inplace(layout, scores, budget, idx, kept, k, v, pos, preserve_order, ws, ws_bytes,
+                                 stream) -> int:
+    return lib().jacap_select_compact_inplace(ctypes.byref(layout), scores, budget, idx, kept, k, v, pos,
+                                              preserve_order, ws, ws_bytes, stream)
 
 
 def jacap_compact_inplace(layout, k, v, pos, idx, budget, preserve_order, ws, ws_bytes, stream) -> int:

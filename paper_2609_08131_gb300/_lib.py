@@ -95,6 +95,7 @@ EXPORTS = [
     "jacap_score_stats",
     "jacap_stats_update",
     "jacap_compact_inplace",
+    "jacap_select_compact_inplace",
     "jacap_select",
     "jacap_select_compact",
     "jacap_compact",

@@ -16,7 +16,6 @@ from . import (
     JACAP_F32,
     JACAP_OK,
     jacap_compact,
-    jacap_compact_inplace,
     jacap_device_status,
     jacap_layout,
     jacap_params,
@@ -26,6 +25,7 @@ from . import (
     jacap_score_stats,
     jacap_select,
     jacap_select_compact,
+    jacap_select_compact_inplace,
     jacap_stats_update,
     jacap_status_string,
     jacap_workspace_offsets,
@@ -343,8 +343,8 @@ class DecodeEvictor:
         """Score request s's full slot with the running statistics, select the
         budget best tokens and compact them in place to rows 0 .. budget - 1.
         ``events``: JACAP_SCORE_KERNELS + 1 torch.cuda.Event recorded around
-        the scoring kernels; ``tail``: two more, recorded after the selection
-        and after the compaction."""
+        the scoring kernels; ``tail``: one more, recorded after the selection
+        with its in-place compaction (one launch)."""
         if self.lengths[s] != self.cap:
             raise RuntimeError("only a full slot is evicted")
         lay, st = self.slot, _stream(stream)
@@ -356,14 +356,11 @@ class DecodeEvictor:
         k, v, pos = _ptr(self.k[s]), _ptr(self.v[s]), _ptr(self.pos[s])
         _check(jacap_score_stats(lay, self.params, stats, counts, k, v, _ptr(self.scores), _ptr(self.ws),
                                  self.ws.numel(), st, handles), "jacap_score_stats")
-        _check(jacap_select(lay, _ptr(self.scores), self.budget, _ptr(self.idx), _ptr(self.kept), _ptr(self.ws),
-                            self.ws.numel(), st), "jacap_select")
+        _check(jacap_select_compact_inplace(lay, _ptr(self.scores), self.budget, _ptr(self.idx), _ptr(self.kept), k,
+                                            v, pos, self.preserve_order, _ptr(self.ws), self.ws.numel(), st),
+               "jacap_select_compact_inplace")
         if tail is not None:
             tail[0].record(stream)
-        _check(jacap_compact_inplace(lay, k, v, pos, _ptr(self.idx), self.budget, self.preserve_order, _ptr(self.ws),
-                                     self.ws.numel(), st), "jacap_compact_inplace")
-        if tail is not None:
-            tail[1].record(stream)
         self.lengths[s] = self.budget
         self.events += 1
 

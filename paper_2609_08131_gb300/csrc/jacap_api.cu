@@ -379,6 +379,38 @@ jacap_status jacap_compact_inplace(const jacap_layout* layout, void* k, void* v,
                                          (cudaStream_t)stream));
 }
 
+jacap_status jacap_select_compact_inplace(const jacap_layout* layout, const float* scores, int32_t budget,
+                                          int32_t* idx, int32_t* kept, void* k, void* v, int32_t* pos,
+                                          int32_t preserve_order, void* ws, size_t ws_bytes, void* stream) {
+  jacap_status st = check_layout(layout);
+  if (st != JACAP_OK) return st;
+  if (scores == nullptr || idx == nullptr || kept == nullptr || k == nullptr || v == nullptr || ws == nullptr ||
+      budget < 1 || (preserve_order != 0 && preserve_order != 1))
+    return JACAP_ERR_INVALID_ARG;
+  if (((uintptr_t)scores & 3u) != 0 || ((uintptr_t)idx & 3u) != 0 || ((uintptr_t)kept & 3u) != 0 ||
+      ((uintptr_t)pos & 3u) != 0 || !aligned16(k) || !aligned16(v))
+    return JACAP_ERR_INVALID_ARG;
+  Dims dm;
+  make_dims(layout, nullptr, dm);
+  const Carve c = carve(dm);
+  if (((uintptr_t)ws & 255u) != 0 || ws_bytes < c.total) return JACAP_ERR_WORKSPACE;
+  int sms = 0;
+  if ((st = check_device(&sms)) != JACAP_OK) return st;
+  const Ws w = make_ws(ws, c);
+  const int64_t units = (int64_t)dm.L * dm.Hkv * dm.S;
+  const int dt = layout->dtype == JACAP_BF16 ? 1 : 0;
+  const cudaStream_t s = (cudaStream_t)stream;
+  if (!preserve_order)  // hole filling inside the selection kernel
+    return map_cuda(launch_select(dm, w, layout->cu_seqlens, scores, budget, idx, kept, layout->max_seqlen,
+                                  persistent_grid(units, sms, 2), s, dt, nullptr, nullptr, nullptr, nullptr, k, v,
+                                  pos));
+  // ascending order moves every kept row: its own launch after the selection
+  if ((st = map_cuda(launch_select(dm, w, layout->cu_seqlens, scores, budget, idx, kept, layout->max_seqlen,
+                                   persistent_grid(units, sms, 2), s))) != JACAP_OK)
+    return st;
+  return map_cuda(launch_compact_inplace(dm, w, dt, layout->cu_seqlens, k, v, pos, idx, budget, 1, s));
+}
+
 jacap_status jacap_select(const jacap_layout* layout, const float* scores, int32_t budget, int32_t* idx,
                           int32_t* kept, void* ws, size_t ws_bytes, void* stream) {
   jacap_status st = check_layout(layout);

@@ -53,12 +53,14 @@ cudaError_t launch_gram(const CUtensorMap& vmap, const Dims& dm, const Ws& ws, i
 cudaError_t launch_factor(const Dims& dm, const Ws& ws, const float* out_factor, cudaStream_t st);
 cudaError_t launch_score(const CUtensorMap& vmap, const Dims& dm, const Ws& ws, int dtype, const void* v,
                          const int32_t* cu, float* scores, int grid, cudaStream_t st);
-// k == nullptr: selection only; otherwise the kept rows of k and v (dtype 1 =
-// bf16, 0 = float32) are also copied into k_out and v_out, as launch_compact does
+// Selection only when k and kio are null. With k: the kept rows of k and v
+// (dtype 1 = bf16, 0 = float32) are also copied into k_out and v_out, as
+// launch_compact does. With kio: the holes of kio, vio (and pos) are filled in
+// place, as launch_compact_inplace does without preserve_order.
 cudaError_t launch_select(const Dims& dm, const Ws& ws, const int32_t* cu, const float* scores, int budget,
                           int32_t* idx, int32_t* kept, int max_seqlen, int grid, cudaStream_t st, int dtype = 1,
                           const void* k = nullptr, const void* v = nullptr, void* k_out = nullptr,
-                          void* v_out = nullptr);
+                          void* v_out = nullptr, void* kio = nullptr, void* vio = nullptr, int32_t* pos = nullptr);
 cudaError_t launch_compact(const Dims& dm, int dtype, const int32_t* cu, const void* k, const void* v,
                            const int32_t* idx, int budget, void* k_out, void* v_out, cudaStream_t st);
 cudaError_t launch_stats_update(const Dims& dm, int dtype, const void* q, float* stats, int32_t* counts, int reset,

@@ -15,7 +15,8 @@
 //
 // After the TOP-B selection the cache of a request is compacted in place so
 // that the kept rows occupy rows 0 .. kept - 1 of the request's range, in one
-// of two ways (one CTA per unit in both):
+// of two ways (one CTA per unit in both; jacap_inplace.cuh holds the per-unit
+// code, which the selection kernel also runs right after selecting a unit):
 //  - ascending order (the order of jacap_compact): every kept row moves to
 //    its rank. The rows move in chunks; every chunk is read completely before
 //    any of it is written (a barrier in between). Because the kept positions
@@ -30,6 +31,7 @@
 //    below `kept`, the evicted row r between the (i-1)-th and i-th of them is
 //    hole number r - i and receives row idx[f + r - i].
 #include "jacap_dev.cuh"
+#include "jacap_inplace.cuh"
 #include "jacap_internal.h"
 
 namespace jacap {
@@ -98,28 +100,23 @@ __global__ void __launch_bounds__(D)
 }
 
 constexpr int CI_THREADS = 256;
-constexpr int CI_CHUNK_BYTES = 16384;  // per tensor and chunk
 
-// One CTA per unit u = (l Hkv + g) S + s, the order of jacap_select's idx.
+// One CTA per unit u = (l Hkv + g) S + s, the order of jacap_select's idx. The
+// kept positions come from the caller: a unit whose positions do not ascend
+// strictly within [0, n) is left untouched and flagged.
 template <typename T>
 __global__ void __launch_bounds__(CI_THREADS)
     compact_inplace_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu, T* k, T* v, int32_t* pos,
                            const int32_t* __restrict__ idx, int budget) {
   pdl_wait();
-  constexpr int RB = D * (int)sizeof(T) / 16;  // 16-byte pieces per row
-  constexpr int CH = CI_CHUNK_BYTES / (D * (int)sizeof(T));
-  constexpr int PER = CH * RB / CI_THREADS;    // pieces per thread and tensor
-  static_assert(CH * RB % CI_THREADS == 0 && CH <= CI_THREADS, "chunk shape");
   if (status_failed(ws)) return;
   const int u = blockIdx.x;
   const int s = u % dm.S, plane = u / dm.S;
-  const int l = plane / dm.Hkv, g = plane % dm.Hkv;
   const int tid = threadIdx.x;
   const int64_t t0 = cu[s];
   const int64_t n = (int64_t)cu[s + 1] - t0;
   const int kept = (int)(n < (int64_t)budget ? n : (int64_t)budget);
   const int32_t* ix = idx + (int64_t)u * budget;
-  // the kept positions must ascend strictly within [0, n): then idx[r] >= r
   int bad = 0;
   for (int r = tid; r < kept; r += CI_THREADS) {
     const int32_t x = ix[r];
@@ -129,55 +126,19 @@ __global__ void __launch_bounds__(CI_THREADS)
     if (tid == 0) flag(ws, ST_INVALID);
     return;
   }
-  const int64_t rowoff = (int64_t)l * dm.kv_sl + (int64_t)g * dm.kv_sh;
-  uint4* kb = (uint4*)(k + rowoff);
-  uint4* vb = (uint4*)(v + rowoff);
-  const int64_t st16 = dm.kv_st * (int64_t)sizeof(T) / 16;  // token stride in 16-byte pieces
-  int32_t* pb = pos != nullptr ? pos + (int64_t)plane * dm.Ntot : nullptr;
-  for (int c0 = 0; c0 < kept; c0 += CH) {
-    uint4 kr[PER], vr[PER];
-    int32_t pr = 0;
-#pragma unroll
-    for (int e = 0; e < PER; ++e) {
-      const int q = e * CI_THREADS + tid, r = c0 + q / RB, piece = q % RB;
-      if (r < kept) {
-        const int32_t x = ix[r];
-        if (x != r) {
-          kr[e] = kb[(t0 + x) * st16 + piece];
-          vr[e] = vb[(t0 + x) * st16 + piece];
-        }
-      }
-    }
-    if (pb != nullptr && tid < CH && c0 + tid < kept) pr = pb[t0 + ix[c0 + tid]];
-    __syncthreads();  // the whole chunk is read before any of it is written
-#pragma unroll
-    for (int e = 0; e < PER; ++e) {
-      const int q = e * CI_THREADS + tid, r = c0 + q / RB, piece = q % RB;
-      if (r < kept && ix[r] != r) {
-        kb[(t0 + r) * st16 + piece] = kr[e];
-        vb[(t0 + r) * st16 + piece] = vr[e];
-      }
-    }
-    if (pb != nullptr && tid < CH && c0 + tid < kept) pb[t0 + c0 + tid] = pr;
-  }
+  compact_ordered_unit<T, CI_THREADS>(dm, plane, t0, kept, k, v, pos, ix);
 }
 
-// Hole filling (see the header comment). c(p) = idx[p] - p counts the evicted
-// rows below kept position p and does not decrease, so hole j lies after the
-// i = #{p < f : c(p) <= j} kept positions below it, at row j + i. One warp per
-// hole (lanes over the 16-byte pieces of the row); the holes are independent.
 template <typename T>
 __global__ void __launch_bounds__(CI_THREADS)
     fill_holes_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu, T* k, T* v, int32_t* pos,
                       const int32_t* __restrict__ idx, int budget) {
   pdl_wait();
-  constexpr int RB = D * (int)sizeof(T) / 16;
   __shared__ int s_f;
   if (status_failed(ws)) return;
   const int u = blockIdx.x;
   const int s = u % dm.S, plane = u / dm.S;
-  const int l = plane / dm.Hkv, g = plane % dm.Hkv;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int tid = threadIdx.x;
   const int64_t t0 = cu[s];
   const int64_t n = (int64_t)cu[s + 1] - t0;
   const int kept = (int)(n < (int64_t)budget ? n : (int64_t)budget);
@@ -195,25 +156,7 @@ __global__ void __launch_bounds__(CI_THREADS)
     if (tid == 0) flag(ws, ST_INVALID);
     return;
   }
-  const int f = s_f, holes = kept - f;
-  const int64_t rowoff = (int64_t)l * dm.kv_sl + (int64_t)g * dm.kv_sh;
-  uint4* kb = (uint4*)(k + rowoff);
-  uint4* vb = (uint4*)(v + rowoff);
-  const int64_t st16 = dm.kv_st * (int64_t)sizeof(T) / 16;
-  int32_t* pb = pos != nullptr ? pos + (int64_t)plane * dm.Ntot : nullptr;
-  for (int j = warp; j < holes; j += CI_THREADS / 32) {
-    int lo = 0, hi = f;  // first p in [0, f) with c(p) > j (f if none)
-    while (lo < hi) {
-      const int mid = (lo + hi) >> 1;
-      if (ix[mid] - mid <= j) lo = mid + 1; else hi = mid;
-    }
-    const int64_t dst = t0 + j + lo, src = t0 + ix[f + j];
-    for (int piece = lane; piece < RB; piece += 32) {
-      kb[dst * st16 + piece] = kb[src * st16 + piece];
-      vb[dst * st16 + piece] = vb[src * st16 + piece];
-    }
-    if (pb != nullptr && lane == 0) pb[dst] = pb[src];
-  }
+  fill_holes_unit<T, CI_THREADS>(dm, plane, t0, kept, s_f, k, v, pos, ix);
 }
 
 template <typename T>

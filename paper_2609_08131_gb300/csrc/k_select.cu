@@ -20,11 +20,16 @@
 // dense [L][Hkv][S][B][d] output; rows of -1 (or of a position outside the
 // request) are zero-filled, so no index value can make it read out of bounds.
 //
-// With GATHER, select_kernel does that copy itself for each unit as soon as
-// the unit's positions are emitted (same rows, same zero fill), so the
-// retained rows stream while other CTAs are still selecting and the pass
-// needs no separate compaction launch.
+// select_kernel can also finish each unit itself as soon as its positions are
+// emitted, so the rows move while other CTAs are still selecting and no
+// separate compaction launch follows: MODE 1 copies the kept rows into k_out,
+// v_out (the work of compact_kernel, same zero fill); MODE 2 fills the holes
+// of the cache in place (jacap_inplace.cuh, as jacap_compact_inplace does).
+// MODE 0 only selects. (The in-place compaction in ascending order moves
+// every kept row; it stays a launch of its own, whose small CTAs keep more
+// bytes in flight per SM than one 1024-thread selection CTA per unit could.)
 #include "jacap_dev.cuh"
+#include "jacap_inplace.cuh"
 #include "jacap_internal.h"
 
 namespace jacap {
@@ -77,11 +82,13 @@ __device__ __forceinline__ void gather_unit(const Dims& dm, int plane, int64_t s
   }
 }
 
-template <int KPT, typename E, bool GATHER>
+template <int KPT, typename E, int MODE>
 __global__ void __launch_bounds__(SE_THREADS)
     select_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu, const float* __restrict__ scores, int B,
                   int32_t* __restrict__ idx, int32_t* __restrict__ kept, const E* __restrict__ k,
-                  const E* __restrict__ v, E* __restrict__ k_out, E* __restrict__ v_out) {
+                  const E* __restrict__ v, E* __restrict__ k_out, E* __restrict__ v_out, E* kio, E* vio,
+                  int32_t* pos) {
+  constexpr bool GATHER = MODE == 1;
   pdl_wait();
   constexpr int SE_KPT = KPT;
   constexpr int SE_SLAB = SE_THREADS * KPT;  // warp w holds positions 32 KPT w .. + 32 KPT - 1 of a slab
@@ -222,8 +229,18 @@ __global__ void __launch_bounds__(SE_THREADS)
       __syncthreads();  // the totals in hist are read before the next slab rewrites them
     }
     // (the barrier that ends the last slab also orders the emitted positions
-    // before the gather reads them)
+    // before they are read back here)
     if constexpr (GATHER) gather_unit<E>(dm, plane, start, end, true, k, v, out, B, u, k_out, v_out);
+    if constexpr (MODE == 2) {
+      // f = the kept positions below B (they ascend: a binary search)
+      int lo = 0, hi = B;
+      while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (out[mid] < B) lo = mid + 1; else hi = mid;
+      }
+      fill_holes_unit<E, SE_THREADS>(dm, plane, start, B, lo, kio, vio, pos, out);
+    }
+    if constexpr (MODE == 2) __syncthreads();  // the unit's rows have moved before `out` is reused
   }
 }
 
@@ -258,29 +275,47 @@ __global__ void __launch_bounds__(256)
 template <int KPT>
 static cudaError_t launch_select_kpt(const Dims& dm, const Ws& ws, const int32_t* cu, const float* scores, int budget,
                                      int32_t* idx, int32_t* kept, int dtype, const void* k, const void* v,
-                                     void* k_out, void* v_out, int grid, cudaStream_t st) {
+                                     void* k_out, void* v_out, void* kio, void* vio, int32_t* pos, int grid,
+                                     cudaStream_t st) {
   using bf = __nv_bfloat16;
+  if (kio != nullptr) {  // hole filling in place
+    if (dtype == 1)
+      return launch_pdl(dm.pdl != 0, select_kernel<KPT, bf, 2>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget,
+                        idx, kept, (const bf*)nullptr, (const bf*)nullptr, (bf*)nullptr, (bf*)nullptr, (bf*)kio,
+                        (bf*)vio, pos);
+    return launch_pdl(dm.pdl != 0, select_kernel<KPT, float, 2>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget,
+                      idx, kept, (const float*)nullptr, (const float*)nullptr, (float*)nullptr, (float*)nullptr,
+                      (float*)kio, (float*)vio, pos);
+  }
   if (k == nullptr)
-    return launch_pdl(dm.pdl != 0, select_kernel<KPT, bf, false>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget,
-                      idx, kept, (const bf*)nullptr, (const bf*)nullptr, (bf*)nullptr, (bf*)nullptr);
+    return launch_pdl(dm.pdl != 0, select_kernel<KPT, bf, 0>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget,
+                      idx, kept, (const bf*)nullptr, (const bf*)nullptr, (bf*)nullptr, (bf*)nullptr, (bf*)nullptr,
+                      (bf*)nullptr, (int32_t*)nullptr);
   if (dtype == 1)
-    return launch_pdl(dm.pdl != 0, select_kernel<KPT, bf, true>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget,
-                      idx, kept, (const bf*)k, (const bf*)v, (bf*)k_out, (bf*)v_out);
-  return launch_pdl(dm.pdl != 0, select_kernel<KPT, float, true>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget,
-                    idx, kept, (const float*)k, (const float*)v, (float*)k_out, (float*)v_out);
+    return launch_pdl(dm.pdl != 0, select_kernel<KPT, bf, 1>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget,
+                      idx, kept, (const bf*)k, (const bf*)v, (bf*)k_out, (bf*)v_out, (bf*)nullptr, (bf*)nullptr,
+                      (int32_t*)nullptr);
+  return launch_pdl(dm.pdl != 0, select_kernel<KPT, float, 1>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget,
+                    idx, kept, (const float*)k, (const float*)v, (float*)k_out, (float*)v_out, (float*)nullptr,
+                    (float*)nullptr, (int32_t*)nullptr);
 }
 
 cudaError_t launch_select(const Dims& dm, const Ws& ws, const int32_t* cu, const float* scores, int budget,
                           int32_t* idx, int32_t* kept, int max_seqlen, int grid, cudaStream_t st, int dtype,
-                          const void* k, const void* v, void* k_out, void* v_out) {
+                          const void* k, const void* v, void* k_out, void* v_out, void* kio, void* vio,
+                          int32_t* pos) {
   if (max_seqlen <= SE_THREADS * 4)
-    JACAP_TRY(launch_select_kpt<4>(dm, ws, cu, scores, budget, idx, kept, dtype, k, v, k_out, v_out, grid, st));
+    JACAP_TRY(launch_select_kpt<4>(dm, ws, cu, scores, budget, idx, kept, dtype, k, v, k_out, v_out, kio, vio, pos,
+                                   grid, st));
   else if (max_seqlen <= SE_THREADS * 8)
-    JACAP_TRY(launch_select_kpt<8>(dm, ws, cu, scores, budget, idx, kept, dtype, k, v, k_out, v_out, grid, st));
+    JACAP_TRY(launch_select_kpt<8>(dm, ws, cu, scores, budget, idx, kept, dtype, k, v, k_out, v_out, kio, vio, pos,
+                                   grid, st));
   else if (max_seqlen <= SE_THREADS * 16)
-    JACAP_TRY(launch_select_kpt<16>(dm, ws, cu, scores, budget, idx, kept, dtype, k, v, k_out, v_out, grid, st));
+    JACAP_TRY(launch_select_kpt<16>(dm, ws, cu, scores, budget, idx, kept, dtype, k, v, k_out, v_out, kio, vio, pos,
+                                    grid, st));
   else
-    JACAP_TRY(launch_select_kpt<32>(dm, ws, cu, scores, budget, idx, kept, dtype, k, v, k_out, v_out, grid, st));
+    JACAP_TRY(launch_select_kpt<32>(dm, ws, cu, scores, budget, idx, kept, dtype, k, v, k_out, v_out, kio, vio, pos,
+                                    grid, st));
   return cudaGetLastError();
 }
 
