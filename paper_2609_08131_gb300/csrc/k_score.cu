@@ -240,7 +240,13 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
 }
 
 // ------------------------------------------------------------ SIMT fp32 ---
-constexpr int SF_THREADS = 128;
+// Two threads per token (lanes 2 t and 2 t + 1): thread `half` forms the
+// output rows r of the quads r / 4 = half, half + 2, ... (the two halves of
+// the triangle get about the same work), four rows at once so their
+// multiply-add chains interleave, and the pair adds its squared norms.
+// L^{-1} is stored with zeros above the diagonal, so a quad may run its
+// columns up to its last row.
+constexpr int SF_THREADS = 2 * TILE;
 constexpr int SF_LD = D + 1;
 constexpr size_t score_f32_smem_bytes() { return (size_t)(D * D + TILE * SF_LD) * sizeof(float); }
 
@@ -256,6 +262,7 @@ __global__ void __launch_bounds__(SF_THREADS)
   if (tid == 0) s_skip = status_failed(ws) ? 1 : 0;
   __syncthreads();
   if (s_skip) return;
+  const int tk = tid >> 1, half = tid & 1;
   bool bad = false;
   int64_t loaded = -1;
   Item item;
@@ -279,18 +286,25 @@ __global__ void __launch_bounds__(SF_THREADS)
         vt[r * SF_LD + c4 + 2] = x.z; vt[r * SF_LD + c4 + 3] = x.w;
       }
       __syncthreads();
-      const int64_t tok = t + tid;
-      if (tok < item.t1) {
-        const float* vr = vt + tid * SF_LD;
-        float ssq = 0.f;
-        for (int r = 0; r < D; ++r) {
-          float yv = 0.f;
-          const float* mr = Mi + r * D;
-          // L^{-1} is lower triangular; a full matrix with output directions
-          const int cend = dm.dense_minv ? D - 1 : r;
-          for (int c = 0; c <= cend; ++c) yv = fmaf(mr[c], vr[c], yv);
-          ssq = fmaf(yv, yv, ssq);
+      const float* vr = vt + tk * SF_LD;
+      float ssq = 0.f;
+      for (int r0 = 4 * half; r0 < D; r0 += 8) {
+        const float* m0 = Mi + r0 * D;
+        // a full matrix with output directions
+        const int cend = dm.dense_minv ? D : r0 + 4;
+        float y0 = 0.f, y1 = 0.f, y2 = 0.f, y3 = 0.f;
+        for (int c = 0; c < cend; ++c) {
+          const float x = vr[c];
+          y0 = fmaf(m0[c], x, y0);
+          y1 = fmaf(m0[D + c], x, y1);
+          y2 = fmaf(m0[2 * D + c], x, y2);
+          y3 = fmaf(m0[3 * D + c], x, y3);
         }
+        ssq = fmaf(y0, y0, fmaf(y1, y1, fmaf(y2, y2, fmaf(y3, y3, ssq))));
+      }
+      ssq += __shfl_xor_sync(0xffffffffu, ssq, 1);
+      const int64_t tok = t + tk;
+      if (half == 0 && tok < item.t1) {
         const int64_t o = (int64_t)item.plane * dm.Ntot + tok;
         const float sc = ws.w[o] * ssq;
         scores[o] = sc;
