@@ -113,8 +113,9 @@ typedef struct {
  *                 kappa_h,i = (1/w) sum_j ((q_h,j - mu_h) . k_i)^2 (1/(w-1) with
  *                 cov_unbiased), the O(N d^2) variant of App. B.2. bf16 caches
  *                 with window in {8, 16, 32, 64} and G * window <= 128 use the
- *                 tensor cores; other shapes and float32 caches a much slower
- *                 CUDA-core kernel. It adds a second read of K.
+ *                 tensor cores inside the K pass (K is still read once); other
+ *                 shapes and float32 caches a much slower CUDA-core kernel
+ *                 after the K pass, which reads K a second time.
  * Callers that zero-initialise the two trailing fields get the method.
  */
 typedef struct {
@@ -158,7 +159,8 @@ jacap_status jacap_score(const jacap_layout* layout, const jacap_params* params,
  * or JACAP_SCORE_KERNELS + 1. Kernel order: plan, query statistics, K pass,
  * weights, Gram, factor, scores. With bf16 caches the Gram kernel computes the
  * Eq. 8 weights itself and the weights slot is empty (its two events are
- * recorded back to back).
+ * recorded back to back); with full_covariance the K-pass slot also holds the
+ * CUDA-core kappa kernel when that one runs.
  */
 #define JACAP_SCORE_KERNELS 7
 jacap_status jacap_score_timed(const jacap_layout* layout, const jacap_params* params,
