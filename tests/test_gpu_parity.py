@@ -311,3 +311,28 @@ def test_output_directions_every_unit(dtype):
                 # and the explicit d_o-dimensional output map gives the same scores (push-through)
                 ora_w = oracle_unit(q, K, V, wl.budget, JacapParams(), out_proj=W[layer, g])
                 assert_scores_close(ev.scores[layer, g, a:b].double().cpu().numpy(), ora_w["scores"])
+
+
+def test_pass_replays_from_a_cuda_graph():
+    # the whole pass (scores, selection, compaction) captured once into a CUDA
+    # graph and replayed gives the eager pass's results bit for bit
+    wl, params = SMALL["bf16_gqa4_ragged_tails"]
+    t = generate(wl, DEV)
+    ev = evict(make_cache(t, wl), wl.budget, params)  # eager, also warms every kernel up
+    ref = [x.clone() for x in (ev.scores, ev.idx, ev.kept, ev.k_out, ev.v_out)]
+    for x in (ev.scores, ev.k_out, ev.v_out):
+        x.zero_()
+    ev.idx.fill_(-7)
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(side):
+        with torch.cuda.graph(g, stream=side, capture_error_mode="thread_local"):
+            ev.run(side)
+    torch.cuda.current_stream().wait_stream(side)
+    for _ in range(2):
+        g.replay()
+        torch.cuda.synchronize()
+        ev.check()
+        got = (ev.scores, ev.idx, ev.kept, ev.k_out, ev.v_out)
+        assert all(torch.equal(a, b) for a, b in zip(ref, got))
