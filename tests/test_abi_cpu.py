@@ -110,6 +110,13 @@ def test_bad_params_and_buffers_are_rejected_on_the_host():
     assert J.jacap_score(lay, J.jacap_params(), p, p, p, p, ctypes.c_void_p(0x1010), big, None) == J.JACAP_ERR_WORKSPACE
     assert J.jacap_select(lay, p, 0, p, p, p, big, None) == J.JACAP_ERR_INVALID_ARG
     assert J.jacap_compact(lay, p, p, p, 8, mis, p, None) == J.JACAP_ERR_INVALID_ARG
+    # the fused calls check what the two calls they replace check
+    assert J.jacap_select_compact(lay, p, 0, p, p, p, p, p, p, p, big, None) == J.JACAP_ERR_INVALID_ARG
+    assert J.jacap_select_compact(lay, p, 8, p, p, p, p, mis, p, p, big, None) == J.JACAP_ERR_INVALID_ARG
+    assert J.jacap_select_compact(lay, p, 8, p, p, p, p, p, p, p, big - 1, None) == J.JACAP_ERR_WORKSPACE
+    assert J.jacap_select_compact_inplace(lay, p, 8, p, p, p, p, p, 2, p, big, None) == J.JACAP_ERR_INVALID_ARG
+    assert J.jacap_select_compact_inplace(lay, p, 8, p, p, mis, p, p, 0, p, big, None) == J.JACAP_ERR_INVALID_ARG
+    assert J.jacap_select_compact_inplace(lay, p, 8, p, p, p, p, None, 0, p, big - 1, None) == J.JACAP_ERR_WORKSPACE
     assert J.jacap_device_status(None, None) == J.JACAP_ERR_INVALID_ARG
 
 
