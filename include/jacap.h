@@ -338,6 +338,18 @@ jacap_status jacap_select_compact_inplace(const jacap_layout* layout, const floa
  * first device-side error recorded since the last jacap_score on `ws`. */
 jacap_status jacap_device_status(const void* ws, void* stream);
 
+/*
+ * Self-test of the device-side failure detection (no counterpart in the
+ * paper): enqueues one thread that clears the status word of `ws` and waits,
+ * with the bounded wait every pipeline of the pass uses, on an mbarrier that
+ * nothing ever arrives on. After limit_ns (1 us .. 10 s) the wait gives up,
+ * sets JACAP_ERR_TIMEOUT in the status word and the kernel returns; nothing
+ * faults and the context stays usable, so jacap_device_status then reports
+ * JACAP_ERR_TIMEOUT and the next jacap_score starts clean. ws: >= 64 bytes,
+ * 256-byte aligned (a workspace).
+ */
+jacap_status jacap_selftest_wait(void* ws, size_t ws_bytes, int64_t limit_ns, void* stream);
+
 /* Static English text for a status code (never NULL). */
 const char* jacap_status_string(jacap_status status);
 

@@ -100,6 +100,7 @@ _SIGS = {
     "jacap_stats_update": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, ctypes.c_int32, _P, _P, _P]),
     "jacap_compact_inplace": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, _P, _P, _P, ctypes.c_int32,
                                              ctypes.c_int32, _P, ctypes.c_size_t, _P]),
+    "jacap_selftest_wait": (ctypes.c_int, [_P, ctypes.c_size_t, ctypes.c_int64, _P]),
     "jacap_select_compact_inplace": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, ctypes.c_int32, _P, _P, _P, _P,
                                                     _P, ctypes.c_int32, _P, ctypes.c_size_t, _P]),
     "jacap_device_status": (ctypes.c_int, [_P, _P]),
@@ -156,6 +157,10 @@ def jacap_score_stats(layout, params, stats, counts, k, v, scores, ws, ws_bytes,
 
 def jacap_stats_update(layout, q_new, reset, stats, counts, stream) -> int:
     return lib().jacap_stats_update(ctypes.byref(layout), q_new, int(reset), stats, counts, stream)
+
+
+def jacap_selftest_wait(ws, ws_bytes, limit_ns, stream) -> int:
+    return lib().jacap_selftest_wait(ws, ws_bytes, limit_ns, stream)
 
 
 def jacap_select_compact_inplace(layout, scores, budget, idx, kept, k, v, pos, preserve_order, ws, ws_bytes,

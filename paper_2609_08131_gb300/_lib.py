@@ -100,6 +100,7 @@ EXPORTS = [
     "jacap_select_compact",
     "jacap_compact",
     "jacap_device_status",
+    "jacap_selftest_wait",
     "jacap_status_string",
     "jacap_workspace_offsets",
 ]

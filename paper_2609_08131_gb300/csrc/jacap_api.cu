@@ -471,6 +471,18 @@ jacap_status jacap_compact(const jacap_layout* layout, const void* k, const void
                                  k_out, v_out, (cudaStream_t)stream));
 }
 
+jacap_status jacap_selftest_wait(void* ws, size_t ws_bytes, int64_t limit_ns, void* stream) {
+  if (ws == nullptr || ((uintptr_t)ws & 255u) != 0 || ws_bytes < 64) return JACAP_ERR_INVALID_ARG;
+  if (limit_ns < 1000 || limit_ns > 10000000000LL) return JACAP_ERR_INVALID_ARG;
+  int sms = 0;
+  jacap_status st = check_device(&sms);
+  if (st != JACAP_OK) return st;
+  Ws w;
+  memset(&w, 0, sizeof(w));
+  w.status = (uint32_t*)ws;
+  return map_cuda(launch_selftest_wait(w, (unsigned long long)limit_ns, (cudaStream_t)stream));
+}
+
 jacap_status jacap_device_status(const void* ws, void* stream) {
   if (ws == nullptr) return JACAP_ERR_INVALID_ARG;
   if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess) return JACAP_ERR_CUDA;

@@ -222,17 +222,18 @@ __device__ __forceinline__ bool mbar_try_wait_suspend(uint32_t bar, uint32_t par
 constexpr uint32_t WAIT_SUSPEND_NS = 1000;
 
 // Bounded wait for the phase with the given parity to complete. Returns false
-// (after flagging ST_TIMEOUT) if it did not complete within WAIT_LIMIT_NS, or
-// if *abort became nonzero while waiting.
+// (after flagging ST_TIMEOUT) if it did not complete within limit_ns
+// (WAIT_LIMIT_NS for every wait of the pass), or if *abort became nonzero
+// while waiting.
 static __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, const Ws& ws,
-                                            volatile int* abort) {
+                                            volatile int* abort, unsigned long long limit_ns = WAIT_LIMIT_NS) {
   if (abort != nullptr && *abort) return false;
   const unsigned long long t0 = globaltimer();
   for (uint32_t it = 0;; ++it) {
     if (mbar_try_wait_suspend(bar, parity, WAIT_SUSPEND_NS)) return true;
     if ((it & 7u) == 7u) {
       if (abort != nullptr && *abort) return false;
-      if (globaltimer() - t0 > WAIT_LIMIT_NS) {
+      if (globaltimer() - t0 > limit_ns) {
         flag(ws, ST_TIMEOUT);
         if (abort != nullptr) *abort = 1;
         return false;

@@ -45,6 +45,8 @@ cudaError_t launch_kpass_bf16(const CUtensorMap& kmap, const Dims& dm, const Ws&
 // the K pass runs and launch_kfull (CUDA cores) overwrites its diagonal kappa.
 bool kfull_uses_tensor_cores(const Dims& dm, int dtype);
 cudaError_t launch_kpass_full(const CUtensorMap& kmap, const Dims& dm, const Ws& ws, int grid, cudaStream_t st);
+// one thread waits (bounded by limit_ns) on an mbarrier nothing arrives on
+cudaError_t launch_selftest_wait(const Ws& ws, unsigned long long limit_ns, cudaStream_t st);
 cudaError_t launch_kfull(const CUtensorMap& kmap, const Dims& dm, const Ws& ws, int dtype, const void* k, int grid,
                          cudaStream_t st);
 cudaError_t launch_weights(const Dims& dm, const Ws& ws, const int32_t* cu, int grid, cudaStream_t st);

@@ -66,6 +66,26 @@ __device__ __forceinline__ float ld_elem<__nv_bfloat16>(const __nv_bfloat16* p) 
   return __bfloat162float(*p);
 }
 
+// Self-test of the bounded waits: one thread waits on an mbarrier that nothing
+// arrives on, with the wait code every pipeline of the pass uses but a short
+// limit; on expiry it sets ST_TIMEOUT in the status word (cleared first) and
+// returns. Nothing faults and the context stays usable.
+__global__ void __launch_bounds__(32) selftest_wait_kernel(Ws ws, unsigned long long limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 16; ++i) ws.status[i] = 0u;
+    mbar_init(smem_u32(&bar), 1);
+    fence_mbar_init();
+  }
+  __syncwarp();
+  if (threadIdx.x == 0) mbar_wait_slow(smem_u32(&bar), 0, ws, nullptr, limit_ns);  // phase 0 never completes
+}
+
+cudaError_t launch_selftest_wait(const Ws& ws, unsigned long long limit_ns, cudaStream_t st) {
+  selftest_wait_kernel<<<1, 32, 0, st>>>(ws, limit_ns);
+  return cudaGetLastError();
+}
+
 // One block per (request, layer, query head); thread c owns channel c.
 template <typename T>
 __global__ void __launch_bounds__(D) window_stats_kernel(Dims dm, Ws ws, const T* __restrict__ q) {

@@ -336,3 +336,25 @@ def test_pass_replays_from_a_cuda_graph():
         ev.check()
         got = (ev.scores, ev.idx, ev.kept, ev.k_out, ev.v_out)
         assert all(torch.equal(a, b) for a, b in zip(ref, got))
+
+
+def test_a_wait_that_nothing_ends_expires_and_the_context_stays_usable():
+    # failure detection without a fault: a bounded wait on an mbarrier that
+    # nothing arrives on gives up after its limit, the status word says
+    # timeout, and the next pass on the same workspace runs clean
+    import time
+
+    from paper_2609_08131_gb300 import JACAP_ERR_TIMEOUT, jacap_selftest_wait
+    from paper_2609_08131_gb300.api import _ptr, _stream
+
+    wl = Workload("t", 1, 4, 2, (700, 129), 8, 64, seed=29)
+    t = generate(wl, DEV)
+    ev = Evictor(make_cache(t, wl), wl.budget)
+    t0 = time.time()
+    assert jacap_selftest_wait(_ptr(ev.ws), ev.ws.numel(), 20_000_000, _stream()) == 0
+    assert ev.device_status() == JACAP_ERR_TIMEOUT
+    assert time.time() - t0 < 5.0
+    ev.run()
+    ev.check()
+    for g in range(wl.num_kv_heads):
+        check_unit(ev, t, wl, jacap_params(), 1, 0, g)
