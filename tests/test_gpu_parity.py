@@ -358,3 +358,30 @@ def test_a_wait_that_nothing_ends_expires_and_the_context_stays_usable():
     ev.check()
     for g in range(wl.num_kv_heads):
         check_unit(ev, t, wl, jacap_params(), 1, 0, g)
+
+
+def test_host_cache_pass_with_output_directions_matches_the_device_pass():
+    # HostEvictor hands each layer group its slice of the output factors: the
+    # kept positions and rows equal those of the device-resident pass (both run
+    # the same kernels on the same bytes; only the chunking of a group's
+    # layout may differ, so positions may differ only at near ties)
+    from paper_2609_08131_gb300.api import HostEvictor
+
+    wl = Workload("t", 3, 8, 2, (900, 300), 16, 64, seed=44)
+    t = generate(wl, DEV)
+    _, F = _output_factors(wl, 160, 9, DEV)
+    dev = Evictor(make_cache(t, wl), wl.budget, jacap_params(), out_factor=F)
+    dev.run()
+    dev.check()
+    he = HostEvictor(t.q_win.cpu().pin_memory(), t.k.cpu().pin_memory(), t.v.cpu().pin_memory(), t.cu_seqlens,
+                     list(wl.seqlens), wl.num_q_heads, wl.budget, jacap_params(), group_layers=2, device=DEV,
+                     out_factor=F)
+    he.run()
+    torch.cuda.synchronize()
+    he.check()
+    a, b = he.idx.cpu().reshape(-1, wl.budget).numpy(), dev.idx.cpu().reshape(-1, wl.budget).numpy()
+    differ = sum(len(np.setdiff1d(x, y)) for x, y in zip(a, b))
+    assert differ <= 2, differ
+    if differ == 0:
+        assert_rows_bitwise(dev.k_out, he.k_out)
+        assert_rows_bitwise(dev.v_out, he.v_out)
