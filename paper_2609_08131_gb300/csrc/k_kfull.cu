@@ -309,9 +309,10 @@ __global__ void __launch_bounds__(KX_THREADS, 1)
           for (int h = 0; h < G; ++h) {
             const float lg = dv[h] + dv[G + h] + dv[2 * G + h];
             bad |= !isfinite(lg);
-            // branch-free online update: one of the two exponentials is exp(0)
+            // branch-free online update: one of the two exponentials is exp(0);
+            // both arguments are <= 0 (fast exponential, as in the K pass)
             const float mn = fmaxf(run_m[h], lg);
-            run_s[h] = run_s[h] * expf(run_m[h] - mn) + expf(lg - mn);
+            run_s[h] = run_s[h] * __expf(run_m[h] - mn) + __expf(lg - mn);
             run_m[h] = mn;
             row[h] = lg;
             row[G + h] = kap[h] * invw;

@@ -388,9 +388,11 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
           for (int h = 0; h < G; ++h) {
             lg[h] = dv[h] + dv[G + h] + dv[2 * G + h];
             bad |= !isfinite(lg[h]);
-            // branch-free online update: one of the two exponentials is exp(0)
+            // branch-free online update: one of the two exponentials is exp(0);
+            // both arguments are <= 0, where the fast exponential's relative
+            // error (a few ulp) is far below what the statistics need
             const float mn = fmaxf(run_m[h], lg[h]);
-            run_s[h] = run_s[h] * expf(run_m[h] - mn) + expf(lg[h] - mn);
+            run_s[h] = run_s[h] * __expf(run_m[h] - mn) + __expf(lg[h] - mn);
             run_m[h] = mn;
           }
           store_part<G>(lkp + tok * (2 * G), lg);
