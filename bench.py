@@ -506,9 +506,21 @@ def run_e2e(args, ev, t, stream, world, dist):
     from paper_2609_08131_gb300.api import HostEvictor
 
     c = ev.cache
-    he = HostEvictor(c.q_win.cpu().pin_memory(), c.k.cpu().pin_memory(), c.v.cpu().pin_memory(), c.cu_seqlens,
-                     c.seqlens, c.num_q_heads, ev.budget, ev.params, group_layers=args.e2e_group,
-                     device=c.k.device, out_factor=ev.out_factor)
+    # every rank pins a host copy of its cache; if any rank cannot, all skip
+    # the end-to-end number together (no rank may wait alone at a barrier)
+    he, why = None, ""
+    try:
+        he = HostEvictor(c.q_win.cpu().pin_memory(), c.k.cpu().pin_memory(), c.v.cpu().pin_memory(), c.cu_seqlens,
+                         c.seqlens, c.num_q_heads, ev.budget, ev.params, group_layers=args.e2e_group,
+                         device=c.k.device, out_factor=ev.out_factor)
+    except RuntimeError as e:
+        why = str(e).splitlines()[0][:200]
+    ok = torch.tensor([1 if he is not None else 0], device=c.k.device)
+    if dist is not None:
+        dist.all_reduce(ok, op=dist.ReduceOp.MIN)
+    if int(ok.item()) == 0:
+        return {"unavailable": "pinned host copy of the cache could not be made" + (f": {why}" if why else
+                                                                                      " on every rank")}
     for _ in range(2):
         he.run(stream)
     torch.cuda.synchronize()
