@@ -1,12 +1,15 @@
 // k_select.cu - TOP-B selection (Algorithm 1 step 5) and compaction of the
 // retained cache Z_C (Sec. 3.1).
 //
-// select_kernel: one 1024-thread CTA per unit (grid-stride). Scores are
+// select_kernel: one CTA per unit (grid-stride), of NT = 1024 threads, or of
+// 256 when the longest request has at most 4096 tokens and there are more
+// units than SMs (then four or more CTAs fit an SM and a pass over many short
+// units, as in decoding-stage eviction, runs in one wave). Scores are
 // non-negative float32, so their bit patterns order like unsigned integers.
 // Three radix passes (digits of 11, 11 and 10 bits, most significant first,
 // shared-memory histograms; a pass counts only keys that match the digits
 // found so far) find the B-th largest key T and how many keys equal to T are
-// still needed. The keys are read in slabs of 1024 KPT into registers (KPT
+// still needed. The keys are read in slabs of NT KPT into registers (KPT
 // per lane, all loads in flight together; KPT = 4, 8, 16 or 32, the smallest
 // that holds the longest request in one slab); a request that fits one slab is
 // read once and every pass works on registers. Emission walks the slabs in
@@ -27,25 +30,24 @@
 // of the cache in place (jacap_inplace.cuh, as jacap_compact_inplace does).
 // MODE 0 only selects. (The in-place compaction in ascending order moves
 // every kept row; it stays a launch of its own, whose small CTAs keep more
-// bytes in flight per SM than one 1024-thread selection CTA per unit could.)
+// bytes in flight per SM than one selection CTA per unit could.)
 #include "jacap_dev.cuh"
 #include "jacap_inplace.cuh"
 #include "jacap_internal.h"
 
 namespace jacap {
 
-constexpr int SE_THREADS = 1024;
 
 constexpr int SE_BINS = 2048;
 
 // Keys of slab `sl` into registers: lane's register j holds position
-// sl * 1024 KPT + 32 KPT w + 32 j + lane (coalesced; all loads in flight at
+// sl * NT KPT + 32 KPT w + 32 j + lane (coalesced; all loads in flight at
 // once). KPT keys per lane (4 .. 32) is chosen from the longest request, so a
 // short cache does not carry empty register slots through every pass.
-template <int KPT>
+template <int KPT, int NT>
 __device__ __forceinline__ void load_slab(const uint32_t* key, int n, int sl, int warp, int lane,
                                           uint32_t (&kr)[KPT]) {
-  const int base = sl * SE_THREADS * KPT + warp * (32 * KPT) + lane;
+  const int base = sl * NT * KPT + warp * (32 * KPT) + lane;
 #pragma unroll
   for (int j = 0; j < KPT; ++j) {
     const int i = base + 32 * j;
@@ -57,7 +59,7 @@ __device__ __forceinline__ void load_slab(const uint32_t* key, int n, int sl, in
 // emitted) from K and V into k_out, v_out; -1 or a position outside the
 // request gives a zero row. All threads of the CTA; out was written by them
 // before the barrier that precedes this call.
-template <typename T>
+template <typename T, int NT>
 __device__ __forceinline__ void gather_unit(const Dims& dm, int plane, int64_t start, int64_t end, bool valid,
                                             const T* __restrict__ k, const T* __restrict__ v,
                                             const int32_t* out, int B, int64_t u, T* __restrict__ k_out,
@@ -68,7 +70,7 @@ __device__ __forceinline__ void gather_unit(const Dims& dm, int plane, int64_t s
   uint4* ko = (uint4*)(k_out + u * B * D);
   uint4* vo = (uint4*)(v_out + u * B * D);
 #pragma unroll 2
-  for (int e = threadIdx.x; e < B * CH; e += SE_THREADS) {
+  for (int e = threadIdx.x; e < B * CH; e += NT) {
     const int r = e / CH, c = e % CH;
     const int32_t src = out[r];
     uint4 kk = make_uint4(0, 0, 0, 0), vv = make_uint4(0, 0, 0, 0);
@@ -82,8 +84,8 @@ __device__ __forceinline__ void gather_unit(const Dims& dm, int plane, int64_t s
   }
 }
 
-template <int KPT, typename E, int MODE>
-__global__ void __launch_bounds__(SE_THREADS)
+template <int KPT, typename E, int MODE, int NT>
+__global__ void __launch_bounds__(NT)
     select_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu, const float* __restrict__ scores, int B,
                   int32_t* __restrict__ idx, int32_t* __restrict__ kept, const E* __restrict__ k,
                   const E* __restrict__ v, E* __restrict__ k_out, E* __restrict__ v_out, E* kio, E* vio,
@@ -91,7 +93,8 @@ __global__ void __launch_bounds__(SE_THREADS)
   constexpr bool GATHER = MODE == 1;
   pdl_wait();
   constexpr int SE_KPT = KPT;
-  constexpr int SE_SLAB = SE_THREADS * KPT;  // warp w holds positions 32 KPT w .. + 32 KPT - 1 of a slab
+  constexpr int SE_SLAB = NT * KPT;  // warp w holds positions 32 KPT w .. + 32 KPT - 1 of a slab
+  constexpr int NW = NT / 32;
   __shared__ uint32_t hist[SE_BINS];
   __shared__ uint32_t s_digit, s_need;
   __shared__ int s_skip;
@@ -108,14 +111,14 @@ __global__ void __launch_bounds__(SE_THREADS)
     int32_t* out = idx + (int64_t)u * B;
     const bool valid = !(start < 0 || end < start || end > dm.Ntot);
     if (!valid) {  // malformed cu_seqlens: no reads
-      for (int r = tid; r < B; r += SE_THREADS) out[r] = -1;
+      for (int r = tid; r < B; r += NT) out[r] = -1;
       if (tid == 0) {
         flag(ws, ST_INVALID);
         if (plane == 0) kept[s] = 0;
       }
       if constexpr (GATHER) {
         __syncthreads();
-        gather_unit<E>(dm, plane, start, end, false, k, v, out, B, u, k_out, v_out);
+        gather_unit<E, NT>(dm, plane, start, end, false, k, v, out, B, u, k_out, v_out);
       }
       continue;
     }
@@ -123,27 +126,27 @@ __global__ void __launch_bounds__(SE_THREADS)
     const uint32_t* key = (const uint32_t*)(scores + (int64_t)plane * dm.Ntot + start);
     if (plane == 0 && tid == 0) kept[s] = min(n, B);
     if (n <= B) {
-      for (int r = tid; r < B; r += SE_THREADS) out[r] = r < n ? r : -1;
+      for (int r = tid; r < B; r += NT) out[r] = r < n ? r : -1;
       if constexpr (GATHER) {
         __syncthreads();
-        gather_unit<E>(dm, plane, start, end, true, k, v, out, B, u, k_out, v_out);
+        gather_unit<E, NT>(dm, plane, start, end, true, k, v, out, B, u, k_out, v_out);
       }
       continue;
     }
     const int nslab = (n + SE_SLAB - 1) / SE_SLAB;
     uint32_t kr[SE_KPT];
-    if (nslab == 1) load_slab<KPT>(key, n, 0, warp, lane, kr);  // register-resident for all passes
+    if (nslab == 1) load_slab<KPT, NT>(key, n, 0, warp, lane, kr);  // register-resident for all passes
     // ---- radix select of the B-th largest key: digits [31:21], [20:10], [9:0] ----
     uint32_t prefix = 0, mask = 0, need = (uint32_t)B;
 #pragma unroll 1
     for (int pass = 0; pass < 3; ++pass) {
       const int shift = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
       const uint32_t dmask = pass == 2 ? 1023u : 2047u;
-      for (int b = tid; b < SE_BINS; b += SE_THREADS) hist[b] = 0;
+      for (int b = tid; b < SE_BINS; b += NT) hist[b] = 0;
       __syncthreads();
 #pragma unroll 1
       for (int sl = 0; sl < nslab; ++sl) {
-        if (nslab > 1) load_slab<KPT>(key, n, sl, warp, lane, kr);
+        if (nslab > 1) load_slab<KPT, NT>(key, n, sl, warp, lane, kr);
         const int base = sl * SE_SLAB + warp * (32 * SE_KPT) + lane;
 #pragma unroll
         for (int j = 0; j < SE_KPT; ++j)
@@ -184,7 +187,7 @@ __global__ void __launch_bounds__(SE_THREADS)
     uint32_t gt_run = 0, eq_run = 0;  // kept-greater and equal keys before this slab
 #pragma unroll 1
     for (int sl = 0; sl < nslab; ++sl) {
-      if (nslab > 1) load_slab<KPT>(key, n, sl, warp, lane, kr);
+      if (nslab > 1) load_slab<KPT, NT>(key, n, sl, warp, lane, kr);
       const int base = sl * SE_SLAB + warp * (32 * SE_KPT) + lane;
       uint32_t gt = 0, eq = 0;
 #pragma unroll
@@ -195,12 +198,12 @@ __global__ void __launch_bounds__(SE_THREADS)
       }
       if (lane == 0) {
         hist[warp] = gt;  // the histogram is free again: it holds the warp totals
-        hist[32 + warp] = eq;
+        hist[NW + warp] = eq;
       }
       __syncthreads();
       uint32_t gt_before = gt_run, eq_before = eq_run, gt_all = 0, eq_all = 0;
-      for (int w = 0; w < 32; ++w) {
-        const uint32_t g = hist[w], e = hist[32 + w];
+      for (int w = 0; w < NW; ++w) {
+        const uint32_t g = hist[w], e = hist[NW + w];
         if (w < warp) {
           gt_before += g;
           eq_before += e;
@@ -230,7 +233,7 @@ __global__ void __launch_bounds__(SE_THREADS)
     }
     // (the barrier that ends the last slab also orders the emitted positions
     // before they are read back here)
-    if constexpr (GATHER) gather_unit<E>(dm, plane, start, end, true, k, v, out, B, u, k_out, v_out);
+    if constexpr (GATHER) gather_unit<E, NT>(dm, plane, start, end, true, k, v, out, B, u, k_out, v_out);
     if constexpr (MODE == 2) {
       // f = the kept positions below B (they ascend: a binary search)
       int lo = 0, hi = B;
@@ -238,7 +241,7 @@ __global__ void __launch_bounds__(SE_THREADS)
         const int mid = (lo + hi) >> 1;
         if (out[mid] < B) lo = mid + 1; else hi = mid;
       }
-      fill_holes_unit<E, SE_THREADS>(dm, plane, start, B, lo, kio, vio, pos, out);
+      fill_holes_unit<E, NT>(dm, plane, start, B, lo, kio, vio, pos, out);
     }
     if constexpr (MODE == 2) __syncthreads();  // the unit's rows have moved before `out` is reused
   }
@@ -272,7 +275,7 @@ __global__ void __launch_bounds__(256)
   }
 }
 
-template <int KPT>
+template <int KPT, int NT>
 static cudaError_t launch_select_kpt(const Dims& dm, const Ws& ws, const int32_t* cu, const float* scores, int budget,
                                      int32_t* idx, int32_t* kept, int dtype, const void* k, const void* v,
                                      void* k_out, void* v_out, void* kio, void* vio, int32_t* pos, int grid,
@@ -280,22 +283,22 @@ static cudaError_t launch_select_kpt(const Dims& dm, const Ws& ws, const int32_t
   using bf = __nv_bfloat16;
   if (kio != nullptr) {  // hole filling in place
     if (dtype == 1)
-      return launch_pdl(dm.pdl != 0, select_kernel<KPT, bf, 2>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget,
+      return launch_pdl(dm.pdl != 0, select_kernel<KPT, bf, 2, NT>, grid, NT, 0, st, dm, ws, cu, scores, budget,
                         idx, kept, (const bf*)nullptr, (const bf*)nullptr, (bf*)nullptr, (bf*)nullptr, (bf*)kio,
                         (bf*)vio, pos);
-    return launch_pdl(dm.pdl != 0, select_kernel<KPT, float, 2>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget,
+    return launch_pdl(dm.pdl != 0, select_kernel<KPT, float, 2, NT>, grid, NT, 0, st, dm, ws, cu, scores, budget,
                       idx, kept, (const float*)nullptr, (const float*)nullptr, (float*)nullptr, (float*)nullptr,
                       (float*)kio, (float*)vio, pos);
   }
   if (k == nullptr)
-    return launch_pdl(dm.pdl != 0, select_kernel<KPT, bf, 0>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget,
+    return launch_pdl(dm.pdl != 0, select_kernel<KPT, bf, 0, NT>, grid, NT, 0, st, dm, ws, cu, scores, budget,
                       idx, kept, (const bf*)nullptr, (const bf*)nullptr, (bf*)nullptr, (bf*)nullptr, (bf*)nullptr,
                       (bf*)nullptr, (int32_t*)nullptr);
   if (dtype == 1)
-    return launch_pdl(dm.pdl != 0, select_kernel<KPT, bf, 1>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget,
+    return launch_pdl(dm.pdl != 0, select_kernel<KPT, bf, 1, NT>, grid, NT, 0, st, dm, ws, cu, scores, budget,
                       idx, kept, (const bf*)k, (const bf*)v, (bf*)k_out, (bf*)v_out, (bf*)nullptr, (bf*)nullptr,
                       (int32_t*)nullptr);
-  return launch_pdl(dm.pdl != 0, select_kernel<KPT, float, 1>, grid, SE_THREADS, 0, st, dm, ws, cu, scores, budget,
+  return launch_pdl(dm.pdl != 0, select_kernel<KPT, float, 1, NT>, grid, NT, 0, st, dm, ws, cu, scores, budget,
                     idx, kept, (const float*)k, (const float*)v, (float*)k_out, (float*)v_out, (float*)nullptr,
                     (float*)nullptr, (int32_t*)nullptr);
 }
@@ -304,18 +307,23 @@ cudaError_t launch_select(const Dims& dm, const Ws& ws, const int32_t* cu, const
                           int32_t* idx, int32_t* kept, int max_seqlen, int grid, cudaStream_t st, int dtype,
                           const void* k, const void* v, void* k_out, void* v_out, void* kio, void* vio,
                           int32_t* pos) {
-  if (max_seqlen <= SE_THREADS * 4)
-    JACAP_TRY(launch_select_kpt<4>(dm, ws, cu, scores, budget, idx, kept, dtype, k, v, k_out, v_out, kio, vio, pos,
-                                   grid, st));
-  else if (max_seqlen <= SE_THREADS * 8)
-    JACAP_TRY(launch_select_kpt<8>(dm, ws, cu, scores, budget, idx, kept, dtype, k, v, k_out, v_out, kio, vio, pos,
-                                   grid, st));
-  else if (max_seqlen <= SE_THREADS * 16)
-    JACAP_TRY(launch_select_kpt<16>(dm, ws, cu, scores, budget, idx, kept, dtype, k, v, k_out, v_out, kio, vio, pos,
-                                    grid, st));
-  else
-    JACAP_TRY(launch_select_kpt<32>(dm, ws, cu, scores, budget, idx, kept, dtype, k, v, k_out, v_out, kio, vio, pos,
-                                    grid, st));
+#define JACAP_SELECT(KPT, NT)                                                                                   \
+  JACAP_TRY((launch_select_kpt<KPT, NT>(dm, ws, cu, scores, budget, idx, kept, dtype, k, v, k_out, v_out, kio, vio, \
+                                        pos, grid, st)))
+  // small CTAs only pay off when the 1024-thread ones would need more than one
+  // wave (one per SM fits); for a few units the larger CTA finishes each sooner
+  int dev = 0, sms = 0;
+  JACAP_TRY(cudaGetDevice(&dev));
+  JACAP_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+  const bool small = (int64_t)dm.L * dm.Hkv * dm.S > sms;
+  if (small && max_seqlen <= 256 * 4) JACAP_SELECT(4, 256);
+  else if (small && max_seqlen <= 256 * 8) JACAP_SELECT(8, 256);
+  else if (small && max_seqlen <= 256 * 16) JACAP_SELECT(16, 256);
+  else if (max_seqlen <= 1024 * 4) JACAP_SELECT(4, 1024);
+  else if (max_seqlen <= 1024 * 8) JACAP_SELECT(8, 1024);
+  else if (max_seqlen <= 1024 * 16) JACAP_SELECT(16, 1024);
+  else JACAP_SELECT(32, 1024);
+#undef JACAP_SELECT
   return cudaGetLastError();
 }
 
