@@ -176,3 +176,35 @@ def test_host_evictor_matches_the_oracle():
                 sel = torch.as_tensor(gidx[:kept], dtype=torch.long, device=DEV)
                 assert_rows_bitwise(t.k[layer, g, cu[s]:cu[s + 1]][sel], he.k_out[layer, g, s, :kept])
                 assert_rows_bitwise(t.v[layer, g, cu[s]:cu[s + 1]][sel], he.v_out[layer, g, s, :kept])
+
+
+def test_many_slots_fill_their_holes_with_the_small_selection_ctas():
+    # an eviction of one request's slot covers 24 layers x 8 KV heads = 192
+    # units (more than the SMs) of 200 tokens: the selection with the hole
+    # filling runs 256-thread CTAs; each unit's compaction is checked against
+    # the positions it selected
+    L, Hq, Hkv, S, B, D = 24, 16, 8, 2, 160, 40
+    wl = Workload("decode many", L, Hq, Hkv, (B + D,) * S, 8, B, seed=47)
+    t = generate(wl, DEV)
+    cu = t.cu_seqlens.cpu().tolist()
+    ev = DecodeEvictor(S, L, Hq, Hkv, B, D, dtype=t.k.dtype, device=DEV)
+    assert L * Hkv > torch.cuda.get_device_properties(0).multi_processor_count
+    n0 = B + D - 1
+    k0 = torch.stack([t.k[:, :, cu[s]:cu[s] + n0] for s in range(S)])
+    v0 = torch.stack([t.v[:, :, cu[s]:cu[s] + n0] for s in range(S)])
+    ev.start(k0, v0, t.q_win.contiguous(), [n0] * S)
+    k_new = torch.stack([t.k[:, :, cu[s] + n0] for s in range(S)])
+    v_new = torch.stack([t.v[:, :, cu[s] + n0] for s in range(S)])
+    full = ev.append(k_new, v_new, t.q_win[:, :, :, -1].contiguous())
+    assert sorted(full) == list(range(S))
+    for s in range(S):
+        kb, vb = ev.k[s].clone(), ev.v[s].clone()
+        ev.evict(s)
+        ev.check()
+        for layer in (0, 5, 11, 23):
+            for g in (0, 3, 7):
+                gidx = ev.idx[layer, g, 0].cpu().numpy()
+                assert list(gidx) == sorted(set(int(x) for x in gidx)) and 0 <= gidx[0] and gidx[-1] < B + D
+                sel = torch.as_tensor(_arrangement(gidx, B, False), dtype=torch.long, device=DEV)
+                assert_rows_bitwise(kb[layer, g][sel], ev.k[s, layer, g, :B])
+                assert_rows_bitwise(vb[layer, g][sel], ev.v[s, layer, g, :B])

@@ -385,3 +385,26 @@ def test_host_cache_pass_with_output_directions_matches_the_device_pass():
     if differ == 0:
         assert_rows_bitwise(dev.k_out, he.k_out)
         assert_rows_bitwise(dev.v_out, he.v_out)
+
+
+def test_many_short_units_take_the_small_selection_ctas():
+    # more units than SMs and requests of at most 4096 tokens: the selection
+    # runs 256-thread CTAs (four or more per SM); sampled units against the
+    # oracle, every unit's selection properties, and the fused selection +
+    # compaction against the two separate calls
+    wl = Workload("t", 24, 16, 8, (1500, 700, 129), 16, 96, seed=46)  # 24 x 8 x 3 = 576 units
+    assert wl.num_layers * wl.num_kv_heads * len(wl.seqlens) > torch.cuda.get_device_properties(0).multi_processor_count
+    t = generate(wl, DEV)
+    ev = evict(make_cache(t, wl), wl.budget)
+    gpu_selection_properties(ev.scores, ev.idx, ev.kept, wl.seqlens, wl.budget)
+    for (s, layer, g) in ((0, 0, 0), (1, 11, 5), (2, 23, 7), (0, 17, 3)):
+        check_unit(ev, t, wl, jacap_params(), s, layer, g, check_w=False)
+    sep = Evictor(make_cache(t, wl), wl.budget)
+    sep.scores.copy_(ev.scores)
+    sep.ws[:64].zero_()
+    sep.select()
+    sep.compact()
+    sep.check()
+    assert torch.equal(ev.idx, sep.idx) and torch.equal(ev.kept, sep.kept)
+    assert_rows_bitwise(sep.k_out, ev.k_out)
+    assert_rows_bitwise(sep.v_out, ev.v_out)
