@@ -408,3 +408,18 @@ def test_many_short_units_take_the_small_selection_ctas():
     assert torch.equal(ev.idx, sep.idx) and torch.equal(ev.kept, sep.kept)
     assert_rows_bitwise(sep.k_out, ev.k_out)
     assert_rows_bitwise(sep.v_out, ev.v_out)
+
+
+def test_full_size_full_covariance():
+    # the K pass with the full-covariance kappa on the 32-layer 32K-token
+    # cache (every CTA runs several units, one image per run): sampled units
+    # against the oracle, every unit's selection properties
+    wl = config(2)
+    t = generate(wl, DEV)
+    params = jacap_params(full_covariance=1)
+    ev = evict(make_cache(t, wl), wl.budget, params)
+    gpu_selection_properties(ev.scores, ev.idx, ev.kept, wl.seqlens, wl.budget)
+    for (layer, g) in ((0, 0), (31, 7), (13, 4)):
+        check_unit(ev, t, wl, params, 0, layer, g, check_w=False)
+    del ev, t
+    torch.cuda.empty_cache()
