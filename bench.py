@@ -509,10 +509,16 @@ def run_e2e(args, ev, t, stream, world, dist):
     # every rank pins a host copy of its cache; if any rank cannot, all skip
     # the end-to-end number together (no rank may wait alone at a barrier)
     he, why = None, ""
+
+    def pinned(x):  # straight into pinned memory: no pageable intermediate copy
+        h = torch.empty(x.shape, dtype=x.dtype, pin_memory=True)
+        h.copy_(x)
+        return h
+
     try:
-        he = HostEvictor(c.q_win.cpu().pin_memory(), c.k.cpu().pin_memory(), c.v.cpu().pin_memory(), c.cu_seqlens,
-                         c.seqlens, c.num_q_heads, ev.budget, ev.params, group_layers=args.e2e_group,
-                         device=c.k.device, out_factor=ev.out_factor)
+        he = HostEvictor(pinned(c.q_win), pinned(c.k), pinned(c.v), c.cu_seqlens, c.seqlens, c.num_q_heads,
+                         ev.budget, ev.params, group_layers=args.e2e_group, device=c.k.device,
+                         out_factor=ev.out_factor)
     except RuntimeError as e:
         why = str(e).splitlines()[0][:200]
     ok = torch.tensor([1 if he is not None else 0], device=c.k.device)
