@@ -198,9 +198,16 @@ jacap_status jacap_score_out(const jacap_layout* layout, const jacap_params* par
  *  - Layouts whose jacap_workspace_size() exceeds JACAP_STATIC_SCRATCH_BYTES
  *    are refused with JACAP_ERR_WORKSPACE before any CUDA call; an invalid
  *    or unsupported layout gives the status jacap_score would.
- *  - The first call on a device (that device current) looks up the scratch
- *    address with cudaGetSymbolAddress, which loads the module's static memory;
- *    make that first call before capturing the stream into a graph.
+ *  - Set-up: the first call on a device (that device current) looks up the
+ *    scratch address with cudaGetSymbolAddress, which loads the module's
+ *    static memory, and caches it with the id of the current CUDA context; a
+ *    call that finds another context current (after cudaDeviceReset, or a
+ *    primary context released and retained again) looks it up afresh. Make
+ *    the first call on each device before capturing a stream into a graph.
+ *  - Footprint: every device context that loads libjacap's module holds the
+ *    JACAP_STATIC_SCRATCH_BYTES array resident until the context ends, whether
+ *    or not it ever calls this function (with CUDA_MODULE_LOADING=EAGER from
+ *    the library's first use; with lazy loading once the module is loaded).
  *  - scratch_out (may be NULL) receives the scratch's device address; it is
  *    laid out as a workspace (see jacap_workspace_offsets) and can be passed
  *    as `ws` to jacap_select and jacap_device_status. Its status word is reset

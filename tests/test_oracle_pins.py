@@ -347,3 +347,41 @@ def test_theorem1_objective_of_the_jacap_set_is_reported():
     got = obj(out["idx"])
     assert got <= best + 1e-12
     assert got > 0
+
+
+def test_theorem1_capacity_two_tokens_scalar_closed_form():
+    # d_k = d_o = 1, two tokens: S = a1 a2 [[1, -1], [-1, 1]], so
+    # J = a1 a2 (u1 - u2)(k1 - k2) and the capacity is
+    # 1/2 log(1 + lambda J^2 / sigma^2), with a1 = logistic((k1 - k2) mu).
+    k1, k2, u1, u2, mu, lam, sig2 = 1.3, -0.4, 0.7, -1.1, 0.8, 2.5, 0.6
+    a1 = expit((k1 - k2) * mu)
+    jac = a1 * (1 - a1) * (u1 - u2) * (k1 - k2)
+    want = 0.5 * math.log1p(lam * jac * jac / sig2)
+    got = T.jacobian_capacity(np.array([[u1], [u2]]), np.array([[k1], [k2]]), np.array([mu]), np.array([lam]),
+                              noise=np.array([[sig2]]))
+    assert got == pytest.approx(want, rel=1e-13)
+
+
+def test_theorem1_capacity_is_the_gaussian_channel_information():
+    # Theorem 1's objective is the mutual information of y = J q + e with
+    # q ~ N(mu, Lambda) and e ~ N(0, Sigma): 1/2 [logdet(J Lambda J^T + Sigma)
+    # - logdet(Sigma)]. J comes here from central differences of Eq. 3, with
+    # d_o != d_k and a non-identity Sigma, so a transposed Jacobian, a dropped
+    # 1/2 or Sigma applied on the wrong side all fail.
+    r = rng(29)
+    n, dk, do = 6, 5, 3
+    K = r.normal(size=(n, dk))
+    U = r.normal(size=(n, do))
+    mu = r.normal(size=dk)
+    lam = r.uniform(0.5, 2.0, size=dk)
+    A = r.normal(size=(do, do))
+    Sig = A @ A.T + 0.5 * np.eye(do)
+    h = 1e-5
+    Jfd = np.zeros((do, dk))
+    for c in range(dk):
+        e = np.zeros(dk)
+        e[c] = h
+        Jfd[:, c] = (T.retained_map(U, K, mu + e) - T.retained_map(U, K, mu - e)) / (2 * h)
+    want = 0.5 * (np.linalg.slogdet(Jfd @ np.diag(lam) @ Jfd.T + Sig)[1] - np.linalg.slogdet(Sig)[1])
+    got = T.jacobian_capacity(U, K, mu, lam, noise=Sig)
+    assert got == pytest.approx(want, rel=1e-7)

@@ -1,7 +1,7 @@
 """jacap_score_static: the scoring pass on the library's static scratch.
 
 The GPU tests call it twice in a row through the C ABI and compare both
-results with jacap_score on a caller-allocated workspace. The file is named to
+results with jacap_score on a caller-allocated workspace, bit for bit. The file is named to
 be collected last, so the static scratch is first touched after every other
 test has run; it passes alone as well. The host-side refusals need no GPU.
 """
@@ -61,7 +61,10 @@ def test_static_scratch_matches_caller_workspace_twice(name):
         assert st == JACAP_OK, (call, st)
         assert scratch != 0 and scratch % 256 == 0
         assert jacap_device_status(ctypes.c_void_p(scratch), stream) == JACAP_OK
+        # same kernels on the same bytes with fixed-order reductions: the
+        # scores are bit for bit those of the caller-workspace pass
         assert_scores_close(out.double().cpu().numpy(), ref, f"static scores, call {call}")
+        assert torch.equal(out.view(torch.int32), ev.scores.view(torch.int32)), f"static scores, call {call}"
     # The returned scratch serves as the workspace of jacap_select.
     idx = torch.empty_like(ev.idx)
     kept = torch.empty_like(ev.kept)
