@@ -36,7 +36,11 @@ FALLBACK_HBM_GBS = 6800.0
 
 def parse():
     p = argparse.ArgumentParser()
-    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--gpus", type=int, default=1,
+                   help="ranks (one GPU each); without a launcher's environment (WORLD_SIZE) the script "
+                        "re-runs itself under torch.distributed.run with this many ranks")
+    p.add_argument("--backend", default="nccl", choices=["nccl", "gloo"],
+                   help="process-group backend of the multi-rank run (gloo: CPU-only checks of the launcher)")
     p.add_argument("--steps", type=int, default=500)
     p.add_argument("--warmup", type=int, default=10)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
@@ -50,8 +54,11 @@ def parse():
     p.add_argument("--out-proj", type=int, default=0, metavar="D_O",
                    help="use true output directions u = W v with synthetic W (D_O x 128) per plane")
     p.add_argument("--decode", type=int, default=0, metavar="B",
-                   help="measure decoding-stage eviction instead: one Llama-3-8B-shaped request whose cache slot "
-                        "of B + interval tokens is scored with running query statistics and compacted to B")
+                   help="measure decoding-stage eviction instead: one request whose cache slot of B + interval "
+                        "tokens is scored with running query statistics and compacted to B")
+    p.add_argument("--decode-model", default="nemotron-7b", choices=["nemotron-7b", "llama-3-8b"],
+                   help="head layout of the decoding benchmark: Nemotron-7B (28 layers, 28 query / 4 KV heads, "
+                        "the paper's decoding-stage model) or Llama-3-8B (32 layers, 32 / 8)")
     p.add_argument("--interval", type=int, default=128, help="decoding-stage eviction interval (tokens)")
     p.add_argument("--preserve-order", action="store_true",
                    help="decoding-stage eviction: compact to ascending slot order instead of filling the holes")
@@ -63,6 +70,12 @@ def parse():
     p.add_argument("--no-graph", action="store_true", help="skip timing the pass replayed from a CUDA graph")
     p.add_argument("--layers", type=int, default=None,
                    help="override the layer count (small profiling captures; the line reports it)")
+    p.add_argument("--extra-configs", default="4",
+                   help="comma-separated evaluation configurations measured after the headline one in the same "
+                        "run and reported under extra_configs ('' for none)")
+    p.add_argument("--extra-steps", type=int, default=100)
+    p.add_argument("--ref-seconds", type=float, default=150.0,
+                   help="reference arm: CPU seconds the whole --steps + --warmup run is sized to")
     return p.parse_args()
 
 
@@ -84,6 +97,8 @@ def aggregate_ranks(t_ms: float, tokens_layers: int, dist=None, device=None):
         import torch
 
         world = dist.get_world_size()
+        if dist.get_backend() == "gloo":
+            device = "cpu"
         x = torch.tensor([float(t_ms)], dtype=torch.float64, device=device)
         dist.all_reduce(x, op=dist.ReduceOp.MAX)
         t_ms = float(x.item())
@@ -222,6 +237,14 @@ def oracle_sample(wl, budget, seconds, device, tensors=None, weighting="jacobian
 
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
+    if int(os.environ.get("WORLD_SIZE", "1")) > 1:
+        # the ranks meet once over gloo (host only: the oracle uses no GPU);
+        # then rank 0 alone runs the oracle and the others exit without work
+        import torch.distributed as dist
+
+        dist.init_process_group("gloo")
+        dist.barrier()
+        dist.destroy_process_group()
     if rank != 0:
         return 0
     from oracle import JacapParams, oracle_unit
@@ -238,8 +261,8 @@ def run_reference(args):
     P = JacapParams(linear_weighting=args.weighting == "linear", full_covariance=args.covariance == "full")
     oracle_unit(Q64, K64[:2048], V64[:2048], budget, P)
     per_tok = (time.perf_counter() - t0) / 2048
-    target = 150.0 / max(1, args.steps + args.warmup)
-    m = int(max(256, min(n_full, target / per_tok)))
+    target = args.ref_seconds / max(1, args.steps + args.warmup)
+    m = int(max(min(256, n_full), min(n_full, target / per_tok)))
     for _ in range(args.warmup):
         oracle_unit(Q64, K64[:m], V64[:m], budget, P)
     times = []
@@ -256,7 +279,7 @@ def run_reference(args):
         "metric": METRIC,
         "value": value,
         "unit": UNIT,
-        "n_gpus": args.gpus,
+        "n_gpus": int(os.environ.get("WORLD_SIZE", "1")),
         "steps": args.steps,
         "warmup": args.warmup,
         "ms_per_step": avg * 1e3,
@@ -290,7 +313,7 @@ def run_ours(args):
         import torch.distributed as dist
 
         torch.cuda.set_device(local)
-        dist.init_process_group("nccl")
+        dist.init_process_group(args.backend)
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
 
@@ -410,6 +433,12 @@ def run_ours(args):
     tokens_layers = sum(t.seqlens) * L
     alg_pass = wl.algorithmic_bytes(budget)
 
+    extra = []
+    for x in [c for c in args.extra_configs.split(",") if c.strip()]:
+        if int(x) == args.config and not args.layers:
+            continue
+        extra.append(measure_config(int(x), args, dev, dist, rank, peaks()[0]))
+
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         v_cpu, desc, wall = oracle_sample(wl, budget, args.cpu_seconds, dev, tensors=t, weighting=args.weighting,
@@ -458,6 +487,7 @@ def run_ours(args):
             "gpu_launches": K * (7 + (1 if args.covariance == "full" and not full_cov_fused else 0)
                                  + (0 if fused_weights else 1)),
             "clocks": clocks,
+            "extra_configs": extra,
             "cpu_baseline": cpu,
             "e2e": e2e,
         }
@@ -465,6 +495,83 @@ def run_ours(args):
     if dist is not None:
         dist.destroy_process_group()
     return 0
+
+
+def measure_config(index, args, dev, dist, rank, hbm):
+    """One more evaluation configuration in the same run: the plain pass timed
+    over --extra-steps steps (CUDA events around them), per-kernel durations
+    from as many steps with an event between kernels, clocks sampled during
+    both, and the pass roofline. The cache is freed afterwards."""
+    import torch
+
+    from paper_2609_08131_gb300 import SCORE_KERNEL_NAMES, jacap_params
+    from paper_2609_08131_gb300.api import Cache, Evictor
+    from paper_2609_08131_gb300.workloads import config, generate
+    from dataclasses import replace
+
+    wl = config(index)
+    wl = replace(wl, seed=wl.seed + 1000 * rank)
+    budget = wl.budget
+    t = generate(wl, dev)
+    ev = Evictor(Cache(t.q_win, t.k, t.v, t.cu_seqlens, t.seqlens, wl.num_q_heads), budget, jacap_params())
+    stream = torch.cuda.current_stream(dev)
+    for _ in range(max(3, args.warmup)):
+        ev.run()
+    ev.check()
+    K = max(1, args.extra_steps)
+    nk = len(SCORE_KERNEL_NAMES)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(nk + 2)] for _ in range(K)]
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    for e in [x for row in evs for x in row] + [a, b]:
+        e.record(stream)
+    torch.cuda.synchronize()
+    sampler = ClockSampler(dev.index)
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    sampler.start()
+    a.record(stream)
+    for _ in range(K):
+        ev.run()
+    b.record(stream)
+    torch.cuda.synchronize()
+    t_ms = a.elapsed_time(b) / K
+    for i in range(K):
+        ev.score(events=evs[i][:nk + 1])
+        ev.select_compact()
+        evs[i][nk + 1].record(stream)
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    ev.check()
+    kern = {name: sum(evs[i][j].elapsed_time(evs[i][j + 1]) for i in range(K)) / K
+            for j, name in enumerate(SCORE_KERNEL_NAMES)}
+    kern["select_compact"] = sum(evs[i][nk].elapsed_time(evs[i][nk + 1]) for i in range(K)) / K
+    L = t.k.shape[0]
+    value, t_ms, world = aggregate_ranks(t_ms, sum(t.seqlens) * L, dist, dev)
+    alg = wl.algorithmic_bytes(budget)
+    out = {
+        "config": index,
+        "workload": wl.name,
+        "layers": wl.num_layers, "q_heads": wl.num_q_heads, "kv_heads": wl.num_kv_heads,
+        "seqlens": list(wl.seqlens) if len(wl.seqlens) <= 4 else f"{len(wl.seqlens)} requests, sum {wl.total_tokens}",
+        "window": wl.window, "budget": budget, "cache_dtype": wl.dtype,
+        "steps": K,
+        "value": value,
+        "unit": UNIT,
+        "ms_per_step": t_ms,
+        "pass_roofline": {
+            "algorithmic_bytes": alg,
+            "achieved_gbs": alg / (t_ms * 1e-3) / 1e9,
+            "frac_of_8tbs": alg / (t_ms * 1e-3) / 1e9 / NOMINAL_HBM_GBS,
+            "frac_of_measured": alg / (t_ms * 1e-3) / 1e9 / hbm,
+        },
+        "kernel_ms": kern,
+        "clocks": clocks,
+        "gpu_launches": K * (7 + (0 if wl.dtype == "bf16" else 1)),
+    }
+    del ev, t
+    torch.cuda.empty_cache()
+    return out
 
 
 def time_cuda_graph(ev, stream, dev, K):
@@ -573,8 +680,10 @@ def run_e2e(args, ev, t, stream, world, dist):
 def run_decode(args):
     """Decoding-stage eviction events (reading R16) on one GPU.
 
-    One request of the Llama-3-8B shape (32 layers, 32 query / 8 KV heads)
-    with a full slot of B + interval tokens; each timed step is one eviction
+    One request of the Nemotron-7B head layout (28 layers, 28 query / 4 KV
+    heads; the paper's decoding-stage model) or, with --decode-model
+    llama-3-8b, of the Llama-3-8B one (32 layers, 32 / 8), with a full slot of
+    B + interval tokens; each timed step is one eviction
     event: the scoring pass with running statistics, TOP-B and the in-place
     compaction. After an event the slot is marked full again (its free rows
     still hold earlier tokens), so every event scores B + interval tokens."""
@@ -588,8 +697,10 @@ def run_decode(args):
     torch.cuda.set_device(dev)
     B, D = args.decode, args.interval
     cap = B + D
-    L, Hq, Hkv, w = 32, 32, 8, 32
-    wl = Workload(f"decoding-stage eviction, Llama-3-8B-shaped, reserved tokens B={B}, interval {D}", L, Hq, Hkv,
+    # Nemotron-7B: 28 layers, 28 query / 4 KV heads (G = 7), head_dim 128
+    L, Hq, Hkv, w = (28, 28, 4, 32) if args.decode_model == "nemotron-7b" else (32, 32, 8, 32)
+    shape = "Nemotron-7B-shaped" if args.decode_model == "nemotron-7b" else "Llama-3-8B-shaped"
+    wl = Workload(f"decoding-stage eviction, {shape}, reserved tokens B={B}, interval {D}", L, Hq, Hkv,
                   (cap,), w + 1, B, seed=40)
     t = generate(wl, dev)
     ev = DecodeEvictor(1, L, Hq, Hkv, B, D, dtype=t.k.dtype, params=jacap_params(), device=dev,
@@ -673,8 +784,35 @@ def run_decode(args):
     return 0
 
 
+def free_port() -> int:
+    import socket
+
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def launch_ranks(args) -> int:
+    """`--gpus N` (N > 1) outside a launcher: run this script again under
+    torch.distributed.run with N ranks on this node (one GPU each, rendezvous
+    on 127.0.0.1); rank 0 prints the JSON line. Returns the launcher's status."""
+    if args.impl == "ours" and args.backend == "nccl":
+        import torch
+
+        have = torch.cuda.device_count()
+        if have < args.gpus:
+            print(f"bench.py: --gpus {args.gpus} needs {args.gpus} GPUs, this node has {have}", file=sys.stderr)
+            return 2
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", f"--nproc-per-node={args.gpus}",
+           "--master-addr", "127.0.0.1", "--master-port", str(free_port()), os.path.abspath(__file__),
+           *sys.argv[1:]]
+    return subprocess.call(cmd)
+
+
 def main():
     args = parse()
+    if args.gpus > 1 and "WORLD_SIZE" not in os.environ:
+        return launch_ranks(args)
     if args.impl == "reference":
         return run_reference(args)
     if args.decode:

@@ -37,7 +37,7 @@ jacap_status check_layout(const jacap_layout* L) {
   if (L->num_q_heads % L->num_kv_heads != 0) return JACAP_ERR_INVALID_ARG;
   const int G = L->num_q_heads / L->num_kv_heads;
   if (L->head_dim != D) return JACAP_ERR_UNSUPPORTED;
-  if (G != 1 && G != 2 && G != 4 && G != 8) return JACAP_ERR_UNSUPPORTED;
+  if (G > G_MAX) return JACAP_ERR_UNSUPPORTED;
   const int64_t el16 = L->dtype == JACAP_BF16 ? 8 : 4;  // elements per 16 bytes
   const int64_t kv[3] = {L->kv_stride_layer, L->kv_stride_head, L->kv_stride_token};
   const int64_t qs[4] = {L->q_stride_seq, L->q_stride_layer, L->q_stride_head, L->q_stride_pos};

@@ -124,6 +124,62 @@ struct ItemStream {
   }
 };
 
+// Largest GQA group (query heads per KV head) the kernels are compiled for.
+constexpr int G_MAX = 8;
+
+// The logits/kappa rows hold 2G floats per token: l_h at [0, G), kappa_h at
+// [G, 2G). A row starts on a multiple of 2G floats from a 1 KB-aligned base, so
+// it is 16-byte aligned for even G and 8-byte aligned for odd G; the kappa
+// half (G floats further) keeps 16 bytes only when G % 4 == 0.
+template <int G>
+struct LkAlign {
+  static constexpr int ROW = G % 2 == 0 ? 4 : 2;                      // floats
+  static constexpr int KAPPA = G % 4 == 0 ? 4 : (G % 2 == 0 ? 2 : 1);  // floats
+};
+
+// dst[0 .. N) = v with the widest stores an alignment of A floats (1, 2 or 4)
+// allows.
+template <int N, int A>
+__device__ __forceinline__ void store_floats(float* dst, const float* v) {
+  int e = 0;
+  if constexpr (A >= 4) {
+#pragma unroll
+    for (; e + 4 <= N; e += 4) *(float4*)(dst + e) = make_float4(v[e], v[e + 1], v[e + 2], v[e + 3]);
+  }
+  if constexpr (A >= 2) {
+#pragma unroll
+    for (; e + 2 <= N; e += 2) *(float2*)(dst + e) = make_float2(v[e], v[e + 1]);
+  }
+#pragma unroll
+  for (; e < N; ++e) dst[e] = v[e];
+}
+
+// v[0 .. N) = src[0 .. N) with the widest loads an alignment of A floats allows.
+template <int N, int A>
+__device__ __forceinline__ void load_floats(float* v, const float* src) {
+  int e = 0;
+  if constexpr (A >= 4) {
+#pragma unroll
+    for (; e + 4 <= N; e += 4) {
+      const float4 x = *(const float4*)(src + e);
+      v[e] = x.x;
+      v[e + 1] = x.y;
+      v[e + 2] = x.z;
+      v[e + 3] = x.w;
+    }
+  }
+  if constexpr (A >= 2) {
+#pragma unroll
+    for (; e + 2 <= N; e += 2) {
+      const float2 x = *(const float2*)(src + e);
+      v[e] = x.x;
+      v[e + 1] = x.y;
+    }
+  }
+#pragma unroll
+  for (; e < N; ++e) v[e] = src[e];
+}
+
 // Programmatic dependent launch. A kernel launched with the programmatic
 // stream-serialization attribute is set up while the previous kernel of the
 // stream still runs and is scheduled as its CTAs exit (no kernel here triggers

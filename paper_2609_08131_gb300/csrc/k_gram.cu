@@ -85,17 +85,7 @@ __global__ void __launch_bounds__(WT_THREADS) weight_kernel(Dims dm, Ws ws, cons
       for (int q = 0; q < 4; ++q) {
         const int64_t tok = t4 + q * WT_THREADS;
         const float* src = ws.lk + (base + (tok < item.t1 ? tok : t4)) * (2 * G);
-        if constexpr ((2 * G) % 4 == 0) {
-#pragma unroll
-          for (int e = 0; e < 2 * G; e += 4) {
-            const float4 q4 = *(const float4*)(src + e);
-            lk[q][e] = q4.x; lk[q][e + 1] = q4.y; lk[q][e + 2] = q4.z; lk[q][e + 3] = q4.w;
-          }
-        } else {
-          const float2 q2 = *(const float2*)src;
-          lk[q][0] = q2.x;
-          lk[q][1] = q2.y;
-        }
+        load_floats<2 * G, LkAlign<G>::ROW>(lk[q], src);
       }
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
@@ -154,8 +144,11 @@ constexpr uint32_t GR_IDESC = idesc_bf16_f32(128, 128, 0, 1);
 template <int G>
 struct GrCfg {
   static constexpr int LK_BYTES = TILE * 2 * G * 4 + 16;  // a tile's logits/kappa rows (+ alignment slack)
-  static constexpr int VST = G == 8 ? 5 : 6;              // stages in flight
-  static constexpr size_t SMEM = 1024 + (size_t)VST * (GR_V_BYTES + GR_W_BYTES + LK_BYTES) + 256;
+  static constexpr size_t smem_for(int stages) {
+    return 1024 + (size_t)stages * (GR_V_BYTES + GR_W_BYTES + LK_BYTES) + 256;
+  }
+  static constexpr int VST = smem_for(6) <= 232448 ? 6 : 5;  // stages in flight
+  static constexpr size_t SMEM = smem_for(VST);
   static_assert(SMEM <= 232448, "shared memory");
 };
 
@@ -409,17 +402,9 @@ __global__ void __launch_bounds__(GR_THREADS, 1)
           uint32_t word = 0u;
           if (i < lt.nvalid) {
             float r[2 * G];
-            if constexpr ((2 * G) % 4 == 0) {  // 16-byte aligned rows (off = 0 for G >= 2)
-#pragma unroll
-              for (int e = 0; e < 2 * G; e += 4) {
-                const float4 x = *(const float4*)(rows + i * 2 * G + e);
-                r[e] = x.x; r[e + 1] = x.y; r[e + 2] = x.z; r[e + 3] = x.w;
-              }
-            } else {
-              const float2 x = *(const float2*)(rows + i * 2 * G);
-              r[0] = x.x;
-              r[1] = x.y;
-            }
+            // the staged copy keeps the rows' global alignment (off is the
+            // row start's distance from the 16-byte boundary below it)
+            load_floats<2 * G, LkAlign<G>::ROW>(r, rows + i * 2 * G);
             float wt = 0.f;
             if (dm.linear) {
 #pragma unroll
@@ -577,7 +562,11 @@ cudaError_t launch_weights(const Dims& dm, const Ws& ws, const int32_t* cu, int 
   switch (dm.G) {
     case 1: return launch_weights_g<1>(dm, ws, cu, grid, st);
     case 2: return launch_weights_g<2>(dm, ws, cu, grid, st);
+    case 3: return launch_weights_g<3>(dm, ws, cu, grid, st);
     case 4: return launch_weights_g<4>(dm, ws, cu, grid, st);
+    case 5: return launch_weights_g<5>(dm, ws, cu, grid, st);
+    case 6: return launch_weights_g<6>(dm, ws, cu, grid, st);
+    case 7: return launch_weights_g<7>(dm, ws, cu, grid, st);
     case 8: return launch_weights_g<8>(dm, ws, cu, grid, st);
     default: return cudaErrorInvalidValue;
   }
@@ -599,7 +588,11 @@ cudaError_t launch_gram(const CUtensorMap& vmap, const Dims& dm, const Ws& ws, i
     switch (dm.G) {
       case 1: return launch_gram_bf16<1>(vmap, dm, ws, cu, grid, st);
       case 2: return launch_gram_bf16<2>(vmap, dm, ws, cu, grid, st);
+      case 3: return launch_gram_bf16<3>(vmap, dm, ws, cu, grid, st);
       case 4: return launch_gram_bf16<4>(vmap, dm, ws, cu, grid, st);
+      case 5: return launch_gram_bf16<5>(vmap, dm, ws, cu, grid, st);
+      case 6: return launch_gram_bf16<6>(vmap, dm, ws, cu, grid, st);
+      case 7: return launch_gram_bf16<7>(vmap, dm, ws, cu, grid, st);
       case 8: return launch_gram_bf16<8>(vmap, dm, ws, cu, grid, st);
       default: return cudaErrorInvalidValue;
     }

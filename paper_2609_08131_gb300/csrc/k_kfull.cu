@@ -319,12 +319,7 @@ __global__ void __launch_bounds__(KX_THREADS, 1)
             bad |= !isfinite(row[G + h]);
           }
           float* dst = lkp + tok * (2 * G);
-          if constexpr (G >= 2) {
-#pragma unroll
-            for (int e = 0; e < 2 * G; e += 4) *(float4*)(dst + e) = make_float4(row[e], row[e + 1], row[e + 2], row[e + 3]);
-          } else {
-            *(float2*)dst = make_float2(row[0], row[1]);
-          }
+          store_floats<2 * G, LkAlign<G>::ROW>(dst, row);
         }
       }
       // ---- softmax statistics of a run, at its last chunk; the run's other
@@ -455,7 +450,11 @@ cudaError_t launch_kpass_full(const CUtensorMap& kmap, const Dims& dm, const Ws&
   switch (dm.G) {
     case 1: return launch_kpf_g<1>(kmap, dm, ws, grid, st);
     case 2: return launch_kpf_g<2>(kmap, dm, ws, grid, st);
+    case 3: return launch_kpf_g<3>(kmap, dm, ws, grid, st);
     case 4: return launch_kpf_g<4>(kmap, dm, ws, grid, st);
+    case 5: return launch_kpf_g<5>(kmap, dm, ws, grid, st);
+    case 6: return launch_kpf_g<6>(kmap, dm, ws, grid, st);
+    case 7: return launch_kpf_g<7>(kmap, dm, ws, grid, st);
     case 8: return launch_kpf_g<8>(kmap, dm, ws, grid, st);
     default: return cudaErrorInvalidValue;
   }

@@ -38,7 +38,6 @@ constexpr int KB_KAPPA_WARP0 = 2, KB_READ_WARP0 = 10, KB_BUILD_WARP = 14;
 
 template <int G>
 struct KbCfg {
-  static constexpr int STAGES = G == 8 ? 5 : 6;        // K tiles in flight
   static constexpr int NB = (3 * G <= 16) ? 16 : 32;  // MMA N = rows of the mu' image
   static constexpr int IMG_ATOM = NB * 128;            // bytes per 64-channel atom
   static constexpr int IMG_BYTES = 2 * IMG_ATOM;
@@ -46,8 +45,12 @@ struct KbCfg {
   static constexpr int KRED_FLOATS = 2 * 4 * 4 * G * 32;  // [group][token subset][writer][G][32]
   static constexpr uint32_t IDESC = idesc_bf16_f32(128, NB, 0, 0);
   static_assert(KB_NACC * NB <= (int)KB_TMEM_COLS, "tensor memory budget");
-  static constexpr size_t SMEM = 1024 + (size_t)STAGES * KB_TILE_BYTES + 2 * IMG_BYTES + 2 * LAM_BYTES +
-                                 KRED_FLOATS * 4 + 4 * 2 * G * 4 + 512;
+  static constexpr size_t smem_for(int stages) {
+    return 1024 + (size_t)stages * KB_TILE_BYTES + 2 * IMG_BYTES + 2 * LAM_BYTES + KRED_FLOATS * 4 + 4 * 2 * G * 4 +
+           512;
+  }
+  static constexpr int STAGES = smem_for(6) <= 232448 ? 6 : 5;  // K tiles in flight
+  static constexpr size_t SMEM = smem_for(STAGES);
 };
 
 // mu' image of one item: rows n = part * G + h hold part (0 hi, 1 mid, 2 lo) of
@@ -80,56 +83,51 @@ __device__ __forceinline__ void build_split_image(uint8_t* im, const float* src,
 
 // Partial kappa over channel quarter `cq` (chunks 4 cq .. 4 cq + 3 of 8
 // channels) for the four token rows lane + 32 j of a staged tile:
-// part[j][h] = sum_c lambda_h,c k_c^2. Each lambda load feeds four tokens.
+// part[j][h] = sum_c lambda_h,c k_c^2. Each lambda load feeds JB tokens: all
+// four for G = 1, 2, 4; for other groups two passes over the quarter take two
+// tokens each, which halves the accumulators held at once (and keeps them in
+// registers).
 template <int G>
 __device__ __forceinline__ void kappa_quarter(uint32_t kt, uint32_t lam, int lane, int cq, float (&part)[4][G]) {
-  float2 acc[4][G];
+  constexpr int JB = (G <= 2 || G == 4) ? 4 : 2;
 #pragma unroll
-  for (int j = 0; j < 4; ++j)
+  for (int j0 = 0; j0 < 4; j0 += JB) {
+    float2 acc[JB][G];
 #pragma unroll
-    for (int h = 0; h < G; ++h) acc[j][h] = make_float2(0.f, 0.f);
+    for (int j = 0; j < JB; ++j)
+#pragma unroll
+      for (int h = 0; h < G; ++h) acc[j][h] = make_float2(0.f, 0.f);
 #pragma unroll 1
-  for (int cc = 4 * cq; cc < 4 * cq + 4; ++cc) {
-    float4 l0[G], l1[G];
-#pragma unroll
-    for (int h = 0; h < G; ++h) {
-      l0[h] = lds_f128(lam + (h * D + 8 * cc) * 4);
-      l1[h] = lds_f128(lam + (h * D + 8 * cc + 4) * 4);
-    }
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const uint4 r = lds_u128(kt + (cc >> 3) * KB_BOX + sw128_off(lane + 32 * j, cc & 7));
-      const uint32_t w[4] = {r.x, r.y, r.z, r.w};
-      float2 sq[4];
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const float2 x = make_float2(bf16lo(w[q]), bf16hi(w[q]));
-        sq[q] = __fmul2_rn(x, x);  // exact: 8-bit significands
-      }
+    for (int cc = 4 * cq; cc < 4 * cq + 4; ++cc) {
+      float4 l0[G], l1[G];
 #pragma unroll
       for (int h = 0; h < G; ++h) {
-        acc[j][h] = __ffma2_rn(sq[0], make_float2(l0[h].x, l0[h].y), acc[j][h]);
-        acc[j][h] = __ffma2_rn(sq[1], make_float2(l0[h].z, l0[h].w), acc[j][h]);
-        acc[j][h] = __ffma2_rn(sq[2], make_float2(l1[h].x, l1[h].y), acc[j][h]);
-        acc[j][h] = __ffma2_rn(sq[3], make_float2(l1[h].z, l1[h].w), acc[j][h]);
+        l0[h] = lds_f128(lam + (h * D + 8 * cc) * 4);
+        l1[h] = lds_f128(lam + (h * D + 8 * cc + 4) * 4);
+      }
+#pragma unroll
+      for (int j = 0; j < JB; ++j) {
+        const uint4 r = lds_u128(kt + (cc >> 3) * KB_BOX + sw128_off(lane + 32 * (j0 + j), cc & 7));
+        const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+        float2 sq[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const float2 x = make_float2(bf16lo(w[q]), bf16hi(w[q]));
+          sq[q] = __fmul2_rn(x, x);  // exact: 8-bit significands
+        }
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+          acc[j][h] = __ffma2_rn(sq[0], make_float2(l0[h].x, l0[h].y), acc[j][h]);
+          acc[j][h] = __ffma2_rn(sq[1], make_float2(l0[h].z, l0[h].w), acc[j][h]);
+          acc[j][h] = __ffma2_rn(sq[2], make_float2(l1[h].x, l1[h].y), acc[j][h]);
+          acc[j][h] = __ffma2_rn(sq[3], make_float2(l1[h].z, l1[h].w), acc[j][h]);
+        }
       }
     }
-  }
 #pragma unroll
-  for (int j = 0; j < 4; ++j)
+    for (int j = 0; j < JB; ++j)
 #pragma unroll
-    for (int h = 0; h < G; ++h) part[j][h] = acc[j][h].x + acc[j][h].y;
-}
-
-template <int G>
-__device__ __forceinline__ void store_part(float* dst, const float (&v)[G]) {
-  if constexpr (G % 4 == 0) {
-#pragma unroll
-    for (int h = 0; h < G; h += 4) *(float4*)(dst + h) = make_float4(v[h], v[h + 1], v[h + 2], v[h + 3]);
-  } else if constexpr (G == 2) {
-    *(float2*)dst = make_float2(v[0], v[1]);
-  } else {
-    dst[0] = v[0];
+      for (int h = 0; h < G; ++h) part[j0 + j][h] = acc[j][h].x + acc[j][h].y;
   }
 }
 
@@ -340,7 +338,7 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
           }
           named_barrier_sync(bar_id, 128);  // the slots may be rewritten after this
           const int64_t tok = t + lane + 32 * cq;
-          if (tok < item.t1) store_part<G>(lkp + tok * (2 * G), kap);
+          if (tok < item.t1) store_floats<G, LkAlign<G>::KAPPA>(lkp + tok * (2 * G), kap);
         }
       }
       cont = is.next_same_unit(item);
@@ -395,7 +393,7 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
             run_s[h] = run_s[h] * __expf(run_m[h] - mn) + __expf(lg[h] - mn);
             run_m[h] = mn;
           }
-          store_part<G>(lkp + tok * (2 * G), lg);
+          store_floats<G, LkAlign<G>::ROW>(lkp + tok * (2 * G), lg);
         }
       }
       // ---- softmax statistics of a run, at its last chunk; the run's other
@@ -457,7 +455,11 @@ cudaError_t launch_kpass_bf16(const CUtensorMap& kmap, const Dims& dm, const Ws&
   switch (dm.G) {
     case 1: return launch_g<1>(kmap, dm, ws, cu, grid, st);
     case 2: return launch_g<2>(kmap, dm, ws, cu, grid, st);
+    case 3: return launch_g<3>(kmap, dm, ws, cu, grid, st);
     case 4: return launch_g<4>(kmap, dm, ws, cu, grid, st);
+    case 5: return launch_g<5>(kmap, dm, ws, cu, grid, st);
+    case 6: return launch_g<6>(kmap, dm, ws, cu, grid, st);
+    case 7: return launch_g<7>(kmap, dm, ws, cu, grid, st);
     case 8: return launch_g<8>(kmap, dm, ws, cu, grid, st);
     default: return cudaErrorInvalidValue;
   }

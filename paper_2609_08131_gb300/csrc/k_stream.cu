@@ -304,14 +304,7 @@ __global__ void __launch_bounds__(KP_THREADS, 1)
           }
         }
         float* dst = ws.lk + ((int64_t)item.plane * dm.Ntot + tok) * (2 * G);
-        if constexpr ((2 * G) % 4 == 0) {
-#pragma unroll
-          for (int e = 0; e < 2 * G; e += 4)
-            *(float4*)(dst + e) = make_float4(out[e], out[e + 1], out[e + 2], out[e + 3]);
-        } else {
-#pragma unroll
-          for (int e = 0; e < 2 * G; ++e) dst[e] = out[e];
-        }
+        store_floats<2 * G, LkAlign<G>::ROW>(dst, out);
       }
     }
     // chunk statistics: combine the 128 per-thread (max, sum) pairs per head
@@ -373,7 +366,11 @@ static cudaError_t launch_kpass_t(const CUtensorMap& kmap, const Dims& dm, const
   switch (dm.G) {
     case 1: return launch_kpass_tg<T, 1>(kmap, dm, ws, cu, grid, st);
     case 2: return launch_kpass_tg<T, 2>(kmap, dm, ws, cu, grid, st);
+    case 3: return launch_kpass_tg<T, 3>(kmap, dm, ws, cu, grid, st);
     case 4: return launch_kpass_tg<T, 4>(kmap, dm, ws, cu, grid, st);
+    case 5: return launch_kpass_tg<T, 5>(kmap, dm, ws, cu, grid, st);
+    case 6: return launch_kpass_tg<T, 6>(kmap, dm, ws, cu, grid, st);
+    case 7: return launch_kpass_tg<T, 7>(kmap, dm, ws, cu, grid, st);
     case 8: return launch_kpass_tg<T, 8>(kmap, dm, ws, cu, grid, st);
     default: return cudaErrorInvalidValue;
   }

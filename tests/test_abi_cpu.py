@@ -66,7 +66,6 @@ def test_workspace_size_is_positive_and_monotone():
 
 @pytest.mark.parametrize("field,value,expect", [
     ("head_dim", 64, J.JACAP_ERR_UNSUPPORTED),
-    ("num_q_heads", 6, J.JACAP_ERR_UNSUPPORTED),       # G = 3
     ("num_q_heads", 7, J.JACAP_ERR_INVALID_ARG),       # not a multiple
     ("num_q_heads", 32, J.JACAP_ERR_UNSUPPORTED),      # G = 16
     ("window", 0, J.JACAP_ERR_INVALID_ARG),
@@ -90,6 +89,13 @@ def test_invalid_layouts_are_rejected_on_the_host(field, value, expect):
     assert st == expect
     st = J.jacap_compact(lay, p, p, p, 8, p, p, None)
     assert st == expect
+
+
+@pytest.mark.parametrize("group", range(1, 9))
+def test_every_gqa_ratio_up_to_eight_is_accepted(group):
+    # Hq = G Hkv for G = 1 .. 8 (Qwen3-14B has G = 5, Nemotron-7B G = 7)
+    lay = good_layout(num_q_heads=group * good_layout().num_kv_heads)
+    assert J.jacap_workspace_size(lay, 8) > 0
 
 
 def test_bad_params_and_buffers_are_rejected_on_the_host():

@@ -37,6 +37,9 @@ CASES = {
                                  True),
     "bf16_gqa8_long_slot": (1, 8, 1, (700,), 16, 40, 512, 200, "bf16", jacap_params(), 34, False),
     "bf16_gqa8_long_slot_ordered": (1, 8, 1, (700,), 16, 40, 512, 200, "bf16", jacap_params(), 34, True),
+    # Nemotron-7B's heads (28 q / 4 kv, G = 7), the paper's decoding-stage model
+    "bf16_gqa7_nemotron_heads": (2, 28, 4, (60, 45), 8, 60, 40, 16, "bf16", jacap_params(), 35, False),
+    "f32_gqa5_ordered": (1, 10, 2, (30,), 4, 25, 24, 8, "f32", jacap_params(tau=2.0), 36, True),
 }
 
 

@@ -84,6 +84,24 @@ SMALL = {
                           jacap_params(full_covariance=1)),
     "f32_mha_linear_weighting": (Workload("t", 1, 4, 4, (900,), 8, 64, dtype="f32", seed=20),
                                  jacap_params(linear_weighting=1, cov_unbiased=1)),
+    # GQA ratios of the paper's other models: Qwen3-14B (40 q / 8 kv heads,
+    # G = 5) and Nemotron-7B (28 q / 4 kv heads, G = 7), plus G = 3 and 6.
+    # Odd G gives 8-byte aligned logits/kappa rows and 4-byte aligned kappa halves.
+    "bf16_gqa5_qwen3_14b_heads": (Workload("t", 2, 40, 8, (1200, 333), 32, 128, seed=41), jacap_params()),
+    "bf16_gqa7_nemotron_heads": (Workload("t", 2, 28, 4, (1500, 129), 32, 128, seed=42), jacap_params()),
+    "bf16_gqa3_tau1": (Workload("t", 1, 6, 2, (800, 257), 16, 64, seed=43), jacap_params(tau=1.0)),
+    "bf16_gqa6_unbiased": (Workload("t", 1, 12, 2, (700, 130), 16, 64, seed=44), jacap_params(cov_unbiased=1)),
+    "bf16_gqa7_peaky_linear": (Workload("t", 1, 14, 2, (650, 3), 8, 40, seed=45), jacap_params(linear_weighting=1)),
+    "f32_gqa5": (Workload("t", 1, 10, 2, (600, 77), 16, 64, dtype="f32", seed=46), jacap_params(tau=0.7)),
+    "f32_gqa7": (Workload("t", 1, 14, 2, (500, 70), 8, 32, dtype="f32", seed=47), jacap_params()),
+    # full covariance: tensor-core kernel with G w = 96, 80, 112 centred queries
+    # (the last with a 32-row mu' image), CUDA-core kernel with G w = 192
+    "bf16_gqa3_full_cov_w32": (Workload("t", 1, 6, 2, (900, 100), 32, 64, seed=48), jacap_params(full_covariance=1)),
+    "bf16_gqa5_full_cov_w16": (Workload("t", 1, 10, 2, (700,), 16, 64, seed=49), jacap_params(full_covariance=1)),
+    "bf16_gqa7_full_cov_w16": (Workload("t", 1, 14, 2, (640, 33), 16, 64, seed=50),
+                               jacap_params(full_covariance=1, tau=2.0)),
+    "bf16_gqa6_full_cov_w32_simt": (Workload("t", 1, 12, 2, (500,), 32, 64, seed=51),
+                                    jacap_params(full_covariance=1)),
 }
 
 
