@@ -605,9 +605,10 @@ def time_cuda_graph(ev, stream, dev, K):
 
 def run_e2e(args, ev, t, stream, world, dist):
     """Same metric through the public API with the cache in pinned host memory
-    (``api.HostEvictor``): every step copies the whole cache host->device in
-    layer groups, overlapped with the pass over the previous group, and reads
-    the kept positions back."""
+    (``jacap_evict_host`` via ``api.HostEvictor``): every step copies the whole
+    cache host->device in layer groups, overlapped with the pass over the
+    previous group, and brings the kept positions and the retained K and V rows
+    back to host memory."""
     import torch
 
     from paper_2609_08131_gb300.api import HostEvictor
@@ -640,12 +641,14 @@ def run_e2e(args, ev, t, stream, world, dist):
     # the host link on its own: one layer group's K copied host -> device
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     grp = he.k_h[:he.gl]
+    probe = torch.empty(grp.shape, dtype=grp.dtype, device=c.k.device)
     a.record(stream)
     for _ in range(3):
-        he.kb[0].copy_(grp, non_blocking=True)
+        probe.copy_(grp, non_blocking=True)
     b.record(stream)
     torch.cuda.synchronize()
     link_gbs = 3 * grp.numel() * grp.element_size() / (a.elapsed_time(b) * 1e-3) / 1e9
+    del probe
     if dist is not None:
         dist.barrier()
     a.record(stream)
@@ -674,7 +677,8 @@ def run_e2e(args, ev, t, stream, world, dist):
     return {"value": sum(t.seqlens) * L * world / (ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": he.h2d_bytes,
             "d2h_bytes_per_step": he.d2h_bytes, "ms_per_step": ms, "steps": n, "group_layers": he.gl,
             "idx_differ_vs_resident": differ, "h2d_link_gbs": link_gbs,
-            "h2d_bound_ms": he.h2d_bytes / (link_gbs * 1e9) * 1e3}
+            "h2d_bound_ms": he.h2d_bytes / (link_gbs * 1e9) * 1e3, "api": "jacap_evict_host (C ABI)",
+            "returns": "kept positions and the retained K and V rows, in pinned host memory"}
 
 
 def run_decode(args):

@@ -27,7 +27,7 @@
  *    the static scratch of jacap_score_static).
  *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
  *    All work is enqueued asynchronously on it; nothing synchronises except
- *    jacap_device_status().
+ *    jacap_device_status() and jacap_evict_host().
  *  - Host-side validation happens before anything is enqueued; on any error
  *    status nothing has been launched. A failed launch returns JACAP_ERR_CUDA.
  *  - Problems only the device can see (a malformed cu_seqlens array, a
@@ -50,7 +50,7 @@ extern "C" {
 typedef enum {
   JACAP_OK = 0,
   JACAP_ERR_INVALID_ARG = 1, /* bad pointer, size, stride, alignment or layout   */
-  JACAP_ERR_UNSUPPORTED = 2, /* head_dim != 128, group size not in {1,2,4,8},
+  JACAP_ERR_UNSUPPORTED = 2, /* head_dim != 128, group size above 8,
                                 ridge = 0, or a device older than sm_103a       */
   JACAP_ERR_WORKSPACE = 3,   /* workspace too small or misaligned               */
   JACAP_ERR_CUDA = 4,        /* a CUDA runtime/driver call or launch failed     */
@@ -72,7 +72,9 @@ typedef enum { JACAP_F32 = 0, JACAP_BF16 = 1 } jacap_dtype;
  *  dtype   type of K, V and Q_win (all three share it).
  *
  * Requirements (else JACAP_ERR_INVALID_ARG / _UNSUPPORTED): head_dim == 128;
- * num_q_heads % num_kv_heads == 0 with a ratio in {1,2,4,8}; window >= 1;
+ * num_q_heads % num_kv_heads == 0 with a ratio G = num_q_heads / num_kv_heads
+ * of 1 to 8 (e.g. G = 4 for Llama-3-8B, 5 for Qwen3-14B, 7 for Nemotron-7B;
+ * larger groups give JACAP_ERR_UNSUPPORTED); window >= 1;
  * every stride a multiple of 8 elements (16-byte rows) and K, V, Q_win 16-byte
  * aligned; kv_stride_token >= head_dim; num_seqs >= 1; total_tokens >= 1 and
  * < 2^31; max_seqlen >= every n_s. cu_seqlens must satisfy cu[0] = 0,
@@ -340,6 +342,49 @@ jacap_status jacap_compact_inplace(const jacap_layout* layout, void* k, void* v,
 jacap_status jacap_select_compact_inplace(const jacap_layout* layout, const float* scores, int32_t budget,
                                           int32_t* idx, int32_t* kept, void* k, void* v, int32_t* pos,
                                           int32_t preserve_order, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * Eviction of a cache held in host memory (an offloaded KV cache, Sec. 3.1):
+ * the whole pass of jacap_score + jacap_select (+ jacap_compact) on caches that
+ * stay in host memory, with the kept positions (and optionally the retained
+ * rows Z_C) written back to host memory. Unlike the other entry points it
+ * returns only when everything is done (both streams synchronised).
+ *
+ * The layers travel in groups of `group_layers` through two device buffers
+ * carved from `dev_buf`: while group g is scored, selected and compacted on
+ * `stream`, group g + 1 is copied host -> device on `copy_stream`, so the
+ * device holds at most two groups and the pass overlaps the copies.
+ *  layout       as for jacap_score, except: cu_seqlens is a HOST pointer
+ *               (copied into dev_buf), and the host arrays must be dense:
+ *               K, V [num_layers][num_kv_heads][total_tokens][128] and Q_win
+ *               [num_seqs][num_layers][num_q_heads][window][128] (strides as
+ *               those shapes give), else JACAP_ERR_INVALID_ARG.
+ *  q_win_host, k_host, v_host  host memory; page-locked (cudaHostAlloc /
+ *               cudaHostRegister) for the copies to overlap the pass.
+ *  out_factor   device, optional: the per-plane factors of jacap_score_out
+ *               (NULL: u = v).
+ *  idx_host     host int32 [num_layers][num_kv_heads][num_seqs][budget], as
+ *               jacap_select writes idx; kept_host host int32 [num_seqs].
+ *  k_out_host, v_out_host  host [num_layers][num_kv_heads][num_seqs][budget][128]
+ *               in the cache dtype, as jacap_compact writes them; both NULL to
+ *               skip the rows (positions only), else both non-NULL.
+ *  dev_buf      device memory the caller owns, 1024-byte aligned, at least
+ *               jacap_host_buffer_size() bytes; holds the two group buffers,
+ *               the workspace and the group outputs. The library allocates no
+ *               device memory; it creates and destroys four CUDA events.
+ *  copy_stream  a second stream for the host -> device copies; NULL (or equal
+ *               to `stream`) runs everything in order on `stream`.
+ * Returns the first error of the host checks, of a CUDA call, or of a group's
+ * device status word (JACAP_ERR_INVALID_ARG, _NONFINITE, _TIMEOUT as from
+ * jacap_device_status).
+ */
+size_t jacap_host_buffer_size(const jacap_layout* layout, int32_t budget, int32_t group_layers,
+                              int32_t copy_rows);
+jacap_status jacap_evict_host(const jacap_layout* layout, const jacap_params* params, int32_t budget,
+                              int32_t group_layers, const void* q_win_host, const void* k_host,
+                              const void* v_host, const float* out_factor, int32_t* idx_host,
+                              int32_t* kept_host, void* k_out_host, void* v_out_host, void* dev_buf,
+                              size_t dev_bytes, void* stream, void* copy_stream);
 
 /* Synchronises `stream`, then reads the workspace status word: JACAP_OK or the
  * first device-side error recorded since the last jacap_score on `ws`. */

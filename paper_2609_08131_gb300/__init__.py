@@ -104,6 +104,10 @@ _SIGS = {
     "jacap_select_compact_inplace": (ctypes.c_int, [ctypes.POINTER(jacap_layout), _P, ctypes.c_int32, _P, _P, _P, _P,
                                                     _P, ctypes.c_int32, _P, ctypes.c_size_t, _P]),
     "jacap_device_status": (ctypes.c_int, [_P, _P]),
+    "jacap_host_buffer_size": (ctypes.c_size_t, [ctypes.POINTER(jacap_layout), ctypes.c_int32, ctypes.c_int32,
+                                                 ctypes.c_int32]),
+    "jacap_evict_host": (ctypes.c_int, [ctypes.POINTER(jacap_layout), ctypes.POINTER(jacap_params), ctypes.c_int32,
+                                        ctypes.c_int32, _P, _P, _P, _P, _P, _P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "jacap_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "jacap_workspace_offsets": (ctypes.c_int, [ctypes.POINTER(jacap_layout), ctypes.c_int32,
                                                ctypes.POINTER(jacap_ws_offsets)]),
@@ -197,6 +201,18 @@ def jacap_select_compact(layout, scores, budget, idx, kept, k, v, k_out, v_out, 
 
 def jacap_compact(layout, k, v, idx, budget, k_out, v_out, stream) -> int:
     return lib().jacap_compact(ctypes.byref(layout), k, v, idx, budget, k_out, v_out, stream)
+
+
+def jacap_host_buffer_size(layout: jacap_layout, budget: int, group_layers: int, copy_rows: int) -> int:
+    return lib().jacap_host_buffer_size(ctypes.byref(layout), budget, group_layers, copy_rows)
+
+
+def jacap_evict_host(layout, params, budget, group_layers, q_win_host, k_host, v_host, out_factor, idx_host,
+                     kept_host, k_out_host, v_out_host, dev_buf, dev_bytes, stream, copy_stream) -> int:
+    """Host-cache eviction (``layout.cu_seqlens`` is a host pointer here); blocks until done."""
+    return lib().jacap_evict_host(ctypes.byref(layout), ctypes.byref(params), budget, group_layers, q_win_host,
+                                  k_host, v_host, out_factor, idx_host, kept_host, k_out_host, v_out_host, dev_buf,
+                                  dev_bytes, stream, copy_stream)
 
 
 def jacap_device_status(ws, stream) -> int:

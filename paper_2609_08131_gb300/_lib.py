@@ -23,7 +23,7 @@ BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libjacap.so")
 
 SOURCES = ["jacap_api.cu", "k_stream.cu", "k_kpass.cu", "k_gram.cu", "k_factor.cu", "k_score.cu", "k_select.cu",
-           "jacap_static.cu", "k_kfull.cu", "k_decode.cu"]
+           "jacap_static.cu", "k_kfull.cu", "k_decode.cu", "jacap_host.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
           "-I" + INCLUDE, "-I" + CSRC]
@@ -44,16 +44,36 @@ def _sources_mtime() -> float:
     return max(os.path.getmtime(f) for f in files)
 
 
+def build_flags() -> list:
+    """Optional build variants, from the environment of the build:
+    JACAP_NVTX=1 marks every kernel launch with an NVTX range (tracing);
+    JACAP_CHECKED=1 makes the persistent kernels validate every work-item
+    record against the cache bounds and report violations in the status word."""
+    extra = []
+    if os.environ.get("JACAP_NVTX") == "1":
+        extra.append("-DJACAP_NVTX")
+    if os.environ.get("JACAP_CHECKED") == "1":
+        extra.append("-DJACAP_CHECKED")
+    return extra
+
+
+def _stamp() -> str:
+    return " ".join(ARCH + CFLAGS + build_flags())
+
+
 def build(verbose: bool = False, force: bool = False) -> str:
     """Compile and link libjacap.so; returns its path."""
-    if not force and os.path.exists(LIB) and os.path.getmtime(LIB) >= _sources_mtime():
+    stamp_path = os.path.join(BUILD, "flags.txt")
+    same_flags = os.path.exists(stamp_path) and open(stamp_path).read() == _stamp()
+    if not force and same_flags and os.path.exists(LIB) and os.path.getmtime(LIB) >= _sources_mtime():
         return LIB
     os.makedirs(BUILD, exist_ok=True)
     cc = nvcc()
+    extra = build_flags()
 
     def compile_one(src):
         obj = os.path.join(BUILD, src.replace(".cu", ".o"))
-        cmd = [cc, *ARCH, *CFLAGS, "-c", os.path.join(CSRC, src), "-o", obj]
+        cmd = [cc, *ARCH, *CFLAGS, *extra, "-c", os.path.join(CSRC, src), "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError(f"nvcc failed for {src}:\n{r.stdout}\n{r.stderr}")
@@ -69,6 +89,8 @@ def build(verbose: bool = False, force: bool = False) -> str:
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
     os.replace(tmp, LIB)
+    with open(stamp_path, "w") as f:
+        f.write(_stamp())
     return LIB
 
 
@@ -103,4 +125,6 @@ EXPORTS = [
     "jacap_selftest_wait",
     "jacap_status_string",
     "jacap_workspace_offsets",
+    "jacap_host_buffer_size",
+    "jacap_evict_host",
 ]

@@ -17,6 +17,8 @@ from . import (
     JACAP_OK,
     jacap_compact,
     jacap_device_status,
+    jacap_evict_host,
+    jacap_host_buffer_size,
     jacap_layout,
     jacap_params,
     jacap_score,
@@ -376,28 +378,27 @@ class DecodeEvictor:
 
 
 class HostEvictor:
-    """Eviction of a cache held in pinned host memory (an offloaded cache).
+    """Eviction of a cache held in pinned host memory (an offloaded cache),
+    through ``jacap_evict_host``.
 
-    The layers go to the device in groups of ``group_layers`` through two
-    device buffers: while group g is scored, selected and compacted on the
-    compute stream, group g + 1 is copied on a copy stream, so the device never
-    holds more than two groups and the pass overlaps the host->device copies.
-    A buffer is refilled once the pass over its previous group has finished,
-    which lets the next ``run()``'s first copies overlap this one's last pass.
+    The library moves the layers to the device in groups of ``group_layers``
+    through two device buffers: while group g is scored, selected and
+    compacted on the compute stream, group g + 1 is copied on a copy stream.
+    Each ``run()`` returns when the kept positions (and, with ``copy_rows``,
+    the retained K and V rows) are in host memory.
 
-    q_win_h [S, L, Hq, w, 128], k_h and v_h [L, Hkv, N, 128]: pinned host
-    tensors (contiguous); cu_seqlens: int32 [S + 1] (host or device), fixed
-    with ``seqlens`` at construction like the layout; ``out_factor``: optional
-    float32 [L][Hkv][128][128] device tensor, as for ``Evictor``. The host
-    tensors are read while the copies execute: leave them unchanged until the
-    stream has been synchronised. After ``run()`` the device tensors
-    idx [L, Hkv, S, B], kept [S] and k_out, v_out [L, Hkv, S, B, 128] hold the
-    result and ``idx_h`` / ``kept_h`` (pinned host) the kept positions once the
-    stream is synchronised.
+    q_win_h [S, L, Hq, w, 128], k_h and v_h [L, Hkv, N, 128]: contiguous
+    tensors in pinned host memory; cu_seqlens: int32 [S + 1] (host or device),
+    fixed with ``seqlens`` at construction like the layout; ``out_factor``:
+    optional float32 [L][Hkv][128][128] device tensor, as for ``Evictor``.
+    After ``run()``: ``idx_h`` [L, Hkv, S, B], ``kept_h`` [S] and, with
+    ``copy_rows``, ``k_out_h``, ``v_out_h`` [L, Hkv, S, B, 128] (pinned host).
+    The only device memory is one buffer of ``jacap_host_buffer_size`` bytes.
     """
 
     def __init__(self, q_win_h, k_h, v_h, cu_seqlens, seqlens, num_q_heads: int, budget: int,
-                 params: jacap_params | None = None, group_layers: int = 8, device="cuda", out_factor=None):
+                 params: jacap_params | None = None, group_layers: int = 8, device="cuda", out_factor=None,
+                 copy_rows: bool = True):
         dev = torch.device(device)
         for name, t in (("q_win_h", q_win_h), ("k_h", k_h), ("v_h", v_h)):
             if t.device.type != "cpu" or not t.is_pinned() or not t.is_contiguous():
@@ -413,78 +414,45 @@ class HostEvictor:
         self.L, self.S, self.gl = L, S, max(1, min(int(group_layers), L))
         self.q_h, self.k_h, self.v_h = q_win_h, k_h, v_h
         self.budget = int(budget)
-        self.params = params
+        self.params = params if params is not None else jacap_params()
         self.num_q_heads = num_q_heads
         self.seqlens = list(seqlens)
-        self.cu = torch.as_tensor(cu_seqlens, dtype=torch.int32).to(dev)
-        gl = self.gl
-        self.kb = [torch.empty((gl, Hkv, N, d), dtype=k_h.dtype, device=dev) for _ in range(2)]
-        self.vb = [torch.empty_like(self.kb[0]) for _ in range(2)]
-        self._qrow = tuple(q_win_h.shape[2:])
-        self.qb = [torch.empty(S * gl * q_win_h[0, 0].numel(), dtype=q_win_h.dtype, device=dev) for _ in range(2)]
-        self._ev = {}  # one Evictor per buffer and group size (the last group may be shorter)
-        self.idx = torch.empty((L, Hkv, S, self.budget), dtype=torch.int32, device=dev)
-        self.kept = torch.empty((S,), dtype=torch.int32, device=dev)
-        self.k_out = torch.empty((L, Hkv, S, self.budget, d), dtype=k_h.dtype, device=dev)
-        self.v_out = torch.empty_like(self.k_out)
-        self.idx_h = torch.empty(self.idx.shape, dtype=torch.int32).pin_memory()
-        self.kept_h = torch.empty(self.kept.shape, dtype=torch.int32).pin_memory()
+        self.copy_rows = bool(copy_rows)
+        self.cu_h = torch.as_tensor(cu_seqlens, dtype=torch.int32).cpu().contiguous()
+        self.lay = Cache(q_win_h, k_h, v_h, self.cu_h, self.seqlens, num_q_heads).layout()  # cu_seqlens: host
+        nbytes = jacap_host_buffer_size(self.lay, self.budget, self.gl, 1 if self.copy_rows else 0)
+        if nbytes == 0:
+            raise JacapError(1, "jacap_host_buffer_size")
+        self.dev_buf = torch.empty(nbytes + 1024, dtype=torch.uint8, device=dev)
+        off = (-self.dev_buf.data_ptr()) % 1024
+        self.dev_buf = self.dev_buf[off:off + nbytes]
+        self.idx_h = torch.empty((L, Hkv, S, self.budget), dtype=torch.int32).pin_memory()
+        self.kept_h = torch.empty((S,), dtype=torch.int32).pin_memory()
+        self.k_out_h = self.v_out_h = None
+        if self.copy_rows:
+            self.k_out_h = torch.empty((L, Hkv, S, self.budget, d), dtype=k_h.dtype).pin_memory()
+            self.v_out_h = torch.empty_like(self.k_out_h).pin_memory()
         self.copy_stream = torch.cuda.Stream(device=dev)
-        self._done = [torch.cuda.Event(), torch.cuda.Event()]
-        self._copied = [torch.cuda.Event(), torch.cuda.Event()]
-        self._used = [False, False]
-
-    def _qview(self, b, n):
-        per = 1
-        for x in self._qrow:
-            per *= x
-        return self.qb[b][:self.S * n * per].view(self.S, n, *self._qrow)
-
-    def _evictor(self, b, n):
-        key = (b, n)
-        if key not in self._ev:
-            c = Cache(self._qview(b, n), self.kb[b][:n], self.vb[b][:n], self.cu, self.seqlens, self.num_q_heads)
-            of = None if self.out_factor is None else self.out_factor[:n]
-            self._ev[key] = Evictor(c, self.budget, self.params, out_factor=of)
-        return self._ev[key]
 
     @property
     def h2d_bytes(self) -> int:
-        """Bytes one ``run()`` copies host->device."""
+        """Bytes one ``run()`` copies host->device (the cache and its window; cu_seqlens aside)."""
         return sum(t.numel() * t.element_size() for t in (self.q_h, self.k_h, self.v_h))
 
     @property
     def d2h_bytes(self) -> int:
-        """Bytes one ``run()`` copies device->host."""
-        return (self.idx_h.numel() + self.kept_h.numel()) * 4
+        """Bytes one ``run()`` copies device->host: positions, kept counts and, with copy_rows, the rows."""
+        rows = 0 if not self.copy_rows else 2 * self.k_out_h.numel() * self.k_out_h.element_size()
+        return (self.idx_h.numel() + self.kept_h.numel()) * 4 + rows
 
     def run(self, stream=None):
-        comp = stream if stream is not None else torch.cuda.current_stream()
-        cs = self.copy_stream
-        for g, l0 in enumerate(range(0, self.L, self.gl)):
-            n = min(self.gl, self.L - l0)
-            b = g & 1
-            with torch.cuda.stream(cs):
-                if self._used[b]:
-                    cs.wait_event(self._done[b])  # the pass over the buffer's previous group is finished
-                self.kb[b][:n].copy_(self.k_h[l0:l0 + n], non_blocking=True)
-                self.vb[b][:n].copy_(self.v_h[l0:l0 + n], non_blocking=True)
-                qv = self._qview(b, n)
-                for s in range(self.S):
-                    qv[s].copy_(self.q_h[s, l0:l0 + n], non_blocking=True)
-                self._copied[b].record(cs)
-            comp.wait_event(self._copied[b])
-            ev = self._evictor(b, n)
-            ev.bind_outputs(self.idx[l0:l0 + n], self.kept, self.k_out[l0:l0 + n], self.v_out[l0:l0 + n])
-            if self.out_factor is not None:
-                ev.out_factor = self.out_factor[l0:l0 + n]
-            ev.run(comp)
-            self._done[b].record(comp)
-            self._used[b] = True
-        with torch.cuda.stream(comp):
-            self.idx_h.copy_(self.idx, non_blocking=True)
-            self.kept_h.copy_(self.kept, non_blocking=True)
+        of = _ptr(self.out_factor) if self.out_factor is not None else ctypes.c_void_p(0)
+        st = jacap_evict_host(self.lay, self.params, self.budget, self.gl, _ptr(self.q_h), _ptr(self.k_h),
+                              _ptr(self.v_h), of, _ptr(self.idx_h), _ptr(self.kept_h),
+                              _ptr(self.k_out_h), _ptr(self.v_out_h), _ptr(self.dev_buf), self.dev_buf.numel(),
+                              _stream(stream), _stream(self.copy_stream))
+        _check(st, "jacap_evict_host")
 
     def check(self, stream=None):
-        for ev in self._ev.values():
-            ev.check(stream)
+        """Errors are returned by ``run()`` itself (it raises); nothing more to read."""
+        return None

@@ -289,10 +289,28 @@ jacap_status score_pass(const jacap_layout* layout, const jacap_params* params, 
   const int64_t items = pass_items(layout, dm);
   const int dt = bf ? 1 : 0;
   const int32_t* cu = layout->cu_seqlens;
+  // hook(i): the boundary before kernel i (optional timing event; with
+  // -DJACAP_NVTX the end of kernel i-1's trace range and the start of i's)
+  static const char* const kTrace[JACAP_SCORE_KERNELS] = {"jacap/plan",  "jacap/query_stats", "jacap/k_pass",
+                                                          "jacap/weights", "jacap/gram",      "jacap/factor",
+                                                          "jacap/scores"};
+  int traced = -1;
   auto hook = [&](int i) -> jacap_status {
+    if (traced >= 0) trace_pop();
+    traced = -1;
+    if (i < JACAP_SCORE_KERNELS) {
+      trace_push(kTrace[i]);
+      traced = i;
+    }
     if (num_events == 0) return JACAP_OK;
     return map_cuda(cudaEventRecord((cudaEvent_t)events[i], s));
   };
+  struct TraceGuard {  // closes an open range on an early return
+    int& t;
+    ~TraceGuard() {
+      if (t >= 0) trace_pop();
+    }
+  } trace_guard{traced};
   if ((st = hook(0)) != JACAP_OK || (st = map_cuda(launch_plan(dm, w, cu, s))) != JACAP_OK) return st;
   if ((st = hook(1)) != JACAP_OK ||
       (st = map_cuda(running ? launch_stats_moments(dm, w, stats, counts, s)
@@ -400,6 +418,7 @@ jacap_status jacap_select_compact_inplace(const jacap_layout* layout, const floa
   const int64_t units = (int64_t)dm.L * dm.Hkv * dm.S;
   const int dt = layout->dtype == JACAP_BF16 ? 1 : 0;
   const cudaStream_t s = (cudaStream_t)stream;
+  const TraceRange trace("jacap/select_compact_inplace");
   if (!preserve_order)  // hole filling inside the selection kernel
     return map_cuda(launch_select(dm, w, layout->cu_seqlens, scores, budget, idx, kept, layout->max_seqlen,
                                   persistent_grid(units, sms, 2), s, dt, nullptr, nullptr, nullptr, nullptr, k, v,
@@ -427,6 +446,7 @@ jacap_status jacap_select(const jacap_layout* layout, const float* scores, int32
   if ((st = check_device(&sms)) != JACAP_OK) return st;
   const Ws w = make_ws(ws, c);
   const int64_t units = (int64_t)dm.L * dm.Hkv * dm.S;
+  const TraceRange trace("jacap/select");
   return map_cuda(launch_select(dm, w, layout->cu_seqlens, scores, budget, idx, kept, layout->max_seqlen,
                                 persistent_grid(units, sms, 2), (cudaStream_t)stream));
 }
@@ -450,6 +470,7 @@ jacap_status jacap_select_compact(const jacap_layout* layout, const float* score
   if ((st = check_device(&sms)) != JACAP_OK) return st;
   const Ws w = make_ws(ws, c);
   const int64_t units = (int64_t)dm.L * dm.Hkv * dm.S;
+  const TraceRange trace("jacap/select_compact");
   return map_cuda(launch_select(dm, w, layout->cu_seqlens, scores, budget, idx, kept, layout->max_seqlen,
                                 persistent_grid(units, sms, 2), (cudaStream_t)stream,
                                 layout->dtype == JACAP_BF16 ? 1 : 0, k, v, k_out, v_out));
@@ -467,6 +488,7 @@ jacap_status jacap_compact(const jacap_layout* layout, const void* k, const void
   if ((st = check_device(&sms)) != JACAP_OK) return st;
   Dims dm;
   make_dims(layout, nullptr, dm);
+  const TraceRange trace("jacap/compact");
   return map_cuda(launch_compact(dm, layout->dtype == JACAP_BF16 ? 1 : 0, layout->cu_seqlens, k, v, idx, budget,
                                  k_out, v_out, (cudaStream_t)stream));
 }

@@ -99,7 +99,18 @@ struct ItemStream {
   int64_t i, end;
   int ctot;
   int4 rec;
+#ifdef JACAP_CHECKED
+  int64_t ntot;
+  int nseq, nplanes;
+  uint32_t* status;
+#endif
   __device__ __forceinline__ ItemStream(const Dims& dm, const Ws& ws, int64_t part, int64_t parts) : tab(ws.chunks) {
+#ifdef JACAP_CHECKED
+    ntot = dm.Ntot;
+    nseq = dm.S;
+    nplanes = dm.L * dm.Hkv;
+    status = ws.status;
+#endif
     ctot = ws.plan[0];
     const int64_t total = (int64_t)dm.L * dm.Hkv * ctot;
     i = part * total / parts;
@@ -113,6 +124,16 @@ struct ItemStream {
     it.t1 = rec.y;
     it.seq = rec.z;
     it.cidx = rec.w;
+#ifdef JACAP_CHECKED
+    // checked build: a record outside the cache ends this CTA's items and is
+    // reported (ST_INVALID) instead of being streamed
+    if (it.t0 < 0 || it.t1 <= it.t0 || it.t1 > ntot || it.seq < 0 || it.seq >= nseq || it.cidx < 0 ||
+        it.cidx >= ctot || it.plane >= nplanes) {
+      atomicOr(status, 1u);
+      i = end;
+      return false;
+    }
+#endif
     ++i;
     if (i < end) rec = tab[i % ctot];
     return true;

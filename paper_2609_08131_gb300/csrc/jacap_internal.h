@@ -7,6 +7,25 @@
 
 namespace jacap {
 
+// Tracing: built with -DJACAP_NVTX (JACAP_NVTX=1 in the environment of the
+// build), the host side marks each kernel's launch with an NVTX range named
+// "jacap/<step>" so a profiler timeline groups the GPU work by step of the
+// pass; otherwise the ranges compile to nothing.
+#ifdef JACAP_NVTX
+#include <nvtx3/nvToolsExt.h>
+inline void trace_push(const char* name) { nvtxRangePushA(name); }
+inline void trace_pop() { nvtxRangePop(); }
+#else
+inline void trace_push(const char*) {}
+inline void trace_pop() {}
+#endif
+struct TraceRange {
+  explicit TraceRange(const char* name) { trace_push(name); }
+  ~TraceRange() { trace_pop(); }
+  TraceRange(const TraceRange&) = delete;
+  TraceRange& operator=(const TraceRange&) = delete;
+};
+
 // Returns a failed CUDA call's error from the enclosing launcher.
 #define JACAP_TRY(call)                     \
   do {                                      \

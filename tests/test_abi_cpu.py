@@ -145,3 +145,43 @@ def test_workspace_offsets_are_inside_the_workspace():
 def test_python_binding_names_match_the_c_abi():
     for name in _lib.EXPORTS:
         assert callable(getattr(J, name))
+
+
+def test_host_cache_entry_checks_on_the_host():
+    # jacap_evict_host: dense host layouts only; every refusal comes before any
+    # CUDA call (the buffer size query needs no GPU either)
+    lay = good_layout()
+    p = ctypes.c_void_p(0x1000)
+    null = ctypes.c_void_p(0)
+    prm = J.jacap_params()
+    with_rows = J.jacap_host_buffer_size(lay, 8, 1, 1)
+    no_rows = J.jacap_host_buffer_size(lay, 8, 1, 0)
+    one_layer = good_layout(num_layers=1, kv_stride_layer=2 * 500 * 128, q_stride_seq=8 * 16 * 128)
+    assert with_rows > no_rows > J.jacap_workspace_size(one_layer, 8) > 0  # a group's workspace + buffers
+    assert J.jacap_host_buffer_size(lay, 8, 2, 1) > with_rows  # two layers per group buffer
+    assert J.jacap_host_buffer_size(lay, 8, 1, 2) == 0
+    assert J.jacap_host_buffer_size(lay, 0, 1, 1) == 0
+    padded = good_layout(kv_stride_token=136)  # a valid device layout, but not a dense host array
+    assert J.jacap_workspace_size(padded, 8) > 0 and J.jacap_host_buffer_size(padded, 8, 1, 1) == 0
+    args = lambda lay, b, gl, q, k_out, v_out, buf, nbytes: J.jacap_evict_host(  # noqa: E731
+        lay, prm, b, gl, q, p, p, null, p, p, k_out, v_out, buf, nbytes, null, null)
+    assert args(padded, 8, 1, p, p, p, p, 1 << 40) == J.JACAP_ERR_INVALID_ARG
+    assert args(good_layout(num_q_heads=32), 8, 1, p, p, p, p, 1 << 40) == J.JACAP_ERR_UNSUPPORTED  # G = 16
+    assert args(good_layout(head_dim=64), 8, 1, p, p, p, p, 1 << 40) == J.JACAP_ERR_UNSUPPORTED
+    assert args(lay, 8, 1, null, p, p, p, 1 << 40) == J.JACAP_ERR_INVALID_ARG  # no window
+    assert args(lay, 8, 1, p, p, null, p, 1 << 40) == J.JACAP_ERR_INVALID_ARG  # rows: both or neither
+    assert args(lay, 8, 0, p, p, p, p, 1 << 40) == J.JACAP_ERR_INVALID_ARG
+    assert args(lay, 8, 1, p, p, p, p, with_rows - 1) == J.JACAP_ERR_WORKSPACE
+    assert args(lay, 8, 1, p, p, p, ctypes.c_void_p(0x1100), 1 << 40) == J.JACAP_ERR_WORKSPACE  # 256-B aligned
+
+
+def test_tracing_and_checked_variants_compile(tmp_path):
+    # JACAP_NVTX=1 / JACAP_CHECKED=1 builds: the host side with its NVTX ranges
+    # and a persistent kernel with the checked work-item stream compile for sm_103a
+    import subprocess
+
+    for src in ("jacap_api.cu", "k_stream.cu"):
+        cmd = [_lib.nvcc(), *_lib.ARCH, *_lib.CFLAGS, "-DJACAP_NVTX", "-DJACAP_CHECKED", "-c",
+               os.path.join(_lib.CSRC, src), "-o", str(tmp_path / (src + ".o"))]
+        r = subprocess.run(cmd, capture_output=True, text=True)
+        assert r.returncode == 0, r.stderr[-2000:]

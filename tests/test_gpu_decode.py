@@ -11,6 +11,8 @@ running statistics with numpy moments of the history, and the eviction steps
 with ``decode_run``'s schedule.
 """
 
+import ctypes
+
 import numpy as np
 import pytest
 import torch
@@ -18,7 +20,7 @@ import torch
 from oracle import JacapParams, oracle_unit
 from oracle.decode_oracle import decode_run
 from paper_2609_08131_gb300 import jacap_params
-from paper_2609_08131_gb300.api import DecodeEvictor
+from paper_2609_08131_gb300.api import Cache, DecodeEvictor, Evictor
 from paper_2609_08131_gb300.workloads import Workload, generate
 
 from parity import assert_rows_bitwise, assert_scores_close, assert_selection
@@ -38,7 +40,7 @@ CASES = {
     "bf16_gqa8_long_slot": (1, 8, 1, (700,), 16, 40, 512, 200, "bf16", jacap_params(), 34, False),
     "bf16_gqa8_long_slot_ordered": (1, 8, 1, (700,), 16, 40, 512, 200, "bf16", jacap_params(), 34, True),
     # Nemotron-7B's heads (28 q / 4 kv, G = 7), the paper's decoding-stage model
-    "bf16_gqa7_nemotron_heads": (2, 28, 4, (60, 45), 8, 60, 40, 16, "bf16", jacap_params(), 35, False),
+    "bf16_gqa7_nemotron_heads": (2, 28, 4, (50, 45), 8, 60, 40, 16, "bf16", jacap_params(), 35, False),
     "f32_gqa5_ordered": (1, 10, 2, (30,), 4, 25, 24, 8, "f32", jacap_params(tau=2.0), 36, True),
 }
 
@@ -150,8 +152,9 @@ def test_compaction_refuses_positions_that_do_not_ascend():
 
 
 def test_host_evictor_matches_the_oracle():
-    # a cache in pinned host memory, evicted in layer groups of 2 through two
-    # device buffers (the groups' copies overlap the previous group's pass)
+    # a cache in pinned host memory, evicted through jacap_evict_host in layer
+    # groups of 2 through two device buffers (the groups' copies overlap the
+    # previous group's pass); positions and retained rows come back to the host
     from oracle import JacapParams as JP
     from paper_2609_08131_gb300.api import HostEvictor
     from paper_2609_08131_gb300.workloads import unit_arrays
@@ -161,13 +164,18 @@ def test_host_evictor_matches_the_oracle():
     he = HostEvictor(t.q_win.cpu().pin_memory(), t.k.cpu().pin_memory(), t.v.cpu().pin_memory(),
                      t.cu_seqlens, list(wl.seqlens), wl.num_q_heads, wl.budget, jacap_params(),
                      group_layers=2, device=DEV)
-    for _ in range(2):  # the second run reuses the buffers
+    first = None
+    for _ in range(2):  # the second run reuses the buffers and must repeat the first bit for bit
+        he.idx_h.fill_(-7)
+        he.k_out_h.fill_(3)
         he.run()
-        torch.cuda.synchronize()
-        he.check()
+        if first is None:
+            first = (he.idx_h.clone(), he.k_out_h.clone(), he.v_out_h.clone())
+    assert torch.equal(first[0], he.idx_h)
+    assert_rows_bitwise(first[1], he.k_out_h)
+    assert_rows_bitwise(first[2], he.v_out_h)
     cu = t.cu_seqlens.cpu().tolist()
     assert he.kept_h.tolist() == [min(n, wl.budget) for n in wl.seqlens]
-    assert torch.equal(he.idx_h, he.idx.cpu())
     for layer in range(wl.num_layers):
         for g in range(wl.num_kv_heads):
             for s in range(len(wl.seqlens)):
@@ -176,9 +184,35 @@ def test_host_evictor_matches_the_oracle():
                 gidx = he.idx_h[layer, g, s].numpy()
                 assert_selection(gidx, cu[s + 1] - cu[s], wl.budget, ora["scores"], ora["idx"])
                 kept = min(cu[s + 1] - cu[s], wl.budget)
-                sel = torch.as_tensor(gidx[:kept], dtype=torch.long, device=DEV)
-                assert_rows_bitwise(t.k[layer, g, cu[s]:cu[s + 1]][sel], he.k_out[layer, g, s, :kept])
-                assert_rows_bitwise(t.v[layer, g, cu[s]:cu[s + 1]][sel], he.v_out[layer, g, s, :kept])
+                sel = torch.as_tensor(gidx[:kept], dtype=torch.long)
+                assert_rows_bitwise(t.k[layer, g, cu[s]:cu[s + 1]].cpu()[sel], he.k_out_h[layer, g, s, :kept])
+                assert_rows_bitwise(t.v[layer, g, cu[s]:cu[s + 1]].cpu()[sel], he.v_out_h[layer, g, s, :kept])
+                assert bool((he.k_out_h[layer, g, s, kept:] == 0).all())
+
+
+def test_host_evictor_positions_only_on_one_stream():
+    # copy_rows off and a single stream (no copy stream): positions only, in order
+    from paper_2609_08131_gb300 import jacap_evict_host
+    from paper_2609_08131_gb300.api import HostEvictor, _ptr, _stream
+
+    wl = Workload("host cache", 3, 12, 2, (500, 77, 640), 8, 48, seed=42)
+    t = generate(wl, DEV)
+    he = HostEvictor(t.q_win.cpu().pin_memory(), t.k.cpu().pin_memory(), t.v.cpu().pin_memory(),
+                     t.cu_seqlens, list(wl.seqlens), wl.num_q_heads, wl.budget, jacap_params(tau=2.0),
+                     group_layers=2, device=DEV, copy_rows=False)
+    assert he.d2h_bytes == (he.idx_h.numel() + he.kept_h.numel()) * 4
+    he.run()
+    two = he.idx_h.clone()
+    st = jacap_evict_host(he.lay, he.params, he.budget, he.gl, _ptr(he.q_h), _ptr(he.k_h), _ptr(he.v_h),
+                          ctypes.c_void_p(0), _ptr(he.idx_h), _ptr(he.kept_h), ctypes.c_void_p(0),
+                          ctypes.c_void_p(0), _ptr(he.dev_buf), he.dev_buf.numel(), _stream(), ctypes.c_void_p(0))
+    assert st == 0
+    assert torch.equal(two, he.idx_h)
+    dev = Evictor(Cache(t.q_win, t.k, t.v, t.cu_seqlens, t.seqlens, wl.num_q_heads), wl.budget,
+                  jacap_params(tau=2.0))
+    dev.run()
+    a, b = he.idx_h.reshape(-1, wl.budget).numpy(), dev.idx.cpu().reshape(-1, wl.budget).numpy()
+    assert sum(len(np.setdiff1d(x, y)) for x, y in zip(a, b)) <= 2
 
 
 def test_many_slots_fill_their_holes_with_the_small_selection_ctas():

@@ -19,6 +19,7 @@ from paper_2609_08131_gb300 import jacap_params
 from paper_2609_08131_gb300.api import Cache, Evictor, evict
 from paper_2609_08131_gb300.workloads import Workload, config, generate, unit_arrays
 
+from oracle_pool import run_units
 from parity import assert_rows_bitwise, assert_scores_close, assert_selection, gpu_selection_properties
 
 pytestmark = pytest.mark.gpu
@@ -258,26 +259,59 @@ def test_config1_every_unit():
     gpu_selection_properties(ev.scores, ev.idx, ev.kept, wl.seqlens, wl.budget)
 
 
-def _sample_units(wl, count):
-    S = len(wl.seqlens)
-    cands = [(0, 0, 0), (S - 1, wl.num_layers - 1, wl.num_kv_heads - 1),
-             (S // 2, wl.num_layers // 2, wl.num_kv_heads // 2), (S // 3, 7 % wl.num_layers, 3 % wl.num_kv_heads)]
+def _spread_units(wl, count):
+    """`count` units (request, layer, KV head): the first and the last layer and
+    KV head, the shortest and the longest request, the rest drawn with a fixed
+    seed."""
+    S, L, H = len(wl.seqlens), wl.num_layers, wl.num_kv_heads
     out = []
-    for c in cands:
-        if c not in out:
-            out.append(c)
+
+    def add(u):
+        if u not in out:
+            out.append(u)
+
+    for s in dict.fromkeys([int(np.argmin(wl.seqlens)), int(np.argmax(wl.seqlens)), 0, S - 1]):
+        add((s, 0, 0))
+        add((s, L - 1, H - 1))
+    add((0, 0, H - 1))
+    add((0, L - 1, 0))
+    r = np.random.default_rng(1000 + S * 100 + L)
+    while len(out) < count:
+        add((int(r.integers(S)), int(r.integers(L)), int(r.integers(H))))
     return out[:count]
 
 
-@pytest.mark.parametrize("index,samples", [(2, 3), (3, 2), (4, 2), (5, 3)])
+def _check_sampled_units(t, wl, evs, units):
+    """Scores, TOP-B sets (for every evictor's budget) and kept rows of `units`
+    against the oracle, run on a pool of processes."""
+    budgets = sorted({e.budget for e in evs})
+    arrays = [tuple(x.astype(np.float32) for x in unit_arrays(t, wl.num_q_heads, s, layer, g))
+              for (s, layer, g) in units]
+    results = run_units(arrays, budgets)
+    cu = t.cu_seqlens.cpu().tolist()
+    for (s, layer, g), (ora_scores, ora_idx) in zip(units, results):
+        a, b = cu[s], cu[s + 1]
+        gs = evs[0].scores[layer, g, a:b].double().cpu().numpy()
+        assert_scores_close(gs, ora_scores, f"scores of unit {(s, layer, g)}")
+        for ev in evs:
+            gidx = ev.idx[layer, g, s].cpu().numpy()
+            assert_selection(gidx, b - a, ev.budget, ora_scores, ora_idx[ev.budget])
+            kept = min(b - a, ev.budget)
+            sel = torch.as_tensor(gidx[:kept], dtype=torch.long, device=t.k.device)
+            assert_rows_bitwise(t.k[layer, g, a:b][sel], ev.k_out[layer, g, s, :kept])
+            assert_rows_bitwise(t.v[layer, g, a:b][sel], ev.v_out[layer, g, s, :kept])
+
+
+@pytest.mark.parametrize("index,samples", [(2, 8), (3, 8), (4, 16), (5, 16)])
 def test_full_size_config(index, samples):
     wl = config(index)
     t = generate(wl, DEV)
     ev = evict(make_cache(t, wl), wl.budget)
     gpu_selection_properties(ev.scores, ev.idx, ev.kept, wl.seqlens, wl.budget)
-    for (s, layer, g) in _sample_units(wl, samples):
-        check_unit(ev, t, wl, jacap_params(), s, layer, g, check_w=False)
+    evs = [ev]
     if index == 2:
+        # the other two budgets of the configuration: selection (and compaction)
+        # on the same scores, as separate calls and as the fused call
         for b in (128, 2048):
             ev2 = Evictor(make_cache(t, wl), b)
             ev2.scores.copy_(ev.scores)
@@ -290,7 +324,9 @@ def test_full_size_config(index, samples):
             assert_rows_bitwise(k2, ev2.k_out)
             assert_rows_bitwise(v2, ev2.v_out)
             del k2, v2
-    del ev, t
+            evs.append(ev2)
+    _check_sampled_units(t, wl, evs, _spread_units(wl, samples))
+    del ev, evs, t
     torch.cuda.empty_cache()
 
 
@@ -395,14 +431,12 @@ def test_host_cache_pass_with_output_directions_matches_the_device_pass():
                      list(wl.seqlens), wl.num_q_heads, wl.budget, jacap_params(), group_layers=2, device=DEV,
                      out_factor=F)
     he.run()
-    torch.cuda.synchronize()
-    he.check()
-    a, b = he.idx.cpu().reshape(-1, wl.budget).numpy(), dev.idx.cpu().reshape(-1, wl.budget).numpy()
+    a, b = he.idx_h.reshape(-1, wl.budget).numpy(), dev.idx.cpu().reshape(-1, wl.budget).numpy()
     differ = sum(len(np.setdiff1d(x, y)) for x, y in zip(a, b))
     assert differ <= 2, differ
     if differ == 0:
-        assert_rows_bitwise(dev.k_out, he.k_out)
-        assert_rows_bitwise(dev.v_out, he.v_out)
+        assert_rows_bitwise(dev.k_out, he.k_out_h)
+        assert_rows_bitwise(dev.v_out, he.v_out_h)
 
 
 def test_many_short_units_take_the_small_selection_ctas():
