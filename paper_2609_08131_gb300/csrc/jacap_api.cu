@@ -58,11 +58,14 @@ jacap_status check_layout(const jacap_layout* L) {
 // per CTA differ by one item at most: with ~27 items per CTA on 152 SMs the
 // last item costs under 4 % of a pass. Items of one unit that follow each
 // other in a CTA's range share one partial Gram and one factor image.
+#ifndef JACAP_TARGET_ITEMS
+#define JACAP_TARGET_ITEMS 4096
+#endif
 int pick_chunk(const jacap_layout* L) {
   const int64_t planes = (int64_t)L->num_layers * L->num_kv_heads;
   for (int c = 16384; c > TILE; c >>= 1) {
     const int64_t items = planes * (L->total_tokens / c + L->num_seqs);
-    if (items >= 4096) return c;
+    if (items >= JACAP_TARGET_ITEMS) return c;
   }
   return TILE;
 }
