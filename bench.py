@@ -60,6 +60,8 @@ def parse():
                    help="head layout of the decoding benchmark: Nemotron-7B (28 layers, 28 query / 4 KV heads, "
                         "the paper's decoding-stage model) or Llama-3-8B (32 layers, 32 / 8)")
     p.add_argument("--interval", type=int, default=128, help="decoding-stage eviction interval (tokens)")
+    p.add_argument("--decode-requests", type=int, default=1,
+                   help="decoding-stage eviction: requests whose slots fill on the same step (one pass for all)")
     p.add_argument("--preserve-order", action="store_true",
                    help="decoding-stage eviction: compact to ascending slot order instead of filling the holes")
     p.add_argument("--e2e-steps", type=int, default=10)
@@ -699,24 +701,36 @@ def run_decode(args):
 
     dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", "0")))
     torch.cuda.set_device(dev)
-    B, D = args.decode, args.interval
+    B, D, S = args.decode, args.interval, max(1, args.decode_requests)
     cap = B + D
     # Nemotron-7B: 28 layers, 28 query / 4 KV heads (G = 7), head_dim 128
     L, Hq, Hkv, w = (28, 28, 4, 32) if args.decode_model == "nemotron-7b" else (32, 32, 8, 32)
     shape = "Nemotron-7B-shaped" if args.decode_model == "nemotron-7b" else "Llama-3-8B-shaped"
-    wl = Workload(f"decoding-stage eviction, {shape}, reserved tokens B={B}, interval {D}", L, Hq, Hkv,
-                  (cap,), w + 1, B, seed=40)
+    wl = Workload(f"decoding-stage eviction, {shape}, reserved tokens B={B}, interval {D}, {S} request(s) "
+                  "filling together", L, Hq, Hkv, (cap,) * S, w + 1, B, seed=40)
     t = generate(wl, dev)
-    ev = DecodeEvictor(1, L, Hq, Hkv, B, D, dtype=t.k.dtype, params=jacap_params(), device=dev,
+    ev = DecodeEvictor(S, L, Hq, Hkv, B, D, dtype=t.k.dtype, params=jacap_params(), device=dev,
                        preserve_order=args.preserve_order)
-    ev.start(t.k[:, :, :cap - 1].unsqueeze(0), t.v[:, :, :cap - 1].unsqueeze(0),
-             t.q_win[:, :, :, :w].contiguous(), [cap - 1])
+    kk = t.k.view(L, Hkv, S, cap, 128).permute(2, 0, 1, 3, 4)
+    vv = t.v.view(L, Hkv, S, cap, 128).permute(2, 0, 1, 3, 4)
+    ev.start(kk[:, :, :, :cap - 1], vv[:, :, :, :cap - 1], t.q_win[:, :, :, :w].contiguous(), [cap - 1] * S)
     q_new = t.q_win[:, :, :, w].contiguous()
-    ev.append(t.k[:, :, cap - 1].unsqueeze(0), t.v[:, :, cap - 1].unsqueeze(0), q_new)
+    ev.append(kk[:, :, :, cap - 1], vv[:, :, :, cap - 1], q_new)
     stream = torch.cuda.current_stream(dev)
+    everyone = list(range(S))
+
+    def refill():
+        ev.lengths = [cap] * S
+
+    def event(events=None, tail=None):  # all S slots in one pass
+        refill()
+        if S == 1:
+            ev.evict(0, events=events, tail=tail)
+        else:
+            ev._evict_group(0, S, None, events, tail)
+
     for _ in range(max(3, args.warmup)):
-        ev.lengths[0] = cap
-        ev.evict(0)
+        event()
     ev.check()
     K = args.steps
     nk = len(SCORE_KERNEL_NAMES)
@@ -731,16 +745,14 @@ def run_decode(args):
     # their launch while the previous one runs) ...
     start.record(stream)
     for i in range(K):
-        ev.lengths[0] = cap
-        ev.evict(0)
+        event()
     stop.record(stream)
     torch.cuda.synchronize()
     t_ms = start.elapsed_time(stop) / K
     # ... and again with an event between kernels for the breakdown
     start.record(stream)
     for i in range(K):
-        ev.lengths[0] = cap
-        ev.evict(0, events=evs[i][:nk + 1], tail=evs[i][nk + 1:])
+        event(events=evs[i][:nk + 1], tail=evs[i][nk + 1:])
     stop.record(stream)
     torch.cuda.synchronize()
     t_ms_events = start.elapsed_time(stop) / K
@@ -758,11 +770,11 @@ def run_decode(args):
     b.record(stream)
     torch.cuda.synchronize()
     upd_us = a.elapsed_time(b) / M * 1e3
-    kv_bytes = 2 * L * Hkv * cap * 128 * t.k.element_size()
+    kv_bytes = 2 * L * Hkv * S * cap * 128 * t.k.element_size()
     line = {
         "mode": "decode",
         "metric": "decoding-stage eviction: cached tokens x layers scored per second (1 GB300)",
-        "value": cap * L / (t_ms * 1e-3),
+        "value": S * cap * L / (t_ms * 1e-3),
         "unit": "tokens/s",
         "ms_per_event": t_ms,
         "ms_per_event_with_kernel_events": t_ms_events,
@@ -773,7 +785,8 @@ def run_decode(args):
         "dtype": "bf16",
         "data": "synthetic",
         "config": {"workload": wl.name, "layers": L, "q_heads": Hq, "kv_heads": Hkv, "head_dim": 128,
-                   "slot_tokens": cap, "budget": B, "interval": D, "statistics": "running, all queries seen",
+                   "requests": S, "slot_tokens": cap, "budget": B, "interval": D,
+                   "statistics": "running, all queries seen",
                    "compaction": "ascending order" if args.preserve_order else "hole filling",
                    "l2": f"inputs larger than L2: each event reads K and V of the slot ({kv_bytes / 1e6:.0f} MB)"},
         "kernel_ms": kern,

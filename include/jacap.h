@@ -307,8 +307,14 @@ jacap_status jacap_score_stats(const jacap_layout* layout, const jacap_params* p
  * bit, in rows 0 .. kept - 1 of the request's token range; rows from kept on
  * are left as they were (free for the next tokens). kept = min(n_s, budget).
  *  k, v  device, the layout; written in place.
- *  pos   device int32 [num_layers][num_kv_heads][total_tokens] or NULL: a
- *        per-token tag (e.g. the original position) moved with the rows.
+ *  pos   device int32 or NULL: a per-token tag (e.g. the original position)
+ *        moved with the rows, laid out like K with one int32 per token row:
+ *        tag (l, g, t) at l*(kv_stride_layer/kv_stride_token)
+ *        + g*(kv_stride_head/kv_stride_token) + t. For a dense K
+ *        [num_layers][num_kv_heads][total_tokens][128] that is a dense
+ *        [num_layers][num_kv_heads][total_tokens]; with pos the layer and head
+ *        strides must be multiples of the token stride (else
+ *        JACAP_ERR_INVALID_ARG).
  *  preserve_order
  *        1: row r receives idx[r] (ascending order, as jacap_compact); up to
  *           `kept` rows move, in chunks that are read whole before any row of

@@ -226,17 +226,22 @@ class DecodeEvictor:
     with those statistics and compacted in place back to ``budget`` tokens
     (by default by moving the kept rows from past the budget into the evicted
     rows, so the slot order is not the token order; ``pos`` records it).
+    Requests that fill on the same decode step and sit next to each other are
+    evicted together in one pass (one launch of each kernel for all of them).
 
-    Buffers (device):
-      k, v    [S, L, Hkv, cap, 128], cap = budget + interval; request s holds
-              its ``lengths[s]`` tokens in rows 0 .. lengths[s] - 1
-      pos     int32 [S, L, Hkv, cap]: the id of every cached token (the
+    Buffers (device), stored [L, Hkv, S, cap(, 128)] so that neighbouring
+    requests form one cache layout, exposed request-major:
+      k, v    [S, L, Hkv, cap, 128] views, cap = budget + interval; request s
+              holds its ``lengths[s]`` tokens in rows 0 .. lengths[s] - 1
+      pos     int32 [S, L, Hkv, cap] view: the id of every cached token (the
               prefill tokens are 0 .. n0 - 1, decode step t of a request adds
               n0 + t); it moves with the rows
       stats   float32 [S, L, Hq, 2, 128] (mean, M2), counts int32 [S, L, Hq]
+    After an eviction of requests a .. b - 1, ``scores`` [L, Hkv, (b - a) cap]
+    and ``idx`` [L, Hkv, b - a, budget] hold that pass's scores and positions.
     Writing a decode step's k, v into the slot is the model's cache write (a
-    plain copy here); the statistics, the scoring pass, the selection and the
-    compaction run in libjacap's kernels.
+    plain indexed copy here); the statistics, the scoring pass, the selection
+    and the compaction run in libjacap's kernels.
     """
 
     def __init__(self, num_seqs: int, num_layers: int, num_q_heads: int, num_kv_heads: int, budget: int,
@@ -258,40 +263,62 @@ class DecodeEvictor:
         self.preserve_order = bool(preserve_order)
         dev = torch.device(device)
         S, L, Hq, Hkv, cap, d = self.S, self.L, self.Hq, self.Hkv, self.cap, 128
-        self.k = torch.zeros((S, L, Hkv, cap, d), dtype=dtype, device=dev)
-        self.v = torch.zeros_like(self.k)
-        self.pos = torch.full((S, L, Hkv, cap), -1, dtype=torch.int32, device=dev)
+        self._k = torch.zeros((L, Hkv, S, cap, d), dtype=dtype, device=dev)
+        self._v = torch.zeros_like(self._k)
+        self._pos = torch.full((L, Hkv, S, cap), -1, dtype=torch.int32, device=dev)
+        self.k = self._k.permute(2, 0, 1, 3, 4)
+        self.v = self._v.permute(2, 0, 1, 3, 4)
+        self.pos = self._pos.permute(2, 0, 1, 3)
         self.stats = torch.zeros((S, L, Hq, 2, d), dtype=torch.float32, device=dev)
         self.counts = torch.zeros((S, L, Hq), dtype=torch.int32, device=dev)
         self.lengths = [0] * S
         self.next_id = [0] * S
-        self.events = 0
-        self.cu = torch.tensor([0, cap], dtype=torch.int32, device=dev)
+        self.events = 0   # request evictions
+        self.passes = 0   # scoring passes (one per group of neighbouring requests)
+        self.cu = torch.arange(0, (S + 1) * cap, cap, dtype=torch.int32, device=dev)
+        self._layouts = {}
         # one request's slot as a cache of cap tokens
-        self.slot = self._layout(1, window=1, q_strides=(d, d, d, d))
+        self.slot = self._group_layout(1)
         # one query per (request, layer, head), [S, L, Hq, 128] contiguous
         self.step_layout = self._layout(S, window=1, q_strides=(L * Hq * d, Hq * d, d, d))
-        nbytes = jacap_workspace_size(self.slot, self.budget)
-        if nbytes == 0:
+        # one workspace serves every group size (the work-item size depends on it)
+        sizes = [jacap_workspace_size(self._group_layout(n), self.budget) for n in range(1, S + 1)]
+        if min(sizes) == 0:
             raise JacapError(1, "jacap_workspace_size")
+        nbytes = max(sizes)
         self.ws = torch.empty(nbytes, dtype=torch.uint8, device=dev)
-        self.scores = torch.empty((L, Hkv, cap), dtype=torch.float32, device=dev)
-        self.idx = torch.empty((L, Hkv, 1, self.budget), dtype=torch.int32, device=dev)
-        self.kept = torch.empty((1,), dtype=torch.int32, device=dev)
+        self._scores = torch.empty(L * Hkv * S * cap, dtype=torch.float32, device=dev)
+        self._idx = torch.empty(L * Hkv * S * self.budget, dtype=torch.int32, device=dev)
+        self._kept = torch.empty((S,), dtype=torch.int32, device=dev)
+        self._views(1)
+
+    def _views(self, n):
+        L, Hkv = self.L, self.Hkv
+        self.scores = self._scores[:L * Hkv * n * self.cap].view(L, Hkv, n * self.cap)
+        self.idx = self._idx[:L * Hkv * n * self.budget].view(L, Hkv, n, self.budget)
+        self.kept = self._kept[:n]
 
     def _layout(self, num_seqs, window, q_strides) -> jacap_layout:
         lay = jacap_layout()
         lay.num_seqs = num_seqs
         lay.cu_seqlens = self.cu.data_ptr()
         lay.max_seqlen = self.cap
-        lay.total_tokens = self.cap
+        lay.total_tokens = num_seqs * self.cap
         lay.num_layers, lay.num_q_heads, lay.num_kv_heads, lay.head_dim = self.L, self.Hq, self.Hkv, 128
         lay.window = window
         lay.dtype = JACAP_BF16 if self.dtype == torch.bfloat16 else JACAP_F32
-        st = self.k.stride()
-        lay.kv_stride_layer, lay.kv_stride_head, lay.kv_stride_token = st[1], st[2], st[3]
+        st = self._k.stride()  # [L, Hkv, S, cap, 128]
+        lay.kv_stride_layer, lay.kv_stride_head, lay.kv_stride_token = st[0], st[1], st[3]
         lay.q_stride_seq, lay.q_stride_layer, lay.q_stride_head, lay.q_stride_pos = q_strides
         return lay
+
+    def _group_layout(self, n) -> jacap_layout:
+        """n neighbouring requests' slots as one cache: request j of the group is
+        tokens j cap .. (j + 1) cap - 1 (the storage puts them next to each
+        other on the token axis of every (layer, KV head) plane)."""
+        if n not in self._layouts:
+            self._layouts[n] = self._layout(n, window=1, q_strides=(128, 128, 128, 128))
+        return self._layouts[n]
 
     def _merge(self, q, reset: bool, stream=None):
         """q: [S, L, Hq, m, 128] queries (the slot dtype, channel contiguous)."""
@@ -321,15 +348,19 @@ class DecodeEvictor:
         """One decode step for every request: k_new, v_new [S, L, Hkv, 128],
         q_new [S, L, Hq, 128]. Returns the requests whose cache is now full
         (each must be evicted before its next append)."""
-        for s in range(self.S):
-            if self.lengths[s] >= self.cap:
-                raise RuntimeError(f"request {s} is full; evict it first")
-            t = self.lengths[s]
-            self.k[s, :, :, t].copy_(k_new[s])
-            self.v[s, :, :, t].copy_(v_new[s])
-            self.pos[s, :, :, t] = self.next_id[s]
-            self.lengths[s] += 1
-            self.next_id[s] += 1
+        full = [s for s in range(self.S) if self.lengths[s] >= self.cap]
+        if full:
+            raise RuntimeError(f"request {full[0]} is full; evict it first")
+        dev = self._k.device
+        rows = torch.tensor(self.lengths, dtype=torch.long, device=dev)
+        reqs = torch.arange(self.S, device=dev)
+        # one indexed copy per tensor for all requests (each writes its next free row)
+        self._k[:, :, reqs, rows] = k_new.permute(1, 2, 0, 3).to(self.dtype)
+        self._v[:, :, reqs, rows] = v_new.permute(1, 2, 0, 3).to(self.dtype)
+        ids = torch.tensor(self.next_id, dtype=torch.int32, device=dev)
+        self._pos[:, :, reqs, rows] = ids.view(1, 1, self.S).expand(self.L, self.Hkv, self.S)
+        self.lengths = [n + 1 for n in self.lengths]
+        self.next_id = [n + 1 for n in self.next_id]
         self.merge_queries(q_new, stream)
         return [s for s in range(self.S) if self.lengths[s] >= self.cap]
 
@@ -347,15 +378,31 @@ class DecodeEvictor:
         ``events``: JACAP_SCORE_KERNELS + 1 torch.cuda.Event recorded around
         the scoring kernels; ``tail``: one more, recorded after the selection
         with its in-place compaction (one launch)."""
-        if self.lengths[s] != self.cap:
-            raise RuntimeError("only a full slot is evicted")
-        lay, st = self.slot, _stream(stream)
+        self._evict_group(s, s + 1, stream, events, tail)
+
+    def evict_many(self, requests, stream=None):
+        """Evict every listed (full) request; neighbouring requests go through
+        one pass together. Returns the groups (first, end) that were evicted."""
+        groups = []
+        for s in sorted(set(requests)):
+            if groups and groups[-1][1] == s:
+                groups[-1][1] = s + 1
+            else:
+                groups.append([s, s + 1])
+        for a, b in groups:
+            self._evict_group(a, b, stream)
+        return [tuple(g) for g in groups]
+
+    def _evict_group(self, a, b, stream=None, events=None, tail=None):
+        if any(self.lengths[s] != self.cap for s in range(a, b)):
+            raise RuntimeError("only full slots are evicted")
+        n = b - a
+        lay, st = self._group_layout(n), _stream(stream)
         handles = [e.cuda_event for e in events] if events is not None else []
-        off_stats = s * self.L * self.Hq * 2 * 128 * 4
-        off_counts = s * self.L * self.Hq * 4
-        stats = ctypes.c_void_p(self.stats.data_ptr() + off_stats)
-        counts = ctypes.c_void_p(self.counts.data_ptr() + off_counts)
-        k, v, pos = _ptr(self.k[s]), _ptr(self.v[s]), _ptr(self.pos[s])
+        stats = ctypes.c_void_p(self.stats[a].data_ptr())
+        counts = ctypes.c_void_p(self.counts[a].data_ptr())
+        k, v, pos = _ptr(self._k[0, 0, a]), _ptr(self._v[0, 0, a]), _ptr(self._pos[0, 0, a])
+        self._views(n)
         _check(jacap_score_stats(lay, self.params, stats, counts, k, v, _ptr(self.scores), _ptr(self.ws),
                                  self.ws.numel(), st, handles), "jacap_score_stats")
         _check(jacap_select_compact_inplace(lay, _ptr(self.scores), self.budget, _ptr(self.idx), _ptr(self.kept), k,
@@ -363,14 +410,15 @@ class DecodeEvictor:
                "jacap_select_compact_inplace")
         if tail is not None:
             tail[0].record(stream)
-        self.lengths[s] = self.budget
-        self.events += 1
+        for s in range(a, b):
+            self.lengths[s] = self.budget
+        self.events += n
+        self.passes += 1
 
     def step(self, k_new, v_new, q_new, stream=None):
-        """append() then evict() every request that became full."""
+        """append() then evict every request that became full (neighbours together)."""
         full = self.append(k_new, v_new, q_new, stream)
-        for s in full:
-            self.evict(s, stream)
+        self.evict_many(full, stream)
         return full
 
     def check(self, stream=None):

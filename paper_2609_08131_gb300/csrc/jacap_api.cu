@@ -195,6 +195,12 @@ bool encode_kv_map(CUtensorMap* map, const jacap_layout* L, const void* base) {
 
 jacap_status map_cuda(cudaError_t e) { return e == cudaSuccess ? JACAP_OK : JACAP_ERR_CUDA; }
 
+// The per-token tags `pos` follow K's layer and head strides in units of its
+// token stride, which must therefore divide them.
+bool pos_layout_ok(const jacap_layout* L, const int32_t* pos) {
+  return pos == nullptr || (L->kv_stride_layer % L->kv_stride_token == 0 && L->kv_stride_head % L->kv_stride_token == 0);
+}
+
 // CTAs for `items` work items with at most per_sm CTAs per SM: each CTA takes
 // a contiguous range, so the grid is chosen to split the items as evenly as
 // the cap allows (ceil(items / cap) items for every CTA but the last few).
@@ -387,6 +393,7 @@ jacap_status jacap_compact_inplace(const jacap_layout* layout, void* k, void* v,
     return JACAP_ERR_INVALID_ARG;
   if (!aligned16(k) || !aligned16(v) || ((uintptr_t)idx & 3u) != 0 || ((uintptr_t)pos & 3u) != 0)
     return JACAP_ERR_INVALID_ARG;
+  if (!pos_layout_ok(layout, pos)) return JACAP_ERR_INVALID_ARG;
   if ((int64_t)layout->num_layers * layout->num_kv_heads * layout->num_seqs >= ((int64_t)1 << 31))
     return JACAP_ERR_INVALID_ARG;
   Dims dm;
@@ -411,6 +418,7 @@ jacap_status jacap_select_compact_inplace(const jacap_layout* layout, const floa
   if (((uintptr_t)scores & 3u) != 0 || ((uintptr_t)idx & 3u) != 0 || ((uintptr_t)kept & 3u) != 0 ||
       ((uintptr_t)pos & 3u) != 0 || !aligned16(k) || !aligned16(v))
     return JACAP_ERR_INVALID_ARG;
+  if (!pos_layout_ok(layout, pos)) return JACAP_ERR_INVALID_ARG;
   Dims dm;
   make_dims(layout, nullptr, dm);
   const Carve c = carve(dm);

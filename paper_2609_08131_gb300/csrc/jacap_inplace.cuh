@@ -28,7 +28,8 @@ __device__ __forceinline__ void compact_ordered_unit(const Dims& dm, int plane, 
   uint4* kb = (uint4*)(k + rowoff);
   uint4* vb = (uint4*)(v + rowoff);
   const int64_t st16 = dm.kv_st * (int64_t)sizeof(T) / 16;  // token stride in 16-byte pieces
-  int32_t* pb = pos != nullptr ? pos + (int64_t)plane * dm.Ntot : nullptr;
+  // the tags follow the layout of K with one int32 per token row
+  int32_t* pb = pos != nullptr ? pos + (int64_t)l * (dm.kv_sl / dm.kv_st) + (int64_t)g * (dm.kv_sh / dm.kv_st) : nullptr;
   for (int c0 = 0; c0 < kept; c0 += CH) {
     uint4 kr[PER], vr[PER];
     int32_t pr = 0;
@@ -74,7 +75,8 @@ __device__ __forceinline__ void fill_holes_unit(const Dims& dm, int plane, int64
   uint4* kb = (uint4*)(k + rowoff);
   uint4* vb = (uint4*)(v + rowoff);
   const int64_t st16 = dm.kv_st * (int64_t)sizeof(T) / 16;
-  int32_t* pb = pos != nullptr ? pos + (int64_t)plane * dm.Ntot : nullptr;
+  // the tags follow the layout of K with one int32 per token row
+  int32_t* pb = pos != nullptr ? pos + (int64_t)l * (dm.kv_sl / dm.kv_st) + (int64_t)g * (dm.kv_sh / dm.kv_st) : nullptr;
   for (int j = warp; j < holes; j += NT / 32) {
     int lo = 0, hi = f;  // first p in [0, f) with c(p) > j (f if none)
     while (lo < hi) {

@@ -130,6 +130,69 @@ def test_decode_evictions_match_the_oracle_event_by_event(name):
     assert ev.events == sum(len(v) for v in event_steps.values()) > 0
 
 
+@pytest.mark.parametrize("ordered", [False, True])
+def test_requests_that_fill_together_are_evicted_in_one_pass(ordered):
+    # three of four requests start with equal prefills, so they fill on the same
+    # decode step; the neighbouring two of them (0, 1) share one pass, request
+    # 3 gets its own, and request 2 fills alone five steps earlier. Every unit
+    # of every request is checked against the oracle
+    # on the exact slot contents before the eviction, and the tags move with
+    # the rows.
+    L, Hq, Hkv, B, D, w, T = 2, 12, 2, 40, 16, 8, 20
+    n0s = (40, 40, 45, 40)
+    S, G, cap = len(n0s), Hq // Hkv, B + D
+    wl = Workload("decode batch", L, Hq, Hkv, tuple(n + T for n in n0s), w + T, B, seed=37)
+    t = generate(wl, DEV)
+    cu = t.cu_seqlens.cpu().tolist()
+    k0 = torch.zeros((S, L, Hkv, max(n0s), 128), dtype=t.k.dtype, device=DEV)
+    v0 = torch.zeros_like(k0)
+    for s, n in enumerate(n0s):
+        k0[s, :, :, :n] = t.k[:, :, cu[s]:cu[s] + n]
+        v0[s, :, :, :n] = t.v[:, :, cu[s]:cu[s] + n]
+    ev = DecodeEvictor(S, L, Hq, Hkv, B, D, dtype=t.k.dtype, device=DEV, preserve_order=ordered)
+    ev.start(k0, v0, t.q_win[:, :, :, :w].contiguous(), list(n0s))
+    q_all = t.q_win.double().cpu().numpy()
+    P = JacapParams()
+    batched = 0
+    for step in range(T):
+        rows = [cu[s] + n0s[s] + step for s in range(S)]
+        k_new = torch.stack([t.k[:, :, r] for r in rows])
+        v_new = torch.stack([t.v[:, :, r] for r in rows])
+        full = ev.append(k_new, v_new, t.q_win[:, :, :, w + step].contiguous())
+        if not full:
+            continue
+        before = {s: (ev.k[s].clone(), ev.v[s].clone(), ev.pos[s].clone()) for s in full}
+        runs = []  # the groups evict_many forms: maximal runs of neighbouring requests
+        for s in full:
+            if runs and runs[-1][-1] == s - 1:
+                runs[-1].append(s)
+            else:
+                runs.append([s])
+        for run in runs:
+            # one run per call, so the scores and positions of each pass can be read
+            assert ev.evict_many(run) == [(run[0], run[-1] + 1)]
+            a, b = run[0], run[-1] + 1
+            ev.check()
+            batched += b - a > 1
+            for j, s in enumerate(range(a, b)):
+                kb, vb, pb = before[s]
+                hist = q_all[s, :, :, :w + step + 1]
+                for layer in range(L):
+                    for g in range(Hkv):
+                        K = kb[layer, g].double().cpu().numpy()
+                        V = vb[layer, g].double().cpu().numpy()
+                        ora = oracle_unit(hist[layer, g * G:(g + 1) * G], K, V, B, P)
+                        sc = ev.scores[layer, g, j * cap:(j + 1) * cap].double().cpu().numpy()
+                        assert_scores_close(sc, ora["scores"], f"step {step} request {s} unit ({layer}, {g})")
+                        gidx = ev.idx[layer, g, j].cpu().numpy()
+                        assert_selection(gidx, cap, B, ora["scores"], ora["idx"])
+                        sel = torch.as_tensor(_arrangement(gidx, B, ordered), dtype=torch.long, device=DEV)
+                        assert_rows_bitwise(kb[layer, g][sel], ev.k[s, layer, g, :B])
+                        assert_rows_bitwise(vb[layer, g][sel], ev.v[s, layer, g, :B])
+                        assert torch.equal(pb[layer, g][sel], ev.pos[s, layer, g, :B])
+    assert batched >= 1 and ev.events > ev.passes
+
+
 def test_compaction_refuses_positions_that_do_not_ascend():
     # a hand-made index list with a repeat: the unit is left untouched and the
     # status word says invalid argument (no out-of-range access is possible:
