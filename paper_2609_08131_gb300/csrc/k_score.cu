@@ -7,7 +7,8 @@
 // only channels 0-63: the first four K-steps are N = 128 MMAs, the last four
 // N = 64 MMAs into columns 64-127. The image's zero quarter (rows 0-63 of
 // channels 64-127) is not copied into shared memory, which leaves room for a
-// fourth V stage. V comes straight from the TMA-staged tile.
+// fourth V stage. V comes straight from the TMA-staged tile; a warp of its
+// own loads the images, so the V ring never waits behind an image slot.
 // Each epilogue thread owns one token (one TMEM lane) and reduces
 // ||y||^2 = sum_j D[j]^2 in fp32, then multiplies by w_i. The tensor-memory accumulator
 // is double-buffered so the epilogue of tile i overlaps the MMAs of tile i+1,
@@ -20,9 +21,9 @@
 
 namespace jacap {
 
-constexpr int SC_THREADS = 192;  // warp 0: TMA, warp 1: MMA, warps 2-5: epilogue
+constexpr int SC_THREADS = 224;  // warp 0: V tiles (TMA), warp 1: MMA, warps 2-5: epilogue, warp 6: images
 template <bool DENSE> __host__ __device__ constexpr int sc_stages() { return DENSE ? 3 : 4; }  // V tiles in flight
-constexpr int SC_IMGS = 2;  // L^{-1} image buffers
+template <bool DENSE> __host__ __device__ constexpr int sc_imgs() { return 2; }  // L^{-1} image buffers
 constexpr int SC_BOX = 16384;
 constexpr int SC_TILE_BYTES = 2 * SC_BOX;
 constexpr int SC_M_BYTES = 65536;
@@ -37,7 +38,7 @@ constexpr int SC_MT_BYTES = 49152;
 template <bool DENSE> __host__ __device__ constexpr int sc_img_bytes() { return DENSE ? SC_M_BYTES : SC_MT_BYTES; }
 template <bool DENSE>
 constexpr size_t score_bf16_smem_bytes() {
-  return 1024 + SC_IMGS * sc_img_bytes<DENSE>() + sc_stages<DENSE>() * SC_TILE_BYTES + 256;
+  return 1024 + sc_imgs<DENSE>() * sc_img_bytes<DENSE>() + sc_stages<DENSE>() * SC_TILE_BYTES + 256;
 }
 
 // DENSE: the score matrix is a full 128 x 128 (output directions) rather than
@@ -48,6 +49,7 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
                       float* __restrict__ scores) {
   pdl_wait();
   constexpr int SC_STAGES = sc_stages<DENSE>();
+  constexpr int SC_IMGS = sc_imgs<DENSE>();
   constexpr int IMG = sc_img_bytes<DENSE>();
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -97,28 +99,11 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
   if (warp == 0) {
     if (lane == 0) {
       prefetch_tmap(&vmap);
-      uint32_t it = 0, nrun = 0;
-      bool ok = true, cont = false;
+      uint32_t it = 0;
+      bool ok = true;
       Item item;
       for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); ok && is.next(item);) {
         const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
-        const int64_t u = (int64_t)item.plane * dm.S + item.seq;
-        if (!cont) {  // a new unit: its image, into the buffer of the run SC_IMGS runs back
-          const int mp = nrun % SC_IMGS;
-          if (nrun >= SC_IMGS && !mbar_wait(smem_u32(&mempty[mp]), ((nrun / SC_IMGS) & 1) ^ 1, ws, abort)) break;
-          mbar_arrive_expect_tx(smem_u32(&mfull[mp]), IMG);
-          const uint8_t* src = ws.minv_img + u * SC_M_BYTES;
-          uint8_t* dst = mimg + mp * IMG;
-          if (DENSE) {
-            bulk_g2s(smem_u32(dst), src, SC_M_BYTES, smem_u32(&mfull[mp]));
-          } else {
-            bulk_g2s(smem_u32(dst), src, 32768, smem_u32(&mfull[mp]));
-            bulk_g2s(smem_u32(dst + 32768), src + 32768 + 8192, 8192, smem_u32(&mfull[mp]));
-            bulk_g2s(smem_u32(dst + 40960), src + 32768 + 24576, 8192, smem_u32(&mfull[mp]));
-          }
-          ++nrun;
-        }
-        cont = is.next_same_unit(item);
         for (int64_t t = item.t0; t < item.t1; t += TILE) {
           const int st = it % SC_STAGES;
           if (it >= (uint32_t)SC_STAGES &&
@@ -135,7 +120,34 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
       }
       for (uint32_t k = (it > (uint32_t)SC_STAGES ? it - SC_STAGES : 0); k < it; ++k)
         mbar_wait(smem_u32(&vfull[k % SC_STAGES]), (k / SC_STAGES) & 1, ws, nullptr);
-      for (uint32_t k = (nrun > SC_IMGS ? nrun - SC_IMGS : 0); k < nrun; ++k)
+    }
+  } else if (warp == 6) {
+    // ------------------- the L^{-1} image of each run, into the buffer of the run SC_IMGS runs back
+    // (a warp of its own, so the V tiles never wait behind an image slot)
+    if (lane == 0) {
+      uint32_t nrun = 0;
+      bool cont = false;
+      Item item;
+      for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
+        const bool same = cont;
+        cont = is.next_same_unit(item);
+        if (same) continue;
+        const int64_t u = (int64_t)item.plane * dm.S + item.seq;
+        const int mp = nrun % SC_IMGS;
+        if (nrun >= SC_IMGS && !mbar_wait(smem_u32(&mempty[mp]), ((nrun / SC_IMGS) & 1) ^ 1, ws, abort)) break;
+        mbar_arrive_expect_tx(smem_u32(&mfull[mp]), IMG);
+        const uint8_t* src = ws.minv_img + u * SC_M_BYTES;
+        uint8_t* dst = mimg + mp * IMG;
+        if (DENSE) {
+          bulk_g2s(smem_u32(dst), src, SC_M_BYTES, smem_u32(&mfull[mp]));
+        } else {
+          bulk_g2s(smem_u32(dst), src, 32768, smem_u32(&mfull[mp]));
+          bulk_g2s(smem_u32(dst + 32768), src + 32768 + 8192, 8192, smem_u32(&mfull[mp]));
+          bulk_g2s(smem_u32(dst + 40960), src + 32768 + 24576, 8192, smem_u32(&mfull[mp]));
+        }
+        ++nrun;
+      }
+      for (uint32_t k = (nrun > (uint32_t)SC_IMGS ? nrun - SC_IMGS : 0); k < nrun; ++k)
         mbar_wait(smem_u32(&mfull[k % SC_IMGS]), (k / SC_IMGS) & 1, ws, nullptr);
     }
   } else if (warp == 1) {
@@ -195,7 +207,7 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
       umma_commit(smem_u32(mdone));
       mbar_wait(smem_u32(mdone), 0, ws, nullptr);
     }
-  } else {
+  } else if (warp < 6) {
     const int quarter = warp & 3;
     const int y = quarter * 32 + lane;  // token row of the tile == TMEM lane
     uint32_t it = 0;
