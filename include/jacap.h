@@ -133,7 +133,11 @@ typedef struct {
  * (budget is accepted for forward compatibility and may be any value >= 1).
  * Returns 0 if the layout is invalid. The workspace must be 256-byte aligned;
  * it holds the status word and every intermediate (mu, lambda, logits, kappa,
- * w, partial Grams, the factor of A). */
+ * w, partial Grams, the factor of A): about 36 bytes per token and KV head of
+ * every layer (G = 4) plus 192 KB per unit. Units are independent, so a caller
+ * short of memory can run the calls over groups of layers (a layout with
+ * num_layers = the group size and K, V, Q_win pointers advanced to the group's
+ * first layer) with one workspace sized for a group. */
 size_t jacap_workspace_size(const jacap_layout* layout, int32_t budget);
 
 /*

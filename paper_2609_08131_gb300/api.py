@@ -102,10 +102,17 @@ class Evictor:
     """Owns the workspace and output buffers for repeated passes over caches
     of one shape; ``run()`` enqueues score, select and compact."""
 
-    def __init__(self, cache: Cache, budget: int, params: jacap_params | None = None, out_factor=None):
+    def __init__(self, cache: Cache, budget: int, params: jacap_params | None = None, out_factor=None,
+                 layer_group: int | None = None):
         """``out_factor``: optional float32 [L][Hkv][128][128] device tensor of
         factors F with F^T F = W^T W for the output maps W (u_i = W v_i);
-        None uses the proxy u_i = v_i."""
+        None uses the proxy u_i = v_i.
+
+        ``layer_group``: run the pass over groups of this many layers, one
+        after the other on the same stream, with a workspace sized for one
+        group instead of the whole cache (units are independent, so the kept
+        sets are those of one pass up to near ties; the workspace takes ~36
+        bytes per token and KV head of every layer it covers)."""
         self.cache = cache
         self.budget = int(budget)
         self.params = params if params is not None else jacap_params()
@@ -117,7 +124,16 @@ class Evictor:
         self.out_factor = out_factor
         self.lay = cache.layout()
         dev = cache.k.device
-        nbytes = jacap_workspace_size(self.lay, self.budget)
+        L = cache.k.shape[0]
+        gl = L if layer_group is None else max(1, min(int(layer_group), L))
+        self.groups = [(l0, min(gl, L - l0)) for l0 in range(0, L, gl)]
+        self._glay = {}
+        for _, n in self.groups:
+            if n not in self._glay:
+                lay = cache.layout()
+                lay.num_layers = n
+                self._glay[n] = lay
+        nbytes = max(jacap_workspace_size(lay, self.budget) for lay in self._glay.values())
         if nbytes == 0:
             raise JacapError(1, "jacap_workspace_size")
         self.ws = torch.empty(nbytes, dtype=torch.uint8, device=dev)
@@ -174,8 +190,34 @@ class Evictor:
                                     self.ws.numel(), _stream(stream)), "jacap_select_compact")
 
     def run(self, stream=None):
-        self.score(stream)
-        self.select_compact(stream)
+        if len(self.groups) == 1:
+            self.score(stream)
+            self.select_compact(stream)
+            return
+        # layer groups: the same calls on sub-layouts whose data pointers start
+        # at the group's first layer, writing the group's slices of the outputs
+        c, st = self.cache, _stream(stream)
+        ek, eq = c.k.element_size(), c.q_win.element_size()
+        ws, wn = _ptr(self.ws), self.ws.numel()
+        for l0, n in self.groups:
+            lay = self._glay[n]
+            koff, qoff = l0 * self.lay.kv_stride_layer * ek, l0 * self.lay.q_stride_layer * eq
+            k = ctypes.c_void_p(c.k.data_ptr() + koff)
+            v = ctypes.c_void_p(c.v.data_ptr() + koff)
+            q = ctypes.c_void_p(c.q_win.data_ptr() + qoff)
+            scores = _ptr(self.scores[l0:l0 + n])
+            if self.out_factor is not None:
+                _check(jacap_score_out(lay, self.params, q, k, v, _ptr(self.out_factor[l0:l0 + n]), scores, ws, wn,
+                                       st, []), "jacap_score_out")
+            else:
+                _check(jacap_score(lay, self.params, q, k, v, scores, ws, wn, st), "jacap_score")
+            _check(jacap_select_compact(lay, scores, self.budget, _ptr(self.idx[l0:l0 + n]), _ptr(self.kept), k, v,
+                                        _ptr(self.k_out[l0:l0 + n]), _ptr(self.v_out[l0:l0 + n]), ws, wn, st),
+                   "jacap_select_compact")
+            # a later group's first kernel clears the status word: surface a
+            # problem of this group first
+            if self.device_status(stream) != JACAP_OK:
+                _check(self.device_status(stream), f"device status (layers {l0} .. {l0 + n - 1})")
 
     def device_status(self, stream=None) -> int:
         return jacap_device_status(_ptr(self.ws), _stream(stream))

@@ -148,6 +148,22 @@ def test_intermediates_match_the_oracle():
                                            rtol=1e-4, atol=1e-6)
 
 
+def test_layer_groups_bound_the_workspace_and_match_the_oracle():
+    # the pass over groups of 2 of 5 layers with a workspace sized for a group
+    wl = Workload("t", 5, 12, 2, (900, 333), 16, 64, seed=31)
+    t = generate(wl, DEV)
+    whole = Evictor(make_cache(t, wl), wl.budget)
+    ev = Evictor(make_cache(t, wl), wl.budget, layer_group=2)
+    assert ev.ws.numel() < whole.ws.numel() and [n for _, n in ev.groups] == [2, 2, 1]
+    ev.run()
+    ev.check()
+    for s in range(len(wl.seqlens)):
+        for layer in range(wl.num_layers):
+            for g in range(wl.num_kv_heads):
+                check_unit(ev, t, wl, jacap_params(), s, layer, g, check_w=False)
+    gpu_selection_properties(ev.scores, ev.idx, ev.kept, wl.seqlens, wl.budget)
+
+
 def test_repeat_calls_are_bitwise_deterministic():
     wl = Workload("t", 2, 8, 2, (1500, 700), 16, 64, seed=22)
     t = generate(wl, DEV)
