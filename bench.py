@@ -45,6 +45,8 @@ def parse():
     p.add_argument("--warmup", type=int, default=10)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--config", type=int, default=2)
+    p.add_argument("--schedule", default="auto", choices=["auto", "separate", "fused"],
+                   help="Gram / factor / scores as separate kernels or one fused launch (auto: the library's choice)")
     p.add_argument("--budget", type=int, default=None)
     p.add_argument("--weighting", default="jacobian", choices=["jacobian", "linear"],
                    help="Eq. 8 softmax-aware weights (the method) or the linear S = I surrogate")
@@ -298,6 +300,31 @@ def run_reference(args):
     return 0
 
 
+# The fused schedule runs the Gram, the factor and the scores as one launch,
+# timed in the Gram's slot of jacap_score_timed.
+FUSED_NAME = "gram_factor_scores"
+SCHEDULES = {"auto": 0, "separate": 1, "fused": 2}
+
+
+def fused_kernel_names(kern, schedule):
+    if schedule != 2:
+        return kern
+    out = {}
+    for k, v in kern.items():
+        if k == "gram":
+            out[FUSED_NAME] = v
+        elif k not in ("factor", "scores"):
+            out[k] = v
+    return out
+
+
+def schedule_desc(schedule, roles):
+    if schedule != 2:
+        return {"kind": "separate kernels"}
+    return {"kind": "fused Gram-factor-scores launch", "factor_ctas": roles[0], "gram_ctas": roles[1],
+            "score_ctas": roles[2], "v_tiles_kept_in_l2_per_item": roles[3]}
+
+
 # -------------------------------------------------------------------- ours --
 def run_ours(args):
     import torch
@@ -336,7 +363,8 @@ def run_ours(args):
         W = torch.randn(wl.num_layers * wl.num_kv_heads, args.out_proj, 128, generator=gen, device=dev) / 128 ** 0.5
         out_factor = torch.linalg.qr(W, mode="r").R.reshape(wl.num_layers, wl.num_kv_heads, 128, 128).contiguous()
     ev = Evictor(cache, budget, jacap_params(linear_weighting=1 if args.weighting == "linear" else 0,
-                                             full_covariance=1 if args.covariance == "full" else 0),
+                                             full_covariance=1 if args.covariance == "full" else 0,
+                                             schedule=SCHEDULES[args.schedule]),
                  out_factor=out_factor)
     stream = torch.cuda.current_stream(dev)
 
@@ -406,6 +434,8 @@ def run_ours(args):
             kern[name] += ev_score[i][j].elapsed_time(ev_score[i][j + 1])
         kern["select_compact"] += ev_score[i][nk].elapsed_time(ev_tail[i][0])
     kern = {k: v / KB for k, v in kern.items()}
+    schedule, roles = ev.schedule_info()
+    kern = fused_kernel_names(kern, schedule)
 
     L, Hkv, N, d = t.k.shape
     es = t.k.element_size()
@@ -427,6 +457,10 @@ def run_ours(args):
         # scores read; retained K, V rows read and written
         "select_compact": L * Hkv * N * 4 + 4 * kept_rows * d * es,
     }
+    if schedule == 2:  # one launch: V read once (its second read is extra traffic), scores written
+        for k in ("gram", "scores"):
+            del alg_kernel[k]
+        alg_kernel[FUSED_NAME] = kv_bytes + L * Hkv * N * 4
     if not fused_weights:
         alg_kernel["weights"] = L * Hkv * N * (8 * G + 4)  # logits + kappa read, w written
     dom = max(alg_kernel, key=lambda k: kern[k])
@@ -484,10 +518,12 @@ def run_ours(args):
             "ms_per_step_with_kernel_events": t_ms_events,
             "ms_per_step_cuda_graph": graph_ms,
             # plan, query statistics, K pass (with the full-covariance kappa when that
-            # runs on the tensor cores), [full covariance on the CUDA cores],
-            # [weights: float32 only], Gram, factor, scores, selection + compaction
-            "gpu_launches": K * (7 + (1 if args.covariance == "full" and not full_cov_fused else 0)
-                                 + (0 if fused_weights else 1)),
+            # runs on the tensor cores), [full covariance on the CUDA cores], unit
+            # softmax statistics, [weights: float32 only], Gram, factor, scores (or the
+            # three as one fused launch), selection + compaction
+            "gpu_launches": K * (8 + (1 if args.covariance == "full" and not full_cov_fused else 0)
+                                 + (0 if fused_weights else 1) - (2 if schedule == 2 else 0)),
+            "schedule": schedule_desc(schedule, roles),
             "clocks": clocks,
             "extra_configs": extra,
             "cpu_baseline": cpu,
@@ -515,7 +551,8 @@ def measure_config(index, args, dev, dist, rank, hbm):
     wl = replace(wl, seed=wl.seed + 1000 * rank)
     budget = wl.budget
     t = generate(wl, dev)
-    ev = Evictor(Cache(t.q_win, t.k, t.v, t.cu_seqlens, t.seqlens, wl.num_q_heads), budget, jacap_params())
+    ev = Evictor(Cache(t.q_win, t.k, t.v, t.cu_seqlens, t.seqlens, wl.num_q_heads), budget,
+                 jacap_params(schedule=SCHEDULES[args.schedule]))
     stream = torch.cuda.current_stream(dev)
     for _ in range(max(3, args.warmup)):
         ev.run()
@@ -548,6 +585,8 @@ def measure_config(index, args, dev, dist, rank, hbm):
     kern = {name: sum(evs[i][j].elapsed_time(evs[i][j + 1]) for i in range(K)) / K
             for j, name in enumerate(SCORE_KERNEL_NAMES)}
     kern["select_compact"] = sum(evs[i][nk].elapsed_time(evs[i][nk + 1]) for i in range(K)) / K
+    schedule, roles = ev.schedule_info()
+    kern = fused_kernel_names(kern, schedule)
     L = t.k.shape[0]
     value, t_ms, world = aggregate_ranks(t_ms, sum(t.seqlens) * L, dist, dev)
     alg = wl.algorithmic_bytes(budget)
@@ -569,7 +608,8 @@ def measure_config(index, args, dev, dist, rank, hbm):
         },
         "kernel_ms": kern,
         "clocks": clocks,
-        "gpu_launches": K * (7 + (0 if wl.dtype == "bf16" else 1)),
+        "gpu_launches": K * (8 + (0 if wl.dtype == "bf16" else 1) - (2 if schedule == 2 else 0)),
+        "schedule": schedule_desc(schedule, roles),
     }
     del ev, t
     torch.cuda.empty_cache()
@@ -761,6 +801,8 @@ def run_decode(args):
     kern = {name: sum(evs[i][j].elapsed_time(evs[i][j + 1]) for i in range(K)) / K
             for j, name in enumerate(SCORE_KERNEL_NAMES)}
     kern["select_compact_inplace"] = sum(evs[i][nk].elapsed_time(evs[i][nk + 1]) for i in range(K)) / K
+    schedule, roles = ev.schedule_info()
+    kern = fused_kernel_names(kern, schedule)
     # one decode step's statistics update (one query per layer and head)
     M = 200
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -793,9 +835,11 @@ def run_decode(args):
         "stats_update_us_per_decode_step": upd_us,
         "event_hbm_fraction": {"kv_bytes": kv_bytes, "of_8tbs": kv_bytes / (t_ms * 1e-3) / 8e12},
         "clocks": clocks,
-        # plan, query statistics, K pass, Gram (with the weights), factor, scores,
-        # selection with the hole filling (ascending order: a second launch)
-        "gpu_launches_per_event": 7 + (1 if args.preserve_order else 0),
+        # plan, query statistics, K pass, unit softmax statistics, Gram (with the
+        # weights), factor, scores (or the three fused), selection with the hole
+        # filling (ascending order: a second launch)
+        "gpu_launches_per_event": 8 + (1 if args.preserve_order else 0) - (2 if schedule == 2 else 0),
+        "schedule": schedule_desc(schedule, roles),
     }
     print(json.dumps(line))
     return 0

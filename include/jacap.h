@@ -97,7 +97,7 @@ typedef struct {
 } jacap_layout;
 
 /*
- * Method switches. Defaults {10.0f, 1, 1, 0, 0, 0}:
+ * Method switches. Defaults {10.0f, 1, 1, 0, 0, 0, 0}:
  *  tau            temperature of the pool softmax (Sec. 3.4; Sec. 4.4 reports
  *                 the best accuracy near 10). Must be finite and > 0.
  *  weight_div_dk  1: keep the 1/d_k factor of Eq. 8; 0: drop it (Alg. 1 step 2
@@ -118,7 +118,21 @@ typedef struct {
  *                 tensor cores inside the K pass (K is still read once); other
  *                 shapes and float32 caches a much slower CUDA-core kernel
  *                 after the K pass, which reads K a second time.
- * Callers that zero-initialise the two trailing fields get the method.
+ *  schedule       how the Gram (Eq. 9), the factor of A and the scores (Eq. 10)
+ *                 are run; every choice computes the same quantities (the
+ *                 partial Grams may be summed in another order, within the
+ *                 float32 rounding of the pass). 0: automatic (currently
+ *                 the separate kernels, the faster schedule on GB300 for
+ *                 every shape measured); 1: three separate kernels, each over
+ *                 the whole cache; 2: fused, one persistent cooperative
+ *                 launch whose CTAs take the three roles and hand each unit
+ *                 from one role to the next as soon as it is ready, so that
+ *                 part of the score role's read of V hits L2 (bf16 caches
+ *                 only; float32 caches and jacap_score_out use separate
+ *                 kernels whatever the value). Other values:
+ *                 JACAP_ERR_INVALID_ARG.
+ * Callers that zero-initialise the trailing fields get the method with the
+ * automatic schedule.
  */
 typedef struct {
   float tau;
@@ -127,7 +141,17 @@ typedef struct {
   int32_t cov_unbiased;
   int32_t linear_weighting;
   int32_t full_covariance;
+  int32_t schedule;
 } jacap_params;
+
+/* The schedule (jacap_params.schedule) that jacap_score, jacap_score_timed,
+ * jacap_score_stats and jacap_evict_host would run for `layout` and `params`
+ * on the current device: 1 (separate kernels) or 2 (fused). With the fused
+ * schedule, roles[0..3] (if not NULL) receive its CTAs per role (factor, Gram,
+ * score) and the V tiles per Gram work item loaded with the L2 evict_last
+ * policy; zeros otherwise. Returns the schedule, or -(jacap_status) for an
+ * invalid layout or params or an unsupported device. No GPU work. */
+int32_t jacap_schedule_info(const jacap_layout* layout, const jacap_params* params, int32_t* roles);
 
 /* Bytes of device workspace jacap_score/jacap_select need for `layout`
  * (budget is accepted for forward compatibility and may be any value >= 1).
@@ -148,10 +172,11 @@ size_t jacap_workspace_size(const jacap_layout* layout, int32_t budget);
  *  ws, ws_bytes device workspace of at least jacap_workspace_size() bytes.
  * Enqueues: a planning kernel (which also resets the status word), query
  * statistics, a streaming pass
- * over K (logits, kappa, softmax statistics), the Eq. 8 weights (inside the
- * weighted-Gram pass for bf16 caches), the weighted-Gram pass over V (tensor
- * cores for bf16), the Cholesky factor and inverse of A, and the quadratic
- * forms.
+ * over K (logits, kappa, softmax statistics), the merge of each unit's softmax
+ * normaliser, the Eq. 8 weights (inside the weighted-Gram pass for bf16
+ * caches), the weighted-Gram pass over V (tensor cores for bf16), the Cholesky
+ * factor and inverse of A, and the quadratic forms (the last three as one
+ * launch with the fused schedule).
  */
 jacap_status jacap_score(const jacap_layout* layout, const jacap_params* params,
                          const void* q_win, const void* k, const void* v, float* scores,
@@ -163,10 +188,13 @@ jacap_status jacap_score(const jacap_layout* layout, const jacap_params* params,
  * events[num_events - 1] after the last one. `events` holds cudaEvent_t
  * handles (as void*) created by the caller; num_events must be 0 (no hooks)
  * or JACAP_SCORE_KERNELS + 1. Kernel order: plan, query statistics, K pass,
- * weights, Gram, factor, scores. With bf16 caches the Gram kernel computes the
- * Eq. 8 weights itself and the weights slot is empty (its two events are
- * recorded back to back); with full_covariance the K-pass slot also holds the
- * CUDA-core kappa kernel when that one runs.
+ * weights, Gram, factor, scores. The weights slot holds the merge of each
+ * unit's softmax normaliser and, for float32 caches, the Eq. 8 weights (with
+ * bf16 caches the Gram kernel computes them itself); with full_covariance the
+ * K-pass slot also holds the CUDA-core kappa kernel when that one runs. With
+ * the fused schedule (jacap_params.schedule) the Gram slot holds the one launch
+ * that runs the Gram, the factor and the scores, and the factor and scores
+ * slots are empty (their events are recorded back to back).
  */
 #define JACAP_SCORE_KERNELS 7
 jacap_status jacap_score_timed(const jacap_layout* layout, const jacap_params* params,

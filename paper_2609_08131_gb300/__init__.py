@@ -62,10 +62,15 @@ class jacap_params(ctypes.Structure):
         ("cov_unbiased", ctypes.c_int32),
         ("linear_weighting", ctypes.c_int32),
         ("full_covariance", ctypes.c_int32),
+        ("schedule", ctypes.c_int32),
     ]
 
-    def __init__(self, tau=10.0, weight_div_dk=1, ridge=1, cov_unbiased=0, linear_weighting=0, full_covariance=0):
-        super().__init__(tau, weight_div_dk, ridge, cov_unbiased, linear_weighting, full_covariance)
+    # values of ``schedule``
+    AUTO, SEPARATE, FUSED = 0, 1, 2
+
+    def __init__(self, tau=10.0, weight_div_dk=1, ridge=1, cov_unbiased=0, linear_weighting=0, full_covariance=0,
+                 schedule=0):
+        super().__init__(tau, weight_div_dk, ridge, cov_unbiased, linear_weighting, full_covariance, schedule)
 
 
 class jacap_ws_offsets(ctypes.Structure):
@@ -109,6 +114,8 @@ _SIGS = {
     "jacap_evict_host": (ctypes.c_int, [ctypes.POINTER(jacap_layout), ctypes.POINTER(jacap_params), ctypes.c_int32,
                                         ctypes.c_int32, _P, _P, _P, _P, _P, _P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "jacap_status_string": (ctypes.c_char_p, [ctypes.c_int]),
+    "jacap_schedule_info": (ctypes.c_int32, [ctypes.POINTER(jacap_layout), ctypes.POINTER(jacap_params),
+                                             ctypes.POINTER(ctypes.c_int32)]),
     "jacap_workspace_offsets": (ctypes.c_int, [ctypes.POINTER(jacap_layout), ctypes.c_int32,
                                                ctypes.POINTER(jacap_ws_offsets)]),
 }
@@ -124,6 +131,14 @@ def lib() -> ctypes.CDLL:
             fn.argtypes = args
         h._jacap_typed = True
     return h
+
+
+def jacap_schedule_info(layout: jacap_layout, params: jacap_params):
+    """(schedule, (factor CTAs, Gram CTAs, score CTAs, kept V tiles per item)) that the scoring
+    entry points would run on the current device; schedule < 0 is -(jacap_status)."""
+    roles = (ctypes.c_int32 * 4)()
+    sched = lib().jacap_schedule_info(ctypes.byref(layout), ctypes.byref(params), roles)
+    return sched, tuple(roles)
 
 
 def jacap_workspace_size(layout: jacap_layout, budget: int) -> int:

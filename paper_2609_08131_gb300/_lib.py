@@ -23,7 +23,7 @@ BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libjacap.so")
 
 SOURCES = ["jacap_api.cu", "k_stream.cu", "k_kpass.cu", "k_gram.cu", "k_factor.cu", "k_score.cu", "k_select.cu",
-           "jacap_static.cu", "k_kfull.cu", "k_decode.cu", "jacap_host.cu"]
+           "jacap_static.cu", "k_kfull.cu", "k_decode.cu", "jacap_host.cu", "k_fused.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
           "-I" + INCLUDE, "-I" + CSRC]
@@ -48,12 +48,17 @@ def build_flags() -> list:
     """Optional build variants, from the environment of the build:
     JACAP_NVTX=1 marks every kernel launch with an NVTX range (tracing);
     JACAP_CHECKED=1 makes the persistent kernels validate every work-item
-    record against the cache bounds and report violations in the status word."""
+    record against the cache bounds and report violations in the status word;
+    JACAP_TRACE=1 records the fused schedule's per-unit timeline (%globaltimer
+    stamps of each role's first and last work on the unit) in a section
+    appended to the workspace."""
     extra = []
     if os.environ.get("JACAP_NVTX") == "1":
         extra.append("-DJACAP_NVTX")
     if os.environ.get("JACAP_CHECKED") == "1":
         extra.append("-DJACAP_CHECKED")
+    if os.environ.get("JACAP_TRACE") == "1":
+        extra.append("-DJACAP_TRACE")
     return extra
 
 
@@ -110,6 +115,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
 
 EXPORTS = [
     "jacap_workspace_size",
+    "jacap_schedule_info",
     "jacap_score",
     "jacap_score_timed",
     "jacap_score_static",

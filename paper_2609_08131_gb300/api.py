@@ -21,6 +21,7 @@ from . import (
     jacap_host_buffer_size,
     jacap_layout,
     jacap_params,
+    jacap_schedule_info,
     jacap_score,
     jacap_score_timed,
     jacap_score_out,
@@ -144,6 +145,18 @@ class Evictor:
         self.kept = torch.empty((S,), dtype=torch.int32, device=dev)
         self.k_out = torch.empty((L, Hkv, S, self.budget, d), dtype=cache.k.dtype, device=dev)
         self.v_out = torch.empty_like(self.k_out)
+
+    def schedule_info(self):
+        """(schedule, roles) of the scoring pass on the current device: 1 = separate kernels,
+        2 = fused (roles = factor, Gram and score CTAs, V tiles per item kept in L2); see
+        jacap_schedule_info. With output directions the pass always uses separate kernels."""
+        if self.out_factor is not None:
+            return 1, (0, 0, 0, 0)
+        lay = self._glay[self.groups[0][1]]
+        sched, roles = jacap_schedule_info(lay, self.params)
+        if sched < 0:
+            raise JacapError(-sched, "jacap_schedule_info")
+        return sched, roles
 
     def bind_outputs(self, idx, kept, k_out, v_out):
         """Write the results into caller-owned device tensors (views into a
@@ -434,6 +447,15 @@ class DecodeEvictor:
         for a, b in groups:
             self._evict_group(a, b, stream)
         return [tuple(g) for g in groups]
+
+    def schedule_info(self, requests: int | None = None):
+        """(schedule, roles) of the scoring pass over ``requests`` slots evicted together
+        (default: all), as jacap_schedule_info reports it."""
+        lay = self._group_layout(self.S if requests is None else int(requests))
+        sched, roles = jacap_schedule_info(lay, self.params)
+        if sched < 0:
+            raise JacapError(-sched, "jacap_schedule_info")
+        return sched, roles
 
     def _evict_group(self, a, b, stream=None, events=None, tail=None):
         if any(self.lengths[s] != self.cap for s in range(a, b)):

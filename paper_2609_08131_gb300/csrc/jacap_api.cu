@@ -6,6 +6,8 @@
 #include <algorithm>
 #include <cudaTypedefs.h>
 #include <math.h>
+#include <stdio.h>
+#include <stdlib.h>
 #include <string.h>
 
 #include "jacap.h"
@@ -20,8 +22,9 @@ constexpr size_t ALIGN = 1024;
 inline size_t align_up(size_t x) { return (x + ALIGN - 1) & ~(ALIGN - 1); }
 
 struct Carve {
-  size_t status, plan, chunks, counters, mu, lam, qdev, lk, cstats, w, gpart, pflag, gram, minv, minv_img,
-      total;
+  size_t status, plan, chunks, counters, mu, lam, qdev, lk, cstats, ustats, w, gpart, pflag, gram, minv,
+      minv_img, total;
+  size_t units, trace;
 };
 
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
@@ -104,10 +107,11 @@ Carve carve(const Dims& dm) {
   const size_t planes = (size_t)dm.L * dm.Hkv;
   const size_t units = planes * dm.S;
   size_t o = 0;
+  c.units = units;
   c.status = o; o = align_up(o + 64);
   c.plan = o; o = align_up(o + ((size_t)dm.S + 2) * 4);
   c.chunks = o; o = align_up(o + (size_t)dm.c_cap * 16);
-  c.counters = o; o = align_up(o + units * 4);
+  c.counters = o; o = align_up(o + units * 8);  // gcount and fdone of the fused schedule
   c.mu = o; o = align_up(o + (size_t)dm.S * dm.L * dm.Hq * D * 4);
   c.lam = o; o = align_up(o + (size_t)dm.S * dm.L * dm.Hq * D * 4);
   // centred window queries: fp32 rows, or the bf16 hi/lo image (512 bytes per padded row)
@@ -115,12 +119,18 @@ Carve carve(const Dims& dm) {
   c.qdev = o; o = align_up(o + (size_t)dm.S * dm.L * dm.Hkv * qrows * 512);
   c.lk = o; o = align_up(o + planes * (size_t)dm.Ntot * 2 * dm.G * 4 + 16);  // + tail of 16-byte rounded copies
   c.cstats = o; o = align_up(o + planes * (size_t)dm.c_cap * dm.G * 2 * 4);
+  c.ustats = o; o = align_up(o + units * (size_t)dm.G * 2 * 4);
   c.w = o; o = align_up(o + planes * (size_t)dm.Ntot * 4);
   c.gpart = o; o = align_up(o + planes * (size_t)dm.c_cap * D * D * 4);
   c.pflag = o; o = align_up(o + planes * (size_t)dm.c_cap * 4);
   c.gram = o; o = align_up(o + units * D * D * 4);
   c.minv = o; o = align_up(o + units * D * D * 4);
   c.minv_img = o; o = align_up(o + units * 65536);
+#ifdef JACAP_TRACE
+  c.trace = o; o = align_up(o + units * TR_SLOTS * 8);  // trace builds: the fused schedule's timeline, last
+#else
+  c.trace = 0;
+#endif
   c.total = o;
   return c;
 }
@@ -131,19 +141,22 @@ Ws make_ws(void* base, const Carve& c) {
   ws.status = (uint32_t*)(b + c.status);
   ws.plan = (int32_t*)(b + c.plan);
   ws.chunks = (int4*)(b + c.chunks);
-  ws.counters = (int32_t*)(b + c.counters);
+  ws.gcount = (int32_t*)(b + c.counters);
+  ws.fdone = ws.gcount + c.units;  // right after gcount: the plan kernel zeroes 2 x units words
   ws.mu = (float*)(b + c.mu);
   ws.lam = (float*)(b + c.lam);
   ws.qdev = (float*)(b + c.qdev);
   ws.qimg = b + c.qdev;
   ws.lk = (float*)(b + c.lk);
   ws.cstats = (float*)(b + c.cstats);
+  ws.ustats = (float*)(b + c.ustats);
   ws.w = (float*)(b + c.w);
   ws.gpart = (float*)(b + c.gpart);
   ws.pflag = (int32_t*)(b + c.pflag);
   ws.gram = (float*)(b + c.gram);
   ws.minv = (float*)(b + c.minv);
   ws.minv_img = b + c.minv_img;
+  ws.trace = c.trace != 0 ? (unsigned long long*)(b + c.trace) : nullptr;
   return ws;
 }
 
@@ -209,6 +222,85 @@ int persistent_grid(int64_t items, int sms, int per_sm) {
   if (items <= cap) return items < 1 ? 1 : (int)items;
   const int64_t per = (items + cap - 1) / cap;
   return (int)((items + per - 1) / per);
+}
+
+// The fused schedule (k_fused.cu). Cost model in SM-microseconds: a 128-token
+// tile costs the Gram role its 16 MMAs of N = 128 (1024 tensor cycles) and
+// the score role its MMAs (SC_TILE_CYCLES), both at ~1.7 G useful cycles/s;
+// a factor CTA takes ~30 us per unit. The factor role gets enough CTAs to
+// keep pace (at most a quarter of the SMs), the rest split between Gram and
+// score in proportion to their cost per tile.
+constexpr double FU_GRAM_US = 1024.0 / 1700.0;
+constexpr double FU_SCORE_US = 880.0 / 1700.0;
+constexpr double FU_FACTOR_US = 30.0;
+
+double fused_tiles(const jacap_layout* L, const Dims& dm) {
+  return (double)dm.L * dm.Hkv * ((double)L->total_tokens / TILE + 0.5 * dm.S);
+}
+
+FusedRoles fused_roles(const jacap_layout* L, const Dims& dm, int sms) {
+  const double units = (double)dm.L * dm.Hkv * dm.S, tiles = fused_tiles(L, dm);
+  int nf = 1;
+  for (int iter = 0; iter < 4; ++iter) {
+    const double t = tiles * (FU_GRAM_US + FU_SCORE_US) / (sms - nf);
+    nf = std::min(std::max((int)ceil(units * FU_FACTOR_US / t), 1), sms / 4);
+  }
+  const int rest = sms - nf;
+  const int ng = std::min(std::max((int)lround(rest * FU_GRAM_US / (FU_GRAM_US + FU_SCORE_US)), 1), rest - 1);
+  FusedRoles r{nf, ng, rest - ng};
+  // tuning override: JACAP_FUSED_ROLES="nf,ng" (the score role takes the other SMs)
+  if (const char* e = getenv("JACAP_FUSED_ROLES")) {
+    int a = 0, b = 0;
+    if (sscanf(e, "%d,%d", &a, &b) == 2 && a >= 1 && b >= 1 && a + b < sms) r = FusedRoles{a, b, sms - a - b};
+  }
+  return r;
+}
+
+// V tiles per Gram item left in L2 (evict_last) for the score role: the
+// evict_last lines in flight (about ng + ns items and nf units' worth of
+// items) stay within 60 % of L2.
+int fused_keep_tiles(const Dims& dm, const FusedRoles& r, double items_per_unit) {
+  int dev = 0, l2 = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, dev) != cudaSuccess)
+    l2 = 0;
+  const double span = r.ng + r.ns + r.nf * items_per_unit;  // items whose kept tiles are in flight
+  int keep = (int)(0.6 * l2 / (span * 32768.0));
+  if (const char* e = getenv("JACAP_KEEP_TILES")) keep = atoi(e);  // tuning override (< 0: no L2 hints)
+  return std::min(std::max(keep, -1), dm.chunk / TILE);
+}
+
+// Items a fused-role CTA takes at a time: about 8 partial Grams per unit for
+// the factor to sum, runs of at most 8192 tokens (a unit's items should finish
+// close in time, for L2).
+int fused_run_items(const Dims& dm, double items_per_unit) {
+  const int by_parts = (int)(items_per_unit / 8.0);
+  int r = std::max(1, std::min(by_parts, 8192 / dm.chunk));
+  if (const char* e = getenv("JACAP_RUN_ITEMS")) r = std::max(1, atoi(e));  // tuning override
+  return r;
+}
+
+// The automatic choice is the separate kernels. Measured on GB300 (config 2:
+// 32 layers x 8 KV heads, n = 32768) the fused launch takes 0.96 ms against
+// 0.80 ms for the Gram, the factor and the scores apart: a unit stays ~150 us
+// between its first Gram tile and its last score tile, so at the pass's rate
+// of V far more than L2 is in flight and only ~12 % of the second read hits
+// L2, while the roles' fill and drain (~80 us each) add to a pass whose
+// separate kernels already run at the effective HBM rate.
+bool fused_pays(const jacap_layout*, const Dims&, int) { return false; }
+
+// 2 (fused, with its roles and kept tiles) or 1 (separate kernels) for a
+// validated layout and params.
+int pick_schedule(const jacap_layout* L, const jacap_params* P, const Dims& dm, int sms, bool dense,
+                  FusedRoles* roles, int* keep, int* run) {
+  const bool fused = L->dtype == JACAP_BF16 && !dense && sms >= 8 &&
+                     (P->schedule == 2 || (P->schedule == 0 && fused_pays(L, dm, sms)));
+  if (!fused) return 1;
+  *roles = fused_roles(L, dm, sms);
+  const double per_plane =
+      L->num_seqs == 1 ? ceil((double)L->total_tokens / dm.chunk) : (double)L->total_tokens / dm.chunk + 0.5 * dm.S;
+  *keep = fused_keep_tiles(dm, *roles, per_plane / dm.S);
+  *run = fused_run_items(dm, per_plane / dm.S);
+  return 2;
 }
 
 // Work items of the pass (plane x chunk): exact for one request, otherwise the
@@ -278,6 +370,7 @@ jacap_status score_pass(const jacap_layout* layout, const jacap_params* params, 
   if (!running && params->cov_unbiased && layout->window < 2) return JACAP_ERR_INVALID_ARG;
   if (params->linear_weighting != 0 && params->linear_weighting != 1) return JACAP_ERR_INVALID_ARG;
   if (params->full_covariance != 0 && params->full_covariance != 1) return JACAP_ERR_INVALID_ARG;
+  if (params->schedule < 0 || params->schedule > 2) return JACAP_ERR_INVALID_ARG;
   if (params->ridge != 1 || (running && params->full_covariance != 0)) return JACAP_ERR_UNSUPPORTED;
   if ((!running && !aligned16(q_win)) || !aligned16(k) || !aligned16(v) || ((uintptr_t)scores & 3u) != 0 ||
       (out_factor != nullptr && !aligned16(out_factor)) || (running && (!aligned16(stats) || ((uintptr_t)counts & 3u))))
@@ -334,10 +427,24 @@ jacap_status score_pass(const jacap_layout* layout, const jacap_params* params, 
   if (dm.full_cov && !fused_full &&  // overwrites the K pass's diagonal kappa; timed with the K pass
       (st = map_cuda(launch_kfull(kmap, dm, w, dt, k, persistent_grid(items, sms, 2), s))) != JACAP_OK)
     return st;
+  // each unit's softmax normaliser from the K pass's chunk statistics (timed with the weights)
+  if ((st = hook(3)) != JACAP_OK || (st = map_cuda(launch_unit_stats(dm, w, s))) != JACAP_OK) return st;
+  FusedRoles roles{0, 0, 0};
+  int keep = 0, run = 1;
+  if (pick_schedule(layout, params, dm, sms, out_factor != nullptr, &roles, &keep, &run) == 2) {
+    // the Gram, the factor and the scores in one launch (timed as the Gram)
+    Dims fd = dm;
+    fd.fused = 1;
+    fd.keep_tiles = keep;
+    fd.run_items = run;
+    if ((st = hook(4)) != JACAP_OK ||
+        (st = map_cuda(launch_fused(vmap, fd, w, scores, roles, s))) != JACAP_OK || (st = hook(5)) != JACAP_OK ||
+        (st = hook(6)) != JACAP_OK || (st = hook(7)) != JACAP_OK)
+      return st;
+    return JACAP_OK;
+  }
   // (bf16 caches: the Gram kernel computes the weights from the K pass's rows)
-  if ((st = hook(3)) != JACAP_OK ||
-      (!bf && (st = map_cuda(launch_weights(dm, w, cu, persistent_grid(items, sms, 8), s))) != JACAP_OK))
-    return st;
+  if (!bf && (st = map_cuda(launch_weights(dm, w, cu, persistent_grid(items, sms, 8), s))) != JACAP_OK) return st;
   if ((st = hook(4)) != JACAP_OK ||
       (st = map_cuda(launch_gram(vmap, dm, w, dt, v, cu, persistent_grid(items, sms, bf ? 1 : 4), s))) != JACAP_OK)
     return st;
@@ -359,6 +466,26 @@ jacap_status jacap_score_out(const jacap_layout* layout, const jacap_params* par
                              size_t ws_bytes, void* stream, void* const* events, int32_t num_events) {
   return score_pass(layout, params, q_win, nullptr, nullptr, k, v, out_factor, scores, ws, ws_bytes, stream, events,
                     num_events);
+}
+
+int32_t jacap_schedule_info(const jacap_layout* layout, const jacap_params* params, int32_t* roles) {
+  jacap_status st = check_layout(layout);
+  if (st != JACAP_OK) return -(int32_t)st;
+  if (params == nullptr || params->schedule < 0 || params->schedule > 2) return -(int32_t)JACAP_ERR_INVALID_ARG;
+  int sms = 0;
+  if ((st = check_device(&sms)) != JACAP_OK) return -(int32_t)st;
+  Dims dm;
+  make_dims(layout, params, dm);
+  FusedRoles r{0, 0, 0};
+  int keep = 0, run = 1;
+  const int sched = pick_schedule(layout, params, dm, sms, false, &r, &keep, &run);
+  if (roles != nullptr) {
+    roles[0] = r.nf;
+    roles[1] = r.ng;
+    roles[2] = r.ns;
+    roles[3] = keep;
+  }
+  return sched;
 }
 
 jacap_status jacap_score_stats(const jacap_layout* layout, const jacap_params* params, const float* stats,

@@ -43,6 +43,10 @@ struct Dims {
   int full_cov;       // 1: kappa with the full window covariance of the queries (App. B.2)
   int kf_rp;          // full covariance on the tensor cores: rows per split part of the query image (else 0)
   int pdl;            // 1: launch with programmatic stream serialization (0 when timing events sit between kernels)
+  int fused;          // 1: the Gram, the factor and the scores run as roles of one persistent launch (k_fused.cu)
+  int keep_tiles;     // fused: V tiles of each Gram item loaded with the L2 evict_last policy (the score
+                      // role reads them again soon after); the item's other tiles are loaded evict_first
+  int run_items;      // fused: consecutive items a role's CTA takes at a time (one partial Gram per run)
 };
 
 // Rows per split part of the full-covariance query image of one KV head's
@@ -59,7 +63,9 @@ struct Ws {
   uint32_t* status;   // [16] status word + first failing unit
   int32_t* plan;      // [0] = chunks per plane C_tot, [1 .. S+1] = chunk prefix per request
   int4* chunks;       // [c_cap] chunk r of every plane: {t0, t1, request, r}
-  int32_t* counters;  // [units] per-unit completion counters (reserved)
+  int32_t* gcount;    // [units] fused schedule: Gram progress of a unit (each item adds 1 for its weights
+                      // and 1 for its partial Gram; complete at 2 x the unit's chunk count)
+  int32_t* fdone;     // [units] fused schedule: 1 once the unit's factor (G, L^{-1} and its image) is written
   float* mu;          // [S][L][Hq][D]  mu / (tau sqrt d)
   float* lam;         // [S][L][Hq][D]  diagonal of Lambda_Q
   float* qdev;        // [S][L][Hq][window][D]  centred window queries q_j - mu (full covariance, CUDA cores)
@@ -67,6 +73,7 @@ struct Ws {
                       // shares qdev's section
   float* lk;          // [L*Hkv][Ntot][2G]  logits then kappa per query head of the group
   float* cstats;      // [L*Hkv][c_cap][G][2]  per-chunk (max, sum exp(l - max))
+  float* ustats;      // [units][G][2]  the unit's softmax normaliser per head: (M_h, 1 / Z_h)
   float* w;           // [L*Hkv][Ntot]  Eq. 8 weights summed over the group
   float* gpart;       // [L*Hkv][c_cap][D/32][D][32]  partial Grams: (m, n) at ((n/32) D + m) 32 + n%32,
                       // lower 32 x 32 blocks only; one per run of a CTA's consecutive chunks of a unit,
@@ -75,7 +82,15 @@ struct Ws {
   float* gram;        // [units][D][D]  sum_i w_i v_i v_i^T
   float* minv;        // [units][D][D]  L^{-1} (float32, lower triangular)
   uint8_t* minv_img;  // [units][65536]  L^{-1} as bf16 hi/lo, shared-memory image for the score MMA
+  unsigned long long* trace;  // [units][8] timeline of the fused schedule (JACAP_TRACE builds only, else null)
 };
+
+// Timeline of the fused schedule, per unit (JACAP_TRACE builds; %globaltimer
+// ns): slot 0 first Gram tile issued (min), 1 last Gram partial published
+// (max), 2 factor start (its wait done), 3 factor published, 4 first score
+// image acquired (min), 5 last score tile finished (max), 6 first score MMA
+// issued (min). The plan kernel resets the slots.
+enum { TR_GRAM0 = 0, TR_GRAM1, TR_FAC0, TR_FAC1, TR_SC_IMG, TR_SC1, TR_SC_MMA, TR_SLOTS = 8 };
 
 // A unit is (plane p = l*Hkv + g, request s); its index is p*S + s.
 struct Item {
@@ -104,7 +119,14 @@ struct ItemStream {
   int nseq, nplanes;
   uint32_t* status;
 #endif
-  __device__ __forceinline__ ItemStream(const Dims& dm, const Ws& ws, int64_t part, int64_t parts) : tab(ws.chunks) {
+  // Strided (the fused schedule): the items are cut into runs of R =
+  // dm.run_items consecutive items and CTA `part` of `parts` walks runs part,
+  // part + parts, ..., so the CTAs of a role sweep the units in order together
+  // and each unit's items finish close in time.
+  int64_t run_end, skip, runlen;
+  __device__ __forceinline__ ItemStream(const Dims& dm, const Ws& ws, int64_t part, int64_t parts,
+                                        bool strided = false)
+      : tab(ws.chunks) {
 #ifdef JACAP_CHECKED
     ntot = dm.Ntot;
     nseq = dm.S;
@@ -113,8 +135,20 @@ struct ItemStream {
 #endif
     ctot = ws.plan[0];
     const int64_t total = (int64_t)dm.L * dm.Hkv * ctot;
-    i = part * total / parts;
-    end = (part + 1) * total / parts;
+    if (strided) {
+      const int64_t R = dm.run_items > 0 ? dm.run_items : 1;
+      i = part * R;
+      run_end = i + R;
+      skip = (parts - 1) * R;
+      runlen = R;
+      end = total;
+    } else {
+      i = part * total / parts;
+      end = (part + 1) * total / parts;
+      run_end = end;
+      skip = 0;
+      runlen = 0;
+    }
     if (i < end) rec = tab[i % ctot];
   }
   __device__ __forceinline__ bool next(Item& it) {
@@ -134,7 +168,10 @@ struct ItemStream {
       return false;
     }
 #endif
-    ++i;
+    if (++i == run_end) {
+      i += skip;
+      run_end = i + runlen;
+    }
     if (i < end) rec = tab[i % ctot];
     return true;
   }
@@ -252,6 +289,20 @@ __device__ __forceinline__ unsigned long long globaltimer() {
   return t;
 }
 
+#ifdef JACAP_TRACE
+__device__ __forceinline__ void trace_min(const Ws& ws, int64_t u, int slot) {
+  if (ws.trace != nullptr) atomicMin(ws.trace + u * TR_SLOTS + slot, globaltimer());
+}
+__device__ __forceinline__ void trace_max(const Ws& ws, int64_t u, int slot) {
+  if (ws.trace != nullptr) atomicMax(ws.trace + u * TR_SLOTS + slot, globaltimer());
+}
+#define JACAP_TRACE_MIN(ws, u, slot) trace_min(ws, u, slot)
+#define JACAP_TRACE_MAX(ws, u, slot) trace_max(ws, u, slot)
+#else
+#define JACAP_TRACE_MIN(ws, u, slot) ((void)0)
+#define JACAP_TRACE_MAX(ws, u, slot) ((void)0)
+#endif
+
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
 }
@@ -345,6 +396,80 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t
       "cp.async.bulk.shared::cta.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
       "l"(src), "r"(bytes), "r"(bar)
       : "memory");
+}
+
+// L2 eviction-priority policies for the .L2::cache_hint forms of the copies
+// below (per instruction; no device-wide L2 setting is touched).
+__device__ __forceinline__ uint64_t policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ uint64_t policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+// tma_load_4d with an L2 cache policy.
+__device__ __forceinline__ void tma_load_4d_hint(uint32_t dst, const CUtensorMap* map, int c0, int c1, int c2,
+                                                 int c3, uint32_t bar, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cta.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3, %4, %5}], [%6], %7;" ::"r"(dst),
+      "l"(map), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(bar), "l"(policy)
+      : "memory");
+}
+
+// bulk_g2s with an L2 cache policy.
+__device__ __forceinline__ void bulk_g2s_hint(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar,
+                                              uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.shared::cta.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::"r"(
+          dst),
+      "l"(src), "r"(bytes), "r"(bar), "l"(policy)
+      : "memory");
+}
+
+// Cross-CTA progress flags of the fused schedule. A producer's threads store
+// their results, each makes them visible device-wide (__threadfence), the
+// producers meet at a barrier, and one of them adds to (or sets) the flag with
+// release semantics; a consumer reads the flag with acquire semantics. Data
+// that the consumer then reads with bulk copies (the async proxy) is ordered
+// after the acquire by fence_proxy_async_global.
+__device__ __forceinline__ int ld_acquire_gpu(const int32_t* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void red_add_release_gpu(int32_t* p, int v) {
+  asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ void st_release_gpu(int32_t* p, int v) {
+  asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+// Bounded wait until *p >= target (acquire). Gives up, returning false, when
+// the pass has failed elsewhere (status word set), when *abort is set, or
+// after WAIT_LIMIT_NS (then it records ST_TIMEOUT and sets *abort).
+static __device__ __noinline__ bool wait_count(const int32_t* p, int target, const Ws& ws, volatile int* abort) {
+  if (ld_acquire_gpu(p) >= target) return true;
+  const unsigned long long t0 = globaltimer();
+  for (uint32_t it = 0;; ++it) {
+    __nanosleep(128);
+    if (ld_acquire_gpu(p) >= target) return true;
+    if ((it & 15u) == 15u) {
+      if ((abort != nullptr && *abort) || status_failed(ws)) return false;
+      if (globaltimer() - t0 > WAIT_LIMIT_NS) {
+        flag(ws, ST_TIMEOUT);
+        if (abort != nullptr) *abort = 1;
+        return false;
+      }
+    }
+  }
 }
 
 __device__ __forceinline__ void prefetch_tmap(const CUtensorMap* map) {

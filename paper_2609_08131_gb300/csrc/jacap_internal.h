@@ -68,12 +68,23 @@ cudaError_t launch_kpass_full(const CUtensorMap& kmap, const Dims& dm, const Ws&
 cudaError_t launch_selftest_wait(const Ws& ws, unsigned long long limit_ns, cudaStream_t st);
 cudaError_t launch_kfull(const CUtensorMap& kmap, const Dims& dm, const Ws& ws, int dtype, const void* k, int grid,
                          cudaStream_t st);
+// The pool-softmax normaliser (M_h, 1 / Z_h) of every unit and query head,
+// merged once from the K pass's chunk statistics into ws.ustats.
+cudaError_t launch_unit_stats(const Dims& dm, const Ws& ws, cudaStream_t st);
 cudaError_t launch_weights(const Dims& dm, const Ws& ws, const int32_t* cu, int grid, cudaStream_t st);
 cudaError_t launch_gram(const CUtensorMap& vmap, const Dims& dm, const Ws& ws, int dtype, const void* v,
                         const int32_t* cu, int grid, cudaStream_t st);
 cudaError_t launch_factor(const Dims& dm, const Ws& ws, const float* out_factor, cudaStream_t st);
 cudaError_t launch_score(const CUtensorMap& vmap, const Dims& dm, const Ws& ws, int dtype, const void* v,
                          const int32_t* cu, float* scores, int grid, cudaStream_t st);
+// The fused schedule (k_fused.cu): CTAs of the factor, Gram and score roles.
+struct FusedRoles {
+  int nf, ng, ns;
+};
+// Gram, factor and scores of a bf16 cache in one cooperative launch of
+// nf + ng + ns CTAs (at most one per SM); dm.keep_tiles set by the caller.
+cudaError_t launch_fused(const CUtensorMap& vmap, const Dims& dm, const Ws& ws, float* scores, const FusedRoles& r,
+                         cudaStream_t st);
 // Selection only when k and kio are null. With k: the kept rows of k and v
 // (dtype 1 = bf16, 0 = float32) are also copied into k_out and v_out, as
 // launch_compact does. With kio: the holes of kio, vio (and pos) are filled in

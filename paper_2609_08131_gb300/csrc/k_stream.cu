@@ -42,6 +42,14 @@ __global__ void __launch_bounds__(256) plan_kernel(Dims dm, Ws ws, const int32_t
     ws.plan[0] = acc;
     s_ctot = acc;
   }
+  // the fused schedule's per-unit progress counters (gcount, then fdone)
+  const int64_t units = (int64_t)dm.L * dm.Hkv * dm.S;
+  for (int64_t i = threadIdx.x; i < 2 * units; i += blockDim.x) ws.gcount[i] = 0;
+#ifdef JACAP_TRACE
+  if (ws.trace != nullptr)
+    for (int64_t i = threadIdx.x; i < TR_SLOTS * units; i += blockDim.x)
+      ws.trace[i] = (i % TR_SLOTS == TR_GRAM0 || i % TR_SLOTS == TR_SC_IMG || i % TR_SLOTS == TR_SC_MMA) ? ~0ull : 0ull;
+#endif
   __syncthreads();
   const int ctot = s_ctot;
   for (int r = threadIdx.x; r < ctot; r += blockDim.x) {

@@ -108,6 +108,11 @@ def test_bad_params_and_buffers_are_rejected_on_the_host():
     assert J.jacap_score(lay, J.jacap_params(weight_div_dk=2), p, p, p, p, p, big, None) == J.JACAP_ERR_INVALID_ARG
     assert J.jacap_score(lay, J.jacap_params(linear_weighting=2), p, p, p, p, p, big, None) == J.JACAP_ERR_INVALID_ARG
     assert J.jacap_score(lay, J.jacap_params(full_covariance=3), p, p, p, p, p, big, None) == J.JACAP_ERR_INVALID_ARG
+    assert J.jacap_score(lay, J.jacap_params(schedule=3), p, p, p, p, p, big, None) == J.JACAP_ERR_INVALID_ARG
+    assert J.jacap_score(lay, J.jacap_params(schedule=-1), p, p, p, p, p, big, None) == J.JACAP_ERR_INVALID_ARG
+    # the schedule query checks its arguments before it asks for a device
+    assert J.jacap_schedule_info(lay, J.jacap_params(schedule=3))[0] == -J.JACAP_ERR_INVALID_ARG
+    assert J.jacap_schedule_info(good_layout(head_dim=64), J.jacap_params())[0] == -J.JACAP_ERR_UNSUPPORTED
     lay1 = good_layout(window=1)
     assert J.jacap_score(lay1, J.jacap_params(cov_unbiased=1), p, p, p, p, p, big, None) == J.JACAP_ERR_INVALID_ARG
     mis = ctypes.c_void_p(0x1008)  # 8-byte aligned only
@@ -176,12 +181,13 @@ def test_host_cache_entry_checks_on_the_host():
 
 
 def test_tracing_and_checked_variants_compile(tmp_path):
-    # JACAP_NVTX=1 / JACAP_CHECKED=1 builds: the host side with its NVTX ranges
-    # and a persistent kernel with the checked work-item stream compile for sm_103a
+    # JACAP_NVTX=1 / JACAP_CHECKED=1 / JACAP_TRACE=1 builds: the host side with
+    # its NVTX ranges and trace section, and a persistent kernel with the checked
+    # work-item stream and the trace resets, compile for sm_103a
     import subprocess
 
     for src in ("jacap_api.cu", "k_stream.cu"):
-        cmd = [_lib.nvcc(), *_lib.ARCH, *_lib.CFLAGS, "-DJACAP_NVTX", "-DJACAP_CHECKED", "-c",
+        cmd = [_lib.nvcc(), *_lib.ARCH, *_lib.CFLAGS, "-DJACAP_NVTX", "-DJACAP_CHECKED", "-DJACAP_TRACE", "-c",
                os.path.join(_lib.CSRC, src), "-o", str(tmp_path / (src + ".o"))]
         r = subprocess.run(cmd, capture_output=True, text=True)
         assert r.returncode == 0, r.stderr[-2000:]

@@ -106,9 +106,20 @@ SMALL = {
 }
 
 
-@pytest.mark.parametrize("name", list(SMALL))
-def test_small_caches_every_unit(name):
+def with_schedule(p, schedule):
+    return jacap_params(p.tau, p.weight_div_dk, p.ridge, p.cov_unbiased, p.linear_weighting, p.full_covariance,
+                        schedule)
+
+
+# every bf16 case under both schedules (separate kernels; the fused persistent
+# launch); float32 caches always take the separate kernels
+SMALL_RUNS = [(n, sch) for n in SMALL for sch in ((1, 2) if SMALL[n][0].dtype == "bf16" else (0,))]
+
+
+@pytest.mark.parametrize("name,schedule", SMALL_RUNS, ids=[f"{n}-s{s}" for n, s in SMALL_RUNS])
+def test_small_caches_every_unit(name, schedule):
     wl, params = SMALL[name]
+    params = with_schedule(params, schedule)
     t = generate(wl, DEV)
     ev = evict(make_cache(t, wl), wl.budget, params)
     for s in range(len(wl.seqlens)):
@@ -118,9 +129,10 @@ def test_small_caches_every_unit(name):
     gpu_selection_properties(ev.scores, ev.idx, ev.kept, wl.seqlens, wl.budget)
 
 
-def test_intermediates_match_the_oracle():
+@pytest.mark.parametrize("schedule", [1, 2])
+def test_intermediates_match_the_oracle(schedule):
     wl = Workload("t", 2, 8, 2, (900, 333), 16, 64, seed=21)
-    params = jacap_params(tau=1.5)
+    params = jacap_params(tau=1.5, schedule=schedule)
     t = generate(wl, DEV)
     ev = evict(make_cache(t, wl), wl.budget, params)
     inter = ev.intermediates()
@@ -164,10 +176,11 @@ def test_layer_groups_bound_the_workspace_and_match_the_oracle():
     gpu_selection_properties(ev.scores, ev.idx, ev.kept, wl.seqlens, wl.budget)
 
 
-def test_repeat_calls_are_bitwise_deterministic():
+@pytest.mark.parametrize("schedule", [1, 2])
+def test_repeat_calls_are_bitwise_deterministic(schedule):
     wl = Workload("t", 2, 8, 2, (1500, 700), 16, 64, seed=22)
     t = generate(wl, DEV)
-    ev = Evictor(make_cache(t, wl), wl.budget)
+    ev = Evictor(make_cache(t, wl), wl.budget, jacap_params(schedule=schedule))
     ev.run()
     ev.check()
     s1, i1 = ev.scores.clone(), ev.idx.clone()
