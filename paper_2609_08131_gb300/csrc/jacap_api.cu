@@ -24,7 +24,7 @@ inline size_t align_up(size_t x) { return (x + ALIGN - 1) & ~(ALIGN - 1); }
 struct Carve {
   size_t status, plan, chunks, counters, mu, lam, qdev, lk, cstats, ustats, w, gpart, pflag, gram, minv,
       minv_img, total;
-  size_t units, trace;
+  size_t units, trace, trace_cta;
 };
 
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
@@ -127,9 +127,11 @@ Carve carve(const Dims& dm) {
   c.minv = o; o = align_up(o + units * D * D * 4);
   c.minv_img = o; o = align_up(o + units * 65536);
 #ifdef JACAP_TRACE
-  c.trace = o; o = align_up(o + units * TR_SLOTS * 8);  // trace builds: the fused schedule's timeline, last
+  c.trace = o; o = align_up(o + units * TR_SLOTS * 8);  // trace builds: the fused schedule's timeline,
+  c.trace_cta = o; o = align_up(o + (size_t)TR_KERNELS * TR_CTAS * TR_CTA_SLOTS * 8);  // then the CTA accounting
 #else
   c.trace = 0;
+  c.trace_cta = 0;
 #endif
   c.total = o;
   return c;
@@ -157,6 +159,7 @@ Ws make_ws(void* base, const Carve& c) {
   ws.minv = (float*)(b + c.minv);
   ws.minv_img = b + c.minv_img;
   ws.trace = c.trace != 0 ? (unsigned long long*)(b + c.trace) : nullptr;
+  ws.trace_cta = c.trace_cta != 0 ? (unsigned long long*)(b + c.trace_cta) : nullptr;
   return ws;
 }
 

@@ -83,6 +83,7 @@ struct Ws {
   float* minv;        // [units][D][D]  L^{-1} (float32, lower triangular)
   uint8_t* minv_img;  // [units][65536]  L^{-1} as bf16 hi/lo, shared-memory image for the score MMA
   unsigned long long* trace;  // [units][8] timeline of the fused schedule (JACAP_TRACE builds only, else null)
+  unsigned long long* trace_cta;  // [TR_KERNELS][TR_CTAS][TR_CTA_SLOTS] per-CTA time accounting (JACAP_TRACE)
 };
 
 // Timeline of the fused schedule, per unit (JACAP_TRACE builds; %globaltimer
@@ -91,6 +92,11 @@ struct Ws {
 // image acquired (min), 5 last score tile finished (max), 6 first score MMA
 // issued (min). The plan kernel resets the slots.
 enum { TR_GRAM0 = 0, TR_GRAM1, TR_FAC0, TR_FAC1, TR_SC_IMG, TR_SC1, TR_SC_MMA, TR_SLOTS = 8 };
+// Per-CTA time accounting of the streaming kernels (JACAP_TRACE builds): for
+// kernel k (TR_K_*) and CTA b, slot j of trace_cta[(k TR_CTAS + b) TR_CTA_SLOTS]
+// sums the ns one role's lane 0 spent in a wait or a busy section (the slot
+// meanings are listed where each kernel records them).
+enum { TR_K_GRAM = 0, TR_K_SCORE = 1, TR_K_KPASS = 2, TR_KERNELS = 3, TR_CTAS = 1024, TR_CTA_SLOTS = 16 };
 
 // A unit is (plane p = l*Hkv + g, request s); its index is p*S + s.
 struct Item {
@@ -298,9 +304,27 @@ __device__ __forceinline__ void trace_max(const Ws& ws, int64_t u, int slot) {
 }
 #define JACAP_TRACE_MIN(ws, u, slot) trace_min(ws, u, slot)
 #define JACAP_TRACE_MAX(ws, u, slot) trace_max(ws, u, slot)
+// time accounting: TRC_T(v) starts a stopwatch, TRC_ADD(acc, v) adds its
+// elapsed ns to acc, TRC_PUT(ws, k, slot, acc) adds acc to the CTA's slot
+#define TRC_DECL(n) unsigned long long trc[n] = {}
+#define TRC_T(v) const unsigned long long v = globaltimer()
+#define TRC_ADD(i, v) (trc[i] += globaltimer() - (v))
+#define TRC_INC(i) (++trc[i])
+#define TRC_PUT(ws, k, n)                                                                                \
+  do {                                                                                                 \
+    if ((ws).trace_cta != nullptr && blockIdx.x < TR_CTAS)                                             \
+      for (int trc_j = 0; trc_j < (n); ++trc_j)                                                        \
+        if (trc[trc_j])                                                                                \
+          atomicAdd((ws).trace_cta + ((size_t)(k) * TR_CTAS + blockIdx.x) * TR_CTA_SLOTS + trc_j, trc[trc_j]); \
+  } while (0)
 #else
 #define JACAP_TRACE_MIN(ws, u, slot) ((void)0)
 #define JACAP_TRACE_MAX(ws, u, slot) ((void)0)
+#define TRC_DECL(n) ((void)0)
+#define TRC_T(v) ((void)0)
+#define TRC_ADD(i, v) ((void)0)
+#define TRC_INC(i) ((void)0)
+#define TRC_PUT(ws, k, n) ((void)0)
 #endif
 
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {

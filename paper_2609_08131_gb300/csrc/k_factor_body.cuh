@@ -41,7 +41,9 @@ constexpr int FB_LD = 36;             // row stride of a 32 x 32 block (floats);
 constexpr int FB_BLK = 32 * FB_LD;    // floats per block
 // 10 lower blocks of A (then L_IJ, and T_II on the diagonal) and 10 blocks of
 // XT (XT_JI at tri(I, J); S_IJ^T there until X_IJ replaces it)
-constexpr size_t FB_SMEM = (size_t)20 * FB_BLK * sizeof(float);
+// 10 lower blocks of A and 10 of XT, then the elimination's buffers (192 floats)
+constexpr int FB_ELIM = 192;
+constexpr size_t FB_SMEM = ((size_t)20 * FB_BLK + FB_ELIM) * sizeof(float);
 
 __device__ __forceinline__ int tri(int i, int j) { return i * (i + 1) / 2 + j; }  // block (i, j), j <= i
 // a partial Gram's lower blocks staged in shared memory: column block nb,
@@ -52,7 +54,12 @@ static_assert(2 * FB_STAGE <= 20 * FB_BLK, "the staging ring fits in the A and X
 // partials in flight: 2 in the factor kernel (two CTAs per SM), 5 in the fused
 // schedule's factor role (one CTA per SM, the shared memory of the Gram role)
 template <bool FUSED> __host__ __device__ constexpr int fb_stages() { return FUSED ? 5 : 2; }
-constexpr size_t FB_FUSED_SMEM = (size_t)fb_stages<true>() * FB_STAGE * sizeof(float);
+// floats before the elimination buffers: the A and XT blocks, or the staging ring if that is longer
+template <bool FUSED> __host__ __device__ constexpr int fb_elim_at() {
+  return 20 * FB_BLK > fb_stages<FUSED>() * FB_STAGE ? 20 * FB_BLK : fb_stages<FUSED>() * FB_STAGE;
+}
+static_assert(fb_elim_at<false>() == 20 * FB_BLK, "the factor kernel's shared memory");
+constexpr size_t FB_FUSED_SMEM = ((size_t)fb_elim_at<true>() + FB_ELIM) * sizeof(float);
 
 // The barrier of the factor's FB_THREADS threads (named barrier 1: in the
 // fused schedule the factor runs on the first FB_THREADS threads of a larger CTA).
@@ -270,7 +277,7 @@ __device__ __forceinline__ void factor_blocked_cta(const Dims& dm, const Ws& ws,
   float* XT = fsm + 10 * FB_BLK;  // tri(I, J): XT_JI = (L^{-1})_IJ^T
   constexpr int NST = fb_stages<FUSED>();
   __shared__ __align__(8) uint64_t s_full[NST];
-  __shared__ __align__(16) float s_elim[192];  // the elimination's row and column buffers, pivots, reciprocals
+  float* s_elim = fsm + fb_elim_at<FUSED>();  // the elimination's row and column buffers, pivots, reciprocals
   __shared__ int s_skip, s_bad, s_np;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) {

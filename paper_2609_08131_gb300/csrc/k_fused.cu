@@ -63,7 +63,7 @@ template <int G>
 static cudaError_t launch_fused_g(const CUtensorMap& vmap, const Dims& dm, const Ws& ws, float* scores,
                                   const FusedRoles& r, cudaStream_t st) {
   constexpr size_t smem = fused_smem_bytes<G>();
-  static_assert(smem + 1024 <= 232448, "shared memory of the fused kernel (1 KB for static variables)");
+  static_assert(smem + 256 <= 232448, "shared memory of the fused kernel (256 B for static variables)");
   cudaError_t e = cudaFuncSetAttribute(fused_gfs_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};

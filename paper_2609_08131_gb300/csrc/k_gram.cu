@@ -37,7 +37,7 @@ template <int G>
 __global__ void __launch_bounds__(WT_THREADS) weight_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu) {
   pdl_wait();
   __shared__ int s_skip;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int tid = threadIdx.x;
   if (tid == 0) s_skip = status_failed(ws) ? 1 : 0;
   __syncthreads();
   if (s_skip) return;

@@ -164,6 +164,9 @@ __device__ __forceinline__ void gram_bf16_body(const CUtensorMap* vmap_p, const 
         keep = policy_evict_last();
         drop = policy_evict_first();
       }
+      // time accounting (trace builds): 0 waits for a free stage, 1 the whole loop
+      TRC_DECL(TR_CTA_SLOTS);
+      TRC_T(tr_all);
       uint32_t it = 0;
       bool ok = true;
       Item item;
@@ -172,11 +175,13 @@ __device__ __forceinline__ void gram_bf16_body(const CUtensorMap* vmap_p, const 
         if (FUSED) JACAP_TRACE_MIN(ws, (int64_t)item.plane * dm.S + item.seq, TR_GRAM0);
         for (int64_t t = item.t0; t < item.t1; t += TILE) {
           const int st = it % GR_VST;
+          TRC_T(tr_w);
           if (it >= (uint32_t)GR_VST &&
               !mbar_wait(smem_u32(&vempty[st]), ((it / GR_VST) & 1) ^ 1, ws, abort)) {
             ok = false;
             break;
           }
+          TRC_ADD(0, tr_w);
           uint8_t* vt = vring + st * GR_V_BYTES;
           const LkTile lt = lk_tile<G>(dm, item, t);
           const uint32_t bar = smem_u32(&vfull[st]);
@@ -194,12 +199,18 @@ __device__ __forceinline__ void gram_bf16_body(const CUtensorMap* vmap_p, const 
           ++it;
         }
       }
+      TRC_ADD(1, tr_all);
+      TRC_PUT(ws, TR_K_GRAM, 2);
       for (uint32_t k = (it > (uint32_t)GR_VST ? it - GR_VST : 0); k < it; ++k)
         mbar_wait(smem_u32(&vfull[k % GR_VST]), (k / GR_VST) & 1, ws, nullptr);
     }
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer ----------
     if (lane == 0) {
+      // time accounting (trace builds): 2 waits for a scaled operand, 3 for a free
+      // accumulator (run start), 4 the whole loop, 5 tiles
+      TRC_DECL(TR_CTA_SLOTS);
+      TRC_T(tr_all);
       uint32_t it = 0, nrun = 0;
       bool ok = true, cont = false, first = true;
       int db = 0;
@@ -209,7 +220,9 @@ __device__ __forceinline__ void gram_bf16_body(const CUtensorMap* vmap_p, const 
         // takes the other buffer once its previous run's epilogue is done
         if (!cont) {
           db = nrun & 1;
+          TRC_T(tr_a);
           if (nrun >= 2 && !mbar_wait(smem_u32(&accempty[db]), ((nrun >> 1) & 1) ^ 1, ws, abort)) break;
+          TRC_ADD(3, tr_a);
           tc_fence_after();
           first = true;
         }
@@ -217,10 +230,13 @@ __device__ __forceinline__ void gram_bf16_body(const CUtensorMap* vmap_p, const 
         for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
           const int vs = it % GR_VST, ab = it & 1;
           // the scaling warps arrive on afull only after the tile's V landed
+          TRC_T(tr_f);
           if (!mbar_wait(smem_u32(&afull[ab]), (it >> 1) & 1, ws, abort)) {
             ok = false;
             break;
           }
+          TRC_ADD(2, tr_f);
+          TRC_INC(5);
           tc_fence_after();
           // B descriptors advance by (byte offset >> 4) in their address field
           const uint64_t b0 = smem_desc_sw128(smem_u32(vring + vs * GR_V_BYTES), GR_BOX, 1024);
@@ -243,6 +259,8 @@ __device__ __forceinline__ void gram_bf16_body(const CUtensorMap* vmap_p, const 
         }
       }
       if (it > 0) mbar_wait(smem_u32(&aempty[(it - 1) & 1]), ((it - 1) >> 1) & 1, ws, nullptr);
+      TRC_ADD(4, tr_all);
+      TRC_PUT(ws, TR_K_GRAM, 6);
     }
   } else if (warp < 10) {
     // ------------------------------------------------- scaling warps ------
@@ -250,14 +268,21 @@ __device__ __forceinline__ void gram_bf16_body(const CUtensorMap* vmap_p, const 
     const int th = (warp - 2) >> 2;      // token half of each tile (blocks 4 th .. 4 th + 3)
     // ldmatrix row addresses: lane l -> matrix l / 8, row l % 8
     const int lm = lane >> 3, lr = lane & 7;
+    // time accounting (trace builds, warp 2): 6 waits for V, 7 for the weights,
+    // 8 for a free operand buffer, 9 scaling, 10 the whole loop
+    TRC_DECL(TR_CTA_SLOTS);
+    TRC_T(tr_all);
     uint32_t it = 0;
     Item item;
     for (ItemStream is(dm, ws, part, parts, FUSED); is.next(item);) {
       for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
         const int vs = it % GR_VST, ab = it & 1;
-        if (!mbar_wait(smem_u32(&vfull[vs]), (it / GR_VST) & 1, ws, abort) ||
-            !mbar_wait(smem_u32(&wready[vs]), (it / GR_VST) & 1, ws, abort))
-          goto scale_done;
+        TRC_T(tr_v);
+        if (!mbar_wait(smem_u32(&vfull[vs]), (it / GR_VST) & 1, ws, abort)) goto scale_done;
+        TRC_ADD(6, tr_v);
+        TRC_T(tr_wr);
+        if (!mbar_wait(smem_u32(&wready[vs]), (it / GR_VST) & 1, ws, abort)) goto scale_done;
+        TRC_ADD(7, tr_wr);
         // weights of this lane's token pairs (rows 2(l%4), 2(l%4)+1 of each
         // 8-token half of its 4 blocks) as bf16 pairs; tokens past the item
         // weigh zero
@@ -274,7 +299,10 @@ __device__ __forceinline__ void gram_bf16_body(const CUtensorMap* vmap_p, const 
             wpl[e] = __byte_perm(x0, x1, 0x7632);  // (lo, lo)
           }
         }
+        TRC_T(tr_ae);
         if (it >= 2 && !mbar_wait(smem_u32(&aempty[ab]), ((it >> 1) & 1) ^ 1, ws, abort)) goto scale_done;
+        TRC_ADD(8, tr_ae);
+        TRC_T(tr_b);
         tc_fence_after();
         const uint32_t vt = smem_u32(vring + vs * GR_V_BYTES);
         const uint32_t acol = tmem + GR_ACOL + 128 * ab;
@@ -308,15 +336,22 @@ __device__ __forceinline__ void gram_bf16_body(const CUtensorMap* vmap_p, const 
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_u32(&afull[ab]));
+        TRC_ADD(9, tr_b);
       }
     }
   scale_done:;
+    TRC_ADD(10, tr_all);
+    if (warp == 2 && lane == 0) TRC_PUT(ws, TR_K_GRAM, 11);
   } else if (warp >= GR_WEIGHT_WARP) {
     // ------------------------------------------------------ weights -------
     // Eq. 8 for the tile's tokens (two per lane of each of the two warps) from the staged logits and
     // kappa: w = wdiv sum_h rho_h^2 kappa_h, rho = alpha_bar (1 - alpha_bar),
     // alpha_bar = exp(l_h - M_h) / Z_h (rho = 1 for the linear surrogate);
     // (M_h, Z_h) merged from the unit's chunk statistics once per run.
+    // time accounting (trace builds, first weight warp): 11 waits for V, 12 the
+    // weights of a tile, 13 the whole loop
+    TRC_DECL(TR_CTA_SLOTS);
+    TRC_T(tr_all);
     uint32_t it = 0;
     bool bad = false, cont = false;
     float u[2 * G];  // M_h, then 1 / Z_h (from the unit-statistics kernel)
@@ -329,7 +364,10 @@ __device__ __forceinline__ void gram_bf16_body(const CUtensorMap* vmap_p, const 
       const int64_t base = (int64_t)item.plane * dm.Ntot;
       for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
         const int vs = it % GR_VST;
+        TRC_T(tr_v);
         if (!mbar_wait(smem_u32(&vfull[vs]), (it / GR_VST) & 1, ws, abort)) goto weights_done;
+        TRC_ADD(11, tr_v);
+        TRC_T(tr_b);
         const LkTile lt = lk_tile<G>(dm, item, t);
         const float* rows = (const float*)(lkring + vs * C::LK_BYTES) + lt.off;
         uint32_t* wout = (uint32_t*)(wring + vs * GR_W_BYTES);
@@ -364,6 +402,7 @@ __device__ __forceinline__ void gram_bf16_body(const CUtensorMap* vmap_p, const 
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_u32(&wready[vs]));
+        TRC_ADD(12, tr_b);
       }
       if (FUSED) {  // this warp's weights of the item are stored: its share of the unit's progress
         __threadfence();
@@ -372,6 +411,8 @@ __device__ __forceinline__ void gram_bf16_body(const CUtensorMap* vmap_p, const 
       }
     }
   weights_done:
+    TRC_ADD(13, tr_all);
+    if (warp == GR_WEIGHT_WARP && lane == 0) TRC_PUT(ws, TR_K_GRAM, 14);
     if (bad) flag(ws, ST_NONFINITE);
   } else {
     // ------------------------------------------------------ epilogue ------

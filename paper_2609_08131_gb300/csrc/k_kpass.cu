@@ -190,15 +190,20 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
       uint32_t it = 0;
       bool ok = true;
       Item item;
+      // time accounting (trace builds): 0 waits for a free stage, 1 the whole loop
+      TRC_DECL(TR_CTA_SLOTS);
+      TRC_T(tr_all);
       for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); ok && is.next(item);) {
         const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
         for (int64_t t = item.t0; t < item.t1; t += TILE) {
           const int st = it % KB_STAGES;
+          TRC_T(tr_w);
           if (it >= (uint32_t)KB_STAGES &&
               !mbar_wait(smem_u32(&empty[st]), ((it / KB_STAGES) & 1) ^ 1, ws, abort)) {
             ok = false;
             break;
           }
+          TRC_ADD(0, tr_w);
           uint8_t* kt = tiles + st * KB_TILE_BYTES;
           mbar_arrive_expect_tx(smem_u32(&full[st]), KB_TILE_BYTES);
           tma_load_4d(smem_u32(kt), &kmap, 0, (int)t, g, l, smem_u32(&full[st]));
@@ -206,6 +211,8 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
           ++it;
         }
       }
+      TRC_ADD(1, tr_all);
+      TRC_PUT(ws, TR_K_KPASS, 2);
       for (uint32_t k = (it > (uint32_t)KB_STAGES ? it - KB_STAGES : 0); k < it; ++k)
         mbar_wait(smem_u32(&full[k % KB_STAGES]), (k / KB_STAGES) & 1, ws, nullptr);
     }
@@ -216,22 +223,31 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
       bool ok = true, cont = false;
       int p = 0;
       Item item;
+      // time accounting (trace builds): 2 waits for an image, 3 for a K tile and a free
+      // logits buffer, 5 the whole loop, 6 tiles
+      TRC_DECL(TR_CTA_SLOTS);
+      TRC_T(tr_all);
       for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); ok && is.next(item);) {
         if (!cont) {
           p = nrun & 1;
+          TRC_T(tr_i);
           if (!mbar_wait(smem_u32(&imgready[p]), (nrun >> 1) & 1, ws, abort)) break;
+          TRC_ADD(2, tr_i);
           tc_fence_after();
         }
         const uint64_t b0 = smem_desc_sw128(smem_u32(img + p * C::IMG_BYTES), 16, 1024);
         for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
           const int st = it % KB_STAGES;
           const int ab = it % KB_NACC;
+          TRC_T(tr_f);
           if (!mbar_wait(smem_u32(&full[st]), (it / KB_STAGES) & 1, ws, abort) ||
               (it >= (uint32_t)KB_NACC &&
                !mbar_wait(smem_u32(&accempty[ab]), ((it / KB_NACC) & 1) ^ 1, ws, abort))) {
             ok = false;
             break;
           }
+          TRC_ADD(3, tr_f);
+          TRC_INC(6);
           tc_fence_after();
           // descriptors advance by (byte offset >> 4) in their address field
           const uint64_t a0 = smem_desc_sw128(smem_u32(tiles + st * KB_TILE_BYTES), 16, 1024);
@@ -254,6 +270,8 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
       }
       // every MMA issued here completes before the CTA tears down tensor memory
       if (it > 0) mbar_wait(smem_u32(&accfull[(it - 1) % KB_NACC]), ((it - 1) / KB_NACC) & 1, ws, nullptr);
+      TRC_ADD(5, tr_all);
+      TRC_PUT(ws, TR_K_KPASS, 7);
     }
   } else if (warp == KB_BUILD_WARP) {
     // ------------------ mu' image and lambda, once per run, one run ahead
@@ -287,6 +305,10 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
     bool bad = false, cont = false;
     int p = 0;
     Item item;
+    // time accounting (trace builds, warp 2): 7 waits for a K tile, 8 its quarter
+    // of kappa, 9 the first group barrier, 10 the reduction and the store, 11 the loop
+    TRC_DECL(TR_CTA_SLOTS);
+    TRC_T(tr_all);
     // A failed wait (which means the abort flag is set) still arrives at the
     // group's named barriers, and the four warps leave together after them.
     // All four see the same runs (the same item stream), so they meet at the
@@ -305,8 +327,12 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
           if ((int)(it & 1) != grp) continue;
           const int st = it % KB_STAGES;
           float part[4][G];
+          TRC_T(tr_f);
           if (mbar_wait(smem_u32(&full[st]), (it / KB_STAGES) & 1, ws, abort)) {
+            TRC_ADD(7, tr_f);
+            TRC_T(tr_k);
             kappa_quarter<G>(smem_u32(tiles + st * KB_TILE_BYTES), lam_s, lane, cq, part);
+            TRC_ADD(8, tr_k);
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&empty[st]));
             // hand the other three token subsets to their owners
@@ -316,7 +342,10 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
 #pragma unroll
                 for (int h = 0; h < G; ++h) slot[((j * 4 + cq) * G + h) * 32 + lane] = part[j][h];
           }
+          TRC_T(tr_b);
           named_barrier_sync(bar_id, 128);
+          TRC_ADD(9, tr_b);
+          TRC_T(tr_r);
           if (*abort) goto kappa_done;
           float kap[G];
 #pragma unroll
@@ -339,6 +368,7 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
           named_barrier_sync(bar_id, 128);  // the slots may be rewritten after this
           const int64_t tok = t + lane + 32 * cq;
           if (tok < item.t1) store_floats<G, LkAlign<G>::KAPPA>(lkp + tok * (2 * G), kap);
+          TRC_ADD(10, tr_r);
         }
       }
       cont = is.next_same_unit(item);
@@ -349,6 +379,8 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
       }
     }
   kappa_done:
+    TRC_ADD(11, tr_all);
+    if (warp == KB_KAPPA_WARP0 && lane == 0) TRC_PUT(ws, TR_K_KPASS, 12);
     if (bad) flag(ws, ST_NONFINITE);
   } else if (warp >= KB_READ_WARP0 && warp < KB_READ_WARP0 + 4) {
     // ------------------------------------------ logits readout + stats ----
@@ -360,6 +392,10 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
     bool bad = false, cont = false;
     float run_m[G], run_s[G];
     Item item;
+    // time accounting (trace builds, first readout warp): 12 waits for logits, 13 the
+    // readout of a tile, 14 the whole loop
+    TRC_DECL(TR_CTA_SLOTS);
+    TRC_T(tr_all);
     for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
       if (!cont) {  // a new run of the unit's consecutive chunks: fresh statistics
 #pragma unroll
@@ -371,7 +407,10 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
       float* lkp = ws.lk + (int64_t)item.plane * dm.Ntot * (2 * G);
       for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
         const int ab = it % KB_NACC;
+        TRC_T(tr_f);
         if (!mbar_wait(smem_u32(&accfull[ab]), (it / KB_NACC) & 1, ws, abort)) break;  // abort: see below
+        TRC_ADD(12, tr_f);
+        TRC_T(tr_b);
         tc_fence_after();
         float dv[C::NB];
         if constexpr (C::NB == 16) tmem_ld16(tmem + ab * C::NB + lanes, dv);
@@ -395,6 +434,7 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
           }
           store_floats<G, LkAlign<G>::ROW>(lkp + tok * (2 * G), lg);
         }
+        TRC_ADD(13, tr_b);
       }
       // ---- softmax statistics of a run, at its last chunk; the run's other
       // chunks get empty statistics (m = -inf, s = 0), which merge as nothing
@@ -429,6 +469,8 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
       named_barrier_sync(1, 128);
     }
   read_done:
+    TRC_ADD(14, tr_all);
+    if (warp == KB_READ_WARP0 && lane == 0) TRC_PUT(ws, TR_K_KPASS, 15);
     if (bad) flag(ws, ST_NONFINITE);
   }
   tc_fence_before();

@@ -8,7 +8,10 @@
 namespace jacap {
 
 
-constexpr int SC_THREADS = 224;  // warp 0: V tiles (TMA), warp 1: MMA, warps 2-5: epilogue, warp 6: images
+// warp 0: V tiles (TMA), 1: MMA, 2-5 and 7-10: epilogue (two warps per tensor-memory
+// lane quarter, each half of the accumulator's columns), 6: images
+constexpr int SC_THREADS = 352;
+constexpr int SC_EPI_B0 = 7;  // first warp of the second epilogue group
 template <bool DENSE> __host__ __device__ constexpr int sc_stages() { return DENSE ? 3 : 4; }  // V tiles in flight
 template <bool DENSE> __host__ __device__ constexpr int sc_imgs() { return 2; }  // L^{-1} image buffers
 constexpr int SC_BOX = 16384;
@@ -36,12 +39,13 @@ constexpr int SC_MT_BYTES = 49152;
 template <bool DENSE> __host__ __device__ constexpr int sc_img_bytes() { return DENSE ? SC_M_BYTES : SC_MT_BYTES; }
 template <bool DENSE>
 constexpr size_t score_bf16_smem_bytes() {
-  return 1024 + sc_imgs<DENSE>() * sc_img_bytes<DENSE>() + sc_stages<DENSE>() * SC_TILE_BYTES + 256;
+  // + 17 mbarriers (136 B, rounded to 144) + the epilogue groups' partial sums (2 x 128 floats)
+  return 1024 + sc_imgs<DENSE>() * sc_img_bytes<DENSE>() + sc_stages<DENSE>() * SC_TILE_BYTES + 144 + 1024;
 }
 
 // DENSE: the score matrix is a full 128 x 128 (output directions) rather than
 // the lower-triangular L^{-1}, so no K-step may be narrowed.
-// The score pass of CTA `part` of `parts` (warps 0-6 work; further warps of
+// The score pass of CTA `part` of `parts` (warps 0-10 work; further warps of
 // the CTA only meet its barriers). FUSED: the role of the fused schedule
 // (k_fused.cu): items strided over the role's CTAs, V tiles loaded with the L2
 // evict_first policy (the Gram role left the first tiles of each item in L2),
@@ -64,6 +68,7 @@ __device__ __forceinline__ void score_bf16_body(const CUtensorMap* vmap_p, const
   uint64_t* mfull = accempty + 2;   // [2]
   uint64_t* mempty = mfull + 2;     // [2]
   uint64_t* mdone = mempty + 2;
+  float* s_part = (float*)(stages + SC_STAGES * SC_TILE_BYTES + 144);  // [2][128] second group's partial sums
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort, s_skip;
 
@@ -77,7 +82,7 @@ __device__ __forceinline__ void score_bf16_body(const CUtensorMap* vmap_p, const
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&accfull[i]), 1);
-      mbar_init(smem_u32(&accempty[i]), 4);
+      mbar_init(smem_u32(&accempty[i]), 8);  // the eight epilogue warps
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&mfull[i]), 1);
@@ -106,15 +111,20 @@ __device__ __forceinline__ void score_bf16_body(const CUtensorMap* vmap_p, const
       uint32_t it = 0;
       bool ok = true;
       Item item;
+      // time accounting (trace builds): 0 waits for a free stage, 1 the whole loop
+      TRC_DECL(TR_CTA_SLOTS);
+      TRC_T(tr_all);
       for (ItemStream is(dm, ws, part, parts, FUSED); ok && is.next(item);) {
         const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
         for (int64_t t = item.t0; t < item.t1; t += TILE) {
           const int st = it % SC_STAGES;
+          TRC_T(tr_w);
           if (it >= (uint32_t)SC_STAGES &&
               !mbar_wait(smem_u32(&vempty[st]), ((it / SC_STAGES) & 1) ^ 1, ws, abort)) {
             ok = false;
             break;
           }
+          TRC_ADD(0, tr_w);
           uint8_t* vt = stages + st * SC_TILE_BYTES;
           mbar_arrive_expect_tx(smem_u32(&vfull[st]), SC_TILE_BYTES);
           if (hints) {
@@ -127,6 +137,8 @@ __device__ __forceinline__ void score_bf16_body(const CUtensorMap* vmap_p, const
           ++it;
         }
       }
+      TRC_ADD(1, tr_all);
+      TRC_PUT(ws, TR_K_SCORE, 2);
       for (uint32_t k = (it > (uint32_t)SC_STAGES ? it - SC_STAGES : 0); k < it; ++k)
         mbar_wait(smem_u32(&vfull[k % SC_STAGES]), (k / SC_STAGES) & 1, ws, nullptr);
     }
@@ -169,10 +181,16 @@ __device__ __forceinline__ void score_bf16_body(const CUtensorMap* vmap_p, const
       bool ok = true, cont = false;
       int mp = 0;
       Item item;
+      // time accounting (trace builds): 2 waits for an image, 3 for a free
+      // accumulator, 4 for a V tile, 5 the whole loop, 6 tiles
+      TRC_DECL(TR_CTA_SLOTS);
+      TRC_T(tr_all);
       for (ItemStream is(dm, ws, part, parts, FUSED); ok && is.next(item);) {
         if (!cont) {
           mp = nrun % SC_IMGS;
+          TRC_T(tr_m);
           if (!mbar_wait(smem_u32(&mfull[mp]), (nrun / SC_IMGS) & 1, ws, abort)) break;
+          TRC_ADD(2, tr_m);
           tc_fence_after();
           if (FUSED) JACAP_TRACE_MIN(ws, (int64_t)item.plane * dm.S + item.seq, TR_SC_MMA);
         }
@@ -180,14 +198,19 @@ __device__ __forceinline__ void score_bf16_body(const CUtensorMap* vmap_p, const
         for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
           const int st = it % SC_STAGES;
           const int ab = it & 1;
+          TRC_T(tr_a);
           if (it >= 2 && !mbar_wait(smem_u32(&accempty[ab]), ((it >> 1) & 1) ^ 1, ws, abort)) {
             ok = false;
             break;
           }
+          TRC_ADD(3, tr_a);
+          TRC_T(tr_v);
           if (!mbar_wait(smem_u32(&vfull[st]), (it / SC_STAGES) & 1, ws, abort)) {
             ok = false;
             break;
           }
+          TRC_ADD(4, tr_v);
+          TRC_INC(6);
           tc_fence_after();
           // descriptors advance by (byte offset >> 4); image rows: hi at row n,
           // lo at row 128 + n (16 KB further) of each 32 KB channel atom
@@ -219,62 +242,111 @@ __device__ __forceinline__ void score_bf16_body(const CUtensorMap* vmap_p, const
       // every MMA issued by this thread has completed before teardown
       umma_commit(smem_u32(mdone));
       mbar_wait(smem_u32(mdone), 0, ws, nullptr);
+      TRC_ADD(5, tr_all);
+      TRC_PUT(ws, TR_K_SCORE, 7);
     }
-  } else if (warp < 6) {
+  } else if (warp < 6 || (warp >= SC_EPI_B0 && warp < SC_EPI_B0 + 4)) {
+    // Epilogue: warp w reads tensor-memory lanes 32 (w % 4) .. + 31 (one token
+    // per thread). Group 0 (warps 2-5) reduces the first half of the
+    // accumulator's columns, group 1 (warps 7-10) the second half and leaves
+    // its partial sums in shared memory; the two warps of a lane quarter meet
+    // at a named barrier (1 + quarter) per tile and group 0 adds, multiplies
+    // by w and stores the score. A warp whose wait failed still meets its
+    // partner at the tile's barrier; both leave after it.
     const int quarter = warp & 3;
+    const int grp = warp < 6 ? 0 : 1;
     const int y = quarter * 32 + lane;  // token row of the tile == TMEM lane
+    constexpr int HALF = sc_acc_cols<DENSE>() / 2;
     uint32_t it = 0;
     bool bad = false, cont = false;
     Item item;
+    // time accounting (trace builds, warp 2): 7 waits for an accumulator,
+    // 8 reading and reducing it, 9 the rest of the tile, 10 the whole loop
+    TRC_DECL(TR_CTA_SLOTS);
+    TRC_T(tr_all);
     for (ItemStream is(dm, ws, part, parts, FUSED); is.next(item);) {
-      if (FUSED && !cont) {  // the unit's weights are complete once its factor is published
-        bool ok = true;
-        if (lane == 0) ok = wait_count(ws.fdone + (int64_t)item.plane * dm.S + item.seq, 1, ws, abort);
-        if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) goto epi_done;
+      bool unit_ok = true;
+      if (FUSED && !cont && grp == 0) {  // the unit's weights are complete once its factor is published
+        if (lane == 0) unit_ok = wait_count(ws.fdone + (int64_t)item.plane * dm.S + item.seq, 1, ws, abort);
+        unit_ok = __shfl_sync(0xffffffffu, unit_ok ? 1 : 0, 0) != 0;
+        if (!unit_ok && lane == 0) *abort = 1;  // the partner leaves after the next barrier
         __syncwarp();  // the lanes' loads of w come after lane 0's acquire
       }
       cont = is.next_same_unit(item);
-      for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
+      // group 0 loads each tile's w two tiles ahead, into two registers used in
+      // turn (the loop takes two tiles per round), so the loads' latency, about
+      // a tile's time, overlaps the reductions of the tiles before them
+      const float* wrow = ws.w + (int64_t)item.plane * dm.Ntot + y;
+      auto wload = [&](int64_t tt) -> float { return (grp == 0 && unit_ok && tt + y < item.t1) ? wrow[tt] : 0.f; };
+      // one tile; false once the epilogue has to stop
+      auto tile = [&](int64_t t, float wt) -> bool {
         const int ab = it & 1;
         const int64_t tok = t + y;
-        const int64_t o = (int64_t)item.plane * dm.Ntot + tok;
-        const float wt = tok < item.t1 ? ws.w[o] : 0.f;  // issued before the wait: hides its latency
-        if (!mbar_wait(smem_u32(&accfull[ab]), (it >> 1) & 1, ws, abort)) goto epi_done;
-        tc_fence_after();
-        const uint32_t trow = tmem + ab * sc_acc_cols<DENSE>() + ((uint32_t)(quarter * 32) << 16);
+        TRC_T(tr_f);
+        const bool ok = unit_ok && mbar_wait(smem_u32(&accfull[ab]), (it >> 1) & 1, ws, abort);
+        TRC_ADD(7, tr_f);
+        TRC_T(tr_r);
         float ssq = 0.f;
-        if (DENSE) {
+        if (ok) {
+          tc_fence_after();
+          const uint32_t trow =
+              tmem + ab * sc_acc_cols<DENSE>() + grp * HALF + ((uint32_t)(quarter * 32) << 16);
+          if (DENSE) {
 #pragma unroll 1
-          for (int cb = 0; cb < 4; ++cb) {
-            float a[32];
-            tmem_ld32(trow + cb * 32, a);
+            for (int cb = 0; cb < HALF / 32; ++cb) {
+              float a[32];
+              tmem_ld32(trow + cb * 32, a);
 #pragma unroll
-            for (int j = 0; j < 32; ++j) ssq = fmaf(a[j], a[j], ssq);
-          }
-        } else {  // y = hi + lo, block by block: columns 32 b + t and 32 b + 16 + t
+              for (int j = 0; j < 32; ++j) ssq = fmaf(a[j], a[j], ssq);
+            }
+          } else {  // y = hi + lo, block by block: columns 32 b + t and 32 b + 16 + t
 #pragma unroll 1
-          for (int cb = 0; cb < 8; ++cb) {
-            float a[32];
-            tmem_ld32(trow + cb * 32, a);
+            for (int cb = 0; cb < HALF / 32; cb += 2) {
+              uint32_t a[32], b2[32];
+              tmem_ld32x2(trow + cb * 32, trow + cb * 32 + 32, a, b2);
 #pragma unroll
-            for (int j = 0; j < 16; ++j) {
-              const float yv = a[j] + a[16 + j];
-              ssq = fmaf(yv, yv, ssq);
+              for (int j = 0; j < 16; ++j) {
+                const float y0 = __uint_as_float(a[j]) + __uint_as_float(a[16 + j]);
+                const float y1 = __uint_as_float(b2[j]) + __uint_as_float(b2[16 + j]);
+                ssq = fmaf(y0, y0, ssq);
+                ssq = fmaf(y1, y1, ssq);
+              }
             }
           }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&accempty[ab]));
+          if (grp == 1) s_part[ab * TILE + y] = ssq;
         }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(smem_u32(&accempty[ab]));
-        if (tok < item.t1) {
-          const float sc = wt * ssq;
-          scores[o] = sc;
+        named_barrier_sync(1 + quarter, 64);
+        TRC_ADD(8, tr_r);
+        if (!ok || *abort) return false;
+        TRC_T(tr_s);
+        if (grp == 0 && tok < item.t1) {
+          const float sc = wt * (ssq + s_part[ab * TILE + y]);
+          scores[(int64_t)item.plane * dm.Ntot + tok] = sc;
           bad |= !isfinite(sc);
         }
+        TRC_ADD(9, tr_s);
+        ++it;
+        return true;
+      };
+      float w0 = wload(item.t0), w1 = wload(item.t0 + TILE);
+      bool go = true;
+      for (int64_t t = item.t0; go && t < item.t1; t += 2 * TILE) {
+        go = tile(t, w0);
+        w0 = wload(t + 2 * TILE);
+        if (go && t + TILE < item.t1) {
+          go = tile(t + TILE, w1);
+          w1 = wload(t + 3 * TILE);
+        }
       }
-      if (FUSED && lane == 0) JACAP_TRACE_MAX(ws, (int64_t)item.plane * dm.S + item.seq, TR_SC1);
+      if (!go) goto epi_done;
+      if (FUSED && grp == 0 && lane == 0) JACAP_TRACE_MAX(ws, (int64_t)item.plane * dm.S + item.seq, TR_SC1);
     }
   epi_done:
+    TRC_ADD(10, tr_all);
+    if (warp == 2 && lane == 0) TRC_PUT(ws, TR_K_SCORE, 11);
     if (bad) flag(ws, ST_NONFINITE);
   }
   tc_fence_before();

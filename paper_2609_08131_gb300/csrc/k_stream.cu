@@ -49,6 +49,8 @@ __global__ void __launch_bounds__(256) plan_kernel(Dims dm, Ws ws, const int32_t
   if (ws.trace != nullptr)
     for (int64_t i = threadIdx.x; i < TR_SLOTS * units; i += blockDim.x)
       ws.trace[i] = (i % TR_SLOTS == TR_GRAM0 || i % TR_SLOTS == TR_SC_IMG || i % TR_SLOTS == TR_SC_MMA) ? ~0ull : 0ull;
+  if (ws.trace_cta != nullptr)
+    for (int64_t i = threadIdx.x; i < (int64_t)TR_KERNELS * TR_CTAS * TR_CTA_SLOTS; i += blockDim.x) ws.trace_cta[i] = 0;
 #endif
   __syncthreads();
   const int ctot = s_ctot;
