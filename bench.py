@@ -45,6 +45,8 @@ def parse():
     p.add_argument("--warmup", type=int, default=10)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--config", type=int, default=2)
+    p.add_argument("--trace-report", action="store_true",
+                   help="diagnostic (a JACAP_TRACE=1 build): print the per-CTA time accounting of one pass, no bench line")
     p.add_argument("--schedule", default="auto", choices=["auto", "separate", "fused"],
                    help="Gram / factor / scores as separate kernels or one fused launch (auto: the library's choice)")
     p.add_argument("--budget", type=int, default=None)
@@ -375,6 +377,16 @@ def run_ours(args):
     for _ in range(max(3, args.warmup)):
         ev.run()
     ev.check()
+    if args.trace_report:
+        from paper_2609_08131_gb300.api import cta_time_accounting
+
+        ev.run()
+        ev.check()
+        print(json.dumps({"mode": "trace report", "config": workload_config(wl, budget, world, args.weighting,
+                                                                              args.out_proj, args.covariance),
+                          "schedule": schedule_desc(*ev.schedule_info()), "cta_time_accounting":
+                          cta_time_accounting(ev)}))
+        return 0
 
     # The end-to-end number first: right after seconds of HBM-saturating passes
     # the host link of these boxes delivers 70-120 GB/s instead of 211 for a

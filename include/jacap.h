@@ -450,9 +450,20 @@ const char* jacap_status_string(jacap_status status);
  *  weights    [num_layers][num_kv_heads][total_tokens]   w_i (Eq. 8 summed over the group)
  *  gram       [num_layers][num_kv_heads][num_seqs][128][128]  sum_i w_i v_i v_i^T
  *  chol_inv   [num_layers][num_kv_heads][num_seqs][128][128]  L^{-1}, A = L L^T
+ * and, in a library built with JACAP_TRACE=1 (0 otherwise; uint64 words):
+ *  trace_timeline  [units][8]  per unit, %globaltimer ns of the fused schedule's
+ *                  first Gram tile, last Gram partial published, factor start,
+ *                  factor published, first score image acquired, last score
+ *                  tile, first score MMA (units = num_layers x num_kv_heads x
+ *                  num_seqs, unit (l, g, s) at (l num_kv_heads + g) num_seqs + s)
+ *  trace_cta       [3][1024][16]  per kernel (K pass 2, Gram 0, scores 1) and
+ *                  CTA, ns its roles spent in each wait and busy section of the
+ *                  last pass, summed over the pass (the slots are documented
+ *                  where the kernels record them)
  * Returns JACAP_ERR_INVALID_ARG for an invalid layout. */
 typedef struct {
   size_t mu_scaled, lambda, weights, gram, chol_inv;
+  size_t trace_timeline, trace_cta;
 } jacap_ws_offsets;
 jacap_status jacap_workspace_offsets(const jacap_layout* layout, int32_t budget, jacap_ws_offsets* out);
 

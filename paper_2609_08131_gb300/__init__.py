@@ -80,6 +80,8 @@ class jacap_ws_offsets(ctypes.Structure):
         ("weights", ctypes.c_size_t),
         ("gram", ctypes.c_size_t),
         ("chol_inv", ctypes.c_size_t),
+        ("trace_timeline", ctypes.c_size_t),
+        ("trace_cta", ctypes.c_size_t),
     ]
 
 

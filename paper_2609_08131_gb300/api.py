@@ -263,6 +263,52 @@ class Evictor:
         }
 
 
+# Slots of the per-CTA time accounting of a JACAP_TRACE build (jacap_ws_offsets.trace_cta):
+# kernel index -> (name, {slot: meaning}); "tiles" counts tiles, every other slot sums ns.
+TRACE_CTA_SLOTS = {
+    2: ("k_pass", {0: "producer: wait for a free stage", 1: "producer: loop", 2: "logits MMA: wait for an image",
+                   3: "logits MMA: wait for a K tile and a free buffer", 5: "logits MMA: loop", 6: "tiles",
+                   7: "kappa warp: wait for a K tile", 8: "kappa warp: its quarter of kappa",
+                   9: "kappa warp: first group barrier", 10: "kappa warp: reduction and store", 11: "kappa warp: loop",
+                   12: "readout warp: wait for logits", 13: "readout warp: readout of a tile",
+                   14: "readout warp: loop"}),
+    0: ("gram", {0: "producer: wait for a free stage", 1: "producer: loop", 2: "MMA: wait for a scaled operand",
+                 3: "MMA: wait for a free accumulator", 4: "MMA: loop", 5: "tiles", 6: "scaling warp: wait for V",
+                 7: "scaling warp: wait for the weights", 8: "scaling warp: wait for a free operand buffer",
+                 9: "scaling warp: scaling", 10: "scaling warp: loop", 11: "weight warp: wait for V",
+                 12: "weight warp: weights of a tile", 13: "weight warp: loop"}),
+    1: ("scores", {0: "producer: wait for a free stage", 1: "producer: loop", 2: "MMA: wait for an image",
+                   3: "MMA: wait for a free accumulator", 4: "MMA: wait for a V tile", 5: "MMA: loop", 6: "tiles",
+                   7: "epilogue warp: wait for an accumulator", 8: "epilogue warp: read, reduce and meet its partner",
+                   9: "epilogue warp: weight and store", 10: "epilogue warp: loop"}),
+}
+
+
+def cta_time_accounting(ev: Evictor) -> dict:
+    """Per-CTA time accounting of the last pass of ``ev`` (a JACAP_TRACE build): for each
+    streaming kernel, the mean over its CTAs of every slot, in us per CTA and ns per tile."""
+    st, off = jacap_workspace_offsets(ev.lay, ev.budget)
+    _check(st, "jacap_workspace_offsets")
+    if off.trace_cta == 0:
+        raise RuntimeError("the library was not built with JACAP_TRACE=1")
+    torch.cuda.synchronize(ev.ws.device)
+    tc = ev.ws[off.trace_cta:off.trace_cta + 3 * 1024 * 16 * 8].view(torch.int64).view(3, 1024, 16).cpu().double()
+    out = {}
+    for k, (name, slots) in TRACE_CTA_SLOTS.items():
+        tile_slot = next(j for j, m in slots.items() if m == "tiles")
+        a = tc[k]
+        a = a[a[:, tile_slot] > 0]
+        if a.shape[0] == 0:
+            continue
+        tiles = a[:, tile_slot].clamp(min=1)
+        rep = {"ctas": int(a.shape[0]), "tiles_per_cta": float(tiles.mean())}
+        for j, m in slots.items():
+            if j != tile_slot:
+                rep[m] = {"us_per_cta": float(a[:, j].mean() / 1e3), "ns_per_tile": float((a[:, j] / tiles).mean())}
+        out[name] = rep
+    return out
+
+
 def evict(cache: Cache, budget: int, params: jacap_params | None = None, check: bool = True) -> Evictor:
     """One eviction pass over a device-resident cache; returns the Evictor
     whose scores / idx / kept / k_out / v_out hold the results."""

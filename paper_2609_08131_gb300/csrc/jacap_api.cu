@@ -336,6 +336,8 @@ jacap_status jacap_workspace_offsets(const jacap_layout* layout, int32_t budget,
   out->weights = c.w;
   out->gram = c.gram;
   out->chol_inv = c.minv;
+  out->trace_timeline = c.trace;
+  out->trace_cta = c.trace_cta;
   return JACAP_OK;
 }
 
