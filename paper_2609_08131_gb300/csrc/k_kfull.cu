@@ -341,9 +341,9 @@ __global__ void __launch_bounds__(KX_THREADS, 1)
           red[rw * 2 * G + G + h] = run_s[h];
         }
       }
-      // a warp that met an abort still arrives here; all four leave together
-      named_barrier_sync(1, 128);
-      if (*abort) goto read_done;
+      // a warp that met an abort still arrives here; the barrier ORs the flag,
+      // so all four leave together
+      if (named_barrier_any(1, 128, *abort != 0)) goto read_done;
       if (rw == 0 && lane < G) {
         const int h = lane;
         float m = -INFINITY, ssum = 0.f;

@@ -310,15 +310,14 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
     TRC_DECL(TR_CTA_SLOTS);
     TRC_T(tr_all);
     // A failed wait (which means the abort flag is set) still arrives at the
-    // group's named barriers, and the four warps leave together after them.
-    // All four see the same runs (the same item stream), so they meet at the
-    // same barriers.
+    // group's named barriers, which OR the flag over the group, so the four
+    // warps leave together after the same barrier. All four see the same runs
+    // (the same item stream), so they meet at the same barriers.
     for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
       if (!cont) {
         p = nrun & 1;
         mbar_wait(smem_u32(&imgready[p]), (nrun >> 1) & 1, ws, abort);
-        named_barrier_sync(bar_id, 128);
-        if (*abort) goto kappa_done;
+        if (named_barrier_any(bar_id, 128, *abort != 0)) goto kappa_done;
       }
       {
         const uint32_t lam_s = smem_u32(lams + p * G * D);
@@ -343,10 +342,10 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
                 for (int h = 0; h < G; ++h) slot[((j * 4 + cq) * G + h) * 32 + lane] = part[j][h];
           }
           TRC_T(tr_b);
-          named_barrier_sync(bar_id, 128);
+          const bool stop = named_barrier_any(bar_id, 128, *abort != 0);
           TRC_ADD(9, tr_b);
           TRC_T(tr_r);
-          if (*abort) goto kappa_done;
+          if (stop) goto kappa_done;
           float kap[G];
 #pragma unroll
           for (int h = 0; h < G; ++h) {
@@ -455,9 +454,9 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
           red[rw * 2 * G + G + h] = run_s[h];
         }
       }
-      // a warp that met an abort still arrives here; all four leave together
-      named_barrier_sync(1, 128);
-      if (*abort) goto read_done;
+      // a warp that met an abort still arrives here; the barrier ORs the flag,
+      // so all four leave together
+      if (named_barrier_any(1, 128, *abort != 0)) goto read_done;
       if (rw == 0 && lane < G) {
         const int h = lane;
         float m = -INFINITY, ssum = 0.f;

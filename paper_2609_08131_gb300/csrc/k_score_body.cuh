@@ -318,9 +318,10 @@ __device__ __forceinline__ void score_bf16_body(const CUtensorMap* vmap_p, const
           if (lane == 0) mbar_arrive(smem_u32(&accempty[ab]));
           if (grp == 1) s_part[ab * TILE + y] = ssq;
         }
-        named_barrier_sync(1 + quarter, 64);
+        // the pair decides together whether to leave (see named_barrier_any)
+        const bool stop = named_barrier_any(1 + quarter, 64, !ok || *abort != 0);
         TRC_ADD(8, tr_r);
-        if (!ok || *abort) return false;
+        if (stop) return false;
         TRC_T(tr_s);
         if (grp == 0 && tok < item.t1) {
           const float sc = wt * (ssq + s_part[ab * TILE + y]);
