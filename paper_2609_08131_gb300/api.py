@@ -281,30 +281,39 @@ TRACE_CTA_SLOTS = {
                    3: "MMA: wait for a free accumulator", 4: "MMA: wait for a V tile", 5: "MMA: loop", 6: "tiles",
                    7: "epilogue warp: wait for an accumulator", 8: "epilogue warp: read, reduce and meet its partner",
                    9: "epilogue warp: weight and store", 10: "epilogue warp: loop"}),
+    3: ("factor", {0: "partial Grams summed into A", 1: "elimination of diagonal block 0",
+                   2: "elimination of diagonal block 1", 3: "elimination of diagonal block 2",
+                   4: "elimination of diagonal block 3", 5: "elimination warp: wait for the other warps",
+                   6: "panels and look-ahead updates", 7: "last inverse phase", 8: "outputs", 9: "units",
+                   10: "whole unit"}),
 }
 
 
 def cta_time_accounting(ev: Evictor) -> dict:
     """Per-CTA time accounting of the last pass of ``ev`` (a JACAP_TRACE build): for each
-    streaming kernel, the mean over its CTAs of every slot, in us per CTA and ns per tile."""
+    streaming kernel and the factor, the mean over its CTAs (the first 1024) of every slot,
+    in us per CTA and ns per 128-token tile (streaming kernels) or per unit (factor)."""
     st, off = jacap_workspace_offsets(ev.lay, ev.budget)
     _check(st, "jacap_workspace_offsets")
     if off.trace_cta == 0:
         raise RuntimeError("the library was not built with JACAP_TRACE=1")
     torch.cuda.synchronize(ev.ws.device)
-    tc = ev.ws[off.trace_cta:off.trace_cta + 3 * 1024 * 16 * 8].view(torch.int64).view(3, 1024, 16).cpu().double()
+    nk = len(TRACE_CTA_SLOTS)
+    tc = ev.ws[off.trace_cta:off.trace_cta + nk * 1024 * 16 * 8].view(torch.int64).view(nk, 1024, 16).cpu().double()
     out = {}
     for k, (name, slots) in TRACE_CTA_SLOTS.items():
-        tile_slot = next(j for j, m in slots.items() if m == "tiles")
+        # the streaming kernels count 128-token tiles, the factor units
+        per = "tile" if "tiles" in slots.values() else "unit"
+        count_slot = next(j for j, m in slots.items() if m == per + "s")
         a = tc[k]
-        a = a[a[:, tile_slot] > 0]
+        a = a[a[:, count_slot] > 0]
         if a.shape[0] == 0:
             continue
-        tiles = a[:, tile_slot].clamp(min=1)
-        rep = {"ctas": int(a.shape[0]), "tiles_per_cta": float(tiles.mean())}
+        cnt = a[:, count_slot].clamp(min=1)
+        rep = {"ctas": int(a.shape[0]), per + "s_per_cta": float(cnt.mean())}
         for j, m in slots.items():
-            if j != tile_slot:
-                rep[m] = {"us_per_cta": float(a[:, j].mean() / 1e3), "ns_per_tile": float((a[:, j] / tiles).mean())}
+            if j != count_slot:
+                rep[m] = {"us_per_cta": float(a[:, j].mean() / 1e3), "ns_per_" + per: float((a[:, j] / cnt).mean())}
         out[name] = rep
     return out
 

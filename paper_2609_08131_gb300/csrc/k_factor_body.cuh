@@ -93,13 +93,15 @@ __device__ __forceinline__ void nt_block(float (&acc)[2][2], const float* P, con
 // pivot row goes to every lane through shared memory: its scaled inverse part
 // (columns < k) from lane k's registers, its A part (columns >= k) as column k
 // of every row (the lower triangle of A; each lane stores its own element).
-// The two values the next step waits for, the pivot p_k and row k + 1's
-// element in column k, also travel by shuffle, so the loop-carried chain is a
-// shuffle, the reciprocal and two multiply-adds rather than a round trip
-// through shared memory (measured alone: 5,500 cycles per block against 8,600
-// with a shuffle per column). rb, cb: two 32-float buffers each (16-byte
-// aligned), alternating by step; piv, pinv: the 32 pivots and their
-// reciprocals. Writes T row-major into `blk` and T^T into `tblk`.
+// The steps are software-pipelined: step k first updates column k + 1 (the
+// next pivot column), sends the next pivot p_{k+1} and row k + 2's element in
+// column k + 1 by shuffle and starts their reciprocal, updates the inverse
+// part, stores the next pivot row, and only then makes the rest of its
+// multiply-adds, which hide the latency of the stores, the shuffles and the
+// reciprocal; the next pivot row is loaded after them. rb, cb: two 32-float
+// buffers each (16-byte aligned), alternating by step; piv, pinv: the 32
+// pivots and their reciprocals. Writes T row-major into `blk` and T^T into
+// `tblk`.
 __device__ __forceinline__ void diag_inverse(float* blk, float* tblk, float* rb, float* cb, float* piv, float* pinv,
                                              int lane, bool& bad) {
   float z[32];
@@ -111,44 +113,73 @@ __device__ __forceinline__ void diag_inverse(float* blk, float* tblk, float* rb,
     z[c + 2] = v.z;
     z[c + 3] = v.w;
   }
+  // step 0's pivot row is column 0 of every row (no inverse part yet)
+  cb[lane] = z[0];
+  float p = __shfl_sync(0xffffffffu, z[0], 0);
+  float rn = __shfl_sync(0xffffffffu, z[0], 1);  // A_{1,0}
+  float inv = recip_nr(p);
+  if (lane == 0) {
+    piv[0] = p;
+    pinv[0] = inv;
+  }
+  __syncwarp();
+  float r[32];
+#pragma unroll
+  for (int c = 0; c < 32; c += 4) {
+    const float4 v = *(const float4*)(cb + c);
+    r[c] = v.x, r[c + 1] = v.y, r[c + 2] = v.z, r[c + 3] = v.w;
+  }
 #pragma unroll
   for (int k = 0; k < 32; ++k) {
-    float* rk = rb + (k & 1) * 32;
-    float* ck = cb + (k & 1) * 32;
-    ck[lane] = z[k];
-    if (lane == k) {
-#pragma unroll
-      for (int c = 0; c < k; c += 4) *(float4*)(rk + c) = make_float4(z[c], z[c + 1], z[c + 2], z[c + 3]);
+    const float m = lane > k ? z[k] * inv : 0.f;
+    float inv_next = 0.f;
+    if (k + 1 < 32) {
+      z[k + 1] = fmaf(-m, rn, z[k + 1]);  // the next pivot column first
+      p = __shfl_sync(0xffffffffu, z[k + 1], k + 1);
+      rn = k + 2 < 32 ? __shfl_sync(0xffffffffu, z[k + 1], k + 2) : 0.f;  // A_{k+2,k+1}
     }
-    const float p = __shfl_sync(0xffffffffu, z[k], k);
-    const float rn = k + 1 < 32 ? __shfl_sync(0xffffffffu, z[k], k + 1) : 0.f;  // A_{k+1,k}
-    __syncwarp();
-    float r[32];
 #pragma unroll
-    for (int c = 0; c < 32; c += 4) {
-      if (c + 4 <= k) {
-        const float4 v = *(const float4*)(rk + c);
-        r[c] = v.x, r[c + 1] = v.y, r[c + 2] = v.z, r[c + 3] = v.w;
-      } else if (c >= k) {
-        const float4 v = *(const float4*)(ck + c);
-        r[c] = v.x, r[c + 1] = v.y, r[c + 2] = v.z, r[c + 3] = v.w;
-      } else {  // the group that holds column k: inverse part below k, A part from k on
-        const float4 u = *(const float4*)(rk + c), v = *(const float4*)(ck + c);
-        const float uu[4] = {u.x, u.y, u.z, u.w}, vv[4] = {v.x, v.y, v.z, v.w};
+    for (int c = 0; c < k; ++c) z[c] = fmaf(-m, r[c], z[c]);  // the inverse part
+    if (k + 1 < 32) {
+      // the pivot row of step k + 1: lane k + 1's inverse part (its columns
+      // <= k are final now) and column k + 1 of every row
+      float* rk = rb + ((k + 1) & 1) * 32;
+      float* ck = cb + ((k + 1) & 1) * 32;
+      ck[lane] = z[k + 1];
+      if (lane == k + 1) {
 #pragma unroll
-        for (int j = 0; j < 4; ++j) r[c + j] = c + j < k ? uu[j] : vv[j];
+        for (int c = 0; c <= k; c += 4) *(float4*)(rk + c) = make_float4(z[c], z[c + 1], z[c + 2], z[c + 3]);
+      }
+      inv_next = recip_nr(p);
+      if (lane == 0) {
+        piv[k + 1] = p;
+        pinv[k + 1] = inv_next;
       }
     }
-    const float inv = recip_nr(p);
-    if (lane == 0) {
-      piv[k] = p;
-      pinv[k] = inv;
-    }
-    const float m = lane > k ? z[k] * inv : 0.f;
-    if (k + 1 < 32) z[k + 1] = fmaf(-m, rn, z[k + 1]);  // the next pivot column first
 #pragma unroll
-    for (int c = 0; c < 32; ++c)
-      if (c != k && c != k + 1) z[c] = fmaf(-m, r[c], z[c]);
+    for (int c = k + 2; c < 32; ++c) z[c] = fmaf(-m, r[c], z[c]);
+    if (k + 1 < 32) {
+      __syncwarp();
+      const float* rk = rb + ((k + 1) & 1) * 32;
+      const float* ck = cb + ((k + 1) & 1) * 32;
+      const int kn = k + 1;
+#pragma unroll
+      for (int c = 0; c < 32; c += 4) {
+        if (c + 4 <= kn) {
+          const float4 v = *(const float4*)(rk + c);
+          r[c] = v.x, r[c + 1] = v.y, r[c + 2] = v.z, r[c + 3] = v.w;
+        } else if (c >= kn) {
+          const float4 v = *(const float4*)(ck + c);
+          r[c] = v.x, r[c + 1] = v.y, r[c + 2] = v.z, r[c + 3] = v.w;
+        } else {  // the group that holds column kn: inverse part below kn, A part from kn on
+          const float4 u = *(const float4*)(rk + c), v = *(const float4*)(ck + c);
+          const float uu[4] = {u.x, u.y, u.z, u.w}, vv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+          for (int j = 0; j < 4; ++j) r[c + j] = c + j < kn ? uu[j] : vv[j];
+        }
+      }
+      inv = inv_next;
+    }
   }
   // T_rc = X_rc / sqrt(p_r), X_rc = -z_c / p_c (c < r), X_rr = 1; the final
   // rows go through shared memory so that few registers stay live
@@ -290,8 +321,16 @@ __device__ __forceinline__ void factor_blocked_cta(const Dims& dm, const Ws& ws,
   const int units = dm.L * dm.Hkv * dm.S;
   uint32_t kk = 0;  // partial stages consumed so far (phases of s_full across units)
   const uint64_t drop = FUSED ? policy_evict_first() : 0;
+  // time accounting (trace builds, thread 0, the elimination warp): 0 the
+  // partial Grams summed into A (and G stored), 1-4 the eliminations of the
+  // diagonal blocks, 5 its waits for the other warps after them, 6 panels and
+  // look-ahead updates, 7 the last inverse phase, 8 the outputs, 9 units,
+  // 10 the whole unit
+  TRC_DECL(TR_CTA_SLOTS);
 #pragma unroll 1
   for (int u = first; u < units; u += stride) {
+  TRC_T(tr_unit);
+  TRC_INC(9);
   const int plane = u / dm.S, s = u % dm.S;
   const int ch0 = ws.plan[1 + s], ch1 = ws.plan[2 + s];
   const float* gp = ws.gpart + ((int64_t)plane * dm.c_cap) * D * D;
@@ -401,6 +440,7 @@ __device__ __forceinline__ void factor_blocked_cta(const Dims& dm, const Ws& ws,
     *(float4*)(dst + 3 * D) = make_float4(r[0].w, r[1].w, r[2].w, r[3].w);
   }
 
+  TRC_ADD(0, tr_unit);
   const int a = tid >> 4, b = tid & 15;
   // the six warps off warp 0's sub-partition (1-3, 5-7) work next to the
   // elimination, so it keeps its issue slots
@@ -413,14 +453,19 @@ __device__ __forceinline__ void factor_blocked_cta(const Dims& dm, const Ws& ws,
 #pragma unroll 1
   for (int K = 0; K < 4; ++K) {
     if (warp == 0) {
+      TRC_T(tr_e);
       diag_inverse(As + tri(K, K) * FB_BLK, XT + tri(K, K) * FB_BLK, s_elim, s_elim + 64, s_elim + 128, s_elim + 160,
                    lane, bad);
+      TRC_ADD(1 + K, tr_e);
     } else if (warp != 4 && K >= 1) {
       trailing_update(As, K - 1, 1, (4 - K) * (5 - K) / 2, vt, 192);
       inv_rows(As, XT, K - 1, vt, 192, 2);
       inv_accumulate(As, XT, K - 1, vt, 192);
     }
+    TRC_T(tr_w);
     fb_all();
+    TRC_ADD(5, tr_w);
+    TRC_T(tr_p);
     // L_IK = A_IK T_KK^T for I > K
     float acc[3][2][2];
 #pragma unroll
@@ -439,14 +484,21 @@ __device__ __forceinline__ void factor_blocked_cta(const Dims& dm, const Ws& ws,
           for (int j = 0; j < 2; ++j) L[(a + 16 * i) * FB_LD + b + 16 * j] = acc[q][i][j];
       }
     fb_all();
-    if (K == 3) break;
+    if (K == 3) {
+      TRC_ADD(6, tr_p);
+      break;
+    }
     // A_{K+1,K+1} -= L_{K+1,K} L_{K+1,K}^T ahead of the rest of the trailing update
     trailing_update(As, K, 0, 1, tid, FB_THREADS);
     fb_all();
+    TRC_ADD(6, tr_p);
   }
 
   // inverse phase 3: X_3J = -T_33 S_3J (all threads)
+  TRC_T(tr_t);
   inv_rows(As, XT, 3, tid, FB_THREADS, 0);
+  TRC_ADD(7, tr_t);
+  TRC_T(tr_o);
   if (bad) s_bad = 1;
 
   // Outputs, 64 rows of L^{-1} at a time, staged row-major in the A blocks
@@ -515,7 +567,10 @@ __device__ __forceinline__ void factor_blocked_cta(const Dims& dm, const Ws& ws,
       JACAP_TRACE_MAX(ws, u, TR_FAC1);
     }
   }
+  TRC_ADD(8, tr_o);
+  TRC_ADD(10, tr_unit);
   }
+  if (tid == 0) TRC_PUT(ws, TR_K_FACTOR, 11);
 }
 
 }  // namespace jacap
