@@ -65,8 +65,15 @@ constexpr size_t FB_FUSED_SMEM = ((size_t)fb_elim_at<true>() + FB_ELIM) * sizeof
 // fused schedule the factor runs on the first FB_THREADS threads of a larger CTA).
 __device__ __forceinline__ void fb_all() { named_barrier_sync(1, FB_THREADS); }
 
-// acc[p][q] += sum_m P[a + 16 p][m] Q[b + 16 q][m]
+// acc[p][q] += sum_m P[a + 16 p][m] Q[b + 16 q][m], with packed fp32x2
+// multiply-adds: the even and the odd m accumulate separately and are added
+// at the end (half the instructions of one chain per output)
 __device__ __forceinline__ void nt_block(float (&acc)[2][2], const float* P, const float* Q, int a, int b) {
+  float2 s[2][2];
+#pragma unroll
+  for (int i = 0; i < 2; ++i)
+#pragma unroll
+    for (int j = 0; j < 2; ++j) s[i][j] = make_float2(0.f, 0.f);
 #pragma unroll
   for (int m = 0; m < 32; m += 4) {
     const float4 p0 = *(const float4*)(P + a * FB_LD + m);
@@ -78,14 +85,14 @@ __device__ __forceinline__ void nt_block(float (&acc)[2][2], const float* P, con
     for (int i = 0; i < 2; ++i)
 #pragma unroll
       for (int j = 0; j < 2; ++j) {
-        float t = acc[i][j];
-        t = fmaf(pv[i].x, qv[j].x, t);
-        t = fmaf(pv[i].y, qv[j].y, t);
-        t = fmaf(pv[i].z, qv[j].z, t);
-        t = fmaf(pv[i].w, qv[j].w, t);
-        acc[i][j] = t;
+        s[i][j] = __ffma2_rn(make_float2(pv[i].x, pv[i].y), make_float2(qv[j].x, qv[j].y), s[i][j]);
+        s[i][j] = __ffma2_rn(make_float2(pv[i].z, pv[i].w), make_float2(qv[j].z, qv[j].w), s[i][j]);
       }
   }
+#pragma unroll
+  for (int i = 0; i < 2; ++i)
+#pragma unroll
+    for (int j = 0; j < 2; ++j) acc[i][j] += s[i][j].x + s[i][j].y;
 }
 
 // T = L^{-1} of one 32 x 32 diagonal block by the elimination described at the
