@@ -456,8 +456,8 @@ const char* jacap_status_string(jacap_status status);
  *                  factor published, first score image acquired, last score
  *                  tile, first score MMA (units = num_layers x num_kv_heads x
  *                  num_seqs, unit (l, g, s) at (l num_kv_heads + g) num_seqs + s)
- *  trace_cta       [4][1024][16]  per kernel (K pass 2, Gram 0, scores 1,
- *                  factor 3) and CTA (the first 1024), ns its roles spent in
+ *  trace_cta       [5][1024][16]  per kernel (K pass 2, Gram 0, scores 1,
+ *                  factor 3, selection 4) and CTA (the first 1024), ns its roles spent in
  *                  each wait and busy section of the last pass, summed over the
  *                  pass (the slots are documented where the kernels record them)
  * Returns JACAP_ERR_INVALID_ARG for an invalid layout. */

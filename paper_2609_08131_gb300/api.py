@@ -286,6 +286,8 @@ TRACE_CTA_SLOTS = {
                    4: "elimination of diagonal block 3", 5: "elimination warp: wait for the other warps",
                    6: "panels and look-ahead updates", 7: "last inverse phase", 8: "outputs", 9: "units",
                    10: "whole unit"}),
+    4: ("selection", {0: "scores loaded", 1: "radix passes", 2: "emission", 3: "rows gathered", 4: "units",
+                      5: "whole unit"}),
 }
 
 

@@ -96,7 +96,8 @@ enum { TR_GRAM0 = 0, TR_GRAM1, TR_FAC0, TR_FAC1, TR_SC_IMG, TR_SC1, TR_SC_MMA, T
 // kernel k (TR_K_*) and CTA b, slot j of trace_cta[(k TR_CTAS + b) TR_CTA_SLOTS]
 // sums the ns one role's lane 0 spent in a wait or a busy section (the slot
 // meanings are listed where each kernel records them).
-enum { TR_K_GRAM = 0, TR_K_SCORE = 1, TR_K_KPASS = 2, TR_K_FACTOR = 3, TR_KERNELS = 4, TR_CTAS = 1024, TR_CTA_SLOTS = 16 };
+enum { TR_K_GRAM = 0, TR_K_SCORE = 1, TR_K_KPASS = 2, TR_K_FACTOR = 3, TR_K_SELECT = 4, TR_KERNELS = 5, TR_CTAS = 1024,
+       TR_CTA_SLOTS = 16 };
 
 // A unit is (plane p = l*Hkv + g, request s); its index is p*S + s.
 struct Item {

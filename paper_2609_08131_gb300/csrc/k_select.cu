@@ -4,7 +4,8 @@
 // select_kernel: one CTA per unit (grid-stride), of NT = 1024 threads, or of
 // 256 when the longest request has at most 4096 tokens and there are more
 // units than SMs (then four or more CTAs fit an SM and a pass over many short
-// units, as in decoding-stage eviction, runs in one wave). Scores are
+// units, as in decoding-stage eviction, runs in one wave), or of 512 (two per
+// SM) for longer requests when there are more than two SMs' worth of units. Scores are
 // non-negative float32, so their bit patterns order like unsigned integers.
 // Three radix passes (digits of 11, 11 and 10 bits, most significant first,
 // shared-memory histograms; a pass counts only keys that match the digits
@@ -69,7 +70,7 @@ __device__ __forceinline__ void gather_unit(const Dims& dm, int plane, int64_t s
   const int64_t base = (int64_t)l * dm.kv_sl + (int64_t)g * dm.kv_sh;
   uint4* ko = (uint4*)(k_out + u * B * D);
   uint4* vo = (uint4*)(v_out + u * B * D);
-#pragma unroll 2
+#pragma unroll 4
   for (int e = threadIdx.x; e < B * CH; e += NT) {
     const int r = e / CH, c = e % CH;
     const int32_t src = out[r];
@@ -85,7 +86,7 @@ __device__ __forceinline__ void gather_unit(const Dims& dm, int plane, int64_t s
 }
 
 template <int KPT, typename E, int MODE, int NT>
-__global__ void __launch_bounds__(NT)
+__global__ void __launch_bounds__(NT, NT == 512 ? 2 : 1)
     select_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu, const float* __restrict__ scores, int B,
                   int32_t* __restrict__ idx, int32_t* __restrict__ kept, const E* __restrict__ k,
                   const E* __restrict__ v, E* __restrict__ k_out, E* __restrict__ v_out, E* kio, E* vio,
@@ -104,7 +105,12 @@ __global__ void __launch_bounds__(NT)
   if (s_skip) return;
   const int units = dm.L * dm.Hkv * dm.S;
   const uint32_t lt = (1u << lane) - 1u;
+  // time accounting (trace builds, thread 0): 0 the scores loaded (one slab),
+  // 1 the radix passes, 2 the emission, 3 the rows gathered, 4 units, 5 the
+  // whole unit (units of more than B tokens)
+  TRC_DECL(TR_CTA_SLOTS);
   for (int u = blockIdx.x; u < units; u += gridDim.x) {
+    TRC_T(tr_u);
     const int plane = u / dm.S, s = u % dm.S;
     const int64_t start = cu[s];
     const int64_t end = cu[s + 1];
@@ -135,7 +141,10 @@ __global__ void __launch_bounds__(NT)
     }
     const int nslab = (n + SE_SLAB - 1) / SE_SLAB;
     uint32_t kr[SE_KPT];
+    TRC_INC(4);
     if (nslab == 1) load_slab<KPT, NT>(key, n, 0, warp, lane, kr);  // register-resident for all passes
+    TRC_ADD(0, tr_u);
+    TRC_T(tr_r);
     // ---- radix select of the B-th largest key: digits [31:21], [20:10], [9:0] ----
     uint32_t prefix = 0, mask = 0, need = (uint32_t)B;
 #pragma unroll 1
@@ -154,10 +163,13 @@ __global__ void __launch_bounds__(NT)
       }
       __syncthreads();
       if (warp == 0) {
-        // lane l sums bins 64 l .. 64 l + 63; suffix sums over lanes locate the
-        // bin holding the need-th largest key, which that lane then finds
+        // lane l sums bins 64 l .. 64 l + 63 (in a rotated order, so that the
+        // lanes' loads fall in different banks); suffix sums over the lanes
+        // locate the group of 64 bins that holds the need-th largest key, and
+        // a second suffix scan over that group (two bins per lane) the bin
         uint32_t c = 0;
-        for (int b = 0; b < 64; ++b) c += hist[64 * lane + b];
+#pragma unroll 8
+        for (int b = 0; b < 64; ++b) c += hist[64 * lane + ((b + lane) & 63)];
         uint32_t suf = c;  // sum over lanes >= lane
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
@@ -165,15 +177,28 @@ __global__ void __launch_bounds__(NT)
           if (lane + o < 32) suf += y;
         }
         const uint32_t above = suf - c;  // keys in bins of higher lanes
-        if (above < need && suf >= need) {  // exactly one lane
-          uint32_t acc = above;
-          int d = 64 * lane + 63;
-          for (; d > 64 * lane; --d) {
-            if (acc + hist[d] >= need) break;
-            acc += hist[d];
-          }
-          s_digit = (uint32_t)d;
-          s_need = need - acc;
+        const uint32_t hit = __ballot_sync(0xffffffffu, above < need && suf >= need);  // exactly one lane
+        const int g = __ffs(hit) - 1;
+        const uint32_t gabove = __shfl_sync(0xffffffffu, above, g);  // keys above the group
+        // bins 64 g + 2 lane (+1), suffix sums from the top of the group down
+        const uint32_t h0 = hist[64 * g + 2 * lane], h1 = hist[64 * g + 2 * lane + 1];
+        const uint32_t c2 = h0 + h1;
+        uint32_t suf2 = c2;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const uint32_t y = __shfl_down_sync(0xffffffffu, suf2, o);
+          if (lane + o < 32) suf2 += y;
+        }
+        const uint32_t a1 = gabove + suf2 - c2;  // keys above bin 2 lane + 1 of the group
+        const uint32_t a0 = a1 + h1;             // keys above bin 2 lane
+        // the bin d with (keys above d) < need <= (keys above d) + hist[d]
+        const bool in1 = a1 < need && a1 + h1 >= need, in0 = a0 < need && a0 + h0 >= need;
+        if (in1) {
+          s_digit = (uint32_t)(64 * g + 2 * lane + 1);
+          s_need = need - a1;
+        } else if (in0) {
+          s_digit = (uint32_t)(64 * g + 2 * lane);
+          s_need = need - a0;
         }
       }
       __syncthreads();
@@ -183,39 +208,60 @@ __global__ void __launch_bounds__(NT)
       __syncthreads();
     }
     const uint32_t T = prefix;  // the B-th largest key; the first `need` keys == T are kept
+    TRC_ADD(1, tr_r);
+    TRC_T(tr_e);
     // ---- emission, slab by slab; in a slab warp w owns positions 32 KPT w .. ----
     uint32_t gt_run = 0, eq_run = 0;  // kept-greater and equal keys before this slab
 #pragma unroll 1
     for (int sl = 0; sl < nslab; ++sl) {
       if (nslab > 1) load_slab<KPT, NT>(key, n, sl, warp, lane, kr);
       const int base = sl * SE_SLAB + warp * (32 * SE_KPT) + lane;
-      uint32_t gt = 0, eq = 0;
+      // the warp's counts of keys > T and == T, and which register slots hold
+      // any key >= T (most hold none: only B of the n keys are kept)
+      uint32_t gt = 0, eq = 0, jmask = 0;
 #pragma unroll
       for (int j = 0; j < SE_KPT; ++j) {
         const bool v = base + 32 * j < n;
-        gt += __popc(__ballot_sync(0xffffffffu, v && kr[j] > T));
-        eq += __popc(__ballot_sync(0xffffffffu, v && kr[j] == T));
+        const uint32_t bg = __ballot_sync(0xffffffffu, v && kr[j] > T);
+        const uint32_t be = __ballot_sync(0xffffffffu, v && kr[j] == T);
+        gt += __popc(bg);
+        eq += __popc(be);
+        if (bg | be) jmask |= 1u << j;
       }
       if (lane == 0) {
         hist[warp] = gt;  // the histogram is free again: it holds the warp totals
         hist[NW + warp] = eq;
       }
       __syncthreads();
-      uint32_t gt_before = gt_run, eq_before = eq_run, gt_all = 0, eq_all = 0;
-      for (int w = 0; w < NW; ++w) {
-        const uint32_t g = hist[w], e = hist[NW + w];
-        if (w < warp) {
-          gt_before += g;
-          eq_before += e;
+      if (warp == 0) {  // exclusive prefixes of the warp totals (lane w: warp w) and the slab totals
+        const uint32_t g = lane < NW ? hist[lane] : 0u, e = lane < NW ? hist[NW + lane] : 0u;
+        uint32_t gs = g, es = e;  // inclusive scans
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const uint32_t y = __shfl_up_sync(0xffffffffu, gs, o), z = __shfl_up_sync(0xffffffffu, es, o);
+          if (lane >= o) {
+            gs += y;
+            es += z;
+          }
         }
-        gt_all += g;
-        eq_all += e;
+        if (lane < NW) {
+          hist[2 * NW + lane] = gs - g;
+          hist[3 * NW + lane] = es - e;
+        }
+        if (lane == 31) {
+          hist[4 * NW] = gs;
+          hist[4 * NW + 1] = es;
+        }
       }
+      __syncthreads();
+      const uint32_t gt_before = gt_run + hist[2 * NW + warp], eq_before = eq_run + hist[3 * NW + warp];
+      const uint32_t gt_all = hist[4 * NW], eq_all = hist[4 * NW + 1];
       // kept before this warp's block: all greater keys plus the equal ones of rank < need
       uint32_t pos = gt_before + min(eq_before, need);
       uint32_t er = eq_before;
 #pragma unroll
       for (int j = 0; j < SE_KPT; ++j) {
+        if (!(jmask & (1u << j))) continue;  // warp-uniform: no key >= T in this slot
         const int i = base + 32 * j;
         const bool v = i < n;
         const uint32_t beq = __ballot_sync(0xffffffffu, v && kr[j] == T);
@@ -233,7 +279,10 @@ __global__ void __launch_bounds__(NT)
     }
     // (the barrier that ends the last slab also orders the emitted positions
     // before they are read back here)
+    TRC_ADD(2, tr_e);
+    TRC_T(tr_g);
     if constexpr (GATHER) gather_unit<E, NT>(dm, plane, start, end, true, k, v, out, B, u, k_out, v_out);
+    TRC_ADD(3, tr_g);
     if constexpr (MODE == 2) {
       // f = the kept positions below B (they ascend: a binary search)
       int lo = 0, hi = B;
@@ -244,7 +293,9 @@ __global__ void __launch_bounds__(NT)
       fill_holes_unit<E, NT>(dm, plane, start, B, lo, kio, vio, pos, out);
     }
     if constexpr (MODE == 2) __syncthreads();  // the unit's rows have moved before `out` is reused
+    TRC_ADD(5, tr_u);
   }
+  if (tid == 0) TRC_PUT(ws, TR_K_SELECT, 6);
 }
 
 template <typename T>
@@ -315,10 +366,17 @@ cudaError_t launch_select(const Dims& dm, const Ws& ws, const int32_t* cu, const
   int dev = 0, sms = 0;
   JACAP_TRY(cudaGetDevice(&dev));
   JACAP_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
-  const bool small = (int64_t)dm.L * dm.Hkv * dm.S > sms;
+  const int64_t units = (int64_t)dm.L * dm.Hkv * dm.S;
+  const bool small = units > sms;
   if (small && max_seqlen <= 256 * 4) JACAP_SELECT(4, 256);
   else if (small && max_seqlen <= 256 * 8) JACAP_SELECT(8, 256);
   else if (small && max_seqlen <= 256 * 16) JACAP_SELECT(16, 256);
+  // more than two waves of 1024-thread CTAs: two 512-thread CTAs per SM (keys
+  // in slabs of 16384, re-read from L2 by each pass) keep twice as many units
+  // going (config 5's 4096 units: 0.95 -> 0.85 ms); with fewer units the
+  // larger CTA finishes each unit sooner (256 units of 131072 tokens: 0.159
+  // against 0.170 ms)
+  else if (units > 2 * (int64_t)sms && max_seqlen > 1024 * 16) JACAP_SELECT(32, 512);
   else if (max_seqlen <= 1024 * 4) JACAP_SELECT(4, 1024);
   else if (max_seqlen <= 1024 * 8) JACAP_SELECT(8, 1024);
   else if (max_seqlen <= 1024 * 16) JACAP_SELECT(16, 1024);
