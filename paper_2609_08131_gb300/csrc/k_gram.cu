@@ -99,8 +99,8 @@ constexpr int GF_LD = D + 4;
 __global__ void __launch_bounds__(GF_THREADS)
     gram_f32_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu, const float* __restrict__ v) {
   pdl_wait();
-  __shared__ float xs[GF_SLAB][GF_LD];  // w_i v_i
-  __shared__ float vs[GF_SLAB][GF_LD];  // v_i
+  __shared__ __align__(16) float xs[GF_SLAB][GF_LD];  // w_i v_i (16-byte rows: GF_LD is a multiple of 4)
+  __shared__ __align__(16) float vs[GF_SLAB][GF_LD];  // v_i
   __shared__ float wsl[GF_SLAB];
   __shared__ int s_skip;
   const int tid = threadIdx.x;
@@ -112,39 +112,39 @@ __global__ void __launch_bounds__(GF_THREADS)
   for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
     const int l = item.plane / dm.Hkv, g = item.plane % dm.Hkv;
     const float* vbase = v + (int64_t)l * dm.kv_sl + (int64_t)g * dm.kv_sh;
-    float acc[8][8];
+    float2 acc[8][4];  // columns (2 q, 2 q + 1) of row p, packed multiply-adds
 #pragma unroll
     for (int a = 0; a < 8; ++a)
 #pragma unroll
-      for (int b = 0; b < 8; ++b) acc[a][b] = 0.f;
+      for (int b = 0; b < 4; ++b) acc[a][b] = make_float2(0.f, 0.f);
     for (int64_t t = item.t0; t < item.t1; t += GF_SLAB) {
       if (tid < GF_SLAB) {
         const int64_t tok = t + tid;
         wsl[tid] = tok < item.t1 ? ws.w[(int64_t)item.plane * dm.Ntot + tok] : 0.f;
       }
       __syncthreads();
-      for (int e = tid; e < GF_SLAB * (D / 4); e += GF_THREADS) {
+#pragma unroll
+      for (int e = tid; e < GF_SLAB * (D / 4); e += GF_THREADS) {  // all loads in flight before the stores
         const int r = e / (D / 4), c4 = (e % (D / 4)) * 4;
         const int64_t tok = t + r;
         float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
         if (tok < item.t1) x = *(const float4*)(vbase + tok * dm.kv_st + c4);
         const float wt = wsl[r];
-        vs[r][c4] = x.x; vs[r][c4 + 1] = x.y; vs[r][c4 + 2] = x.z; vs[r][c4 + 3] = x.w;
-        xs[r][c4] = wt * x.x; xs[r][c4 + 1] = wt * x.y; xs[r][c4 + 2] = wt * x.z; xs[r][c4 + 3] = wt * x.w;
+        *(float4*)&vs[r][c4] = x;
+        *(float4*)&xs[r][c4] = make_float4(wt * x.x, wt * x.y, wt * x.z, wt * x.w);
       }
       __syncthreads();
 #pragma unroll 4
       for (int r = 0; r < GF_SLAB; ++r) {
-        float a[8], b[8];
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          a[q] = vs[r][rb * 8 + q];
-          b[q] = xs[r][cb * 8 + q];
-        }
+        const float4 a0 = *(const float4*)&vs[r][rb * 8], a1 = *(const float4*)&vs[r][rb * 8 + 4];
+        const float4 b0 = *(const float4*)&xs[r][cb * 8], b1 = *(const float4*)&xs[r][cb * 8 + 4];
+        const float a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+        const float2 b[4] = {make_float2(b0.x, b0.y), make_float2(b0.z, b0.w), make_float2(b1.x, b1.y),
+                             make_float2(b1.z, b1.w)};
 #pragma unroll
         for (int p = 0; p < 8; ++p)
 #pragma unroll
-          for (int q = 0; q < 8; ++q) acc[p][q] = fmaf(a[p], b[q], acc[p][q]);
+          for (int q = 0; q < 4; ++q) acc[p][q] = __ffma2_rn(make_float2(a[p], a[p]), b[q], acc[p][q]);
       }
       __syncthreads();
     }
@@ -156,8 +156,8 @@ __global__ void __launch_bounds__(GF_THREADS)
       // (m, n) at ((n / 32) D + m) 32 + n % 32; the 8 columns share one block
       const int m = rb * 8 + p, n0 = cb * 8;
       float* row = dst + ((n0 >> 5) * D + m) * 32 + (n0 & 31);
-      *(float4*)row = make_float4(acc[p][0], acc[p][1], acc[p][2], acc[p][3]);
-      *(float4*)(row + 4) = make_float4(acc[p][4], acc[p][5], acc[p][6], acc[p][7]);
+      *(float4*)row = make_float4(acc[p][0].x, acc[p][0].y, acc[p][1].x, acc[p][1].y);
+      *(float4*)(row + 4) = make_float4(acc[p][2].x, acc[p][2].y, acc[p][3].x, acc[p][3].y);
     }
   }
 }

@@ -39,16 +39,18 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
 // the triangle get about the same work), four rows at once so their
 // multiply-add chains interleave, and the pair adds its squared norms.
 // L^{-1} is stored with zeros above the diagonal, so a quad may run its
-// columns up to its last row.
+// columns up to its last row. Four columns per step: one 16-byte load of each
+// of the quad's rows and of the token's row serves 16 multiply-adds (the
+// staged rows are 16-byte aligned).
 constexpr int SF_THREADS = 2 * TILE;
-constexpr int SF_LD = D + 1;
+constexpr int SF_LD = D + 4;
 constexpr size_t score_f32_smem_bytes() { return (size_t)(D * D + TILE * SF_LD) * sizeof(float); }
 
 __global__ void __launch_bounds__(SF_THREADS)
     score_f32_kernel(Dims dm, Ws ws, const int32_t* __restrict__ cu, const float* __restrict__ v,
                      float* __restrict__ scores) {
   pdl_wait();
-  extern __shared__ float ssm[];
+  extern __shared__ __align__(16) float ssm[];
   float* Mi = ssm;               // [D][D] L^{-1}
   float* vt = ssm + D * D;       // [TILE][SF_LD]
   __shared__ int s_skip;
@@ -66,18 +68,20 @@ __global__ void __launch_bounds__(SF_THREADS)
     const float* vbase = v + (int64_t)l * dm.kv_sl + (int64_t)g * dm.kv_sh;
     __syncthreads();
     if (u != loaded) {
+      // unrolled so that all of a thread's loads are in flight before its stores
       const float* src = ws.minv + u * D * D;
+#pragma unroll
       for (int e = tid * 4; e < D * D; e += SF_THREADS * 4) *(float4*)(Mi + e) = *(const float4*)(src + e);
       loaded = u;
     }
     for (int64_t t = item.t0; t < item.t1; t += TILE) {
       __syncthreads();
+#pragma unroll
       for (int e = tid; e < TILE * (D / 4); e += SF_THREADS) {
         const int r = e / (D / 4), c4 = (e % (D / 4)) * 4;
         float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
         if (t + r < item.t1) x = *(const float4*)(vbase + (t + r) * dm.kv_st + c4);
-        vt[r * SF_LD + c4] = x.x; vt[r * SF_LD + c4 + 1] = x.y;
-        vt[r * SF_LD + c4 + 2] = x.z; vt[r * SF_LD + c4 + 3] = x.w;
+        *(float4*)(vt + r * SF_LD + c4) = x;
       }
       __syncthreads();
       const float* vr = vt + tk * SF_LD;
@@ -87,12 +91,14 @@ __global__ void __launch_bounds__(SF_THREADS)
         // a full matrix with output directions
         const int cend = dm.dense_minv ? D : r0 + 4;
         float y0 = 0.f, y1 = 0.f, y2 = 0.f, y3 = 0.f;
-        for (int c = 0; c < cend; ++c) {
-          const float x = vr[c];
-          y0 = fmaf(m0[c], x, y0);
-          y1 = fmaf(m0[D + c], x, y1);
-          y2 = fmaf(m0[2 * D + c], x, y2);
-          y3 = fmaf(m0[3 * D + c], x, y3);
+        for (int c = 0; c < cend; c += 4) {  // cend is a multiple of 4
+          const float4 x = *(const float4*)(vr + c);
+          const float4 a0 = *(const float4*)(m0 + c), a1 = *(const float4*)(m0 + D + c);
+          const float4 a2 = *(const float4*)(m0 + 2 * D + c), a3 = *(const float4*)(m0 + 3 * D + c);
+          y0 = fmaf(a0.x, x.x, y0), y1 = fmaf(a1.x, x.x, y1), y2 = fmaf(a2.x, x.x, y2), y3 = fmaf(a3.x, x.x, y3);
+          y0 = fmaf(a0.y, x.y, y0), y1 = fmaf(a1.y, x.y, y1), y2 = fmaf(a2.y, x.y, y2), y3 = fmaf(a3.y, x.y, y3);
+          y0 = fmaf(a0.z, x.z, y0), y1 = fmaf(a1.z, x.z, y1), y2 = fmaf(a2.z, x.z, y2), y3 = fmaf(a3.z, x.z, y3);
+          y0 = fmaf(a0.w, x.w, y0), y1 = fmaf(a1.w, x.w, y1), y2 = fmaf(a2.w, x.w, y2), y3 = fmaf(a3.w, x.w, y3);
         }
         ssq = fmaf(y0, y0, fmaf(y1, y1, fmaf(y2, y2, fmaf(y3, y3, ssq))));
       }
