@@ -46,12 +46,16 @@ __device__ __forceinline__ void load_unit_stats(const Dims& dm, const Ws& ws, in
 // as a bf16 pair hi + lo in the stage for the scaling warps. The scaling warps
 // read V transposed with ldmatrix, form w_i v_i = hi + lo with packed bf16
 // arithmetic and store hi and lo as two A operands; two MMAs per 16 tokens
-// accumulate v (hi + lo)^T.
+// accumulate v hi^T and v lo^T, in two accumulators, each chain issued by a
+// warp of its own: one thread's MMAs of N <= 128 follow each other at ~60 ns
+// here whatever their accumulators, while two issuing threads overlap theirs.
+// The epilogue adds the two.
 // The scaling warps share nothing but the mbarriers of the pipeline. A run of
-// consecutive chunks of one unit in a CTA's item range accumulates in one
-// tensor-memory buffer; four epilogue warps copy each finished run's Gram out
-// while the next run accumulates in the other buffer.
-constexpr int GR_THREADS = 512;   // warp 0: TMA, 1: MMA, 2-9: scale, 10-13: epilogue, 14-15: weights
+// consecutive chunks of one unit in a CTA's item range accumulates in the
+// accumulator pair; four epilogue warps copy each finished run's Gram out
+// before the next run starts on it.
+constexpr int GR_THREADS = 544;   // warp 0: TMA, 1 and 16: MMA, 2-9: scale, 10-13: epilogue, 14-15: weights
+constexpr int GR_MMA_LO_WARP = 16;  // issues the v lo^T chain (warp 1 the v hi^T chain)
 constexpr int GR_EPI0 = 10;       // first epilogue warp
 constexpr int GR_WEIGHT_WARP = 14;  // 14 and 15, 64 tokens of each tile each
 constexpr int GR_SCALERS = 256;
@@ -59,8 +63,8 @@ constexpr int GR_BOX = 16384;      // {64 channels, 128 tokens} bf16, 128-byte s
 constexpr int GR_V_BYTES = 2 * GR_BOX;
 constexpr int GR_W_BYTES = 512;    // the tile's weights as bf16 pairs, one word per token
 constexpr uint32_t GR_TMEM_COLS = 512;
-constexpr uint32_t GR_ACOL = 128;  // A buffers: [128 + 128 ab, +64) hi, [+64, +128) lo
-constexpr uint32_t GR_DCOL1 = 384; // accumulators: columns [0, 128) and [384, 512), alternating by item
+constexpr uint32_t GR_DLO = 128;   // accumulators: columns [0, 128) v hi^T, [128, 256) v lo^T
+constexpr uint32_t GR_ACOL = 256;  // A buffers: [256 + 128 ab, +64) hi, [+64, +128) lo
 // M = 128 (channels), N = 128 (channels), A in TMEM (K-major), B MN-major.
 constexpr uint32_t GR_IDESC = idesc_bf16_f32(128, 128, 0, 1);
 
@@ -118,8 +122,8 @@ __device__ __forceinline__ void gram_bf16_body(const CUtensorMap* vmap_p, const 
   uint64_t* wready = vempty + GR_VST;  // the weight warp has written the tile's weights
   uint64_t* afull = wready + GR_VST;
   uint64_t* aempty = afull + 2;
-  uint64_t* accfull = aempty + 2;   // [2]
-  uint64_t* accempty = accfull + 2; // [2]
+  uint64_t* accfull = aempty + 2;   // the run's Gram is complete in the accumulators
+  uint64_t* accempty = accfull + 1; // the epilogue has read them
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort, s_skip;
 
@@ -129,17 +133,15 @@ __device__ __forceinline__ void gram_bf16_body(const CUtensorMap* vmap_p, const 
     s_skip = status_failed(ws) ? 1 : 0;
     for (int i = 0; i < GR_VST; ++i) {
       mbar_init(smem_u32(&vfull[i]), 1);
-      mbar_init(smem_u32(&vempty[i]), 1);
+      mbar_init(smem_u32(&vempty[i]), 2);  // the two MMA warps' commits
       mbar_init(smem_u32(&wready[i]), 2);  // the two weight warps
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&afull[i]), GR_SCALERS / 32);
-      mbar_init(smem_u32(&aempty[i]), 1);
+      mbar_init(smem_u32(&aempty[i]), 2);  // the two MMA warps' commits
     }
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(smem_u32(&accfull[i]), 1);
-      mbar_init(smem_u32(&accempty[i]), 4);  // the epilogue warps
-    }
+    mbar_init(smem_u32(accfull), 2);   // the two MMA warps' commits
+    mbar_init(smem_u32(accempty), 4);  // the epilogue warps
     fence_mbar_init();
   }
   __syncthreads();
@@ -204,29 +206,28 @@ __device__ __forceinline__ void gram_bf16_body(const CUtensorMap* vmap_p, const 
       for (uint32_t k = (it > (uint32_t)GR_VST ? it - GR_VST : 0); k < it; ++k)
         mbar_wait(smem_u32(&vfull[k % GR_VST]), (k / GR_VST) & 1, ws, nullptr);
     }
-  } else if (warp == 1) {
-    // ------------------------------------------------ MMA issuer ----------
+  } else if (warp == 1 || warp == GR_MMA_LO_WARP) {
+    // ------------------------------------------------ MMA issuers ---------
     if (lane == 0) {
+      const bool lo = warp == GR_MMA_LO_WARP;  // the v lo^T chain
       // time accounting (trace builds): 2 waits for a scaled operand, 3 for a free
       // accumulator (run start), 4 the whole loop, 5 tiles
       TRC_DECL(TR_CTA_SLOTS);
       TRC_T(tr_all);
       uint32_t it = 0, nrun = 0;
       bool ok = true, cont = false, first = true;
-      int db = 0;
       Item item;
       for (ItemStream is(dm, ws, part, parts, FUSED); ok && is.next(item);) {
-        // one accumulator per run of consecutive chunks of a unit; a new run
-        // takes the other buffer once its previous run's epilogue is done
+        // a run of consecutive chunks of a unit accumulates in the accumulator
+        // pair; a new run starts on it once the previous run's epilogue has read it
         if (!cont) {
-          db = nrun & 1;
           TRC_T(tr_a);
-          if (nrun >= 2 && !mbar_wait(smem_u32(&accempty[db]), ((nrun >> 1) & 1) ^ 1, ws, abort)) break;
+          if (nrun >= 1 && !mbar_wait(smem_u32(accempty), (nrun - 1) & 1, ws, abort)) break;
           TRC_ADD(3, tr_a);
           tc_fence_after();
           first = true;
         }
-        const uint32_t dacc = tmem + (db ? GR_DCOL1 : 0u);
+        const uint32_t dacc = tmem + (lo ? GR_DLO : 0u);
         for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
           const int vs = it % GR_VST, ab = it & 1;
           // the scaling warps arrive on afull only after the tile's V landed
@@ -240,12 +241,11 @@ __device__ __forceinline__ void gram_bf16_body(const CUtensorMap* vmap_p, const 
           tc_fence_after();
           // B descriptors advance by (byte offset >> 4) in their address field
           const uint64_t b0 = smem_desc_sw128(smem_u32(vring + vs * GR_V_BYTES), GR_BOX, 1024);
-          const uint32_t acol = tmem + GR_ACOL + 128 * ab;
+          const uint32_t acol = tmem + GR_ACOL + 128 * ab + (lo ? 64u : 0u);  // hi or lo
 #pragma unroll
           for (int k = 0; k < TILE / 16; ++k) {  // 16 tokens per MMA
             const uint64_t bd = b0 + (uint64_t)((k * 2048) >> 4);
             umma_f16_ts(dacc, acol + 8 * k, bd, GR_IDESC, (first && k == 0) ? 0u : 1u);
-            umma_f16_ts(dacc, acol + 64 + 8 * k, bd, GR_IDESC, 1u);
           }
           first = false;
           umma_commit(smem_u32(&vempty[vs]));
@@ -254,13 +254,13 @@ __device__ __forceinline__ void gram_bf16_body(const CUtensorMap* vmap_p, const 
         if (!ok) break;
         cont = is.next_same_unit(item);
         if (!cont) {
-          umma_commit(smem_u32(&accfull[db]));
+          umma_commit(smem_u32(accfull));
           ++nrun;
         }
       }
       if (it > 0) mbar_wait(smem_u32(&aempty[(it - 1) & 1]), ((it - 1) >> 1) & 1, ws, nullptr);
       TRC_ADD(4, tr_all);
-      TRC_PUT(ws, TR_K_GRAM, 6);
+      if (!lo) TRC_PUT(ws, TR_K_GRAM, 6);
     }
   } else if (warp < 10) {
     // ------------------------------------------------- scaling warps ------
@@ -306,28 +306,35 @@ __device__ __forceinline__ void gram_bf16_body(const CUtensorMap* vmap_p, const 
         tc_fence_after();
         const uint32_t vt = smem_u32(vring + vs * GR_V_BYTES);
         const uint32_t acol = tmem + GR_ACOL + 128 * ab;
+        // the tile's V fragments of this warp, all eight loads in flight
+        // before any arithmetic or tensor-memory store (each store orders the
+        // code around it); matrices: 0 = (tokens 0-7, ch c0..c0+7),
+        // 1 = (tokens 0-7, c0+8..), 2 = (8-15, c0..), 3 = (8-15, c0+8..)
+        uint32_t r[2][4][4];
+#pragma unroll
+        for (int lh = 0; lh < 2; ++lh)
+#pragma unroll
+          for (int blk = 0; blk < 4; ++blk) {
+            const int b = 4 * th + blk;  // 16-token block of the tile
+            const int c0 = quarter * 32 + lh * 16 + (lm & 1) * 8;
+            const int tokr = 16 * b + (lm >> 1) * 8 + lr;
+            const uint32_t addr = vt + (c0 >> 6) * GR_BOX + sw128_off(tokr, (c0 & 63) >> 3);
+            ldsm_x4_trans(addr, r[lh][blk][0], r[lh][blk][1], r[lh][blk][2], r[lh][blk][3]);
+          }
 #pragma unroll
         for (int lh = 0; lh < 2; ++lh) {
           // one 32-column slab (this warp's 4 token blocks) of hi and of lo,
           // built in registers and written with one wide store each
           uint32_t hi[16], lo[16];
 #pragma unroll
-          for (int blk = 0; blk < 4; ++blk) {
-            const int b = 4 * th + blk;  // 16-token block of the tile
-            // matrices: 0 = (tokens 0-7, ch c0..c0+7), 1 = (tokens 0-7, c0+8..), 2 = (8-15, c0..), 3 = (8-15, c0+8..)
-            const int c0 = quarter * 32 + lh * 16 + (lm & 1) * 8;
-            const int tokr = 16 * b + (lm >> 1) * 8 + lr;
-            const uint32_t addr = vt + (c0 >> 6) * GR_BOX + sw128_off(tokr, (c0 & 63) >> 3);
-            uint32_t r[4];
-            ldsm_x4_trans(addr, r[0], r[1], r[2], r[3]);
+          for (int blk = 0; blk < 4; ++blk)
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
               // w v = hi + lo; registers (r0 = lanes 0-7, r1 = lanes 8-15) of
               // columns 8 blk + 4 (q / 2) ..
               const int e = 4 * blk + 2 * (q >> 1) + (q & 1);
-              bf16x2_scale_split(wph[2 * blk + (q >> 1)], wpl[2 * blk + (q >> 1)], r[q], hi[e], lo[e]);
+              bf16x2_scale_split(wph[2 * blk + (q >> 1)], wpl[2 * blk + (q >> 1)], r[lh][blk][q], hi[e], lo[e]);
             }
-          }
           const uint32_t lanes = (uint32_t)(quarter * 32 + lh * 16) << 16;
           tmem_st_16x128b_x8(acol + lanes + 32 * th, hi);
           tmem_st_16x128b_x8(acol + lanes + 64 + 32 * th, lo);
@@ -342,7 +349,7 @@ __device__ __forceinline__ void gram_bf16_body(const CUtensorMap* vmap_p, const 
   scale_done:;
     TRC_ADD(10, tr_all);
     if (warp == 2 && lane == 0) TRC_PUT(ws, TR_K_GRAM, 11);
-  } else if (warp >= GR_WEIGHT_WARP) {
+  } else if (warp == GR_WEIGHT_WARP || warp == GR_WEIGHT_WARP + 1) {
     // ------------------------------------------------------ weights -------
     // Eq. 8 for the tile's tokens (two per lane of each of the two warps) from the staged logits and
     // kappa: w = wdiv sum_h rho_h^2 kappa_h, rho = alpha_bar (1 - alpha_bar),
@@ -416,11 +423,12 @@ __device__ __forceinline__ void gram_bf16_body(const CUtensorMap* vmap_p, const 
     if (bad) flag(ws, ST_NONFINITE);
   } else {
     // ------------------------------------------------------ epilogue ------
-    // D is a chunk's partial Gram; warp (quarter q) copies rows 32 q .. +31,
-    // each lane its row: 32 consecutive floats per column block, so a lane
-    // writes 128 contiguous bytes per block. The Gram is symmetric and its
-    // consumers read the lower triangle only, so only the column blocks
-    // cb <= q (the lower 32 x 32 blocks) are written.
+    // The accumulator pair holds a run's partial Gram (v hi^T + v lo^T); warp
+    // (quarter q) copies rows 32 q .. +31, each lane its row: 32 consecutive
+    // floats per column block, so a lane writes 128 contiguous bytes per
+    // block. The Gram is symmetric and its consumers read the lower triangle
+    // only, so only the column blocks cb <= q (the lower 32 x 32 blocks) are
+    // written.
     const int quarter = warp & 3;
     const int m = quarter * 32 + lane;
     uint32_t nrun = 0;
@@ -438,23 +446,24 @@ __device__ __forceinline__ void gram_bf16_body(const CUtensorMap* vmap_p, const 
       if (warp == GR_EPI0 && lane == 0) ws.pflag[(int64_t)item.plane * dm.c_cap + item.cidx] = cont ? 0 : 1;
       cont = is.next_same_unit(item);
       if (cont) continue;
-      const int db = nrun & 1;
-      if (!mbar_wait(smem_u32(&accfull[db]), (nrun >> 1) & 1, ws, abort)) break;
+      if (!mbar_wait(smem_u32(accfull), nrun & 1, ws, abort)) break;
       tc_fence_after();
-      const uint32_t trow = tmem + (db ? GR_DCOL1 : 0u) + ((uint32_t)(quarter * 32) << 16);
+      const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
       float* dst = ws.gpart + ((int64_t)item.plane * dm.c_cap + run_cidx) * D * D + (int64_t)m * 32;
 #pragma unroll 1
       for (int cb = 0; cb <= quarter; ++cb) {
-        float a[32];
+        float a[32], b[32];
         tmem_ld32(trow + cb * 32, a);
+        tmem_ld32(trow + GR_DLO + cb * 32, b);
 #pragma unroll
         for (int j = 0; j < 32; j += 4)
-          *(float4*)(dst + cb * D * 32 + j) = make_float4(a[j], a[j + 1], a[j + 2], a[j + 3]);
+          *(float4*)(dst + cb * D * 32 + j) =
+              make_float4(a[j] + b[j], a[j + 1] + b[j + 1], a[j + 2] + b[j + 2], a[j + 3] + b[j + 3]);
       }
       tc_fence_before();
       if (FUSED) __threadfence();  // this warp's rows of the partial (and the pflag entries) are visible
       __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&accempty[db]));
+      if (lane == 0) mbar_arrive(smem_u32(accempty));
       if (FUSED && lane == 0) {
         red_add_release_gpu(ws.gcount + (int64_t)item.plane * dm.S + item.seq, run_items);
         JACAP_TRACE_MAX(ws, (int64_t)item.plane * dm.S + item.seq, TR_GRAM1);
