@@ -269,9 +269,10 @@ TRACE_CTA_SLOTS = {
     2: ("k_pass", {0: "producer: wait for a free stage", 1: "producer: loop", 2: "logits MMA: wait for an image",
                    3: "logits MMA: wait for a K tile and a free buffer", 5: "logits MMA: loop", 6: "tiles",
                    7: "kappa warp: wait for a K tile", 8: "kappa warp: its quarter of kappa",
-                   9: "kappa warp: first group barrier", 10: "kappa warp: reduction and store", 11: "kappa warp: loop",
-                   12: "readout warp: wait for logits", 13: "readout warp: readout of a tile",
-                   14: "readout warp: loop"}),
+                   9: "kappa warp: wait for the group's slot", 10: "kappa warp: partials into the slot",
+                   11: "kappa warp: loop", 12: "readout warp: wait for logits",
+                   13: "readout warp: readout of a tile", 14: "readout warp: loop",
+                   15: "readout warp: wait for the kappa partials"}),
     0: ("gram", {0: "producer: wait for a free stage", 1: "producer: loop", 2: "MMA: wait for a scaled operand",
                  3: "MMA: wait for a free accumulator", 4: "MMA: loop", 5: "tiles", 6: "scaling warp: wait for V",
                  7: "scaling warp: wait for the weights", 8: "scaling warp: wait for a free operand buffer",

@@ -21,9 +21,12 @@
 // unit's consecutive items ahead); 2-9 kappa (two groups of four warps alternate
 // tiles; in a group each warp takes one quarter of the channels for all 128
 // tokens, four per lane, so every lambda value read from shared memory serves
-// four tokens; the quarters are reduce-scattered through shared memory);
-// 10-13 read the logits back from tensor memory (one lane quarter each) and
-// keep the online softmax statistics.
+// four tokens, and writes its partial sums of all four token subsets into the
+// group's slot); 10-13 read the logits back from tensor memory (one lane
+// quarter each), add the four partial kappa of their 32 tokens from the slot,
+// keep the online softmax statistics and store each token's row (logits,
+// kappa) in one piece. Each group has two slots (one for G > 4), handed over
+// with mbarriers, so a group writes one while the readout warps read the other.
 #include "jacap_dev.cuh"
 #include "jacap_internal.h"
 
@@ -42,14 +45,18 @@ struct KbCfg {
   static constexpr int IMG_ATOM = NB * 128;            // bytes per 64-channel atom
   static constexpr int IMG_BYTES = 2 * IMG_ATOM;
   static constexpr int LAM_BYTES = G * D * 4;          // lambda, fp32 [G][128]
-  static constexpr int KRED_FLOATS = 2 * 4 * 4 * G * 32;  // [group][token subset][writer][G][32]
+  // partial-kappa slots per group: two (the group writes one while the readout
+  // warps read the other) when they fit beside five K stages, else one
+  static constexpr int SLOTS = G <= 4 ? 2 : 1;
+  static constexpr int SLOT_FLOATS = 4 * 4 * G * 32;                 // [token subset][writer][G][32]
+  static constexpr int KRED_FLOATS = 2 * SLOTS * SLOT_FLOATS;        // [group][slot]
   static constexpr uint32_t IDESC = idesc_bf16_f32(128, NB, 0, 0);
   static_assert(KB_NACC * NB <= (int)KB_TMEM_COLS, "tensor memory budget");
   static constexpr size_t smem_for(int stages) {
     return 1024 + (size_t)stages * KB_TILE_BYTES + 2 * IMG_BYTES + 2 * LAM_BYTES + KRED_FLOATS * 4 + 4 * 2 * G * 4 +
            512;
   }
-  static constexpr int STAGES = smem_for(6) <= 232448 ? 6 : 5;  // K tiles in flight
+  static constexpr int STAGES = smem_for(6) <= 232448 ? 6 : (smem_for(5) <= 232448 ? 5 : 4);  // K tiles in flight
   static constexpr size_t SMEM = smem_for(STAGES);
 };
 
@@ -150,6 +157,8 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
   uint64_t* accempty = accfull + KB_NACC;
   uint64_t* imgready = accempty + KB_NACC;
   uint64_t* imgfree = imgready + 2;
+  uint64_t* kready = imgfree + 2;            // [group][slot] a tile's partial kappa are in the slot
+  uint64_t* kfree = kready + 2 * C::SLOTS;   // [group][slot] the readout warps have read them
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort, s_skip;
 
@@ -168,6 +177,11 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&imgready[i]), 1);
       mbar_init(smem_u32(&imgfree[i]), 9);  // MMA commit + the eight kappa warps
+
+    }
+    for (int i = 0; i < 2 * C::SLOTS; ++i) {
+      mbar_init(smem_u32(&kready[i]), 4);  // the group's four kappa warps
+      mbar_init(smem_u32(&kfree[i]), 4);   // the four readout warps
     }
     fence_mbar_init();
   }
@@ -296,77 +310,57 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
     }
   } else if (warp >= KB_KAPPA_WARP0 && warp < KB_READ_WARP0) {
     // ------------------------------------------------------ kappa ---------
+    // A group's warp writes its partial kappa of all four token subsets into
+    // the group's slot and signals kready; the readout warp of each subset
+    // adds the four partials (in writer order) and stores the token's row.
     const int kw = warp - KB_KAPPA_WARP0;
     const int grp = kw >> 2;                  // tiles with it % 2 == grp
-    const int cq = kw & 3;                    // channel quarter; also the token subset finished here
-    const int bar_id = 2 + grp;               // the four warps of the group
-    float* slot = kred + grp * (4 * 4 * G * 32);
-    uint32_t it = 0, nrun = 0;
-    bool bad = false, cont = false;
+    const int cq = kw & 3;                    // channel quarter
+    uint32_t it = 0, nrun = 0, ng = 0;        // ng: tiles of this group so far
+    bool cont = false;
     int p = 0;
     Item item;
     // time accounting (trace builds, warp 2): 7 waits for a K tile, 8 its quarter
-    // of kappa, 9 the first group barrier, 10 the reduction and the store, 11 the loop
+    // of kappa, 9 waits for the group's slot, 10 the partials into it, 11 the loop
     TRC_DECL(TR_CTA_SLOTS);
     TRC_T(tr_all);
-    // A failed wait (which means the abort flag is set) still arrives at the
-    // group's named barriers, which OR the flag over the group, so the four
-    // warps leave together after the same barrier. All four see the same runs
-    // (the same item stream), so they meet at the same barriers.
+    // Every wait is bounded and the warps meet at no named barrier, so a warp
+    // whose wait failed (the abort flag is set) leaves on its own.
     for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
       if (!cont) {
         p = nrun & 1;
-        mbar_wait(smem_u32(&imgready[p]), (nrun >> 1) & 1, ws, abort);
-        if (named_barrier_any(bar_id, 128, *abort != 0)) goto kappa_done;
+        if (!mbar_wait(smem_u32(&imgready[p]), (nrun >> 1) & 1, ws, abort)) goto kappa_done;
       }
       {
         const uint32_t lam_s = smem_u32(lams + p * G * D);
-        float* lkp = ws.lk + (int64_t)item.plane * dm.Ntot * (2 * G) + G;
         for (int64_t t = item.t0; t < item.t1; t += TILE, ++it) {
           if ((int)(it & 1) != grp) continue;
           const int st = it % KB_STAGES;
           float part[4][G];
           TRC_T(tr_f);
-          if (mbar_wait(smem_u32(&full[st]), (it / KB_STAGES) & 1, ws, abort)) {
-            TRC_ADD(7, tr_f);
-            TRC_T(tr_k);
-            kappa_quarter<G>(smem_u32(tiles + st * KB_TILE_BYTES), lam_s, lane, cq, part);
-            TRC_ADD(8, tr_k);
-            __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&empty[st]));
-            // hand the other three token subsets to their owners
-#pragma unroll
-            for (int j = 0; j < 4; ++j)
-              if (j != cq)
-#pragma unroll
-                for (int h = 0; h < G; ++h) slot[((j * 4 + cq) * G + h) * 32 + lane] = part[j][h];
-          }
+          if (!mbar_wait(smem_u32(&full[st]), (it / KB_STAGES) & 1, ws, abort)) goto kappa_done;
+          TRC_ADD(7, tr_f);
+          TRC_T(tr_k);
+          kappa_quarter<G>(smem_u32(tiles + st * KB_TILE_BYTES), lam_s, lane, cq, part);
+          TRC_ADD(8, tr_k);
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&empty[st]));
           TRC_T(tr_b);
-          const bool stop = named_barrier_any(bar_id, 128, *abort != 0);
+          // slot b of the group takes its tiles ng = b, b + SLOTS, ...; it is free
+          // once the readout warps have read its previous tile
+          const int b = ng % C::SLOTS, use = ng / C::SLOTS;
+          const int ks = grp * C::SLOTS + b;
+          if (use >= 1 && !mbar_wait(smem_u32(&kfree[ks]), (use - 1) & 1, ws, abort)) goto kappa_done;
           TRC_ADD(9, tr_b);
           TRC_T(tr_r);
-          if (stop) goto kappa_done;
-          float kap[G];
+          float* slot = kred + ks * C::SLOT_FLOATS;
 #pragma unroll
-          for (int h = 0; h < G; ++h) {
-            // own subset cq: add the other quarters' partial sums in writer order
-            float v = 0.f;
+          for (int j = 0; j < 4; ++j)
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-              float x;
-              if (q == cq) {
-                x = part[cq][h];
-              } else {
-                x = slot[((cq * 4 + q) * G + h) * 32 + lane];
-              }
-              v += x;
-            }
-            kap[h] = v;
-            bad |= !isfinite(v);
-          }
-          named_barrier_sync(bar_id, 128);  // the slots may be rewritten after this
-          const int64_t tok = t + lane + 32 * cq;
-          if (tok < item.t1) store_floats<G, LkAlign<G>::KAPPA>(lkp + tok * (2 * G), kap);
+            for (int h = 0; h < G; ++h) slot[((j * 4 + cq) * G + h) * 32 + lane] = part[j][h];
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&kready[ks]));
+          ++ng;
           TRC_ADD(10, tr_r);
         }
       }
@@ -380,7 +374,6 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
   kappa_done:
     TRC_ADD(11, tr_all);
     if (warp == KB_KAPPA_WARP0 && lane == 0) TRC_PUT(ws, TR_K_KPASS, 12);
-    if (bad) flag(ws, ST_NONFINITE);
   } else if (warp >= KB_READ_WARP0 && warp < KB_READ_WARP0 + 4) {
     // ------------------------------------------ logits readout + stats ----
     const int quarter = warp & 3;
@@ -392,7 +385,7 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
     float run_m[G], run_s[G];
     Item item;
     // time accounting (trace builds, first readout warp): 12 waits for logits, 13 the
-    // readout of a tile, 14 the whole loop
+    // readout of a tile (with 15, its wait for the kappa partials), 14 the whole loop
     TRC_DECL(TR_CTA_SLOTS);
     TRC_T(tr_all);
     for (ItemStream is(dm, ws, blockIdx.x, gridDim.x); is.next(item);) {
@@ -417,21 +410,39 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_u32(&accempty[ab]));
+        // kappa of this warp's 32 tokens: the four partials of the tile's group
+        // (the group's slot holds [token subset][writer][G][32]), added in writer order
+        const uint32_t ng = it >> 1;  // the tile is the ng-th of group it % 2
+        const int ks = (int)(it & 1) * C::SLOTS + (int)(ng % C::SLOTS);
+        TRC_T(tr_k);
+        if (!mbar_wait(smem_u32(&kready[ks]), (ng / C::SLOTS) & 1, ws, abort)) break;  // abort: see below
+        TRC_ADD(15, tr_k);
+        const float* slot = kred + ks * C::SLOT_FLOATS;
+        float row[2 * G];  // logits, then kappa
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+          float v = 0.f;
+#pragma unroll
+          for (int q = 0; q < 4; ++q) v += slot[((quarter * 4 + q) * G + h) * 32 + lane];
+          row[G + h] = v;
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&kfree[ks]));
         const int64_t tok = t + y;
         if (tok < item.t1) {
-          float lg[G];
 #pragma unroll
           for (int h = 0; h < G; ++h) {
-            lg[h] = dv[h] + dv[G + h] + dv[2 * G + h];
-            bad |= !isfinite(lg[h]);
+            const float lg = dv[h] + dv[G + h] + dv[2 * G + h];
+            row[h] = lg;
+            bad |= !isfinite(lg) || !isfinite(row[G + h]);
             // branch-free online update: one of the two exponentials is exp(0);
             // both arguments are <= 0, where the fast exponential's relative
             // error (a few ulp) is far below what the statistics need
-            const float mn = fmaxf(run_m[h], lg[h]);
-            run_s[h] = run_s[h] * __expf(run_m[h] - mn) + __expf(lg[h] - mn);
+            const float mn = fmaxf(run_m[h], lg);
+            run_s[h] = run_s[h] * __expf(run_m[h] - mn) + __expf(lg - mn);
             run_m[h] = mn;
           }
-          store_floats<G, LkAlign<G>::ROW>(lkp + tok * (2 * G), lg);
+          store_floats<2 * G, LkAlign<G>::ROW>(lkp + tok * (2 * G), row);
         }
         TRC_ADD(13, tr_b);
       }
@@ -469,7 +480,7 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
     }
   read_done:
     TRC_ADD(14, tr_all);
-    if (warp == KB_READ_WARP0 && lane == 0) TRC_PUT(ws, TR_K_KPASS, 15);
+    if (warp == KB_READ_WARP0 && lane == 0) TRC_PUT(ws, TR_K_KPASS, 16);
     if (bad) flag(ws, ST_NONFINITE);
   }
   tc_fence_before();
