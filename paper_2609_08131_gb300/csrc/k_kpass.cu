@@ -60,6 +60,19 @@ struct KbCfg {
   static constexpr size_t SMEM = smem_for(STAGES);
 };
 
+// The K tile `it` lands on barrier full[kb_full(it)], one per (tile parity,
+// stage). A kappa group takes every other tile, so with an odd number of
+// stages it sees only every other use of a stage; on a barrier per stage its
+// parity wait could not tell "my tile landed" from "the other group's tile in
+// this stage has not landed yet". Per (parity, stage) every waiter sees
+// consecutive phases: the tile's use of its barrier is it / kb_full_period.
+template <int STAGES>
+__device__ __forceinline__ int kb_full(uint32_t it) { return (int)(it & 1) * STAGES + (int)(it % STAGES); }
+template <int STAGES>
+__device__ __forceinline__ uint32_t kb_full_parity(uint32_t it) {
+  return (it / (STAGES % 2 == 0 ? STAGES : 2 * STAGES)) & 1;
+}
+
 // mu' image of one item: rows n = part * G + h hold part (0 hi, 1 mid, 2 lo) of
 // src[h][0..127], K-major with the 128-byte swizzle (two 64-channel atoms).
 template <int G>
@@ -151,8 +164,8 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
   float* lams = (float*)(img + 2 * C::IMG_BYTES);       // [parity][G][128] lambda
   float* kred = lams + 2 * G * D;                        // partial kappa of the upper channel half
   float* red = kred + C::KRED_FLOATS;                    // [4 readout warps][2G]
-  uint64_t* full = (uint64_t*)(red + 4 * 2 * G);
-  uint64_t* empty = full + KB_STAGES;
+  uint64_t* full = (uint64_t*)(red + 4 * 2 * G);  // [tile parity][stage], see kb_full
+  uint64_t* empty = full + 2 * KB_STAGES;
   uint64_t* accfull = empty + KB_STAGES;
   uint64_t* accempty = accfull + KB_NACC;
   uint64_t* imgready = accempty + KB_NACC;
@@ -168,6 +181,7 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
     s_skip = status_failed(ws) ? 1 : 0;
     for (int i = 0; i < KB_STAGES; ++i) {
       mbar_init(smem_u32(&full[i]), 1);
+      mbar_init(smem_u32(&full[KB_STAGES + i]), 1);
       mbar_init(smem_u32(&empty[i]), 5);  // MMA commit + the four kappa warps of the tile
     }
     for (int i = 0; i < KB_NACC; ++i) {
@@ -219,16 +233,17 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
           }
           TRC_ADD(0, tr_w);
           uint8_t* kt = tiles + st * KB_TILE_BYTES;
-          mbar_arrive_expect_tx(smem_u32(&full[st]), KB_TILE_BYTES);
-          tma_load_4d(smem_u32(kt), &kmap, 0, (int)t, g, l, smem_u32(&full[st]));
-          tma_load_4d(smem_u32(kt + KB_BOX), &kmap, 64, (int)t, g, l, smem_u32(&full[st]));
+          const uint32_t fb = smem_u32(&full[kb_full<KB_STAGES>(it)]);
+          mbar_arrive_expect_tx(fb, KB_TILE_BYTES);
+          tma_load_4d(smem_u32(kt), &kmap, 0, (int)t, g, l, fb);
+          tma_load_4d(smem_u32(kt + KB_BOX), &kmap, 64, (int)t, g, l, fb);
           ++it;
         }
       }
       TRC_ADD(1, tr_all);
       TRC_PUT(ws, TR_K_KPASS, 2);
       for (uint32_t k = (it > (uint32_t)KB_STAGES ? it - KB_STAGES : 0); k < it; ++k)
-        mbar_wait(smem_u32(&full[k % KB_STAGES]), (k / KB_STAGES) & 1, ws, nullptr);
+        mbar_wait(smem_u32(&full[kb_full<KB_STAGES>(k)]), kb_full_parity<KB_STAGES>(k), ws, nullptr);
     }
   } else if (warp == 1) {
     // ------------------------------------------------ logits MMA issuer ---
@@ -254,7 +269,7 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
           const int st = it % KB_STAGES;
           const int ab = it % KB_NACC;
           TRC_T(tr_f);
-          if (!mbar_wait(smem_u32(&full[st]), (it / KB_STAGES) & 1, ws, abort) ||
+          if (!mbar_wait(smem_u32(&full[kb_full<KB_STAGES>(it)]), kb_full_parity<KB_STAGES>(it), ws, abort) ||
               (it >= (uint32_t)KB_NACC &&
                !mbar_wait(smem_u32(&accempty[ab]), ((it / KB_NACC) & 1) ^ 1, ws, abort))) {
             ok = false;
@@ -338,7 +353,8 @@ __global__ void __launch_bounds__(KB_THREADS, 1)
           const int st = it % KB_STAGES;
           float part[4][G];
           TRC_T(tr_f);
-          if (!mbar_wait(smem_u32(&full[st]), (it / KB_STAGES) & 1, ws, abort)) goto kappa_done;
+          if (!mbar_wait(smem_u32(&full[kb_full<KB_STAGES>(it)]), kb_full_parity<KB_STAGES>(it), ws, abort))
+            goto kappa_done;
           TRC_ADD(7, tr_f);
           TRC_T(tr_k);
           kappa_quarter<G>(smem_u32(tiles + st * KB_TILE_BYTES), lam_s, lane, cq, part);
