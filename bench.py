@@ -707,19 +707,7 @@ def run_e2e(args, ev, t, stream, world, dist):
         torch.cuda.synchronize()
         return 3 * grp.numel() * grp.element_size() / (a.elapsed_time(b) * 1e-3) / 1e9
 
-    # Right after seconds of heavy GPU work these hosts' copies run at 70-120 GB/s for some
-    # seconds before they return to the link's rate: probe every 0.5 s, for 20 s at most,
-    # until three probes in a row agree within 5 %, and record how long that took.
-    import time
-
-    t_settle = time.perf_counter()
-    rates = [link()]
-    while time.perf_counter() - t_settle < 20.0 and not (
-            len(rates) >= 3 and max(rates[-3:]) <= 1.05 * min(rates[-3:])):
-        time.sleep(0.5)
-        rates.append(link())
-    settle_s = time.perf_counter() - t_settle
-    link_gbs = rates[-1]
+    link_gbs = link()
     if dist is not None:
         dist.barrier()
     a.record(stream)
@@ -750,7 +738,6 @@ def run_e2e(args, ev, t, stream, world, dist):
     return {"value": sum(t.seqlens) * L * world / (ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": he.h2d_bytes,
             "d2h_bytes_per_step": he.d2h_bytes, "ms_per_step": ms, "steps": n, "group_layers": he.gl,
             "idx_differ_vs_resident": differ, "h2d_link_gbs": link_gbs, "h2d_link_after_gbs": link_after_gbs,
-            "h2d_link_first_gbs": rates[0], "h2d_settle_s": round(settle_s, 2),
             "h2d_achieved_gbs": he.h2d_bytes / (ms * 1e-3) / 1e9,
             "h2d_bound_ms": he.h2d_bytes / (link_gbs * 1e9) * 1e3, "api": "jacap_evict_host (C ABI)",
             "returns": "kept positions and the retained K and V rows, in pinned host memory"}
